@@ -1,0 +1,343 @@
+"""CPU oracle for SmartVL's budget-conditioned gated prefill (TEST INFRASTRUCTURE).
+
+This module is test infrastructure. Only the test suite, the smoke check and
+the benchmark's CPU-baseline leg may import it; the product path never does.
+It shares no code with the CUDA library: every step is written here again,
+plainly, from the paper ("Look Less, Think Faster: Joint Token-Compute
+Adaptation for Multimodal LLMs", arXiv 2607.20357).
+
+Arithmetic is float64 throughout. A storage mode rounds the tensors that the
+GPU stores in memory: ``"fp64"`` (no rounding), ``"fp32"`` or ``"bf16"``
+(round-to-nearest-even emulation of bfloat16 storage). Token logits are never
+rounded.
+
+What each function follows:
+
+* ``sinusoidal_encoding`` / ``budget_embedding`` -- Eq. 5 (PE and MLP of the
+  scalar budget, Sec. 3.1), reused on the LLM side (Sec. 3.2).
+* ``token_logits`` -- Sec. 3.1, per-token logits z; the scorer is a per-token
+  MLP conditioned additively on the budget embedding (reading R1).
+* ``prefill_cost_xG`` -- Eq. 8 with integer arithmetic (scaled by G so that
+  alpha_l = (sum_j M_lj)/G is exact); 8D^2 generalised to 4D^2 + 4 D D_kv.
+* ``budget_keep_count`` -- Sec. 3.3 "Inference": the budget projection drops
+  the lowest-confidence visual tokens first, i.e. the largest token count that
+  keeps Eq. 8 within b * C_full (Eq. 2).
+* ``select_kept`` -- Sec. 3.1 inference rule: discard the lowest-confidence
+  tokens, keep the rest as a contiguous sequence in image order.
+* ``pack_sample`` -- Sec. 3 problem statement S = S_text + S_vis; kept visual
+  tokens (through the LLaVA MLP projector) followed by the text tokens, with
+  positions 0..S-1 (Sec. 3.1: RoPE on the compressed contiguous sequence).
+* ``decoder_layer`` -- Sec. 3.2 gating: group j of layer l switches its
+  attention heads and its slice of FFN channels together; alpha_l = 0 skips
+  the layer through its residual connection. Gated-off parts contribute zero
+  (masked-dense definition).
+* ``forward_sample`` / ``forward_batch`` -- the whole path, sample by sample.
+
+Pins (checked by ``tests/test_oracle_pins.py``, all CPU): brute-force subset
+selection, closed-form budget inversion, an operation counter against Eq. 8,
+an independent dense transformer written with library routines, zeroed-weight
+and removed-layer equivalences, shortened-sequence equivalence, batch
+independence, and the paper's "full 8.5T" LLaVA-1.5-7B figure (Sec. 1).
+The accuracy of the learned policy itself is parity unpinned: the paper's
+trained weights are not available, so no printed end-to-end value exists.
+"""
+from __future__ import annotations
+
+import numpy as np
+from scipy.special import erf
+
+OVER_BUDGET = 1  # sample flag: even zero visual tokens exceed the budget
+
+
+# ----------------------------------------------------------------------------
+# storage rounding
+# ----------------------------------------------------------------------------
+def round_bf16(a) -> np.ndarray:
+    """Round to the nearest bfloat16 (ties to even), returned as float64.
+
+    The value is first rounded to float32 (as a float32 accumulator would
+    hold it), then the low 16 bits are rounded away.
+    """
+    f = np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+    u = f.view(np.uint32).astype(np.uint64)
+    nan = np.isnan(f)
+    lsb = (u >> np.uint64(16)) & np.uint64(1)
+    u = (u + np.uint64(0x7FFF) + lsb) & np.uint64(0xFFFF0000)
+    out = u.astype(np.uint32).view(np.float32).astype(np.float64)
+    out[nan] = np.nan
+    return out
+
+
+def make_store(mode: str):
+    if mode == "fp64":
+        return lambda a: np.asarray(a, dtype=np.float64)
+    if mode == "fp32":
+        return lambda a: np.asarray(a, dtype=np.float32).astype(np.float64)
+    if mode == "bf16":
+        return round_bf16
+    raise ValueError(mode)
+
+
+# ----------------------------------------------------------------------------
+# Eq. 5: budget encoding, token controller logits (Sec. 3.1)
+# ----------------------------------------------------------------------------
+def sinusoidal_encoding(b: float, dim: int) -> np.ndarray:
+    """PE(b): dim/2 frequencies 10000^(-2i/dim) of the argument 1000*b;
+    sines in the first half, cosines in the second (reading R2)."""
+    i = np.arange(dim // 2, dtype=np.float64)
+    omega = 10000.0 ** (-2.0 * i / dim)
+    arg = 1000.0 * float(b) * omega
+    return np.concatenate([np.sin(arg), np.cos(arg)])
+
+
+def silu(x):
+    return x / (1.0 + np.exp(-x))
+
+
+def gelu(x):
+    return 0.5 * x * (1.0 + erf(x / np.sqrt(2.0)))
+
+
+def budget_embedding(b: float, w1: np.ndarray, w2: np.ndarray) -> np.ndarray:
+    """e_b = W2 SiLU(W1 PE(b)) (Eq. 5 without the ViT position term)."""
+    pe = sinusoidal_encoding(b, w1.shape[1])
+    return w2 @ silu(w1 @ pe)
+
+
+def token_logits(x: np.ndarray, e_b: np.ndarray, w1: np.ndarray, w2: np.ndarray, c2: float) -> np.ndarray:
+    """z_i = w2 . SiLU(W1 x_i + e_b) + c2 for every visual token row x_i."""
+    hidden = x @ w1.T + e_b[None, :]
+    return silu(hidden) @ w2 + c2
+
+
+# ----------------------------------------------------------------------------
+# Eq. 8: prefill FLOPs, exact in integers (times G)
+# ----------------------------------------------------------------------------
+def effective_groups(layer_gate, group_gate, n_prefix: int) -> np.ndarray:
+    """e_{l,j}: 1 if group j of layer l runs. Prefix layers always run
+    (Sec. 3.2); otherwise the layer bit and the group bit must both be on."""
+    lg = np.asarray(layer_gate).astype(np.int64)
+    gg = np.asarray(group_gate).astype(np.int64)
+    e = (lg[:, None] != 0) & (gg != 0)
+    e[:n_prefix, :] = True
+    return e.astype(np.int64)
+
+
+def prefill_cost_xG(dims, S: int, groups_on) -> int:
+    """G * C(S) of Eq. 8 for one sample.
+
+    groups_on[l] = sum_j M_lj, so alpha_l * G = groups_on[l].  The MHA term
+    8 D^2 is written 4 D^2 + 4 D D_kv (Q, O plus K, V projections).
+    """
+    D, Dkv, Di, V, G = dims.d_model, dims.d_kv, dims.d_ffn, dims.vocab, dims.n_groups
+    per_layer = (4 * D * D + 4 * D * Dkv + 6 * D * Di) * S + 4 * D * S * S
+    total = 0
+    for n_on in groups_on:
+        total += int(n_on) * per_layer
+    return total + G * 2 * D * V * S
+
+
+def budget_keep_count(dims, budget: float, n_vis: int, s_text: int, groups_on, keep_count: int = -1):
+    """Number of visual tokens to keep and the sample flags (Sec. 3.3).
+
+    With keep_count >= 0 the count is min(keep_count, N). Otherwise it is the
+    largest k in [0, N] with C(S_text + k) <= b * C_full, where C_full is
+    Eq. 8 at S = N + S_text with every group on. The comparison is done in
+    float64 on the exact integers G*C; the budget is the float32 value given.
+    """
+    if keep_count >= 0:
+        return min(int(keep_count), n_vis), 0
+    L, G = dims.n_layers, dims.n_groups
+    c_full = prefill_cost_xG(dims, n_vis + s_text, [G] * L)
+    limit = float(np.float32(budget)) * float(c_full)
+    for k in range(n_vis, -1, -1):
+        if float(prefill_cost_xG(dims, s_text + k, groups_on)) <= limit:
+            return k, 0
+    return 0, OVER_BUDGET
+
+
+def select_kept(z: np.ndarray, k: int) -> np.ndarray:
+    """Indices of the k highest logits (equal logits: lower index first),
+    returned in ascending index order."""
+    n = len(z)
+    order = np.lexsort((np.arange(n), -np.asarray(z, dtype=np.float64)))
+    return np.sort(order[:k])
+
+
+# ----------------------------------------------------------------------------
+# decoder pieces
+# ----------------------------------------------------------------------------
+def rmsnorm(x: np.ndarray, gain: np.ndarray, eps: float) -> np.ndarray:
+    ms = np.mean(x * x, axis=-1, keepdims=True)
+    return x / np.sqrt(ms + eps) * gain
+
+
+def rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
+    """Rotary embedding, rotate-half convention: dim i pairs with i + d/2,
+    angle pos * theta^(-2i/d). x is [S, heads, d]."""
+    d = x.shape[-1]
+    half = d // 2
+    inv = theta ** (-2.0 * np.arange(half, dtype=np.float64) / d)
+    ang = pos.astype(np.float64)[:, None] * inv[None, :]
+    cos = np.cos(ang)[:, None, :]
+    sin = np.sin(ang)[:, None, :]
+    x1, x2 = x[..., :half], x[..., half:]
+    return np.concatenate([x1 * cos - x2 * sin, x2 * cos + x1 * sin], axis=-1)
+
+
+def causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
+    """softmax(q k^T / sqrt(d) + causal mask) v for one head; q,k,v are [S, d]."""
+    S, d = q.shape
+    s = (q @ k.T) / np.sqrt(d)
+    s = np.where(np.tril(np.ones((S, S), dtype=bool)), s, -np.inf)
+    s = s - s.max(axis=1, keepdims=True)
+    p = np.exp(s)
+    p = p / p.sum(axis=1, keepdims=True)
+    return p @ v
+
+
+def decoder_layer(X, pos, lw, groups, dims, store):
+    """One gated decoder layer on one sample's rows X [S, D] (Sec. 3.2).
+
+    ``groups`` is e_{l,:} (length G). Head h belongs to group h // (A/G);
+    FFN channel c to group c // (D_int/G) (reading R3). Off groups give zero
+    attention output and zero FFN channels; no rescaling by 1/alpha. With
+    every group off the layer is the identity (residual bypass).
+    """
+    A, Akv, dh, G = dims.n_heads, dims.n_kv_heads, dims.d_head, dims.n_groups
+    S = X.shape[0]
+    if not np.any(groups):
+        return X
+    hpg = A // G
+    xn = store(rmsnorm(X, lw["attn_norm"], dims.rms_eps))
+    q = (xn @ lw["wq"].T).reshape(S, A, dh)
+    k = (xn @ lw["wk"].T).reshape(S, Akv, dh)
+    v = (xn @ lw["wv"].T).reshape(S, Akv, dh)
+    q = store(rope(q, pos, dims.rope_theta))
+    k = store(rope(k, pos, dims.rope_theta))
+    v = store(v)
+    o = np.zeros((S, A, dh))
+    for h in range(A):
+        if groups[h // hpg]:
+            kv = h // (A // Akv)
+            o[:, h, :] = causal_attention(q[:, h, :], k[:, kv, :], v[:, kv, :])
+    o = store(o.reshape(S, A * dh))
+    X = store(X + o @ lw["wo"].T)
+
+    xn = store(rmsnorm(X, lw["ffn_norm"], dims.rms_eps))
+    u = silu(xn @ lw["wg"].T) * (xn @ lw["wu"].T)
+    cpg = dims.d_ffn // G
+    for j in range(G):
+        if not groups[j]:
+            u[:, j * cpg:(j + 1) * cpg] = 0.0
+    u = store(u)
+    return store(X + u @ lw["wd"].T)
+
+
+def project_visual(x, weights, dims, store):
+    """LLaVA MLP projector W2 GELU(W1 x) (identity when no projector)."""
+    if not dims.proj_hidden:
+        return x
+    h = store(gelu(x @ weights["proj_w1"].T))
+    return store(h @ weights["proj_w2"].T)
+
+
+# ----------------------------------------------------------------------------
+# the whole path
+# ----------------------------------------------------------------------------
+def score_select_sample(dims, weights, x, budget, s_text, layer_gate, group_gate, keep_count=-1):
+    """Token controller for one sample: logits, k and ascending kept indices."""
+    e_b = budget_embedding(float(np.float32(budget)), weights["bud_w1"], weights["bud_w2"])
+    z = token_logits(x, e_b, weights["ctrl_w1"], weights["ctrl_w2"], weights["ctrl_c2"])
+    groups_on = effective_groups(layer_gate, group_gate, dims.n_prefix).sum(axis=1)
+    k, flags = budget_keep_count(dims, budget, x.shape[0], s_text, groups_on, keep_count)
+    return z, k, flags, select_kept(z, k)
+
+
+def pack_sample(dims, weights, x, kept, text_ids, store):
+    """[projected kept visual rows (image order)] ++ [text embedding rows]."""
+    vis = project_visual(x[kept], weights, dims, store)
+    txt = weights["embed"][np.asarray(text_ids, dtype=np.int64)]
+    X = np.concatenate([vis, txt], axis=0)
+    return store(X), np.arange(X.shape[0])
+
+
+def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
+                   keep_count=-1, mode="fp32", n_layers=None):
+    """Token controller + pack + gated decoder + final norm + last-row logits.
+
+    ``n_layers`` (default: all) runs only the first layers -- used to bound
+    the oracle's time; the final norm and LM head then apply after them.
+    """
+    store = make_store(mode)
+    z, k, flags, kept = score_select_sample(dims, weights, x, budget, len(text_ids),
+                                            layer_gate, group_gate, keep_count)
+    X, pos = pack_sample(dims, weights, x, kept, text_ids, store)
+    e = effective_groups(layer_gate, group_gate, dims.n_prefix)
+    nl = dims.n_layers if n_layers is None else n_layers
+    for l in range(nl):
+        X = decoder_layer(X, pos, weights["layers"][l], e[l], dims, store)
+    y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
+    logits = make_store("fp64" if mode == "fp64" else "fp32")(weights["lm_head"] @ y)
+    return {"z": z, "k": k, "flags": flags, "kept": kept, "hidden": X, "logits": logits}
+
+
+def forward_batch(dims, weights, batch, mode="fp32", n_layers=None, samples=None):
+    """Run ``forward_sample`` on each sample of a numpy batch dict
+    (keys as produced by the input generator, converted to numpy)."""
+    out = []
+    B = batch["B"]
+    for b in (range(B) if samples is None else samples):
+        v0, v1 = batch["vis_off"][b], batch["vis_off"][b + 1]
+        t0, t1 = batch["text_off"][b], batch["text_off"][b + 1]
+        out.append(forward_sample(
+            dims, weights, batch["vis"][v0:v1], batch["text_ids"][t0:t1], batch["budget"][b],
+            batch["layer_gate"][b], batch["group_gate"][b], int(batch["keep_count"][b]),
+            mode=mode, n_layers=n_layers))
+    return out
+
+
+def executed_flops(dims, n_vis, k, s_text, groups_on, all_logits=False) -> int:
+    """Algorithmic FLOPs that the gated path must execute for one sample:
+    scorer, projector on kept tokens, active projections and FFN, causal
+    attention (2 D S (S+1) alpha) and the LM head."""
+    D, Dkv, Di, V, G = dims.d_model, dims.d_kv, dims.d_ffn, dims.vocab, dims.n_groups
+    S = k + s_text
+    f = 2 * n_vis * dims.c_vis * dims.h_ctrl
+    if dims.proj_hidden:
+        f += 2 * k * (dims.c_vis * dims.proj_hidden + dims.proj_hidden * D)
+    lin = (4 * D * D + 4 * D * Dkv + 6 * D * Di) * S
+    att = 2 * D * S * (S + 1)
+    fl = 0
+    for n_on in groups_on:
+        fl += int(n_on) * (lin + att)
+    assert fl % G == 0
+    f += fl // G
+    f += 2 * D * V * (S if all_logits else 1)
+    return f
+
+
+def to_numpy_weights(w) -> dict:
+    """Convert a weight dict of torch tensors into float64 numpy arrays."""
+    import torch
+
+    def cv(t):
+        if isinstance(t, torch.Tensor):
+            return t.detach().to("cpu", torch.float64).numpy()
+        return t
+
+    out = {k: cv(v) for k, v in w.items() if k != "layers"}
+    out["layers"] = [{k: cv(v) for k, v in lw.items()} for lw in w["layers"]]
+    return out
+
+
+def to_numpy_batch(batch) -> dict:
+    import torch
+    out = {}
+    for k, v in batch.items():
+        if isinstance(v, torch.Tensor):
+            v = v.detach().cpu()
+            out[k] = v.to(torch.float64).numpy() if v.dtype == torch.bfloat16 else v.numpy()
+        else:
+            out[k] = v
+    return out

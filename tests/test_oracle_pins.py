@@ -1,0 +1,387 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: brute force,
+a closed form, an independent dense transformer built from library routines,
+a per-matmul operation tally, or a figure printed in the paper.
+"""
+import itertools
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import smartvl_oracle as O
+from paper_2607_20357_gb300 import synth
+from tests.dense_reference import dense_forward, rope_complex
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+SMALL = synth.ModelDims(n_layers=3, d_model=64, n_heads=4, n_kv_heads=2, d_ffn=128, vocab=50,
+                        n_groups=2, n_prefix=0, c_vis=32, h_ctrl=16, proj_hidden=48,
+                        rms_eps=1e-5, rope_theta=1e4)
+SMALL_ID = synth.reduced(SMALL, c_vis=64, proj_hidden=0, n_kv_heads=4, n_groups=4)
+
+
+def np_weights(dims, seed=3, std=0.08):
+    return O.to_numpy_weights(synth.make_weights(dims, seed, std=std))
+
+
+# ----------------------------------------------------------------------------- primitives
+def test_round_bf16_matches_torch_conversion():
+    rng = np.random.default_rng(0)
+    x = np.concatenate([rng.normal(size=4000) * 10.0 ** rng.integers(-6, 6, size=4000),
+                        [0.0, -0.0, 1.0, 1.00390625, 1.005859375, 65504.0, 3.4e38]])
+    ref = torch.tensor(x, dtype=torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_bf16(x), ref)
+
+
+def test_sinusoidal_encoding_closed_form():
+    pe0 = O.sinusoidal_encoding(0.0, 16)
+    np.testing.assert_array_equal(pe0, np.r_[np.zeros(8), np.ones(8)])
+    pe = O.sinusoidal_encoding(0.37, 64)
+    np.testing.assert_allclose(pe[:32] ** 2 + pe[32:] ** 2, 1.0, atol=1e-14)
+    # first frequency is 1 rad per unit of 1000*b; last is 10000^(-62/64)
+    assert pe[0] == pytest.approx(math.sin(370.0))
+    assert pe[31] == pytest.approx(math.sin(370.0 * 10000 ** (-62 / 64)))
+    assert pe[63] == pytest.approx(math.cos(370.0 * 10000 ** (-62 / 64)))
+
+
+def test_token_logits_match_library_mlp():
+    rng = np.random.default_rng(1)
+    x = rng.normal(size=(20, 32))
+    w1, w2 = rng.normal(size=(16, 32)) * 0.2, rng.normal(size=16)
+    e_b = rng.normal(size=16)
+    ref = (torch.nn.functional.silu(torch.tensor(x) @ torch.tensor(w1).T + torch.tensor(e_b))
+           @ torch.tensor(w2)).numpy() + 0.25
+    np.testing.assert_allclose(O.token_logits(x, e_b, w1, w2, 0.25), ref, rtol=1e-12, atol=1e-12)
+
+
+def test_activation_special_values():
+    assert O.silu(np.array(0.0)) == 0.0
+    assert O.gelu(np.array(0.0)) == 0.0
+    assert O.gelu(np.array(10.0)) == pytest.approx(10.0)
+    assert O.gelu(np.array(1.0)) == pytest.approx(0.8413447460685429)   # Phi(1)
+    assert O.silu(np.array(1.0)) == pytest.approx(1.0 / (1.0 + math.exp(-1.0)))
+
+
+def test_rmsnorm_constant_rows():
+    x = np.full((3, 8), -2.0)
+    g = np.arange(1, 9, dtype=np.float64)
+    out = O.rmsnorm(x, g, 1e-5)
+    np.testing.assert_allclose(out, np.tile(-2.0 / math.sqrt(4.0 + 1e-5) * g, (3, 1)))
+
+
+def test_rope_properties_and_complex_form():
+    rng = np.random.default_rng(2)
+    x = rng.normal(size=(12, 3, 16))
+    pos = np.arange(12)
+    r = O.rope(x, pos, 1e4)
+    np.testing.assert_allclose(np.linalg.norm(r, axis=-1), np.linalg.norm(x, axis=-1), rtol=1e-12)
+    np.testing.assert_allclose(r[0], x[0])
+    ref = rope_complex(torch.tensor(x), torch.tensor(pos), 1e4).numpy()
+    np.testing.assert_allclose(r, ref, rtol=1e-12, atol=1e-12)
+    # relative position: <rope(q, m), rope(k, n)> depends only on m - n
+    q, k = rng.normal(size=16), rng.normal(size=16)
+    qq = O.rope(np.tile(q, (12, 1, 1)), pos, 1e4)[:, 0]
+    kk = O.rope(np.tile(k, (12, 1, 1)), pos, 1e4)[:, 0]
+    assert qq[7] @ kk[3] == pytest.approx(qq[9] @ kk[5], rel=1e-12)
+
+
+def test_causal_attention_softmax_rows():
+    rng = np.random.default_rng(3)
+    q, k = rng.normal(size=(9, 8)), rng.normal(size=(9, 8))
+    v = np.ones((9, 8))
+    np.testing.assert_allclose(O.causal_attention(q, k, v), 1.0, rtol=1e-13)
+    # first row attends only to itself
+    v = rng.normal(size=(9, 8))
+    np.testing.assert_allclose(O.causal_attention(q, k, v)[0], v[0], rtol=1e-13)
+
+
+# ----------------------------------------------------------------------------- selection
+@pytest.mark.parametrize("n", [1, 5, 9, 12])
+def test_select_kept_equals_bruteforce(n):
+    rng = np.random.default_rng(n)
+    for trial in range(4):
+        z = rng.integers(-3, 4, size=n).astype(np.float64)   # many exact ties
+        for k in range(n + 1):
+            best = None
+            for sub in itertools.combinations(range(n), k):
+                key = (-sum(z[list(sub)]), sub)   # max sum, then lowest indices
+                if best is None or key < best:
+                    best = key
+            np.testing.assert_array_equal(O.select_kept(z, k), np.array(best[1], dtype=np.int64))
+
+
+def test_select_kept_permutation_invariance():
+    rng = np.random.default_rng(11)
+    z = rng.normal(size=200)
+    perm = rng.permutation(200)
+    for k in (0, 1, 57, 200):
+        a = set(O.select_kept(z, k).tolist())
+        b = set(perm[O.select_kept(z[perm], k)].tolist())
+        assert a == b and len(a) == k
+
+
+# ----------------------------------------------------------------------------- Eq. 8
+def _matmul_tally_flops(dims, S, n_on_per_layer, causal=False, lm_rows=None):
+    """FLOPs from the list of matmuls one sample's forward performs (2 per MAC).
+    Attention: QK^T and PV per head; Eq. 8 counts every (query, key) pair."""
+    D, Dkv, Di, V, G = dims.d_model, dims.d_kv, dims.d_ffn, dims.vocab, dims.n_groups
+    A, dh = dims.n_heads, dims.d_head
+    total = 0
+    pairs = S * (S + 1) // 2 if causal else S * S
+    for n_on in n_on_per_layer:
+        heads = A * n_on // G
+        chans = Di * n_on // G
+        kv = dims.n_kv_heads * n_on // G
+        macs = S * D * (heads * dh)          # Q
+        macs += 2 * S * D * (kv * dh)        # K, V
+        macs += 2 * heads * pairs * dh       # QK^T and PV
+        macs += S * (heads * dh) * D         # O
+        macs += 2 * S * D * chans            # gate, up
+        macs += S * chans * D                # down
+        total += 2 * macs
+    total += 2 * D * V * (S if lm_rows is None else lm_rows)
+    return total
+
+
+@pytest.mark.parametrize("dims", [SMALL, SMALL_ID, synth.WORKLOADS["llava"].dims, synth.WORKLOADS["qwen"].dims])
+def test_eq8_equals_matmul_tally(dims):
+    G, L = dims.n_groups, dims.n_layers
+    rng = np.random.default_rng(5)
+    for S in (1, 17, 640):
+        n_on = rng.integers(0, G + 1, size=L)
+        assert O.prefill_cost_xG(dims, S, n_on) == G * _matmul_tally_flops(dims, S, n_on)
+
+
+def test_executed_flops_equals_causal_tally():
+    dims = SMALL
+    n_on = [2, 0, 1]
+    k, s_text, n_vis = 9, 5, 20
+    S = k + s_text
+    f = O.executed_flops(dims, n_vis, k, s_text, n_on)
+    extra = 2 * n_vis * dims.c_vis * dims.h_ctrl + 2 * k * (dims.c_vis * dims.proj_hidden + dims.proj_hidden * dims.d_model)
+    assert f == extra + _matmul_tally_flops(dims, S, n_on, causal=True, lm_rows=1)
+
+
+def test_eq8_tiny_and_paper_full_prefill():
+    with open(os.path.join(GOLDEN, "paper_prefill_flops.json")) as fh:
+        gold = json.load(fh)
+    tiny = synth.WORKLOADS["tiny"].dims
+    assert O.prefill_cost_xG(tiny, 80, [4, 4]) // 4 == gold["tiny_full_flops_S80"]["value"]
+    llava = synth.WORKLOADS["llava"].dims
+    S = 576 + 64
+    with_lm = O.prefill_cost_xG(llava, S, [4] * 32) / 4
+    without_lm = with_lm - 2 * llava.d_model * llava.vocab * S
+    paper = gold["llava7b_full_prefill"]["value_tflops"] * 1e12
+    assert abs(without_lm - paper) / paper < 0.005      # 8.504 T
+    assert abs(with_lm - paper) / paper < 0.025         # 8.672 T (Eq. 8 as printed)
+
+
+# ----------------------------------------------------------------------------- budget -> k
+def _closed_form_k(dims, b, n_vis, s_text, n_on):
+    """Invert the quadratic a S^2 + c S <= R with the formula, then step."""
+    D, Dkv, Di, V, G = dims.d_model, dims.d_kv, dims.d_ffn, dims.vocab, dims.n_groups
+    L = dims.n_layers
+    lin = 4 * D * D + 4 * D * Dkv + 6 * D * Di
+    S_full = n_vis + s_text
+    c_full = G * L * (lin * S_full + 4 * D * S_full ** 2) + G * 2 * D * V * S_full
+    R = float(np.float32(b)) * float(c_full)
+    n_sum = int(sum(int(v) for v in n_on))
+    a = 4 * D * n_sum
+    c = lin * n_sum + G * 2 * D * V
+    S = int((-c + math.sqrt(c * c + 4 * a * R)) / (2 * a)) if a > 0 else int(R // c)
+    cost = lambda s: float(a * s * s + c * s)
+    while S + 1 <= S_full and cost(S + 1) <= R:
+        S += 1
+    while S >= s_text and cost(S) > R:
+        S -= 1
+    if S < s_text:
+        return 0, O.OVER_BUDGET
+    return min(S - s_text, n_vis), 0
+
+
+@pytest.mark.parametrize("name", ["tiny", "llava", "qwen", "mixed"])
+def test_budget_k_closed_form_and_bracket(name):
+    dims = synth.WORKLOADS[name].dims
+    rng = np.random.default_rng(7)
+    G, L = dims.n_groups, dims.n_layers
+    for trial in range(25):
+        n_vis = int(rng.integers(0, 700))
+        s_text = int(rng.integers(1, 200))
+        b = float(rng.uniform(0.02, 1.0))
+        lg = (rng.random(L) < 0.8).astype(np.uint8)
+        gg = (rng.random((L, G)) < 0.7).astype(np.uint8)
+        n_on = O.effective_groups(lg, gg, dims.n_prefix).sum(1)
+        k, fl = O.budget_keep_count(dims, b, n_vis, s_text, n_on)
+        assert (k, fl) == _closed_form_k(dims, b, n_vis, s_text, n_on)
+        if fl == 0:
+            c_full = O.prefill_cost_xG(dims, n_vis + s_text, [G] * L)
+            lim = float(np.float32(b)) * c_full
+            assert O.prefill_cost_xG(dims, s_text + k, n_on) <= lim
+            if k < n_vis:
+                assert O.prefill_cost_xG(dims, s_text + k + 1, n_on) > lim
+
+
+def test_budget_one_keeps_everything_and_keep_count_override():
+    dims = synth.WORKLOADS["llava"].dims
+    full = [4] * 32
+    assert O.budget_keep_count(dims, 1.0, 576, 64, full) == (576, 0)
+    assert O.budget_keep_count(dims, 0.3, 576, 64, full, keep_count=32) == (32, 0)
+    assert O.budget_keep_count(dims, 0.3, 20, 64, full, keep_count=32) == (20, 0)
+    # fewer groups on leave room for more tokens
+    half = [2] * 32
+    assert O.budget_keep_count(dims, 0.55, 576, 64, half)[0] == 576
+    assert O.budget_keep_count(dims, 0.5, 576, 64, half)[0] < 576   # LM head is not gated
+    # a budget below the text-only cost keeps nothing and flags the sample
+    assert O.budget_keep_count(dims, 0.01, 576, 64, full) == (0, O.OVER_BUDGET)
+
+
+def test_budget_k_llava_sweep_values():
+    with open(os.path.join(GOLDEN, "budget_k_llava.json")) as fh:
+        gold = json.load(fh)
+    dims = synth.WORKLOADS[gold["workload"]].dims
+    for b, k in gold["k_by_budget"].items():
+        n_on = [dims.n_groups] * dims.n_layers
+        assert O.budget_keep_count(dims, float(b), gold["n_vis"], gold["s_text"], n_on) == (k, 0)
+        assert _closed_form_k(dims, float(b), gold["n_vis"], gold["s_text"], n_on) == (k, 0)
+
+
+def test_prefix_layers_ignore_gates():
+    dims = synth.reduced(SMALL, n_prefix=2)
+    lg = np.array([0, 0, 0], np.uint8)
+    gg = np.zeros((3, 2), np.uint8)
+    e = O.effective_groups(lg, gg, dims.n_prefix)
+    np.testing.assert_array_equal(e, [[1, 1], [1, 1], [0, 0]])
+
+
+# ----------------------------------------------------------------------------- gated forward
+def _sample(dims, seed=0, n_vis=24, s_text=7):
+    rng = np.random.default_rng(seed)
+    x = O.round_bf16(rng.normal(size=(n_vis, dims.c_vis)))
+    ids = rng.integers(0, dims.vocab, size=s_text)
+    return x, ids
+
+
+def _packed_rows(dims, w, x, kept, ids):
+    vis = x[kept]
+    if dims.proj_hidden:
+        vis = O.gelu(vis @ w["proj_w1"].T) @ w["proj_w2"].T
+    return np.concatenate([vis, w["embed"][ids]], 0)
+
+
+@pytest.mark.parametrize("dims", [SMALL, SMALL_ID])
+def test_all_on_keep_all_equals_dense_library_forward(dims):
+    w = np_weights(dims)
+    x, ids = _sample(dims)
+    L, G = dims.n_layers, dims.n_groups
+    out = O.forward_sample(dims, w, x, ids, 1.0, np.ones(L, np.uint8), np.ones((L, G), np.uint8), mode="fp64")
+    assert out["k"] == x.shape[0]
+    X0 = _packed_rows(dims, w, x, np.arange(x.shape[0]), ids)
+    hid, logits = dense_forward(X0, w["layers"], w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(out["hidden"], hid, rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(out["logits"], logits, rtol=1e-10, atol=1e-10)
+
+
+def test_group_off_equals_zeroed_weights():
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 1)
+    L, G = dims.n_layers, dims.n_groups
+    gg = np.ones((L, G), np.uint8)
+    gg[0, 1] = 0
+    gg[2, 0] = 0
+    out = O.forward_sample(dims, w, x, ids, 1.0, np.ones(L, np.uint8), gg, keep_count=10, mode="fp64")
+    wz = {k: v for k, v in w.items()}
+    layers = []
+    hpg, cpg = dims.n_heads // G, dims.d_ffn // G
+    for l, lw in enumerate(w["layers"]):
+        lw = dict(lw)
+        lw["wo"], lw["wd"] = lw["wo"].copy(), lw["wd"].copy()
+        for j in range(G):
+            if not gg[l, j]:
+                lw["wo"][:, j * hpg * dims.d_head:(j + 1) * hpg * dims.d_head] = 0.0
+                lw["wd"][:, j * cpg:(j + 1) * cpg] = 0.0
+        layers.append(lw)
+    X0 = _packed_rows(dims, w, x, out["kept"], ids)
+    hid, logits = dense_forward(X0, layers, w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(out["hidden"], hid, rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(out["logits"], logits, rtol=1e-10, atol=1e-10)
+
+
+def test_all_groups_off_equals_removed_layer_and_layer_gate():
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 2)
+    L, G = dims.n_layers, dims.n_groups
+    gg = np.ones((L, G), np.uint8)
+    gg[1, :] = 0
+    out = O.forward_sample(dims, w, x, ids, 1.0, np.ones(L, np.uint8), gg, keep_count=12, mode="fp64")
+    lg = np.ones(L, np.uint8)
+    lg[1] = 0
+    out2 = O.forward_sample(dims, w, x, ids, 1.0, lg, np.ones((L, G), np.uint8), keep_count=12, mode="fp64")
+    X0 = _packed_rows(dims, w, x, out["kept"], ids)
+    hid, logits = dense_forward(X0, [w["layers"][0], w["layers"][2]], w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(out["hidden"], hid, rtol=1e-10, atol=1e-10)
+    np.testing.assert_array_equal(out["hidden"], out2["hidden"])
+
+
+def test_prefix_layer_runs_even_when_gated_off():
+    dims = synth.reduced(SMALL, n_prefix=1)
+    w = np_weights(dims)
+    x, ids = _sample(dims, 3)
+    L, G = dims.n_layers, dims.n_groups
+    lg = np.ones(L, np.uint8)
+    lg[0] = 0
+    a = O.forward_sample(dims, w, x, ids, 1.0, lg, np.ones((L, G), np.uint8), keep_count=8, mode="fp64")
+    b = O.forward_sample(dims, w, x, ids, 1.0, np.ones(L, np.uint8), np.ones((L, G), np.uint8), keep_count=8, mode="fp64")
+    np.testing.assert_array_equal(a["hidden"], b["hidden"])
+
+
+def test_kept_subset_equals_dense_on_shortened_sequence():
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 4, n_vis=30)
+    L, G = dims.n_layers, dims.n_groups
+    out = O.forward_sample(dims, w, x, ids, 0.6, np.ones(L, np.uint8), np.ones((L, G), np.uint8), mode="fp64")
+    assert 0 < out["k"] < 30
+    # the kept tokens are the top-k logits, in image order, at positions 0..S-1
+    e_b = O.budget_embedding(float(np.float32(0.6)), w["bud_w1"], w["bud_w2"])
+    z = O.token_logits(x, e_b, w["ctrl_w1"], w["ctrl_w2"], 0.0)
+    assert set(out["kept"]) == set(np.argsort(-z)[:out["k"]])
+    X0 = _packed_rows(dims, w, x, np.sort(out["kept"]), ids)
+    hid, logits = dense_forward(X0, w["layers"], w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(out["hidden"], hid, rtol=1e-10, atol=1e-10)
+
+
+def test_storage_modes_are_close_and_ordered():
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 5)
+    L, G = dims.n_layers, dims.n_groups
+    args = (dims, w, x, ids, 0.8, np.ones(L, np.uint8), np.ones((L, G), np.uint8))
+    r64 = O.forward_sample(*args, mode="fp64")
+    r32 = O.forward_sample(*args, mode="fp32")
+    r16 = O.forward_sample(*args, mode="bf16")
+    err = lambda a, b: np.abs(a - b).max() / np.abs(b).max()
+    assert err(r32["hidden"], r64["hidden"]) < 1e-6
+    assert 1e-5 < err(r16["hidden"], r64["hidden"]) < 2e-2
+    np.testing.assert_array_equal(O.round_bf16(r16["hidden"]), r16["hidden"])
+
+
+def test_batch_equals_independent_samples():
+    dims = SMALL
+    w = np_weights(dims)
+    wl = synth.Workload("t", dims, batch=3, n_vis=(10, 20), s_text=(3, 9), budgets=("uniform", 0.3, 1.0),
+                        gates="budget_scaled", features="normal")
+    batch = O.to_numpy_batch(synth.make_batch(wl, 9))
+    outs = O.forward_batch(dims, w, batch, mode="fp64")
+    for b in range(3):
+        v0, v1 = batch["vis_off"][b], batch["vis_off"][b + 1]
+        t0, t1 = batch["text_off"][b], batch["text_off"][b + 1]
+        one = O.forward_sample(dims, w, batch["vis"][v0:v1], batch["text_ids"][t0:t1], batch["budget"][b],
+                               batch["layer_gate"][b], batch["group_gate"][b], mode="fp64")
+        np.testing.assert_array_equal(one["hidden"], outs[b]["hidden"])
