@@ -1,0 +1,205 @@
+/*
+ * svl.h -- C ABI of the GB300 (sm_103a) budget-conditioned gated prefill.
+ *
+ * The library implements the inference hot path of SmartVL ("Look Less, Think
+ * Faster: Joint Token-Compute Adaptation for Multimodal LLMs", arXiv
+ * 2607.20357): the vision-side token controller that scores visual tokens
+ * under a budget and keeps the top k of each sample (Sec. 3.1, Sec. 3.3
+ * "Inference"), the packing of kept visual tokens and text tokens into one
+ * variable-length batch (Sec. 3.1, contiguous RoPE), and the LLM decoder
+ * forward under per-sample layer / head-group gates (Sec. 3.2) where gated-off
+ * work is never issued.
+ *
+ * Conventions shared by every call below.
+ *  - All tensor arguments are DEVICE pointers owned by the caller, unless the
+ *    name says host. bf16 tensors are IEEE bfloat16, row-major, contiguous.
+ *  - Calls that take a stream are asynchronous on it; the library never
+ *    synchronises the stream and never copies device data to the host.
+ *    Counts that depend on data (k, sequence lengths, tile lists) stay on the
+ *    device.
+ *  - The returned status reports argument and shape errors found on the host;
+ *    in that case nothing was launched. Data-dependent errors (a non-finite
+ *    token logit, a device wait that ran out of time) are OR-ed into the
+ *    model's device status word, read with svl_get_device_status().
+ *  - `workspace` is caller-allocated device memory of at least
+ *    svl_workspace_size() bytes, 256-byte aligned. Calls that share a
+ *    workspace must be ordered on one stream.
+ *  - Gates are bytes, 0 = off, anything else = on. For layers l < n_prefix
+ *    the gates are ignored and every group runs (Sec. 3.2 prefix layers).
+ */
+#ifndef SVL_H
+#define SVL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum svl_status {
+  SVL_OK = 0,
+  SVL_ERR_INVALID_ARG = 1,   /* null pointer, negative size, bad enum value */
+  SVL_ERR_SHAPE = 2,         /* sizes inconsistent with the model or the workspace */
+  SVL_ERR_UNSUPPORTED = 3,   /* dims the kernels do not support (see svl_model_create) */
+  SVL_ERR_CUDA = 4,          /* a CUDA runtime call failed */
+  SVL_ERR_NONFINITE = 5,     /* device status bit: a token logit was NaN or infinite */
+  SVL_ERR_TIMEOUT = 6,       /* device status bit: a bounded device wait gave up */
+  SVL_ERR_WORKSPACE = 7      /* workspace null, too small or misaligned */
+} svl_status;
+
+/* Device status word bits (svl_get_device_status). */
+#define SVL_DEV_NONFINITE 0x1u
+#define SVL_DEV_TIMEOUT 0x2u
+#define SVL_DEV_BAD_INDEX 0x4u
+
+/* Per-sample flag bits written by svl_score_select. */
+#define SVL_FLAG_OVER_BUDGET 0x1u /* even zero visual tokens exceed b * C_full */
+
+/* Model dimensions.  Notation of Sec. 3: L layers, width D, A heads, FFN
+ * width D_int, vocabulary V, G head groups, P prefix layers; C_v is the
+ * vision feature width; H the token-controller hidden width.
+ * Supported: D = A * d_head with d_head in {64, 128}; A % G == 0 and
+ * A_kv % G == 0 (each group owns whole KV heads); (D_int / G) % 64 == 0;
+ * (A / G) * d_head % 64 == 0; D, C_v, proj_hidden multiples of 64;
+ * H in {16, 32, ..., 256}; proj_hidden == 0 requires C_v == D. */
+typedef struct svl_model_desc {
+  int32_t n_layers;     /* L */
+  int32_t d_model;      /* D */
+  int32_t n_heads;      /* A */
+  int32_t n_kv_heads;   /* A_kv (GQA when < A) */
+  int32_t d_ffn;        /* D_int (SwiGLU) */
+  int32_t vocab;        /* V */
+  int32_t n_groups;     /* G */
+  int32_t n_prefix;     /* P */
+  int32_t c_vis;        /* C_v */
+  int32_t h_ctrl;       /* H */
+  int32_t proj_hidden;  /* LLaVA projector hidden width; 0 = identity */
+  float rms_eps;
+  float rope_theta;
+  int32_t max_seq;      /* longest per-sample sequence the model will see */
+} svl_model_desc;
+
+/* One decoder layer's weights: device bf16, nn.Linear layout [out, in]. */
+typedef struct svl_layer_weights {
+  const void* wq;         /* [A*d_head, D] */
+  const void* wk;         /* [A_kv*d_head, D] */
+  const void* wv;         /* [A_kv*d_head, D] */
+  const void* wo;         /* [D, A*d_head] */
+  const void* wg;         /* [D_int, D] */
+  const void* wu;         /* [D_int, D] */
+  const void* wd;         /* [D, D_int] */
+  const void* attn_norm;  /* [D] RMSNorm gain */
+  const void* ffn_norm;   /* [D] */
+} svl_layer_weights;
+
+/* All weights: device bf16 unless noted. The model keeps these pointers (it
+ * does not copy them): the caller keeps the memory alive until
+ * svl_model_destroy(). */
+typedef struct svl_weights {
+  const void* ctrl_w1;    /* [H, C_v]  token scorer, first layer */
+  const void* ctrl_w2;    /* [H]       token scorer, output weights */
+  float ctrl_c2;          /*           token scorer, output bias (host value) */
+  const void* bud_w1;     /* [H, H]    budget MLP (Eq. 5) */
+  const void* bud_w2;     /* [H, H] */
+  const void* proj_w1;    /* [proj_hidden, C_v] or NULL */
+  const void* proj_w2;    /* [D, proj_hidden] or NULL */
+  const void* embed;      /* [V, D] token embedding */
+  const void* final_norm; /* [D] */
+  const void* lm_head;    /* [V, D] */
+  const svl_layer_weights* layers; /* HOST array of n_layers entries */
+} svl_weights;
+
+typedef struct svl_model svl_model;
+
+/* Creates a model on the current CUDA device: validates dims, records the
+ * weight pointers, allocates the device status word and the RoPE cos/sin
+ * table (max_seq x d_head/2 float2, computed in double precision).
+ * Returns SVL_ERR_UNSUPPORTED for dims outside the list above. */
+svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* weights, svl_model** out);
+void svl_model_destroy(svl_model* model);
+
+/* Bytes of workspace for batches of up to `max_batch` samples with at most
+ * `max_vis_total` visual and `max_text_total` text tokens in total. */
+size_t svl_workspace_size(const svl_model* model, int32_t max_batch, int64_t max_vis_total,
+                          int64_t max_text_total);
+
+/* (1) Token controller (Sec. 3.1; Sec. 3.3 "Inference"; Eq. 5; Eq. 8).
+ *  Scores every visual token, z_i = w2 . SiLU(W1 x_i + e_b) + c2, with the
+ *  budget embedding e_b = W_b2 SiLU(W_b1 PE(b)); derives k_b as the largest
+ *  count whose Eq. 8 cost (with the sample's gates) stays within b * C_full,
+ *  or min(keep_count[b], N_b) when keep_count[b] >= 0; keeps the k_b highest
+ *  logits (equal logits: lower index first) and writes their indices in
+ *  ascending order, compacted over the batch.
+ *   vis_feats   [n_vis_total, C_v] bf16; sample b owns rows vis_off[b]..vis_off[b+1)
+ *   vis_off     [B+1] int32, vis_off[0] = 0, vis_off[B] = n_vis_total
+ *   text_len    [B] int32 text tokens per sample (S_text)
+ *   budget      [B] float32 b in (0, 1]
+ *   keep_count  [B] int32 or NULL (NULL / negative: derive from the budget)
+ *   layer_gate  [B, L] uint8; group_gate [B, L, G] uint8
+ *  Outputs: scores [n_vis_total] float32; k [B] int32; kept_idx
+ *  [n_vis_total] int32 (first sum(k) entries valid; indices are local to the
+ *  sample); kept_off [B+1] int32; sample_flags [B] uint32. */
+svl_status svl_score_select(svl_model* model, int32_t B, int32_t n_vis_total,
+                            const void* vis_feats, const int32_t* vis_off, const int32_t* text_len,
+                            const float* budget, const int32_t* keep_count,
+                            const uint8_t* layer_gate, const uint8_t* group_gate,
+                            float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off,
+                            uint32_t* sample_flags, void* workspace, size_t workspace_bytes,
+                            void* stream);
+
+/* (2) Pack (Sec. 3 S = S_text + S_vis; Sec. 3.1 contiguous RoPE).
+ *  Sample b's sequence is its kept visual tokens in ascending index order,
+ *  projected by the LLaVA MLP W_p2 GELU(W_p1 x) (identity when proj_hidden
+ *  is 0), followed by the embeddings of its text ids; positions 0..S_b-1.
+ *   text_ids [n_text_total] int32, text_off [B+1] int32
+ *  Outputs: X [T_cap, D] bf16 with T_cap = n_vis_total + n_text_total (rows
+ *  beyond T = sum S_b untouched), cu_seqlens [B+1] int32, pos [T_cap] int32. */
+svl_status svl_pack(svl_model* model, int32_t B, int32_t n_vis_total, int32_t n_text_total,
+                    const void* vis_feats, const int32_t* vis_off, const int32_t* kept_idx,
+                    const int32_t* kept_off, const int32_t* text_ids, const int32_t* text_off,
+                    void* X, int32_t* cu_seqlens, int32_t* pos,
+                    void* workspace, size_t workspace_bytes, void* stream);
+
+#define SVL_LOGITS_LAST 0 /* logits of each sample's last row: [B, V] */
+#define SVL_LOGITS_ALL 1  /* logits of every row: [T_cap, V] */
+
+/* (3) Gated decoder forward (Sec. 3.2; Eq. 3; Eq. 8).
+ *  For each layer l and sample b with e_{b,l,j} = (l < P) or
+ *  (layer_gate[b,l] and group_gate[b,l,j]): RMSNorm; Q,K,V for the heads of
+ *  active groups only, with RoPE; causal attention per active head; output
+ *  projection over the active heads' rows of W_O added to X; RMSNorm; SwiGLU
+ *  over the active groups' FFN channels only; down projection added to X.
+ *  A sample with no active group in a layer is left untouched (residual
+ *  bypass). Then the final RMSNorm and the LM head. X is updated in place
+ *  (on return it holds the final hidden state before the final norm).
+ *   X [T_cap, D] bf16 in/out; cu_seqlens [B+1]; pos [T_cap] (from svl_pack)
+ *   logits float32 [B, V] (LAST) or [T_cap, V] (ALL)
+ *   t_cap: rows of X (n_vis_total + n_text_total of the pack call) */
+svl_status svl_gated_prefill(svl_model* model, int32_t B, int32_t t_cap, void* X,
+                             const int32_t* cu_seqlens, const int32_t* pos,
+                             const uint8_t* layer_gate, const uint8_t* group_gate,
+                             int32_t logits_mode, float* logits,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* Eq. 8 for one sample, host only, no GPU: writes G * C(S) (exact integer
+ * arithmetic, 8 D^2 generalised to 4 D^2 + 4 D D_kv) for S = s_text + s_vis
+ * with the gates given (layer_gate [L], group_gate [L, G]; NULL = all on),
+ * and the FLOPs the gated path executes (causal attention, last-row logits). */
+svl_status svl_flops(const svl_model_desc* desc, int32_t s_text, int32_t s_vis, int32_t n_vis,
+                     const uint8_t* layer_gate, const uint8_t* group_gate,
+                     double* eq8_flops, double* exec_flops);
+
+/* Reads (and clears) the device status word; synchronises `stream`. */
+svl_status svl_get_device_status(svl_model* model, void* stream, uint32_t* code);
+
+const char* svl_status_string(svl_status s);
+
+/* Number of kernels launched by this library since the process started
+ * (host-side counter, used to report launches per step). */
+uint64_t svl_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SVL_H */

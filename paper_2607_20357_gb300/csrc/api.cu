@@ -1,0 +1,670 @@
+// C ABI of the gated prefill: argument checks, model state, workspace layout,
+// tensor-map encoding and the launch sequences of the three stages.
+#include <cudaTypedefs.h>
+
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "gemm.cuh"
+#include "kernels.cuh"
+
+using namespace svl;
+
+struct svl_model {
+  svl_model_desc d;
+  svl_weights w;
+  std::vector<svl_layer_weights> layers;
+  int device = 0;
+  int num_sms = 0;
+  uint32_t* d_status = nullptr;
+  float2* rope_cs = nullptr;
+  // B-operand tensor maps of the weights: per layer q, k, v, o, g, u, d
+  std::vector<CUtensorMap> tm_layer;
+  CUtensorMap tm_ctrl_w1, tm_proj_w1, tm_proj_w2, tm_lm_head;
+};
+
+namespace {
+
+std::atomic<uint64_t> g_launches{0};
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map, K-major rows of `cols` elements, boxes of 64 x 128
+// with 128-byte swizzle (the layout the tcgen05 descriptors expect).
+bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols) {
+  auto fn = encode_fn();
+  if (!fn || !ptr || rows == 0 || cols == 0 || (reinterpret_cast<uintptr_t>(ptr) & 15)) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), 128};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+// Each call keeps its scratch at the start of the workspace: no data flows
+// between calls through the workspace, so the three layouts overlap and the
+// workspace size is the largest of them.
+struct SelLayout {
+  size_t e_b, scalars, kept_local, total;
+};
+struct PackLayout {
+  size_t scalars, stage, hp, row_map, total;
+};
+struct PreLayout {
+  int64_t t_cap;
+  int n_pad, mt_max, qkv_cap, o_cap, gu_cap, dn_cap, attn_cap;
+  size_t xn, q, k, v, ao, hmid, yl, act, seg, qkv, o, gu, dn, attn, counts, total;
+};
+
+struct Bump {
+  size_t off = 0;
+  size_t take(size_t bytes) {
+    size_t o = off;
+    off = align256(off + bytes);
+    return o;
+  }
+};
+
+SelLayout sel_layout(const svl_model_desc& d, int B, int64_t nv) {
+  SelLayout L{};
+  Bump b;
+  L.e_b = b.take(sizeof(float) * B * d.h_ctrl);
+  L.scalars = b.take(64);
+  L.kept_local = b.take(sizeof(int) * std::max<int64_t>(nv, 1));
+  L.total = b.off;
+  return L;
+}
+
+PackLayout pack_layout(const svl_model_desc& d, int64_t nv) {
+  PackLayout L{};
+  Bump b;
+  L.scalars = b.take(64);
+  if (d.proj_hidden) {
+    L.stage = b.take(2 * nv * d.c_vis);
+    L.hp = b.take(2 * nv * d.proj_hidden);
+    L.row_map = b.take(sizeof(int) * std::max<int64_t>(nv, 1));
+  }
+  L.total = b.off;
+  return L;
+}
+
+PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
+  PreLayout L{};
+  const int64_t dh = d.d_model / d.n_heads, dkv = static_cast<int64_t>(d.n_kv_heads) * dh;
+  const int64_t hq = static_cast<int64_t>(d.n_heads) * dh;
+  const int G = d.n_groups;
+  L.t_cap = t_cap;
+  L.n_pad = ((B + 15) / 16) * 16;
+  L.mt_max = static_cast<int>(t_cap / 128 + B + 1);
+  const int qkv_nt = static_cast<int>((hq / 256 + G + 1) + 2 * (dkv / 256 + G + 1));
+  L.qkv_cap = L.mt_max * qkv_nt;
+  L.o_cap = L.mt_max * ((d.d_model + 255) / 256);
+  L.dn_cap = L.o_cap;
+  L.gu_cap = L.mt_max * (d.d_ffn / 128 + G + 1);
+  L.attn_cap = static_cast<int>(d.n_heads * (t_cap / kAttnQ + B + 1));
+  Bump b;
+  L.xn = b.take(2 * t_cap * d.d_model);
+  L.q = b.take(2 * t_cap * hq);
+  L.k = b.take(2 * t_cap * dkv);
+  L.v = b.take(2 * t_cap * dkv);
+  L.ao = b.take(2 * t_cap * hq);
+  L.hmid = b.take(2 * t_cap * d.d_ffn);
+  L.yl = b.take(2 * static_cast<size_t>(L.n_pad) * d.d_model);
+  const size_t nl = d.n_layers;
+  L.act = b.take(nl * B);
+  L.seg = b.take(sizeof(int4) * nl * B);
+  L.qkv = b.take(sizeof(int4) * nl * L.qkv_cap);
+  L.o = b.take(sizeof(int4) * nl * L.o_cap);
+  L.gu = b.take(sizeof(int4) * nl * L.gu_cap);
+  L.dn = b.take(sizeof(int4) * nl * L.dn_cap);
+  L.attn = b.take(sizeof(int4) * nl * L.attn_cap);
+  L.counts = b.take(sizeof(int) * 5 * nl);
+  L.total = b.off;
+  return L;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+svl_status check_ws(void* ws, size_t bytes, size_t need) {
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255)) return SVL_ERR_WORKSPACE;
+  return bytes < need ? SVL_ERR_WORKSPACE : SVL_OK;
+}
+
+GemmParams base_params(const svl_model* m) {
+  GemmParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.status = m->d_status;
+  return p;
+}
+
+int gemm_grid(const svl_model* m, int64_t tiles) {
+  int64_t g = std::min<int64_t>(m->num_sms, tiles);
+  return static_cast<int>(std::max<int64_t>(g, 1));
+}
+
+svl_status launch(EpiKind kind, const svl_model* m, const GemmParams& p, int64_t tiles, cudaStream_t s) {
+  if (tiles <= 0) return SVL_OK;
+  g_launches++;
+  return launch_gemm(kind, p, gemm_grid(m, tiles), s) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
+}
+
+svl_status last_error() { return cudaGetLastError() == cudaSuccess ? SVL_OK : SVL_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+const char* svl_status_string(svl_status s) {
+  switch (s) {
+    case SVL_OK: return "ok";
+    case SVL_ERR_INVALID_ARG: return "invalid argument";
+    case SVL_ERR_SHAPE: return "shape mismatch";
+    case SVL_ERR_UNSUPPORTED: return "unsupported dimensions";
+    case SVL_ERR_CUDA: return "CUDA error";
+    case SVL_ERR_NONFINITE: return "non-finite token logit";
+    case SVL_ERR_TIMEOUT: return "device wait timed out";
+    case SVL_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+  }
+  return "unknown status";
+}
+
+uint64_t svl_launch_count(void) { return g_launches.load(); }
+
+svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, svl_model** out) {
+  if (!desc || !w || !out) return SVL_ERR_INVALID_ARG;
+  *out = nullptr;
+  const svl_model_desc& d = *desc;
+  if (d.n_layers <= 0 || d.d_model <= 0 || d.n_heads <= 0 || d.n_kv_heads <= 0 || d.d_ffn <= 0 || d.vocab <= 0 ||
+      d.n_groups <= 0 || d.n_prefix < 0 || d.c_vis <= 0 || d.h_ctrl <= 0 || d.proj_hidden < 0 || d.max_seq <= 0 ||
+      !(d.rms_eps > 0.f) || !(d.rope_theta > 0.f))
+    return SVL_ERR_INVALID_ARG;
+  if (d.d_model % d.n_heads) return SVL_ERR_UNSUPPORTED;
+  const int dh = d.d_model / d.n_heads;
+  const int G = d.n_groups;
+  if (dh != 64 && dh != 128) return SVL_ERR_UNSUPPORTED;
+  if (G > 8 || d.n_heads % G || d.n_kv_heads % G || d.n_heads % d.n_kv_heads) return SVL_ERR_UNSUPPORTED;
+  if ((d.d_ffn / G) % 64 || d.d_ffn % G) return SVL_ERR_UNSUPPORTED;
+  if (((d.n_heads / G) * dh) % 64) return SVL_ERR_UNSUPPORTED;
+  if (d.d_model % 64 || d.c_vis % 64 || d.proj_hidden % 64) return SVL_ERR_UNSUPPORTED;
+  if (d.h_ctrl % 16 || d.h_ctrl > 256) return SVL_ERR_UNSUPPORTED;
+  if (d.proj_hidden == 0 && d.c_vis != d.d_model) return SVL_ERR_UNSUPPORTED;
+  // Eq. 8 times G must stay exact in double precision at the longest sequence
+  {
+    const double S = d.max_seq, D = d.d_model, Dkv = static_cast<double>(d.n_kv_heads) * dh;
+    const double c = G * d.n_layers * ((4 * D * D + 4 * D * Dkv + 6 * D * d.d_ffn) * S + 4 * D * S * S) +
+                     G * 2.0 * D * d.vocab * S;
+    if (c >= 9.0e15) return SVL_ERR_UNSUPPORTED;
+  }
+  if (!w->ctrl_w1 || !w->ctrl_w2 || !w->bud_w1 || !w->bud_w2 || !w->embed || !w->final_norm || !w->lm_head ||
+      !w->layers)
+    return SVL_ERR_INVALID_ARG;
+  if (d.proj_hidden && (!w->proj_w1 || !w->proj_w2)) return SVL_ERR_INVALID_ARG;
+  if (!encode_fn()) return SVL_ERR_CUDA;
+
+  svl_model* m = new svl_model();
+  m->d = d;
+  m->w = *w;
+  m->layers.assign(w->layers, w->layers + d.n_layers);
+  m->w.layers = m->layers.data();
+  cudaGetDevice(&m->device);
+  cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+  const int64_t dkv = static_cast<int64_t>(d.n_kv_heads) * dh, hq = static_cast<int64_t>(d.n_heads) * dh;
+  bool ok = true;
+  m->tm_layer.resize(static_cast<size_t>(d.n_layers) * 7);
+  for (int l = 0; l < d.n_layers && ok; ++l) {
+    const svl_layer_weights& lw = m->layers[l];
+    if (!lw.wq || !lw.wk || !lw.wv || !lw.wo || !lw.wg || !lw.wu || !lw.wd || !lw.attn_norm || !lw.ffn_norm) {
+      ok = false;
+      break;
+    }
+    CUtensorMap* t = &m->tm_layer[static_cast<size_t>(l) * 7];
+    ok = make_map(t + 0, lw.wq, hq, d.d_model) && make_map(t + 1, lw.wk, dkv, d.d_model) &&
+         make_map(t + 2, lw.wv, dkv, d.d_model) && make_map(t + 3, lw.wo, d.d_model, hq) &&
+         make_map(t + 4, lw.wg, d.d_ffn, d.d_model) && make_map(t + 5, lw.wu, d.d_ffn, d.d_model) &&
+         make_map(t + 6, lw.wd, d.d_model, d.d_ffn);
+  }
+  ok = ok && make_map(&m->tm_ctrl_w1, w->ctrl_w1, d.h_ctrl, d.c_vis) &&
+       make_map(&m->tm_lm_head, w->lm_head, d.vocab, d.d_model);
+  if (ok && d.proj_hidden)
+    ok = make_map(&m->tm_proj_w1, w->proj_w1, d.proj_hidden, d.c_vis) &&
+         make_map(&m->tm_proj_w2, w->proj_w2, d.d_model, d.proj_hidden);
+  if (!ok) {
+    delete m;
+    return SVL_ERR_INVALID_ARG;
+  }
+  if (cudaMalloc(&m->d_status, sizeof(uint32_t)) != cudaSuccess ||
+      cudaMalloc(&m->rope_cs, sizeof(float2) * static_cast<size_t>(d.max_seq) * (dh / 2)) != cudaSuccess) {
+    svl_model_destroy(m);
+    return SVL_ERR_CUDA;
+  }
+  cudaMemset(m->d_status, 0, sizeof(uint32_t));
+  launch_rope_table(m->rope_cs, d.max_seq, dh, static_cast<double>(d.rope_theta), 0);
+  g_launches++;
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    svl_model_destroy(m);
+    return SVL_ERR_CUDA;
+  }
+  *out = m;
+  return SVL_OK;
+}
+
+void svl_model_destroy(svl_model* m) {
+  if (!m) return;
+  if (m->d_status) cudaFree(m->d_status);
+  if (m->rope_cs) cudaFree(m->rope_cs);
+  delete m;
+}
+
+size_t svl_workspace_size(const svl_model* m, int32_t max_batch, int64_t max_vis_total, int64_t max_text_total) {
+  if (!m || max_batch <= 0 || max_vis_total < 0 || max_text_total < 0) return 0;
+  const size_t a = sel_layout(m->d, max_batch, max_vis_total).total;
+  const size_t b = pack_layout(m->d, max_vis_total).total;
+  const size_t c = pre_layout(m->d, max_batch, max_vis_total + max_text_total).total;
+  return std::max(a, std::max(b, c));
+}
+
+svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
+                            const int32_t* vis_off, const int32_t* text_len, const float* budget,
+                            const int32_t* keep_count, const uint8_t* layer_gate, const uint8_t* group_gate,
+                            float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
+                            void* ws, size_t ws_bytes, void* stream) {
+  if (!m || B <= 0 || n_vis_total < 0 || !vis_off || !text_len || !budget || !layer_gate || !group_gate ||
+      !scores || !k || !kept_idx || !kept_off)
+    return SVL_ERR_INVALID_ARG;
+  if (n_vis_total > 0 && (!vis_feats || !aligned16(vis_feats))) return SVL_ERR_INVALID_ARG;
+  const SelLayout L = sel_layout(m->d, B, n_vis_total);
+  svl_status st = check_ws(ws, ws_bytes, L.total);
+  if (st != SVL_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const svl_model_desc& d = m->d;
+  float* e_b = at<float>(ws, L.e_b);
+
+  launch_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.bud_w1),
+                      static_cast<const __nv_bfloat16*>(m->w.bud_w2), d.h_ctrl, B, e_b, s);
+  g_launches++;
+
+  if (n_vis_total > 0) {
+    GemmParams p = base_params(m);
+    if (!make_map(&p.mapA, vis_feats, n_vis_total, d.c_vis)) return SVL_ERR_INVALID_ARG;
+    p.mapB[0] = m->tm_ctrl_w1;
+    p.grid_m = (n_vis_total + kBM - 1) / kBM;
+    p.grid_n = 1;
+    p.bn = d.h_ctrl;
+    p.m_limit = n_vis_total;
+    p.n_limit = d.h_ctrl;
+    p.K = d.c_vis;
+    p.kgroup = d.c_vis;
+    p.out[0] = scores;
+    p.e_b = e_b;
+    p.seg_off = vis_off;
+    p.n_seg = B;
+    p.w2 = static_cast<const __nv_bfloat16*>(m->w.ctrl_w2);
+    p.c2 = m->w.ctrl_c2;
+    st = launch(EPI_SCORE, m, p, p.grid_m, s);
+    if (st != SVL_OK) return st;
+  }
+
+  SelectArgs a;
+  a.scores = scores;
+  a.vis_off = vis_off;
+  a.text_len = text_len;
+  a.budget = budget;
+  a.keep_count = keep_count;
+  a.layer_gate = layer_gate;
+  a.group_gate = group_gate;
+  a.L = d.n_layers;
+  a.G = d.n_groups;
+  a.P = d.n_prefix;
+  a.D = d.d_model;
+  a.Dkv = static_cast<long long>(d.n_kv_heads) * (d.d_model / d.n_heads);
+  a.Di = d.d_ffn;
+  a.V = d.vocab;
+  a.k_out = k;
+  a.flags = sample_flags;
+  a.kept_local = at<int>(ws, L.kept_local);
+  launch_select(a, B, s);
+  g_launches++;
+  launch_compact(B, vis_off, k, a.kept_local, kept_idx, kept_off, at<int>(ws, L.scalars), s);
+  g_launches++;
+  return last_error();
+}
+
+svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text_total, const void* vis_feats,
+                    const int32_t* vis_off, const int32_t* kept_idx, const int32_t* kept_off,
+                    const int32_t* text_ids, const int32_t* text_off, void* X, int32_t* cu_seqlens, int32_t* pos,
+                    void* ws, size_t ws_bytes, void* stream) {
+  if (!m || B <= 0 || n_vis_total < 0 || n_text_total < 0 || !vis_off || !kept_idx || !kept_off || !text_off ||
+      !X || !cu_seqlens || !pos)
+    return SVL_ERR_INVALID_ARG;
+  if ((n_text_total > 0 && !text_ids) || (n_vis_total > 0 && !vis_feats)) return SVL_ERR_INVALID_ARG;
+  if (!aligned16(X) || (vis_feats && !aligned16(vis_feats))) return SVL_ERR_INVALID_ARG;
+  const PackLayout L = pack_layout(m->d, n_vis_total);
+  svl_status st = check_ws(ws, ws_bytes, L.total);
+  if (st != SVL_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const svl_model_desc& d = m->d;
+  const int64_t t_cap = static_cast<int64_t>(n_vis_total) + n_text_total;
+  if (t_cap > INT32_MAX / 2) return SVL_ERR_SHAPE;
+
+  PackArgs a;
+  a.B = B;
+  a.D = d.d_model;
+  a.c_vis = d.c_vis;
+  a.V = d.vocab;
+  a.t_cap = static_cast<int>(t_cap);
+  a.vis = static_cast<const __nv_bfloat16*>(vis_feats);
+  a.vis_off = vis_off;
+  a.kept_idx = kept_idx;
+  a.kept_off = kept_off;
+  a.text_ids = text_ids;
+  a.text_off = text_off;
+  a.embed = static_cast<const __nv_bfloat16*>(m->w.embed);
+  a.X = static_cast<__nv_bfloat16*>(X);
+  a.cu_seqlens = cu_seqlens;
+  a.pos = pos;
+  a.t_total = at<int>(ws, L.scalars) + 1;
+  a.use_projector = d.proj_hidden ? 1 : 0;
+  a.stage = d.proj_hidden ? at<__nv_bfloat16>(ws, L.stage) : nullptr;
+  a.row_map = d.proj_hidden ? at<int>(ws, L.row_map) : nullptr;
+  a.status = m->d_status;
+  launch_pack_offsets(a, s);
+  g_launches++;
+  launch_pack_gather(a, s);
+  g_launches++;
+
+  if (d.proj_hidden && n_vis_total > 0) {
+    GemmParams p = base_params(m);
+    if (!make_map(&p.mapA, a.stage, n_vis_total, d.c_vis)) return SVL_ERR_CUDA;
+    p.mapB[0] = m->tm_proj_w1;
+    p.grid_m = (n_vis_total + kBM - 1) / kBM;
+    p.grid_n = (d.proj_hidden + 255) / 256;
+    p.bn = 256;
+    p.m_limit_dev = kept_off + B;
+    p.m_limit = n_vis_total;
+    p.n_limit = d.proj_hidden;
+    p.K = d.c_vis;
+    p.kgroup = d.c_vis;
+    p.out[0] = at<__nv_bfloat16>(ws, L.hp);
+    p.ld[0] = d.proj_hidden;
+    st = launch(EPI_GELU, m, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s);
+    if (st != SVL_OK) return st;
+
+    GemmParams q = base_params(m);
+    if (!make_map(&q.mapA, at<__nv_bfloat16>(ws, L.hp), n_vis_total, d.proj_hidden)) return SVL_ERR_CUDA;
+    q.mapB[0] = m->tm_proj_w2;
+    q.grid_m = p.grid_m;
+    q.grid_n = (d.d_model + 255) / 256;
+    q.bn = 256;
+    q.m_limit_dev = kept_off + B;
+    q.m_limit = n_vis_total;
+    q.n_limit = d.d_model;
+    q.K = d.proj_hidden;
+    q.kgroup = d.proj_hidden;
+    q.out[0] = X;
+    q.ld[0] = d.d_model;
+    q.row_map = a.row_map;
+    st = launch(EPI_ROWMAP, m, q, static_cast<int64_t>(q.grid_m) * q.grid_n, s);
+    if (st != SVL_OK) return st;
+  }
+  return last_error();
+}
+
+svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                             const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
+                             int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream) {
+  if (!m || B <= 0 || t_cap <= 0 || !X || !cu_seqlens || !pos || !layer_gate || !group_gate || !logits)
+    return SVL_ERR_INVALID_ARG;
+  if (logits_mode != SVL_LOGITS_LAST && logits_mode != SVL_LOGITS_ALL) return SVL_ERR_INVALID_ARG;
+  if (!aligned16(X)) return SVL_ERR_INVALID_ARG;
+  const PreLayout L = pre_layout(m->d, B, t_cap);
+  svl_status st = check_ws(ws, ws_bytes, L.total);
+  if (st != SVL_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const svl_model_desc& d = m->d;
+  const int dh = d.d_model / d.n_heads;
+  const int hq = d.n_heads * dh, dkv = d.n_kv_heads * dh;
+  const int nl = d.n_layers;
+  int* counts = at<int>(ws, L.counts);
+
+  ScheduleArgs sa;
+  sa.B = B;
+  sa.L = nl;
+  sa.G = d.n_groups;
+  sa.P = d.n_prefix;
+  sa.A = d.n_heads;
+  sa.Akv = d.n_kv_heads;
+  sa.dh = dh;
+  sa.D = d.d_model;
+  sa.Di = d.d_ffn;
+  sa.cu_seqlens = cu_seqlens;
+  sa.layer_gate = layer_gate;
+  sa.group_gate = group_gate;
+  sa.act = at<uint8_t>(ws, L.act);
+  sa.seg = at<int4>(ws, L.seg);
+  sa.qkv_tiles = at<int4>(ws, L.qkv);
+  sa.qkv_cap = L.qkv_cap;
+  sa.qkv_count = counts;
+  sa.o_tiles = at<int4>(ws, L.o);
+  sa.o_cap = L.o_cap;
+  sa.o_count = counts + nl;
+  sa.gu_tiles = at<int4>(ws, L.gu);
+  sa.gu_cap = L.gu_cap;
+  sa.gu_count = counts + 2 * nl;
+  sa.dn_tiles = at<int4>(ws, L.dn);
+  sa.dn_cap = L.dn_cap;
+  sa.dn_count = counts + 3 * nl;
+  sa.attn_items = at<int4>(ws, L.attn);
+  sa.attn_cap = L.attn_cap;
+  sa.attn_count = counts + 4 * nl;
+  sa.status = m->d_status;
+  launch_schedule(sa, s);
+  g_launches++;
+
+  __nv_bfloat16* xn = at<__nv_bfloat16>(ws, L.xn);
+  __nv_bfloat16* qb = at<__nv_bfloat16>(ws, L.q);
+  __nv_bfloat16* kb = at<__nv_bfloat16>(ws, L.k);
+  __nv_bfloat16* vb = at<__nv_bfloat16>(ws, L.v);
+  __nv_bfloat16* ao = at<__nv_bfloat16>(ws, L.ao);
+  __nv_bfloat16* hm = at<__nv_bfloat16>(ws, L.hmid);
+  CUtensorMap map_xn, map_ao, map_hm;
+  if (!make_map(&map_xn, xn, t_cap, d.d_model) || !make_map(&map_ao, ao, t_cap, hq) ||
+      !make_map(&map_hm, hm, t_cap, d.d_ffn))
+    return SVL_ERR_CUDA;
+
+  NormArgs na;
+  na.t_cap = t_cap;
+  na.D = d.d_model;
+  na.B = B;
+  na.eps = d.rms_eps;
+  na.X = static_cast<const __nv_bfloat16*>(X);
+  na.Y = xn;
+  na.cu_seqlens = cu_seqlens;
+
+  AttnArgs aa;
+  aa.Q = qb;
+  aa.K = kb;
+  aa.V = vb;
+  aa.O = ao;
+  aa.cap = L.attn_cap;
+  aa.A = d.n_heads;
+  aa.Akv = d.n_kv_heads;
+  aa.dh = dh;
+  aa.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(dh)));
+
+  for (int l = 0; l < nl; ++l) {
+    const svl_layer_weights& lw = m->layers[l];
+    const CUtensorMap* tm = &m->tm_layer[static_cast<size_t>(l) * 7];
+    na.act = sa.act + static_cast<size_t>(l) * B;
+    na.gain = static_cast<const __nv_bfloat16*>(lw.attn_norm);
+    launch_rmsnorm(na, s);
+    g_launches++;
+
+    GemmParams p = base_params(m);
+    p.mapA = map_xn;
+    p.mapB[0] = tm[0];
+    p.mapB[1] = tm[1];
+    p.mapB[2] = tm[2];
+    p.tiles = sa.qkv_tiles + static_cast<size_t>(l) * L.qkv_cap;
+    p.tile_count = counts + l;
+    p.max_tiles = L.qkv_cap;
+    p.K = d.d_model;
+    p.kgroup = d.d_model;
+    p.out[0] = qb;
+    p.out[1] = kb;
+    p.out[2] = vb;
+    p.ld[0] = hq;
+    p.ld[1] = dkv;
+    p.ld[2] = dkv;
+    p.pos = pos;
+    p.rope_cs = m->rope_cs;
+    p.rope_rows = d.max_seq;
+    p.d_head = dh;
+    if ((st = launch(EPI_QKV_ROPE, m, p, L.qkv_cap, s)) != SVL_OK) return st;
+
+    aa.items = sa.attn_items + static_cast<size_t>(l) * L.attn_cap;
+    aa.count = counts + 4 * nl + l;
+    launch_attention(aa, s);
+    g_launches++;
+
+    p = base_params(m);
+    p.mapA = map_ao;
+    p.mapB[0] = tm[3];
+    p.tiles = sa.o_tiles + static_cast<size_t>(l) * L.o_cap;
+    p.tile_count = counts + nl + l;
+    p.max_tiles = L.o_cap;
+    p.K = hq;
+    p.kgroup = hq / d.n_groups;
+    p.out[0] = X;
+    p.ld[0] = d.d_model;
+    if ((st = launch(EPI_RESID, m, p, L.o_cap, s)) != SVL_OK) return st;
+
+    na.gain = static_cast<const __nv_bfloat16*>(lw.ffn_norm);
+    launch_rmsnorm(na, s);
+    g_launches++;
+
+    p = base_params(m);
+    p.mapA = map_xn;
+    p.mapB[0] = tm[4];
+    p.mapB[1] = tm[5];
+    p.b_split = 1;
+    p.tiles = sa.gu_tiles + static_cast<size_t>(l) * L.gu_cap;
+    p.tile_count = counts + 2 * nl + l;
+    p.max_tiles = L.gu_cap;
+    p.K = d.d_model;
+    p.kgroup = d.d_model;
+    p.out[0] = hm;
+    p.ld[0] = d.d_ffn;
+    if ((st = launch(EPI_SWIGLU, m, p, L.gu_cap, s)) != SVL_OK) return st;
+
+    p = base_params(m);
+    p.mapA = map_hm;
+    p.mapB[0] = tm[6];
+    p.tiles = sa.dn_tiles + static_cast<size_t>(l) * L.dn_cap;
+    p.tile_count = counts + 3 * nl + l;
+    p.max_tiles = L.dn_cap;
+    p.K = d.d_ffn;
+    p.kgroup = d.d_ffn / d.n_groups;
+    p.out[0] = X;
+    p.ld[0] = d.d_model;
+    if ((st = launch(EPI_RESID, m, p, L.dn_cap, s)) != SVL_OK) return st;
+  }
+
+  // final norm + LM head
+  na.gain = static_cast<const __nv_bfloat16*>(m->w.final_norm);
+  na.act = nullptr;
+  GemmParams p = base_params(m);
+  if (logits_mode == SVL_LOGITS_LAST) {
+    const int n_pad = ((B + 15) / 16) * 16;
+    na.Y = at<__nv_bfloat16>(ws, L.yl);
+    launch_final_last_rows(na, n_pad, s);
+    g_launches++;
+    p.mapA = m->tm_lm_head;
+    if (!make_map(&p.mapB[0], na.Y, n_pad, d.d_model)) return SVL_ERR_CUDA;
+    p.grid_m = (d.vocab + kBM - 1) / kBM;
+    p.grid_n = (n_pad + 255) / 256;
+    p.bn = std::min(n_pad, 256);
+    p.m_limit = d.vocab;
+    p.n_limit = B;
+    p.K = d.d_model;
+    p.kgroup = d.d_model;
+    p.out[0] = logits;
+    p.ld[0] = d.vocab;
+    if ((st = launch(EPI_LOGITS_T, m, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
+  } else {
+    launch_rmsnorm(na, s);
+    g_launches++;
+    p.mapA = map_xn;
+    p.mapB[0] = m->tm_lm_head;
+    p.grid_m = (t_cap + kBM - 1) / kBM;
+    p.grid_n = (d.vocab + 255) / 256;
+    p.bn = 256;
+    p.m_limit_dev = cu_seqlens + B;
+    p.m_limit = t_cap;
+    p.n_limit = d.vocab;
+    p.K = d.d_model;
+    p.kgroup = d.d_model;
+    p.out[0] = logits;
+    p.ld[0] = d.vocab;
+    if ((st = launch(EPI_F32, m, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
+  }
+  return last_error();
+}
+
+svl_status svl_flops(const svl_model_desc* d, int32_t s_text, int32_t s_vis, int32_t n_vis, const uint8_t* lg,
+                     const uint8_t* gg, double* eq8, double* exec) {
+  if (!d || s_text < 0 || s_vis < 0 || n_vis < 0 || d->n_heads <= 0 || d->n_groups <= 0) return SVL_ERR_INVALID_ARG;
+  const int64_t D = d->d_model, dh = d->d_model / d->n_heads, Dkv = d->n_kv_heads * dh, Di = d->d_ffn, V = d->vocab;
+  const int64_t G = d->n_groups, S = static_cast<int64_t>(s_text) + s_vis;
+  int64_t n_on = 0;
+  for (int l = 0; l < d->n_layers; ++l)
+    for (int j = 0; j < G; ++j)
+      n_on += (l < d->n_prefix || !lg || !gg || (lg[l] && gg[l * G + j])) ? 1 : 0;
+  const int64_t lin = 4 * D * D + 4 * D * Dkv + 6 * D * Di;
+  const int64_t cG = n_on * (lin * S + 4 * D * S * S) + G * 2 * D * V * S;
+  if (eq8) *eq8 = static_cast<double>(cG) / static_cast<double>(G);
+  if (exec) {
+    double f = 2.0 * n_vis * d->c_vis * d->h_ctrl;
+    if (d->proj_hidden) f += 2.0 * s_vis * (static_cast<double>(d->c_vis) * d->proj_hidden + static_cast<double>(d->proj_hidden) * D);
+    f += static_cast<double>(n_on) * (static_cast<double>(lin) * S + 2.0 * D * S * (S + 1)) / G;
+    f += 2.0 * D * V;
+    *exec = f;
+  }
+  return SVL_OK;
+}
+
+svl_status svl_get_device_status(svl_model* m, void* stream, uint32_t* code) {
+  if (!m || !code) return SVL_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(code, m->d_status, sizeof(uint32_t), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return SVL_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return SVL_ERR_CUDA;
+  if (cudaMemsetAsync(m->d_status, 0, sizeof(uint32_t), s) != cudaSuccess) return SVL_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return SVL_ERR_CUDA;
+  return SVL_OK;
+}
+
+}  // extern "C"

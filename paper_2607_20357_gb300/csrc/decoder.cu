@@ -1,0 +1,274 @@
+// Device-side schedule of the gated decoder (Sec. 3.2) and the row kernels
+// around the GEMMs: RMSNorm, final norm of the last rows, RoPE table.
+//
+// For every layer l the schedule kernel turns the gates into work lists, so
+// that gated-off work is never issued and the host never learns k or T:
+//  * e_{b,l,j} = (l < P) or (layer_gate[b,l] and group_gate[b,l,j]);
+//  * consecutive samples with the same non-zero group mask form one row
+//    segment (samples with mask 0 skip the layer: residual bypass);
+//  * QKV tiles cover only the Q/K/V columns of active groups (column runs of
+//    consecutive active groups), gate/up tiles only active FFN channels;
+//    O and down tiles carry the mask so their K loop visits only active
+//    groups' rows of W_O / W_down;
+//  * attention items are (sample, active head, 64-query block).
+#include "kernels.cuh"
+
+namespace svl {
+
+constexpr int kMaxNT = 512;
+
+struct NTile {
+  int n0, ncols, mat;
+};
+
+// Column runs of consecutive active groups, cut into tiles of `step`.
+SVL_DEVINL int build_runs(NTile* out, int cnt, int mask, int G, int width, int step, int mat) {
+  int j = 0;
+  while (j < G) {
+    if (!((mask >> j) & 1)) { ++j; continue; }
+    int j1 = j;
+    while (j1 + 1 < G && ((mask >> (j1 + 1)) & 1)) ++j1;
+    const int c0 = j * width, c1 = (j1 + 1) * width;
+    for (int n0 = c0; n0 < c1 && cnt < kMaxNT; n0 += step) out[cnt++] = {n0, min(step, c1 - n0), mat};
+    j = j1 + 1;
+  }
+  return cnt;
+}
+
+// Emits mt x nt tiles of one segment, n-tiles in bands of kNBand (a band
+// sweeps all m-tiles before the next band starts, so concurrent CTAs share
+// the same weight columns in L2).
+__device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const NTile* nt, int n_nt, int kmask,
+                           uint32_t* status) {
+  const int mt = (r1 - r0 + kBM_SCHED - 1) / kBM_SCHED;
+  const int total = mt * n_nt;
+  for (int t = threadIdx.x; t < total; t += blockDim.x) {
+    const int band = t / (mt * kNBand);
+    const int rem = t - band * mt * kNBand;
+    const int bw = min(kNBand, n_nt - band * kNBand);
+    const int mi = rem / bw;
+    const int ni = band * kNBand + rem % bw;
+    const int m0 = r0 + mi * kBM_SCHED;
+    const int idx = base + t;
+    if (idx >= cap) {
+      report(status, SVL_DEV_BAD_INDEX);
+      continue;
+    }
+    const NTile n = nt[ni];
+    tiles[idx] = make_int4(m0, min(m0 + kBM_SCHED, r1), n.n0, n.ncols | (n.mat << 16) | (kmask << 24));
+  }
+}
+
+__global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
+  __shared__ NTile nt[kMaxNT];
+  __shared__ int s_nseg, s_nnt;
+  __shared__ int s_heads[256];
+  const int l = blockIdx.x, tid = threadIdx.x;
+  const int B = a.B, G = a.G;
+  int4* seg = a.seg + static_cast<size_t>(l) * B;
+  uint8_t* act = a.act + static_cast<size_t>(l) * B;
+
+  if (tid == 0) {
+    int ns = 0;
+    for (int b = 0; b < B; ++b) {
+      int mask = 0;
+      for (int j = 0; j < G; ++j) {
+        const bool e = (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * G + j]);
+        mask |= e ? (1 << j) : 0;
+      }
+      const int r0 = a.cu_seqlens[b], r1 = a.cu_seqlens[b + 1];
+      act[b] = (mask != 0 && r1 > r0) ? 1 : 0;
+      if (mask == 0 || r1 <= r0) continue;
+      if (ns > 0 && seg[ns - 1].z == mask && seg[ns - 1].y == r0) {
+        seg[ns - 1].y = r1;
+      } else {
+        seg[ns] = make_int4(r0, r1, mask, 0);
+        ++ns;
+      }
+    }
+    s_nseg = ns;
+  }
+  __syncthreads();
+  const int nseg = s_nseg;
+  const int hq = (a.A / G) * a.dh, hk = (a.Akv / G) * a.dh;
+
+  // ---- QKV (N-sparse over active groups' Q, K, V columns)
+  int off = 0;
+  for (int s = 0; s < nseg; ++s) {
+    const int4 sg = seg[s];
+    if (tid == 0) {
+      int c = build_runs(nt, 0, sg.z, G, hq, 256, 0);
+      c = build_runs(nt, c, sg.z, G, hk, 256, 1);
+      c = build_runs(nt, c, sg.z, G, hk, 256, 2);
+      s_nnt = c;
+    }
+    __syncthreads();
+    emit_tiles(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, sg.x, sg.y, nt, s_nnt, 0, a.status);
+    off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
+    __syncthreads();
+  }
+  if (tid == 0) a.qkv_count[l] = min(off, a.qkv_cap);
+
+  // ---- O projection (K-sparse: kmask = segment mask), all D columns
+  off = 0;
+  if (tid == 0) s_nnt = build_runs(nt, 0, 1, 1, a.D, 256, 0);
+  __syncthreads();
+  for (int s = 0; s < nseg; ++s) {
+    const int4 sg = seg[s];
+    emit_tiles(a.o_tiles + static_cast<size_t>(l) * a.o_cap, off, a.o_cap, sg.x, sg.y, nt, s_nnt, sg.z, a.status);
+    off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
+  }
+  if (tid == 0) a.o_count[l] = min(off, a.o_cap);
+  // ---- down projection: same tiles shape as O
+  off = 0;
+  for (int s = 0; s < nseg; ++s) {
+    const int4 sg = seg[s];
+    emit_tiles(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, off, a.dn_cap, sg.x, sg.y, nt, s_nnt, sg.z, a.status);
+    off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
+  }
+  if (tid == 0) a.dn_count[l] = min(off, a.dn_cap);
+  __syncthreads();
+
+  // ---- gate/up (N-sparse over active FFN channels, 128 per tile)
+  off = 0;
+  for (int s = 0; s < nseg; ++s) {
+    const int4 sg = seg[s];
+    if (tid == 0) s_nnt = build_runs(nt, 0, sg.z, G, a.Di / G, 128, 0);
+    __syncthreads();
+    emit_tiles(a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, off, a.gu_cap, sg.x, sg.y, nt, s_nnt, 0, a.status);
+    off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
+    __syncthreads();
+  }
+  if (tid == 0) a.gu_count[l] = min(off, a.gu_cap);
+
+  // ---- attention items: per active sample, 64-query blocks (latest first), active heads
+  off = 0;
+  int4* items = a.attn_items + static_cast<size_t>(l) * a.attn_cap;
+  const int hpg = a.A / G;
+  for (int s = 0; s < nseg; ++s) {
+    const int4 sg = seg[s];
+    if (tid == 0) {
+      int nh = 0;
+      for (int j = 0; j < G; ++j)
+        if ((sg.z >> j) & 1)
+          for (int h = 0; h < hpg && nh < 256; ++h) s_heads[nh++] = j * hpg + h;
+      s_nnt = nh;
+    }
+    __syncthreads();
+    const int nh = s_nnt;
+    // samples inside the segment
+    int lo = 0, hi = B;
+    while (hi - lo > 1) {  // first sample of the segment
+      const int mid = (lo + hi) >> 1;
+      if (a.cu_seqlens[mid] <= sg.x) lo = mid; else hi = mid;
+    }
+    for (int b = lo; b < B && a.cu_seqlens[b] < sg.y; ++b) {
+      const int r0 = a.cu_seqlens[b], r1 = a.cu_seqlens[b + 1];
+      if (r1 <= r0) continue;
+      const int nq = (r1 - r0 + kAttnQ - 1) / kAttnQ;
+      const int total = nq * nh;
+      for (int t = tid; t < total; t += blockDim.x) {
+        const int qi = nq - 1 - t / nh;
+        const int h = s_heads[t % nh];
+        const int q0 = r0 + qi * kAttnQ;
+        const int idx = off + t;
+        if (idx < a.attn_cap) items[idx] = make_int4(q0, min(q0 + kAttnQ, r1), r0, h);
+        else report(a.status, SVL_DEV_BAD_INDEX);
+      }
+      off += total;
+    }
+    __syncthreads();
+  }
+  if (tid == 0) a.attn_count[l] = min(off, a.attn_cap);
+}
+
+void launch_schedule(const ScheduleArgs& a, cudaStream_t s) { schedule_kernel<<<a.L, 256, 0, s>>>(a); }
+
+// ---------------------------------------------------------------- RMSNorm
+SVL_DEVINL int find_sample(const int* cu, int B, int r) {
+  int lo = 0, hi = B;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (cu[mid] <= r) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
+SVL_DEVINL void norm_row(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y, int D, float eps,
+                         int lane) {
+  const uint4* xv = reinterpret_cast<const uint4*>(x);
+  const uint4* gv = reinterpret_cast<const uint4*>(g);
+  uint4* yv = reinterpret_cast<uint4*>(y);
+  float ss = 0.f;
+  for (int c = lane; c < D / 8; c += 32) {
+    const uint4 u = xv[c];
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = unpack_bf16x2(w[i]);
+      ss += f.x * f.x + f.y * f.y;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const float inv = rsqrtf(ss / static_cast<float>(D) + eps);
+  for (int c = lane; c < D / 8; c += 32) {
+    const uint4 u = xv[c], gg = gv[c];
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    const uint32_t q[4] = {gg.x, gg.y, gg.z, gg.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = unpack_bf16x2(w[i]), h = unpack_bf16x2(q[i]);
+      o[i] = pack_bf16x2(f.x * inv * h.x, f.y * inv * h.y);
+    }
+    yv[c] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+__global__ void rmsnorm_kernel(NormArgs a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp;
+  const int T = a.cu_seqlens[a.B];
+  if (r >= T || r >= a.t_cap) return;
+  if (a.act && !a.act[find_sample(a.cu_seqlens, a.B, r)]) return;
+  norm_row(a.X + static_cast<size_t>(r) * a.D, a.gain, a.Y + static_cast<size_t>(r) * a.D, a.D, a.eps, lane);
+}
+
+__global__ void final_rows_kernel(NormArgs a, int n_pad) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (b >= n_pad) return;
+  __nv_bfloat16* y = a.Y + static_cast<size_t>(b) * a.D;
+  const int r1 = b < a.B ? a.cu_seqlens[b + 1] : 0, r0 = b < a.B ? a.cu_seqlens[b] : 0;
+  if (b >= a.B || r1 <= r0) {
+    for (int c = lane; c < a.D / 8; c += 32) reinterpret_cast<uint4*>(y)[c] = make_uint4(0, 0, 0, 0);
+    return;
+  }
+  norm_row(a.X + static_cast<size_t>(r1 - 1) * a.D, a.gain, y, a.D, a.eps, lane);
+}
+
+void launch_rmsnorm(const NormArgs& a, cudaStream_t s) {
+  const int grid = (a.t_cap + 7) / 8;
+  if (grid > 0) rmsnorm_kernel<<<grid, 256, 0, s>>>(a);
+}
+
+void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s) {
+  final_rows_kernel<<<(n_pad + 7) / 8, 256, 0, s>>>(a, n_pad);
+}
+
+__global__ void rope_table_kernel(float2* cs, int max_seq, int dh, double theta) {
+  const int half = dh / 2;
+  const long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
+  if (i >= static_cast<long long>(max_seq) * half) return;
+  const int p = static_cast<int>(i / half), f = static_cast<int>(i % half);
+  const double ang = static_cast<double>(p) * pow(theta, -2.0 * f / dh);
+  cs[i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
+}
+
+void launch_rope_table(float2* cs, int max_seq, int dh, double theta, cudaStream_t s) {
+  const long long n = static_cast<long long>(max_seq) * (dh / 2);
+  rope_table_kernel<<<static_cast<int>((n + 255) / 256), 256, 0, s>>>(cs, max_seq, dh, theta);
+}
+
+}  // namespace svl

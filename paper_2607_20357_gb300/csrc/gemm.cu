@@ -1,0 +1,422 @@
+// Persistent warp-specialised tcgen05 GEMM with fused epilogues (sm_103a).
+//
+//   warp 0      one thread issues TMA loads of A (128 x 64) and B (up to
+//               2 x 128 x 64) per stage into a 4-stage shared-memory ring;
+//   warp 1      allocates 512 TMEM columns; one thread issues
+//               tcgen05.mma (M = 128, N <= 256, K = 16 per instruction) and
+//               commits stage releases and accumulator-ready signals;
+//   warps 2-5   epilogue: tcgen05.ld of their 32-lane quarter of the
+//               accumulator, fused math, global stores. Two accumulators
+//               alternate so the epilogue of tile i overlaps tile i+1.
+//
+// Every wait is bounded (kWaitCycles); a time-out sets SVL_DEV_TIMEOUT in the
+// status word, stops all roles, lets in-flight copies land, frees TMEM and
+// returns.
+#include "gemm.cuh"
+
+namespace svl {
+
+struct TileInfo {
+  int m0, m_end, n0, ncols, mat, kmask;
+  bool valid;
+};
+
+SVL_DEVINL int num_tiles(const GemmParams& p) {
+  if (p.tiles) {
+    int n = *p.tile_count;
+    return n < 0 ? 0 : (n > p.max_tiles ? p.max_tiles : n);
+  }
+  return p.grid_m * p.grid_n;
+}
+
+SVL_DEVINL TileInfo get_tile(const GemmParams& p, int t) {
+  TileInfo ti;
+  if (p.tiles) {
+    int4 v = p.tiles[t];
+    ti.m0 = v.x;
+    ti.m_end = v.y;
+    ti.n0 = v.z;
+    ti.ncols = tile_ncols(v.w);
+    ti.mat = tile_mat(v.w);
+    ti.kmask = tile_kmask(v.w);
+    ti.valid = ti.ncols > 0 && ti.m_end > ti.m0 && ti.mat < 3;
+  } else {
+    int mi = t % p.grid_m, ni = t / p.grid_m;
+    int mlim = p.m_limit;
+    if (p.m_limit_dev) mlim = min(mlim, *p.m_limit_dev);
+    ti.m0 = mi * kBM;
+    ti.m_end = min(ti.m0 + kBM, mlim);
+    ti.n0 = ni * p.bn;
+    ti.ncols = min(p.bn, p.n_limit - ti.n0);
+    ti.mat = 0;
+    ti.kmask = 0;
+    ti.valid = ti.m0 < mlim && ti.ncols > 0;
+  }
+  return ti;
+}
+
+SVL_DEVINL bool kblock_on(int kb, int kmask, int kgb) {
+  return kmask == 0 || ((kmask >> (kb / kgb)) & 1);
+}
+
+SVL_DEVINL void set_abort(volatile int* abort, uint32_t* status) {
+  *abort = 1;
+  report(status, SVL_DEV_TIMEOUT);
+}
+
+// ------------------------------------------------------------------ producer
+SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* full,
+                              uint64_t* empty, volatile int* abort) {
+  const int ntiles = num_tiles(p);
+  const int nkb = p.K / kBK, kgb = p.kgroup / kBK;
+  int s = 0;
+  uint32_t ph = 0;
+  for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
+    TileInfo ti = get_tile(p, t);
+    if (!ti.valid) continue;
+    const int halves = p.b_split ? 2 : (ti.ncols > kBHalf ? 2 : 1);
+    const CUtensorMap* mb0 = p.b_split ? &p.mapB[0] : &p.mapB[ti.mat];
+    const CUtensorMap* mb1 = p.b_split ? &p.mapB[1] : &p.mapB[ti.mat];
+    const int y1 = p.b_split ? ti.n0 : ti.n0 + kBHalf;
+    const uint32_t bytes = kABytes + halves * kBHalfBytes;
+    for (int kb = 0; kb < nkb; ++kb) {
+      if (!kblock_on(kb, ti.kmask, kgb)) continue;
+      if (!mbar_wait(&empty[s], ph ^ 1, abort)) {
+        set_abort(abort, p.status);
+        return;
+      }
+      uint8_t* sa = stages + s * kStageBytes;
+      uint8_t* sb = sa + kABytes;
+      mbar_arrive_expect_tx(&full[s], bytes);
+      tma_load_2d(sa, &p.mapA, &full[s], kb * kBK, ti.m0);
+      tma_load_2d(sb, mb0, &full[s], kb * kBK, ti.n0);
+      if (halves == 2) tma_load_2d(sb + kBHalfBytes, mb1, &full[s], kb * kBK, y1);
+      if (++s == kStages) {
+        s = 0;
+        ph ^= 1;
+      }
+    }
+  }
+}
+
+// ------------------------------------------------------------------ MMA issuer
+SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, uint64_t* empty,
+                         uint64_t* tfull, uint64_t* tempty, uint32_t tmem, volatile int* abort) {
+  const int ntiles = num_tiles(p);
+  const int nkb = p.K / kBK, kgb = p.kgroup / kBK;
+  int s = 0, it = 0;
+  uint32_t ph = 0;
+  for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
+    TileInfo ti = get_tile(p, t);
+    if (!ti.valid) continue;
+    const int acc = it & 1;
+    const uint32_t aph = (it >> 1) & 1;
+    if (!mbar_wait(&tempty[acc], aph ^ 1, abort)) {
+      set_abort(abort, p.status);
+      return;
+    }
+    tc_fence_after();
+    const int n = p.b_split ? 2 * kBHalf : ((ti.ncols + 15) & ~15);
+    const uint32_t idesc = idesc_bf16_f32(kBM, n);
+    const uint32_t d = tmem + acc * kAccCols;
+    uint32_t accumulate = 0;
+    for (int kb = 0; kb < nkb; ++kb) {
+      if (!kblock_on(kb, ti.kmask, kgb)) continue;
+      if (!mbar_wait(&full[s], ph, abort)) {
+        set_abort(abort, p.status);
+        return;
+      }
+      tc_fence_after();
+      const uint32_t a0 = smem_u32(stages + s * kStageBytes);
+      const uint32_t b0 = a0 + kABytes;
+#pragma unroll
+      for (int k = 0; k < kBK / 16; ++k) {
+        tc_mma_bf16(d, smem_desc_sw128(a0 + k * 32), smem_desc_sw128(b0 + k * 32), idesc,
+                    accumulate);
+        accumulate = 1;
+      }
+      tc_commit(&empty[s]);
+      if (++s == kStages) {
+        s = 0;
+        ph ^= 1;
+      }
+    }
+    tc_commit(&tfull[acc]);
+    ++it;
+  }
+}
+
+// ------------------------------------------------------------------ epilogues
+SVL_DEVINL void store_bf16(__nv_bfloat16* dst, const float* v, int n /*16 or 32*/) {
+  uint4* d = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (i * 8 < n)
+      d[i] = make_uint4(pack_bf16x2(v[8 * i + 0], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                        pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+  }
+}
+
+SVL_DEVINL void load_bf16(const __nv_bfloat16* src, float* v, int n) {
+  const uint4* s = reinterpret_cast<const uint4*>(src);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (i * 8 < n) {
+      uint4 u = s[i];
+      float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y), c = unpack_bf16x2(u.z), d = unpack_bf16x2(u.w);
+      v[8 * i + 0] = a.x; v[8 * i + 1] = a.y; v[8 * i + 2] = b.x; v[8 * i + 3] = b.y;
+      v[8 * i + 4] = c.x; v[8 * i + 5] = c.y; v[8 * i + 6] = d.x; v[8 * i + 7] = d.y;
+    }
+  }
+}
+
+template <int KIND>
+SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, bool rv,
+                              uint32_t taddr) {
+  float v[32];
+  if constexpr (KIND == EPI_QKV_ROPE) {
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[ti.mat]);
+    const size_t ld = static_cast<size_t>(p.ld[ti.mat]);
+    if (ti.mat < 2) {
+      const int dh = p.d_head, half = dh / 2;
+      int prow = rv ? p.pos[row] : 0;
+      if (prow < 0 || prow >= p.rope_rows) {  // longer than the model's max_seq
+        report(p.status, SVL_DEV_BAD_INDEX);
+        prow = 0;
+      }
+      const float2* cs = p.rope_cs + static_cast<size_t>(prow) * half;
+      float w[32];
+      for (int hb = 0; hb < ti.ncols; hb += dh) {
+        for (int i0 = 0; i0 < half; i0 += 32) {
+          tmem_ld32(taddr + hb + i0, v);
+          tmem_ld32(taddr + hb + half + i0, w);
+          if (rv) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+              const float2 c = cs[i0 + j];
+              const float x1 = v[j], x2 = w[j];
+              v[j] = x1 * c.x - x2 * c.y;
+              w[j] = x2 * c.x + x1 * c.y;
+            }
+            __nv_bfloat16* o = out + static_cast<size_t>(row) * ld + ti.n0 + hb + i0;
+            store_bf16(o, v, 32);
+            store_bf16(o + half, w, 32);
+          }
+        }
+      }
+    } else {
+      for (int c = 0; c < ti.ncols; c += 32) {
+        tmem_ld32(taddr + c, v);
+        if (rv) store_bf16(out + static_cast<size_t>(row) * ld + ti.n0 + c, v, min(32, ti.ncols - c));
+      }
+    }
+  } else if constexpr (KIND == EPI_RESID) {
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
+    const size_t ld = static_cast<size_t>(p.ld[0]);
+    for (int c = 0; c < ti.ncols; c += 32) {
+      tmem_ld32(taddr + c, v);
+      if (rv) {
+        const int n = min(32, ti.ncols - c);
+        __nv_bfloat16* o = out + static_cast<size_t>(row) * ld + ti.n0 + c;
+        float x[32];
+        load_bf16(o, x, n);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] += x[j];
+        store_bf16(o, v, n);
+      }
+    }
+  } else if constexpr (KIND == EPI_SWIGLU) {
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
+    const size_t ld = static_cast<size_t>(p.ld[0]);
+    float u[32];
+    for (int c = 0; c < ti.ncols; c += 32) {
+      tmem_ld32(taddr + c, v);
+      tmem_ld32(taddr + kBHalf + c, u);
+      if (rv) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * u[j];
+        store_bf16(out + static_cast<size_t>(row) * ld + ti.n0 + c, v, min(32, ti.ncols - c));
+      }
+    }
+  } else if constexpr (KIND == EPI_GELU || KIND == EPI_ROWMAP) {
+    __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
+    const size_t ld = static_cast<size_t>(p.ld[0]);
+    const int orow = (KIND == EPI_ROWMAP && rv) ? p.row_map[row] : row;
+    for (int c = 0; c < ti.ncols; c += 32) {
+      tmem_ld32(taddr + c, v);
+      if (rv) {
+        if constexpr (KIND == EPI_GELU) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
+        }
+        store_bf16(out + static_cast<size_t>(orow) * ld + ti.n0 + c, v, min(32, ti.ncols - c));
+      }
+    }
+  } else if constexpr (KIND == EPI_LOGITS_T) {
+    float* out = reinterpret_cast<float*>(p.out[0]);
+    const size_t ld = static_cast<size_t>(p.ld[0]);
+    for (int c = 0; c < ti.ncols; c += 32) {
+      tmem_ld32(taddr + c, v);
+      if (rv) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (c + j < ti.ncols) out[static_cast<size_t>(ti.n0 + c + j) * ld + row] = v[j];
+      }
+    }
+  } else if constexpr (KIND == EPI_F32) {
+    float* out = reinterpret_cast<float*>(p.out[0]);
+    const size_t ld = static_cast<size_t>(p.ld[0]);
+    for (int c = 0; c < ti.ncols; c += 32) {
+      tmem_ld32(taddr + c, v);
+      if (rv) {
+        float* o = out + static_cast<size_t>(row) * ld + ti.n0 + c;
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+          if (c + j < ti.ncols) o[j] = v[j];
+      }
+    }
+  } else if constexpr (KIND == EPI_SCORE) {
+    int b = 0;
+    if (rv) {
+      int lo = 0, hi = p.n_seg;  // find b with seg_off[b] <= row < seg_off[b+1]
+      while (hi - lo > 1) {
+        int mid = (lo + hi) >> 1;
+        if (p.seg_off[mid] <= row) lo = mid; else hi = mid;
+      }
+      b = lo;
+    }
+    const int H = ti.ncols;
+    const float* eb = p.e_b + static_cast<size_t>(b) * H;
+    float z = 0.f;
+    for (int c = 0; c < H; c += 32) {
+      tmem_ld32(taddr + c, v);
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (c + j < H) z += __bfloat162float(p.w2[c + j]) * silu_f(v[j] + eb[c + j]);
+    }
+    if (rv) {
+      z += p.c2;
+      if (!isfinite(z)) report(p.status, SVL_DEV_NONFINITE);
+      reinterpret_cast<float*>(p.out[0])[row] = z;
+    }
+  }
+}
+
+template <int KIND>
+SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem,
+                              volatile int* abort) {
+  const int ntiles = num_tiles(p);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int q = warp & 3;  // TMEM lane quarter this warp may access
+  int it = 0;
+  for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
+    TileInfo ti = get_tile(p, t);
+    if (!ti.valid) continue;
+    const int acc = it & 1;
+    const uint32_t aph = (it >> 1) & 1;
+    const bool ok = mbar_wait(&tfull[acc], aph, abort);
+    __syncwarp();
+    if (!__all_sync(0xffffffffu, ok)) {
+      set_abort(abort, p.status);
+      return;
+    }
+    tc_fence_after();
+    const int row = ti.m0 + q * 32 + lane;
+    const bool rv = row < ti.m_end;
+    const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
+    epilogue_tile<KIND>(p, ti, row, rv, taddr);
+    tc_fence_before();
+    mbar_arrive(&tempty[acc]);
+    ++it;
+  }
+}
+
+// ------------------------------------------------------------------ kernel
+template <int KIND>
+__global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* stages = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(stages + kStages * kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + kStages;
+  uint64_t* tfull = bars + 2 * kStages;
+  uint64_t* tempty = bars + 2 * kStages + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 4);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 4 * 32);
+    }
+    *abort = 0;
+    fence_barrier_init();
+    fence_proxy_async();
+    prefetch_tmap(&p.mapA);
+    prefetch_tmap(&p.mapB[0]);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) producer_loop(p, stages, full, empty, abort);
+  } else if (warp == 1) {
+    if (lane == 0) mma_loop(p, stages, full, empty, tfull, tempty, tmem, abort);
+  } else {
+    epilogue_loop<KIND>(p, tfull, tempty, tmem, abort);
+  }
+
+  __syncwarp();
+  if (*abort) {
+    // Let copies and MMAs already issued land before the CTA lets go of its
+    // shared and tensor memory (about 10 ms; they finish in microseconds).
+    long long t0 = clock64();
+    while (clock64() - t0 < 20000000LL) {
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+template <int KIND>
+static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t stream) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  gemm_kernel<KIND><<<grid, kGemmThreads, kGemmSmem, stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream) {
+  switch (kind) {
+    case EPI_QKV_ROPE: return launch_kind<EPI_QKV_ROPE>(p, grid, stream);
+    case EPI_RESID: return launch_kind<EPI_RESID>(p, grid, stream);
+    case EPI_SWIGLU: return launch_kind<EPI_SWIGLU>(p, grid, stream);
+    case EPI_GELU: return launch_kind<EPI_GELU>(p, grid, stream);
+    case EPI_ROWMAP: return launch_kind<EPI_ROWMAP>(p, grid, stream);
+    case EPI_LOGITS_T: return launch_kind<EPI_LOGITS_T>(p, grid, stream);
+    case EPI_F32: return launch_kind<EPI_F32>(p, grid, stream);
+    case EPI_SCORE: return launch_kind<EPI_SCORE>(p, grid, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace svl

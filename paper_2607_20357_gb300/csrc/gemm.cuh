@@ -1,0 +1,76 @@
+// Persistent tcgen05/TMEM GEMM for sm_103a: C[M,N] = A[M,K] * B[N,K]^T with
+// bf16 K-major operands staged by TMA (128-byte swizzle) and an fp32
+// accumulator in tensor memory, followed by a fused epilogue.
+//
+// Work arrives either as an explicit device tile list (the gated layers: one
+// tile per (row segment, column run) of active groups) or as a dense grid.
+#pragma once
+
+#include "common.cuh"
+
+namespace svl {
+
+constexpr int kBM = 128;           // rows per tile (TMEM lanes)
+constexpr int kBK = 64;            // K per stage: one 128-byte swizzle row
+constexpr int kBHalf = 128;        // B rows per TMA box; a stage holds two
+constexpr int kStages = 4;
+constexpr int kABytes = kBM * kBK * 2;
+constexpr int kBHalfBytes = kBHalf * kBK * 2;
+constexpr int kStageBytes = kABytes + 2 * kBHalfBytes;
+constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2-5 epilogue
+constexpr int kAccCols = 256;      // fp32 columns per accumulator
+constexpr int kTmemCols = 512;     // two accumulators (epilogue overlaps the next tile)
+constexpr int kGemmSmem = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+
+enum EpiKind : int {
+  EPI_QKV_ROPE = 0,  // mat 0/1: RoPE then bf16 store to Q/K; mat 2: bf16 store to V
+  EPI_RESID = 1,     // out[r, n] = bf16(out[r, n] + acc)
+  EPI_SWIGLU = 2,    // out[r, n0 + c] = bf16(SiLU(acc[c]) * acc[128 + c])
+  EPI_GELU = 3,      // out[r, n] = bf16(GELU(acc))
+  EPI_ROWMAP = 4,    // out[row_map[r], n] = bf16(acc)
+  EPI_LOGITS_T = 5,  // out[n, r] = acc (fp32): swapped LM head, r = vocab id, n = sample
+  EPI_F32 = 6,       // out[r, n] = acc (fp32)
+  EPI_SCORE = 7,     // z[r] = sum_h w2[h] SiLU(acc[h] + e_b[sample(r), h]) + c2
+  EPI_COUNT = 8
+};
+
+// Tile encoding (int4): x = m0, y = m_end (rows >= m_end are not stored),
+// z = n0, w = ncols | mat << 16 | kmask << 24 (kmask 0 = every K block).
+SVL_DEVINL int tile_ncols(int w) { return w & 0xFFFF; }
+SVL_DEVINL int tile_mat(int w) { return (w >> 16) & 0xFF; }
+SVL_DEVINL int tile_kmask(int w) { return (w >> 24) & 0xFF; }
+
+struct GemmParams {
+  CUtensorMap mapA;
+  CUtensorMap mapB[3];
+  // explicit tile list (tiles != nullptr) ...
+  const int4* tiles;
+  const int* tile_count;
+  int max_tiles;
+  // ... or dense grid: grid_m x grid_n tiles of kBM x bn
+  int grid_m, grid_n, bn;
+  const int* m_limit_dev;  // rows bound read on the device (nullptr: use m_limit)
+  int m_limit, n_limit;
+  // K loop
+  int K;       // multiple of 64
+  int kgroup;  // K elements per gate group (kmask), multiple of 64
+  int b_split; // 1: B rows 0-127 from mapB[0], rows 128-255 from mapB[1] (gate | up)
+  // epilogue operands
+  void* out[3];
+  int ld[3];
+  const int* row_map;
+  const int* pos;
+  const float2* rope_cs;  // [rope_rows, d_head/2] (cos, sin)
+  int rope_rows;
+  int d_head;
+  const float* e_b;       // [B, H]
+  const int* seg_off;     // [B+1] token offsets per sample (score)
+  int n_seg;
+  const __nv_bfloat16* w2;
+  float c2;
+  uint32_t* status;
+};
+
+cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream);
+
+}  // namespace svl

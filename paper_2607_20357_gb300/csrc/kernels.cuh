@@ -1,0 +1,106 @@
+// Declarations of the non-GEMM kernels and their launchers.
+#pragma once
+
+#include "common.cuh"
+
+namespace svl {
+
+constexpr int kSelectThreads = 512;
+constexpr int kAttnQ = 64;        // query rows per attention work item
+constexpr int kNBand = 8;         // n-tiles per raster band in the tile lists
+constexpr int kBM_SCHED = 128;    // tile rows (the GEMM's M)
+
+struct SelectArgs {
+  const float* scores;
+  const int* vis_off;
+  const int* text_len;
+  const float* budget;
+  const int* keep_count;
+  const uint8_t* layer_gate;
+  const uint8_t* group_gate;
+  int L, G, P;
+  long long D, Dkv, Di, V;
+  int* k_out;
+  uint32_t* flags;
+  int* kept_local;
+};
+
+void launch_budget_embed(const float* budget, const __nv_bfloat16* w1, const __nv_bfloat16* w2, int H, int B,
+                         float* e_b, cudaStream_t s);
+void launch_select(const SelectArgs& a, int B, cudaStream_t s);
+void launch_compact(int B, const int* vis_off, const int* k, const int* kept_local, int* kept_idx, int* kept_off,
+                    int* kept_total, cudaStream_t s);
+
+// ---------------------------------------------------------------- pack
+struct PackArgs {
+  int B, D, c_vis, V;
+  int t_cap;
+  const __nv_bfloat16* vis;
+  const int* vis_off;
+  const int* kept_idx;
+  const int* kept_off;
+  const int* text_ids;
+  const int* text_off;
+  const __nv_bfloat16* embed;
+  __nv_bfloat16* X;
+  int* cu_seqlens;
+  int* pos;
+  int* t_total;            // device scalar: T
+  int use_projector;       // 1: visual rows go to the staging buffer
+  __nv_bfloat16* stage;    // [kept_total, c_vis]
+  int* row_map;            // [kept_total] -> row of X
+  uint32_t* status;
+};
+void launch_pack_offsets(const PackArgs& a, cudaStream_t s);
+void launch_pack_gather(const PackArgs& a, cudaStream_t s);
+
+// ---------------------------------------------------------------- decoder
+struct ScheduleArgs {
+  int B, L, G, P;
+  int A, Akv, dh, D, Di;
+  const int* cu_seqlens;
+  const uint8_t* layer_gate;
+  const uint8_t* group_gate;
+  // per-layer outputs (layer l at offset l * cap)
+  uint8_t* act;             // [L, B] sample active in layer
+  int4* seg;                // [L, B] row segments {r0, r1, mask, 0}
+  int4* qkv_tiles; int qkv_cap; int* qkv_count;
+  int4* o_tiles; int o_cap; int* o_count;
+  int4* gu_tiles; int gu_cap; int* gu_count;
+  int4* dn_tiles; int dn_cap; int* dn_count;
+  int4* attn_items; int attn_cap; int* attn_count;
+  uint32_t* status;
+};
+void launch_schedule(const ScheduleArgs& a, cudaStream_t s);
+
+struct NormArgs {
+  int t_cap, D, B;
+  float eps;
+  const __nv_bfloat16* X;
+  const __nv_bfloat16* gain;
+  __nv_bfloat16* Y;
+  const int* cu_seqlens;
+  const uint8_t* act;     // [B] or nullptr (every row)
+};
+void launch_rmsnorm(const NormArgs& a, cudaStream_t s);
+
+// Final norm of each sample's last row into Y[b] (rows B..n_pad-1 zeroed).
+void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s);
+
+struct AttnArgs {
+  const __nv_bfloat16* Q;   // [T, A*dh]
+  const __nv_bfloat16* K;   // [T, Akv*dh]
+  const __nv_bfloat16* V;
+  __nv_bfloat16* O;         // [T, A*dh]
+  const int4* items;        // {q0, q_end, r0, head}
+  const int* count;
+  int cap;
+  int A, Akv, dh;
+  float scale_log2;         // log2(e) / sqrt(dh)
+};
+void launch_attention(const AttnArgs& a, cudaStream_t s);
+
+// RoPE table: cs[p * half + i] = (cos, sin)(p * theta^(-2i/dh)), double precision.
+void launch_rope_table(float2* cs, int max_seq, int dh, double theta, cudaStream_t s);
+
+}  // namespace svl

@@ -1,0 +1,77 @@
+// Packing (Sec. 3: S = S_text + S_vis; Sec. 3.1: kept tokens form a
+// compressed contiguous sequence with positions 0..S-1). Sample b occupies
+// rows cu_seqlens[b]..cu_seqlens[b+1) of X: kept visual rows in ascending
+// token order, then its text rows.
+#include "kernels.cuh"
+
+namespace svl {
+
+__global__ void pack_offsets_kernel(PackArgs a) {
+  if (threadIdx.x != 0) return;
+  int t = 0;
+  a.cu_seqlens[0] = 0;
+  for (int b = 0; b < a.B; ++b) {
+    const int kb = a.kept_off[b + 1] - a.kept_off[b];
+    const int st = a.text_off[b + 1] - a.text_off[b];
+    t += max(kb, 0) + max(st, 0);
+    if (t > a.t_cap) {
+      report(a.status, SVL_DEV_BAD_INDEX);
+      t = a.t_cap;
+    }
+    a.cu_seqlens[b + 1] = t;
+  }
+  *a.t_total = t;
+}
+
+// One warp per output row.
+__global__ void pack_gather_kernel(PackArgs a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp;
+  const int T = *a.t_total;
+  if (r >= T) return;
+  int lo = 0, hi = a.B;  // sample b with cu[b] <= r < cu[b+1]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (a.cu_seqlens[mid] <= r) lo = mid; else hi = mid;
+  }
+  const int b = lo;
+  const int i = r - a.cu_seqlens[b];
+  const int kb = a.kept_off[b + 1] - a.kept_off[b];
+  if (lane == 0) a.pos[r] = i;
+  const uint4* src;
+  uint4* dst;
+  int width;
+  bool bad = false;
+  if (i < kb) {
+    const int j = a.kept_off[b] + i;
+    const int n_b = a.vis_off[b + 1] - a.vis_off[b];
+    int tok = a.kept_idx[j];
+    if (tok < 0 || tok >= n_b) { bad = true; tok = 0; }
+    src = reinterpret_cast<const uint4*>(a.vis + static_cast<size_t>(a.vis_off[b] + tok) * a.c_vis);
+    width = a.c_vis;
+    if (a.use_projector) {
+      dst = reinterpret_cast<uint4*>(a.stage + static_cast<size_t>(j) * a.c_vis);
+      if (lane == 0) a.row_map[j] = r;
+    } else {
+      dst = reinterpret_cast<uint4*>(a.X + static_cast<size_t>(r) * a.D);
+    }
+  } else {
+    int id = a.text_ids[a.text_off[b] + (i - kb)];
+    if (id < 0 || id >= a.V) { bad = true; id = 0; }
+    src = reinterpret_cast<const uint4*>(a.embed + static_cast<size_t>(id) * a.D);
+    dst = reinterpret_cast<uint4*>(a.X + static_cast<size_t>(r) * a.D);
+    width = a.D;
+  }
+  if (bad && lane == 0) report(a.status, SVL_DEV_BAD_INDEX);
+  for (int c = lane; c < width / 8; c += 32) dst[c] = bad ? make_uint4(0, 0, 0, 0) : src[c];
+}
+
+void launch_pack_offsets(const PackArgs& a, cudaStream_t s) { pack_offsets_kernel<<<1, 32, 0, s>>>(a); }
+
+void launch_pack_gather(const PackArgs& a, cudaStream_t s) {
+  const int rows_per_block = 8;
+  const int grid = (a.t_cap + rows_per_block - 1) / rows_per_block;
+  if (grid > 0) pack_gather_kernel<<<grid, rows_per_block * 32, 0, s>>>(a);
+}
+
+}  // namespace svl

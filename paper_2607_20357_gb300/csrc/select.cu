@@ -1,0 +1,224 @@
+// Token controller (Sec. 3.1; Sec. 3.3 "Inference"): budget embedding,
+// budget -> k from Eq. 8, per-sample top-k by radix select, stable compaction.
+// The token scores themselves come from the tcgen05 GEMM (EPI_SCORE).
+#include "kernels.cuh"
+
+namespace svl {
+
+// e_b = W_b2 SiLU(W_b1 PE(b)), PE(b) = [sin(1000 b w_i) | cos(1000 b w_i)],
+// w_i = 10000^(-2i/H) (Eq. 5). One block per sample, double precision.
+__global__ void budget_embed_kernel(const float* __restrict__ budget, const __nv_bfloat16* __restrict__ w1,
+                                    const __nv_bfloat16* __restrict__ w2, int H, float* __restrict__ e_b) {
+  __shared__ double pe[256];
+  __shared__ double hid[256];
+  const int b = blockIdx.x, i = threadIdx.x;
+  const double bv = static_cast<double>(budget[b]);
+  if (i < H) {
+    const int half = H / 2;
+    const int f = i < half ? i : i - half;
+    const double omega = pow(10000.0, -2.0 * f / H);
+    const double arg = 1000.0 * bv * omega;
+    pe[i] = i < half ? sin(arg) : cos(arg);
+  }
+  __syncthreads();
+  if (i < H) {
+    double s = 0.0;
+    for (int j = 0; j < H; ++j) s += static_cast<double>(__bfloat162float(w1[i * H + j])) * pe[j];
+    hid[i] = s / (1.0 + exp(-s));
+  }
+  __syncthreads();
+  if (i < H) {
+    double s = 0.0;
+    for (int j = 0; j < H; ++j) s += static_cast<double>(__bfloat162float(w2[i * H + j])) * hid[j];
+    e_b[b * H + i] = static_cast<float>(s);
+  }
+}
+
+// Orderable key: unsigned comparison of keys matches float comparison.
+SVL_DEVINL uint32_t order_key(float z) {
+  if (z == 0.0f) z = 0.0f;  // -0 and +0 are equal logits
+  const uint32_t u = __float_as_uint(z);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Exclusive block-wide prefix sum of one int per thread (blockDim.x <= 1024).
+SVL_DEVINL int block_exclusive_scan(int v, int* total, int* warp_sums) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sums[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < nw ? warp_sums[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    if (lane < nw) warp_sums[lane] = w;  // inclusive
+  }
+  __syncthreads();
+  const int base = warp > 0 ? warp_sums[warp - 1] : 0;
+  *total = warp_sums[nw - 1];
+  __syncthreads();
+  return base + x - v;
+}
+
+// One block per sample: k from the budget (largest k with Eq. 8 cost within
+// b * C_full), then the k largest logits (ties: lower index), written in
+// ascending index order to kept_local[vis_off[b] ...].
+__global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
+  __shared__ int hist[256];
+  __shared__ int warp_sums[32];
+  __shared__ int best_k;
+  __shared__ int s_prefix_cnt[2];
+  __shared__ long long n_on_sum;
+
+  const int b = blockIdx.x, tid = threadIdx.x;
+  const int v0 = a.vis_off[b], v1 = a.vis_off[b + 1];
+  const int n = max(0, v1 - v0);
+  const long long s_text = a.text_len[b];
+
+  // ---- k from the budget (Eq. 8, exact integers scaled by G)
+  if (tid == 0) {
+    long long s = 0;
+    for (int l = 0; l < a.L; ++l) {
+      int on = 0;
+      for (int j = 0; j < a.G; ++j) {
+        const bool e = (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * a.G + j]);
+        on += e ? 1 : 0;
+      }
+      s += on;
+    }
+    n_on_sum = s;
+    best_k = -1;
+  }
+  __syncthreads();
+  int k;
+  uint32_t flags = 0;
+  const int kc = a.keep_count ? a.keep_count[b] : -1;
+  if (kc >= 0) {
+    k = min(kc, n);
+  } else {
+    const long long D = a.D, Dkv = a.Dkv, Di = a.Di, V = a.V, G = a.G, L = a.L;
+    const long long lin = 4 * D * D + 4 * D * Dkv + 6 * D * Di;
+    const long long S_full = n + s_text;
+    const long long c_full = G * L * (lin * S_full + 4 * D * S_full * S_full) + G * 2 * D * V * S_full;
+    const double limit = static_cast<double>(a.budget[b]) * static_cast<double>(c_full);
+    long long mine = -1;
+    for (int kk = tid; kk <= n; kk += blockDim.x) {
+      const long long S = s_text + kk;
+      const long long cost = n_on_sum * (lin * S + 4 * D * S * S) + G * 2 * D * V * S;
+      if (static_cast<double>(cost) <= limit) mine = max(mine, static_cast<long long>(kk));
+    }
+    // cost grows with k, so the feasible set is a prefix: take the max
+    if (mine >= 0) atomicMax(&best_k, static_cast<int>(mine));
+    __syncthreads();
+    if (best_k < 0) {
+      k = 0;
+      flags |= SVL_FLAG_OVER_BUDGET;
+    } else {
+      k = best_k;
+    }
+  }
+  if (tid == 0) {
+    a.k_out[b] = k;
+    if (a.flags) a.flags[b] = flags;
+  }
+
+  const float* z = a.scores + v0;
+  int* out = a.kept_local + v0;
+  if (k == 0) return;
+  if (k >= n) {
+    for (int i = tid; i < n; i += blockDim.x) out[i] = i;
+    return;
+  }
+
+  // ---- radix select of the k-th largest key, 8 bits per pass, MSB first
+  uint32_t prefix = 0, mask = 0;
+  int remaining = k;  // keys still to take among those matching `prefix`
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int i = tid; i < n; i += blockDim.x) {
+      const uint32_t key = order_key(z[i]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 0xFF], 1);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int above = 0, d = 255;
+      for (; d > 0; --d) {
+        if (above + hist[d] >= remaining) break;
+        above += hist[d];
+      }
+      s_prefix_cnt[0] = d;
+      s_prefix_cnt[1] = remaining - above;
+    }
+    __syncthreads();
+    prefix |= static_cast<uint32_t>(s_prefix_cnt[0]) << shift;
+    mask |= 0xFFu << shift;
+    remaining = s_prefix_cnt[1];
+    __syncthreads();
+  }
+  const uint32_t tau = prefix;  // key of the k-th largest logit
+  // keys > tau are kept; of the keys == tau, the `remaining` lowest indices
+
+  // ---- ordered pass: ranks of equal keys and output positions by index
+  int eq_before = 0, kept_before = 0;
+  for (int base = 0; base < n; base += blockDim.x) {
+    const int i = base + tid;
+    uint32_t key = 0;
+    if (i < n) key = order_key(z[i]);
+    const int is_eq = (i < n && key == tau) ? 1 : 0;
+    int eq_total;
+    const int eq_rank = eq_before + block_exclusive_scan(is_eq, &eq_total, warp_sums);
+    const int keep = (i < n && (key > tau || (is_eq && eq_rank < remaining))) ? 1 : 0;
+    int keep_total;
+    const int pos = kept_before + block_exclusive_scan(keep, &keep_total, warp_sums);
+    if (keep) out[pos] = i;
+    eq_before += eq_total;
+    kept_before += keep_total;
+  }
+}
+
+// Compacts the per-sample kept lists: kept_off[b] = k_0 + ... + k_{b-1}.
+__global__ void compact_kernel(int B, const int* __restrict__ vis_off, const int* __restrict__ k,
+                               const int* __restrict__ kept_local, int* __restrict__ kept_idx,
+                               int* __restrict__ kept_off, int* __restrict__ kept_total) {
+  __shared__ int off;
+  const int b = blockIdx.x;
+  if (threadIdx.x == 0) {
+    int s = 0;
+    for (int i = 0; i < b; ++i) s += k[i];
+    off = s;
+    kept_off[b] = s;
+    if (b == B - 1) {
+      kept_off[B] = s + k[b];
+      if (kept_total) *kept_total = s + k[b];
+    }
+  }
+  __syncthreads();
+  const int kb = k[b];
+  const int* src = kept_local + vis_off[b];
+  for (int i = threadIdx.x; i < kb; i += blockDim.x) kept_idx[off + i] = src[i];
+}
+
+void launch_budget_embed(const float* budget, const __nv_bfloat16* w1, const __nv_bfloat16* w2, int H, int B,
+                         float* e_b, cudaStream_t s) {
+  budget_embed_kernel<<<B, 256, 0, s>>>(budget, w1, w2, H, e_b);
+}
+
+void launch_select(const SelectArgs& a, int B, cudaStream_t s) {
+  select_kernel<<<B, kSelectThreads, 0, s>>>(a);
+}
+
+void launch_compact(int B, const int* vis_off, const int* k, const int* kept_local, int* kept_idx, int* kept_off,
+                    int* kept_total, cudaStream_t s) {
+  compact_kernel<<<B, 256, 0, s>>>(B, vis_off, k, kept_local, kept_idx, kept_off, kept_total);
+}
+
+}  // namespace svl

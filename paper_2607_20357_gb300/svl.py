@@ -1,0 +1,255 @@
+"""Python binding of libsvl.so (ctypes): the C ABI of ``include/svl.h``.
+
+Every function here only marshals arguments -- torch tensors become device
+pointers, the stream is torch's current CUDA stream -- and calls the C entry
+point of the same name. All computation runs in the library's CUDA kernels.
+There is no fallback: if the library is missing or fails to load, the call
+raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libsvl.so")
+_lib = None
+
+SVL_LOGITS_LAST = 0
+SVL_LOGITS_ALL = 1
+SVL_FLAG_OVER_BUDGET = 1
+SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
+
+SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
+           "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count"]
+
+
+class ModelDesc(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("n_layers", "d_model", "n_heads", "n_kv_heads", "d_ffn", "vocab",
+                                              "n_groups", "n_prefix", "c_vis", "h_ctrl", "proj_hidden")] + \
+               [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float), ("max_seq", ctypes.c_int32)]
+
+
+class LayerWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd", "attn_norm", "ffn_norm")]
+
+
+class Weights(ctypes.Structure):
+    _fields_ = [("ctrl_w1", ctypes.c_void_p), ("ctrl_w2", ctypes.c_void_p), ("ctrl_c2", ctypes.c_float),
+                ("bud_w1", ctypes.c_void_p), ("bud_w2", ctypes.c_void_p), ("proj_w1", ctypes.c_void_p),
+                ("proj_w2", ctypes.c_void_p), ("embed", ctypes.c_void_p), ("final_norm", ctypes.c_void_p),
+                ("lm_head", ctypes.c_void_p), ("layers", ctypes.POINTER(LayerWeights))]
+
+
+def lib():
+    """Loads libsvl.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libsvl.so not built ({LIB_PATH}); run __graft_entry__.build()")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+        L.svl_model_create.argtypes = [ctypes.POINTER(ModelDesc), ctypes.POINTER(Weights), ctypes.POINTER(vp)]
+        L.svl_model_create.restype = ctypes.c_int
+        L.svl_model_destroy.argtypes = [vp]
+        L.svl_model_destroy.restype = None
+        L.svl_workspace_size.argtypes = [vp, i32, i64, i64]
+        L.svl_workspace_size.restype = sz
+        L.svl_score_select.argtypes = [vp, i32, i32] + [vp] * 13 + [sz, vp]
+        L.svl_score_select.restype = ctypes.c_int
+        L.svl_pack.argtypes = [vp, i32, i32, i32] + [vp] * 10 + [sz, vp]
+        L.svl_pack.restype = ctypes.c_int
+        L.svl_gated_prefill.argtypes = [vp, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, sz, vp]
+        L.svl_gated_prefill.restype = ctypes.c_int
+        L.svl_flops.argtypes = [ctypes.POINTER(ModelDesc), i32, i32, i32, vp, vp,
+                                ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
+        L.svl_flops.restype = ctypes.c_int
+        L.svl_get_device_status.argtypes = [vp, vp, ctypes.POINTER(ctypes.c_uint32)]
+        L.svl_get_device_status.restype = ctypes.c_int
+        L.svl_status_string.argtypes = [ctypes.c_int]
+        L.svl_status_string.restype = ctypes.c_char_p
+        L.svl_launch_count.argtypes = []
+        L.svl_launch_count.restype = ctypes.c_uint64
+        _lib = L
+    return _lib
+
+
+class SvlError(RuntimeError):
+    def __init__(self, fn, code):
+        super().__init__(f"{fn}: {lib().svl_status_string(code).decode()} (status {code})")
+        self.code = code
+
+
+def _check(fn, code):
+    if code != 0:
+        raise SvlError(fn, code)
+
+
+def _p(x):
+    """Device (or host) pointer of a tensor / int / None."""
+    if x is None:
+        return None
+    if isinstance(x, torch.Tensor):
+        return ctypes.c_void_p(x.data_ptr())
+    return ctypes.c_void_p(int(x))
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def svl_model_create(desc: ModelDesc, weights: Weights):
+    h = ctypes.c_void_p()
+    _check("svl_model_create", lib().svl_model_create(ctypes.byref(desc), ctypes.byref(weights), ctypes.byref(h)))
+    return h
+
+
+def svl_model_destroy(model):
+    lib().svl_model_destroy(model)
+
+
+def svl_workspace_size(model, max_batch, max_vis_total, max_text_total) -> int:
+    return int(lib().svl_workspace_size(model, int(max_batch), int(max_vis_total), int(max_text_total)))
+
+
+def svl_score_select(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
+                     group_gate, scores, k, kept_idx, kept_off, sample_flags, workspace, workspace_bytes,
+                     stream=None):
+    _check("svl_score_select", lib().svl_score_select(
+        model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
+        _p(layer_gate), _p(group_gate), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags),
+        _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_pack(model, B, n_vis_total, n_text_total, vis_feats, vis_off, kept_idx, kept_off, text_ids, text_off,
+             X, cu_seqlens, pos, workspace, workspace_bytes, stream=None):
+    _check("svl_pack", lib().svl_pack(
+        model, int(B), int(n_vis_total), int(n_text_total), _p(vis_feats), _p(vis_off), _p(kept_idx),
+        _p(kept_off), _p(text_ids), _p(text_off), _p(X), _p(cu_seqlens), _p(pos), _p(workspace),
+        int(workspace_bytes), _stream(stream)))
+
+
+def svl_gated_prefill(model, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, logits_mode, logits,
+                      workspace, workspace_bytes, stream=None):
+    _check("svl_gated_prefill", lib().svl_gated_prefill(
+        model, int(B), int(t_cap), _p(X), _p(cu_seqlens), _p(pos), _p(layer_gate), _p(group_gate),
+        int(logits_mode), _p(logits), _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_flops(desc: ModelDesc, s_text, s_vis, n_vis, layer_gate=None, group_gate=None):
+    """Host-side Eq. 8 (eq8) and executed FLOPs for one sample; gates are
+    CPU uint8 tensors [L] and [L, G] or None (all on)."""
+    eq8, ex = ctypes.c_double(), ctypes.c_double()
+    lg = None if layer_gate is None else ctypes.c_void_p(layer_gate.contiguous().data_ptr())
+    gg = None if group_gate is None else ctypes.c_void_p(group_gate.contiguous().data_ptr())
+    _check("svl_flops", lib().svl_flops(ctypes.byref(desc), int(s_text), int(s_vis), int(n_vis), lg, gg,
+                                        ctypes.byref(eq8), ctypes.byref(ex)))
+    return eq8.value, ex.value
+
+
+def svl_get_device_status(model, stream=None) -> int:
+    code = ctypes.c_uint32()
+    _check("svl_get_device_status", lib().svl_get_device_status(model, _stream(stream), ctypes.byref(code)))
+    return int(code.value)
+
+
+def svl_launch_count() -> int:
+    return int(lib().svl_launch_count())
+
+
+# --------------------------------------------------------------------------- plumbing
+def model_desc(dims, max_seq: int) -> ModelDesc:
+    return ModelDesc(n_layers=dims.n_layers, d_model=dims.d_model, n_heads=dims.n_heads,
+                     n_kv_heads=dims.n_kv_heads, d_ffn=dims.d_ffn, vocab=dims.vocab, n_groups=dims.n_groups,
+                     n_prefix=dims.n_prefix, c_vis=dims.c_vis, h_ctrl=dims.h_ctrl, proj_hidden=dims.proj_hidden,
+                     rms_eps=dims.rms_eps, rope_theta=dims.rope_theta, max_seq=int(max_seq))
+
+
+class GatedPrefill:
+    """Owns a model handle and the device weight tensors it points to.
+
+    ``weights`` is a dict as produced by the input generator, tensors on the
+    CUDA device (bf16, nn.Linear layout). ``run`` allocates the outputs and
+    the workspace with torch and calls the three C entry points in order.
+    """
+
+    def __init__(self, dims, weights: dict, max_seq: int = 8192):
+        self.dims = dims
+        self.w = weights
+        self.desc = model_desc(dims, max_seq)
+        lw = (LayerWeights * dims.n_layers)()
+        for i, l in enumerate(weights["layers"]):
+            lw[i] = LayerWeights(*[l[n].data_ptr() for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd",
+                                                             "attn_norm", "ffn_norm")])
+        self._lw = lw
+        opt = lambda n: weights[n].data_ptr() if n in weights else None
+        self._wts = Weights(weights["ctrl_w1"].data_ptr(), weights["ctrl_w2"].data_ptr(), float(weights["ctrl_c2"]),
+                            weights["bud_w1"].data_ptr(), weights["bud_w2"].data_ptr(), opt("proj_w1"),
+                            opt("proj_w2"), weights["embed"].data_ptr(), weights["final_norm"].data_ptr(),
+                            weights["lm_head"].data_ptr(), lw)
+        self.handle = svl_model_create(self.desc, self._wts)
+        self._ws = None
+        self._ws_key = None
+
+    def close(self):
+        if self.handle:
+            svl_model_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def workspace(self, B, n_vis, n_text, device="cuda"):
+        need = svl_workspace_size(self.handle, B, n_vis, n_text)
+        if self._ws is None or self._ws.numel() < need:
+            self._ws = torch.empty(need, dtype=torch.uint8, device=device)
+        return self._ws, self._ws.numel()
+
+    def alloc_outputs(self, batch: dict, logits_mode: int = SVL_LOGITS_LAST):
+        d = self.dims
+        B = batch["B"]
+        nv = batch["vis"].shape[0]
+        nt = int(batch["text_ids"].shape[0])
+        dev = batch["vis"].device
+        t_cap = nv + nt
+        i32 = dict(dtype=torch.int32, device=dev)
+        return {
+            "scores": torch.empty(max(nv, 1), dtype=torch.float32, device=dev),
+            "k": torch.empty(B, **i32),
+            "kept_idx": torch.empty(max(nv, 1), **i32),
+            "kept_off": torch.empty(B + 1, **i32),
+            "flags": torch.empty(B, dtype=torch.int32, device=dev),
+            "X": torch.empty(max(t_cap, 1), d.d_model, dtype=torch.bfloat16, device=dev),
+            "cu_seqlens": torch.empty(B + 1, **i32),
+            "pos": torch.empty(max(t_cap, 1), **i32),
+            "logits": torch.empty((B if logits_mode == SVL_LOGITS_LAST else max(t_cap, 1)), d.vocab,
+                                  dtype=torch.float32, device=dev),
+            "text_len": (batch["text_off"][1:] - batch["text_off"][:-1]).to(torch.int32).contiguous(),
+        }
+
+    def run(self, batch: dict, out: Optional[dict] = None, logits_mode: int = SVL_LOGITS_LAST, stream=None,
+            stages=("select", "pack", "prefill")):
+        B = batch["B"]
+        nv = batch["vis"].shape[0]
+        nt = int(batch["text_ids"].shape[0])
+        out = out or self.alloc_outputs(batch, logits_mode)
+        ws, wsb = self.workspace(B, nv, nt, batch["vis"].device)
+        if "select" in stages:
+            svl_score_select(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"], batch["budget"],
+                             batch["keep_count"], batch["layer_gate"], batch["group_gate"], out["scores"], out["k"],
+                             out["kept_idx"], out["kept_off"], out["flags"], ws, wsb, stream)
+        if "pack" in stages:
+            svl_pack(self.handle, B, nv, nt, batch["vis"], batch["vis_off"], out["kept_idx"], out["kept_off"],
+                     batch["text_ids"], batch["text_off"], out["X"], out["cu_seqlens"], out["pos"], ws, wsb, stream)
+        if "prefill" in stages:
+            svl_gated_prefill(self.handle, B, max(nv + nt, 1), out["X"], out["cu_seqlens"], out["pos"],
+                              batch["layer_gate"], batch["group_gate"], logits_mode, out["logits"], ws, wsb, stream)
+        return out

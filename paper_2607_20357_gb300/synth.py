@@ -201,19 +201,27 @@ def _features(kind: str, n: int, c: int, g, device):
 
 
 def make_batch(wl: Workload, seed: int, budget: Optional[float] = None, batch: Optional[int] = None,
-               device="cpu", dims: Optional[ModelDims] = None) -> dict:
+               device="cpu", dims: Optional[ModelDims] = None, n_vis_list=None, s_text_list=None,
+               keep_list=None, budget_list=None) -> dict:
     """One seeded batch: features, offsets, text ids, budgets, gates.
 
     ``budget`` overrides the workload's budget spec with one value for the
-    whole batch. Returned tensors live on ``device``; offsets and gates are
+    whole batch; ``n_vis_list`` / ``s_text_list`` / ``keep_list`` /
+    ``budget_list`` fix those per sample (edge cases). Returned tensors live on ``device``; offsets and gates are
     int32/uint8, features bf16, budgets float32.
     """
     dims = dims or wl.dims
-    B = batch or wl.batch
+    B = batch or (len(n_vis_list) if n_vis_list is not None else wl.batch)
     g = _gen(seed, "cpu")
     n_vis = torch.randint(wl.n_vis[0], wl.n_vis[1] + 1, (B,), generator=g)
     s_text = torch.randint(wl.s_text[0], wl.s_text[1] + 1, (B,), generator=g)
-    if budget is not None:
+    if n_vis_list is not None:
+        n_vis = torch.tensor(n_vis_list, dtype=torch.int64)
+    if s_text_list is not None:
+        s_text = torch.tensor(s_text_list, dtype=torch.int64)
+    if budget_list is not None:
+        budgets = torch.tensor(budget_list, dtype=torch.float32)
+    elif budget is not None:
         budgets = torch.full((B,), float(budget))
     elif wl.budgets[0] == "uniform":
         lo, hi = wl.budgets[1], wl.budgets[2]
@@ -241,13 +249,15 @@ def make_batch(wl: Workload, seed: int, budget: Optional[float] = None, batch: O
     fg = _gen(seed * 7919 + 1, device)
     for b in range(B):
         feats.append(_features(wl.features, int(n_vis[b]), dims.c_vis, fg, device).to(torch.bfloat16))
-    vis = torch.cat(feats, 0)
+    vis = torch.cat(feats, 0) if feats else torch.zeros(0, dims.c_vis, dtype=torch.bfloat16, device=device)
     vis_off = torch.zeros(B + 1, dtype=torch.int32)
     vis_off[1:] = torch.cumsum(n_vis, 0).to(torch.int32)
     text_off = torch.zeros(B + 1, dtype=torch.int32)
     text_off[1:] = torch.cumsum(s_text, 0).to(torch.int32)
     text_ids = torch.randint(0, dims.vocab, (int(text_off[-1]),), generator=g, dtype=torch.int64).to(torch.int32)
     keep = torch.full((B,), -1 if wl.keep_count is None else wl.keep_count, dtype=torch.int32)
+    if keep_list is not None:
+        keep = torch.tensor(keep_list, dtype=torch.int32)
     return {
         "B": B,
         "vis": vis,

@@ -1,0 +1,76 @@
+"""Helpers shared by the GPU parity tests: device copies of generated
+inputs, oracle runs on the same inputs, and error measures."""
+import numpy as np
+import torch
+
+from oracle import smartvl_oracle as O
+from paper_2607_20357_gb300 import svl, synth
+
+TIE_BAND = 1e-4
+
+
+def to_device(obj, device="cuda"):
+    if isinstance(obj, torch.Tensor):
+        return obj.to(device)
+    if isinstance(obj, dict):
+        return {k: to_device(v, device) for k, v in obj.items()}
+    if isinstance(obj, list):
+        return [to_device(v, device) for v in obj]
+    return obj
+
+
+def rel_err(got, ref) -> float:
+    """max |got - ref| / max |ref| (norm-wise relative error of a tensor)."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return float(np.abs(got - ref).max() / max(np.abs(ref).max(), 1e-30))
+
+
+def check_selection(gpu_scores, gpu_kept, ref, z_tol=1e-4):
+    """Kept sets agree except for tokens whose oracle logits lie within the
+    tie band of the k-th largest logit. Returns True when identical."""
+    k = ref["k"]
+    ours, theirs = set(gpu_kept.tolist()), set(ref["kept"].tolist())
+    assert len(ours) == k == len(gpu_kept)
+    assert np.all(np.diff(gpu_kept) > 0), "kept indices not strictly ascending"
+    if ours == theirs:
+        return True
+    z = ref["z"]
+    kth = np.sort(z)[::-1][k - 1]
+    for i in ours ^ theirs:
+        assert abs(z[i] - kth) < TIE_BAND, f"token {i}: logit {z[i]} vs k-th {kth}"
+    return False
+
+
+def gpu_topk_valid(scores, kept, k):
+    """The kept set is the k largest of the GPU's own logits, ties to lower index."""
+    n = len(scores)
+    order = sorted(range(n), key=lambda i: (-float(scores[i]), i))
+    assert sorted(order[:k]) == sorted(kept.tolist())
+
+
+class Case:
+    """Seeded model + batch on the GPU and the oracle's view of both."""
+
+    def __init__(self, dims, wl, seed, batch=None, budget=None, max_seq=8192, std=0.02):
+        self.dims = dims
+        w = synth.make_weights(dims, seed, std=std)
+        b = synth.make_batch(wl, seed, budget=budget, batch=batch, dims=dims)
+        self.w_np = O.to_numpy_weights(w)
+        self.b_np = O.to_numpy_batch(b)
+        self.w = to_device(w)
+        self.b = to_device(b)
+        self.model = svl.GatedPrefill(dims, self.w, max_seq=max_seq)
+
+    def run(self, logits_mode=svl.SVL_LOGITS_LAST):
+        out = self.model.run(self.b, logits_mode=logits_mode)
+        torch.cuda.synchronize()
+        status = svl.svl_get_device_status(self.model.handle)
+        assert status == 0, f"device status {status:#x}"
+        return {k: v.cpu() for k, v in out.items()}
+
+    def oracle(self, mode="fp32", samples=None, n_layers=None):
+        return O.forward_batch(self.dims, self.w_np, self.b_np, mode=mode, samples=samples, n_layers=n_layers)
+
+    def close(self):
+        self.model.close()

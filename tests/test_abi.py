@@ -1,0 +1,61 @@
+"""The C-ABI library loads and exports every entry point include/svl.h
+declares; host-only entry points behave (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import smartvl_oracle as O
+from paper_2607_20357_gb300 import svl, synth
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "svl.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?[\w\s\*]+?\b(svl_\w+)\s*\(", text, re.M)))
+
+
+def test_header_declares_the_entry_points():
+    syms = declared_symbols()
+    for name in ("svl_score_select", "svl_pack", "svl_gated_prefill", "svl_model_create", "svl_flops"):
+        assert name in syms
+    assert set(syms) == set(svl.SYMBOLS)
+
+
+def test_library_exports_every_declared_symbol(svl_lib):
+    for name in declared_symbols():
+        assert hasattr(svl_lib, name), name
+
+
+def test_status_strings(svl_lib):
+    for code in range(8):
+        assert svl_lib.svl_status_string(code)
+    assert svl_lib.svl_status_string(0) == b"ok"
+
+
+def test_model_create_rejects_bad_args_without_gpu(svl_lib):
+    h = ctypes.c_void_p()
+    assert svl_lib.svl_model_create(None, None, ctypes.byref(h)) == 1
+    d = svl.model_desc(synth.WORKLOADS["tiny"].dims, 256)
+    d.n_groups = 3  # 4 heads are not divisible into 3 groups
+    w = svl.Weights()
+    assert svl_lib.svl_model_create(ctypes.byref(d), ctypes.byref(w), ctypes.byref(h)) in (1, 3)
+
+
+@pytest.mark.parametrize("name", ["tiny", "llava", "qwen", "mixed"])
+def test_host_flops_match_oracle(svl_lib, name):
+    dims = synth.WORKLOADS[name].dims
+    desc = svl.model_desc(dims, 8192)
+    rng = np.random.default_rng(0)
+    for _ in range(10):
+        s_text, k, n_vis = int(rng.integers(1, 300)), int(rng.integers(0, 600)), 700
+        lg = torch.tensor(rng.random(dims.n_layers) < 0.8, dtype=torch.uint8)
+        gg = torch.tensor(rng.random((dims.n_layers, dims.n_groups)) < 0.7, dtype=torch.uint8)
+        eq8, ex = svl.svl_flops(desc, s_text, k, n_vis, lg, gg)
+        n_on = O.effective_groups(lg.numpy(), gg.numpy(), dims.n_prefix).sum(1)
+        assert eq8 == pytest.approx(O.prefill_cost_xG(dims, s_text + k, n_on) / dims.n_groups, rel=1e-15)
+        assert ex == pytest.approx(O.executed_flops(dims, n_vis, k, s_text, n_on), rel=1e-12)
