@@ -130,6 +130,7 @@ def prefill_cost_xG(dims, S: int, groups_on) -> int:
     8 D^2 is written 4 D^2 + 4 D D_kv (Q, O plus K, V projections).
     """
     D, Dkv, Di, V, G = dims.d_model, dims.d_kv, dims.d_ffn, dims.vocab, dims.n_groups
+    S = int(S)  # Python integers: exact, no fixed-width overflow
     per_layer = (4 * D * D + 4 * D * Dkv + 6 * D * Di) * S + 4 * D * S * S
     total = 0
     for n_on in groups_on:
@@ -145,6 +146,7 @@ def budget_keep_count(dims, budget: float, n_vis: int, s_text: int, groups_on, k
     Eq. 8 at S = N + S_text with every group on. The comparison is done in
     float64 on the exact integers G*C; the budget is the float32 value given.
     """
+    n_vis, s_text = int(n_vis), int(s_text)
     if keep_count >= 0:
         return min(int(keep_count), n_vis), 0
     L, G = dims.n_layers, dims.n_groups
@@ -302,6 +304,7 @@ def executed_flops(dims, n_vis, k, s_text, groups_on, all_logits=False) -> int:
     scorer, projector on kept tokens, active projections and FFN, causal
     attention (2 D S (S+1) alpha) and the LM head."""
     D, Dkv, Di, V, G = dims.d_model, dims.d_kv, dims.d_ffn, dims.vocab, dims.n_groups
+    n_vis, k, s_text = int(n_vis), int(k), int(s_text)
     S = k + s_text
     f = 2 * n_vis * dims.c_vis * dims.h_ctrl
     if dims.proj_hidden:

@@ -385,3 +385,12 @@ def test_batch_equals_independent_samples():
         one = O.forward_sample(dims, w, batch["vis"][v0:v1], batch["text_ids"][t0:t1], batch["budget"][b],
                                batch["layer_gate"][b], batch["group_gate"][b], mode="fp64")
         np.testing.assert_array_equal(one["hidden"], outs[b]["hidden"])
+
+
+def test_eq8_accepts_fixed_width_integers():
+    """Lengths arriving as numpy int32 must not overflow Eq. 8's products."""
+    dims = synth.WORKLOADS["video"].dims
+    a = O.prefill_cost_xG(dims, np.int32(4672), np.full(32, 4, np.int64))
+    assert a == O.prefill_cost_xG(dims, 4672, [4] * 32)
+    assert O.budget_keep_count(dims, 0.25, np.int32(4608), np.int32(64), [4] * 32) == \
+        O.budget_keep_count(dims, 0.25, 4608, 64, [4] * 32)
