@@ -1,0 +1,441 @@
+#!/usr/bin/env python
+"""Benchmark of the budget-conditioned gated prefill on one GB300 per rank.
+
+Workload: LLaVA-1.5-7B-shaped batch -- 16 samples of 576 CLIP ViT-L/14-336
+visual tokens (dim 1024, low-rank + salient clusters) and 64 text tokens,
+MLP projector 1024->4096->4096, 32-layer decoder (d 4096, 32 heads, SwiGLU
+11008, vocab 32000), budgets 25/50/75/100% of full-prefill FLOPs. Weights
+and inputs are synthetic (seeded), the paper's datasets and checkpoints are
+not used.
+
+A step is one pass of the whole path -- svl_score_select, svl_pack,
+svl_gated_prefill -- over one batch; step i uses budget budgets[i % 4].
+Reported value: input tokens per second (sum over samples of visual + text
+tokens before selection) over the K timed steps, summed over ranks.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (test infrastructure, float64
+arithmetic) on a bounded sample of the same workload; it never touches the
+GPU.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2607_20357_gb300 import synth  # noqa: E402
+
+METRIC = "gated-prefill input tokens/sec and executed TFLOP/s (% of bf16 peak) vs budget"
+WORKLOAD = "llava"
+SEED = 1000
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=8)
+    ap.add_argument("--warmup", type=int, default=4)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            p = json.load(fh)
+        return {"hbm_gbs": p["hbm_gbs"], "bf16_tflops": p["bf16_tflops"],
+                "bf16_tflops_sustained": p.get("bf16_tflops_sustained", p["bf16_tflops"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def workload_config(wl, batch):
+    d = wl.dims
+    return {
+        "workload": "LLaVA-1.5-7B-shaped gated prefill: B=16, 576 visual (C_v 1024, MLP projector) + 64 text "
+                    "tokens, 32 layers d4096 h32 ffn11008 V32000, G=4 head groups, budgets 0.25/0.5/0.75/1.0",
+        "batch": batch, "n_vis": wl.n_vis[0], "s_text": wl.s_text[0], "budgets": list(wl.budgets),
+        "layers": d.n_layers, "d_model": d.d_model, "heads": d.n_heads, "d_ffn": d.d_ffn, "vocab": d.vocab,
+        "groups": d.n_groups, "gates": wl.gates,
+        "l2": "not flushed: each step streams 13 GB of weights through the 129 MB L2",
+        "parallelism": "replicas (independent batches per GPU, no collective)",
+    }
+
+
+# --------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "out", "").strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- flops
+def per_kind_flops(dims, k, s_text, lg, gg):
+    """Algorithmic FLOPs per GEMM kind for one batch (executed work only)."""
+    D, Di, G = dims.d_model, dims.d_ffn, dims.n_groups
+    hq, dkv = dims.n_heads * dims.d_head, dims.d_kv
+    f = {"qkv_gemm": 0.0, "o_gemm": 0.0, "gateup_gemm": 0.0, "down_gemm": 0.0, "attention": 0.0}
+    for b in range(len(k)):
+        S = int(k[b]) + int(s_text[b])
+        for l in range(dims.n_layers):
+            on = G if l < dims.n_prefix else int(lg[b, l] != 0) * int((gg[b, l] != 0).sum())
+            a = on / G
+            f["qkv_gemm"] += a * 2 * S * D * (hq + 2 * dkv)
+            f["o_gemm"] += a * 2 * S * hq * D
+            f["gateup_gemm"] += a * 2 * S * D * 2 * Di
+            f["down_gemm"] += a * 2 * S * Di * D
+            f["attention"] += a * 2 * D * S * (S + 1)
+    return f
+
+
+def executed_flops(svl, desc, k, s_text, n_vis, lg, gg):
+    tot = 0.0
+    for b in range(len(k)):
+        _, ex = svl.svl_flops(desc, int(s_text[b]), int(k[b]), int(n_vis[b]), lg[b].contiguous(), gg[b].contiguous())
+        tot += ex
+    return tot
+
+
+def gemm_traffic_record():
+    """Per-launch DRAM bytes of the dominant GEMM from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "gemm_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as fh:
+        rec = json.load(fh)
+    src = os.path.join(ROOT, "paper_2607_20357_gb300", "csrc", "gemm.cu")
+    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    return rec if rec.get("gemm_cu_sha256_16") == h else None
+
+
+# --------------------------------------------------------------------------- CPU oracle sample
+def oracle_sample_seconds(dims, w_np, x, ids, budget, lg, gg, n_layers):
+    """Seconds of the oracle on one sample: front (score/select/pack + final
+    norm + LM head) and n_layers decoder layers."""
+    from oracle import smartvl_oracle as O
+    t0 = time.perf_counter()
+    O.forward_sample(dims, w_np, x, ids, budget, lg, gg, mode="fp32", n_layers=0)
+    t1 = time.perf_counter()
+    O.forward_sample(dims, w_np, x, ids, budget, lg, gg, mode="fp32", n_layers=n_layers)
+    t2 = time.perf_counter()
+    front = t1 - t0
+    return front, max(t2 - t1 - front, 0.0) / max(n_layers, 1), (t2 - t1)
+
+
+def cpu_oracle_baseline(dims, weights_cpu_layers, weights_rest, batch_cpu, budget, n_layers):
+    from oracle import smartvl_oracle as O
+    w = O.to_numpy_weights(dict(weights_rest, layers=weights_cpu_layers))
+    b = 0
+    v0, v1 = int(batch_cpu["vis_off"][b]), int(batch_cpu["vis_off"][b + 1])
+    t0, t1 = int(batch_cpu["text_off"][b]), int(batch_cpu["text_off"][b + 1])
+    x = batch_cpu["vis"][v0:v1].double().numpy()
+    ids = batch_cpu["text_ids"][t0:t1].numpy()
+    lg, gg = batch_cpu["layer_gate"][b].numpy(), batch_cpu["group_gate"][b].numpy()
+    front, per_layer, wall = oracle_sample_seconds(dims, w, x, ids, budget, lg, gg, n_layers)
+    t_full = front + per_layer * dims.n_layers
+    tokens = (v1 - v0) + (t1 - t0)
+    return tokens / t_full, wall + front
+
+
+# --------------------------------------------------------------------------- reference arm
+def run_reference(args, rank, world):
+    """The CPU oracle as the reference arm: one sample per step, layers
+    0-1 of 32 timed and scaled to the full depth."""
+    if rank != 0:
+        return
+    wl = synth.WORKLOADS[WORKLOAD]
+    dims = wl.dims
+    nl = 2
+    w = synth.make_weights(dims, SEED, device="cpu", layers=range(nl))
+    from oracle import smartvl_oracle as O
+    w_np = O.to_numpy_weights(w)
+    batches = [synth.make_batch(wl, SEED, budget=b, batch=1) for b in wl.budgets]
+    times, tokens = [], []
+    for i in range(args.warmup + args.steps):
+        bt = batches[i % len(batches)]
+        x = bt["vis"].double().numpy()
+        ids = bt["text_ids"].numpy()
+        t0 = time.perf_counter()
+        front, per_layer, _ = oracle_sample_seconds(dims, w_np, x, ids, float(bt["budget"][0]),
+                                                    bt["layer_gate"][0].numpy(), bt["group_gate"][0].numpy(), nl)
+        t_full = front + per_layer * dims.n_layers
+        if i >= args.warmup:
+            times.append(t_full)
+            tokens.append(x.shape[0] + ids.shape[0])
+    value = sum(tokens) / sum(times)
+    cores = os.cpu_count()
+    sample = (f"1 sample per step (budget cycling {list(wl.budgets)}); token controller, pack, final norm and "
+              f"LM head timed whole; decoder layers 0-{nl - 1} timed and scaled x{dims.n_layers // nl} to 32 layers")
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(wl, 1), "impl": "reference",
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- our arm
+def run_ours(args, rank, world, local_rank):
+    from paper_2607_20357_gb300 import svl
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    wl = synth.WORKLOADS[WORKLOAD]
+    dims = wl.dims
+    B = wl.batch
+    pk = peaks()
+
+    weights = synth.make_weights(dims, SEED, device=dev)
+    max_seq = wl.n_vis[1] + wl.s_text[1] + 64
+    model = svl.GatedPrefill(dims, weights, max_seq=max_seq)
+    seed = SEED + 17 * rank
+    batches = [synth.make_batch(wl, seed, budget=b, device=dev) for b in wl.budgets]
+    outs = [model.alloc_outputs(bt) for bt in batches]
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        model.run(batches[i % len(batches)], out=outs[i % len(batches)])
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    status = svl.svl_get_device_status(model.handle)
+    if status:
+        raise RuntimeError(f"device status {status:#x} after warm-up")
+
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    launches0 = svl.svl_launch_count()
+    svl.svl_profile_start(model.handle)
+    with ClockSampler(local_rank) as clk:
+        t_wall0 = time.perf_counter()
+        for i in range(args.steps):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter() - t_wall0
+    kern = svl.svl_profile_stop(model.handle)
+    launches = svl.svl_launch_count() - launches0
+    if world > 1:
+        torch.distributed.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = sum(step_ms)
+
+    # per-budget accounting (k read back after the timed region)
+    desc = model.desc
+    per_budget, tokens_total, fexec_total = [], 0, 0.0
+    kind_flops = {}
+    for j, bt in enumerate(batches):
+        nsteps = len(range(j, args.steps, len(batches)))
+        if nsteps == 0:
+            continue
+        k = outs[j]["k"].cpu().numpy()
+        nv = (bt["vis_off"][1:] - bt["vis_off"][:-1]).cpu().numpy()
+        st = (bt["text_off"][1:] - bt["text_off"][:-1]).cpu().numpy()
+        lg, gg = bt["layer_gate"].cpu(), bt["group_gate"].cpu()
+        toks = int(nv.sum() + st.sum())
+        fex = executed_flops(svl, desc, k, st, nv, lg, gg)
+        ms = statistics.mean(step_ms[i] for i in range(j, args.steps, len(batches)))
+        per_budget.append({"budget": float(bt["budget"][0]), "k_mean": float(k.mean()), "ms_per_step": ms,
+                           "tokens_per_s": toks / (ms / 1000.0), "exec_tflops": fex / (ms / 1000.0) / 1e12,
+                           "exec_tflop_per_step": fex / 1e12})
+        tokens_total += toks * nsteps
+        fexec_total += fex * nsteps
+        for kk, v in per_kind_flops(dims, k, st, lg.numpy(), gg.numpy()).items():
+            kind_flops[kk] = kind_flops.get(kk, 0.0) + v * nsteps
+
+    # linear-in-FLOPs check: t(b)/t(1) / (F(b)/F(1)) - 1
+    full = [p for p in per_budget if abs(p["budget"] - 1.0) < 1e-6]
+    if full:
+        for p in per_budget:
+            p["time_vs_flops_ratio_minus_1"] = (p["ms_per_step"] / full[0]["ms_per_step"]) / \
+                (p["exec_tflop_per_step"] / full[0]["exec_tflop_per_step"]) - 1.0
+
+    # dominant kernel roofline (tensor-bound GEMM)
+    gemm_tags = ["qkv_gemm", "o_gemm", "gateup_gemm", "down_gemm"]
+    dom = max(gemm_tags, key=lambda t: kern.get(t, (0, 0.0))[1])
+    n_l, t_l = kern[dom]
+    achieved = kind_flops[dom] / (t_l / 1000.0) / 1e12
+    peak = pk["bf16_tflops_sustained"]
+    traffic_rec = gemm_traffic_record()
+    roofline = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "peak_source": pk["source"] + " bf16 sustained",
+                "launches": n_l, "avg_launch_ms": t_l / n_l,
+                "flops_per_launch": kind_flops[dom] / n_l,
+                "traffic": (traffic_rec or {}).get("dram_bytes_per_launch") if traffic_rec else None}
+    kernels = {t: {"launches": n, "total_ms": ms, "share": ms / max(sum(v[1] for v in kern.values()), 1e-9)}
+               for t, (n, ms) in sorted(kern.items(), key=lambda kv: -kv[1][1])}
+    for t in list(kind_flops):
+        if t in kernels:
+            kernels[t]["tflops"] = kind_flops[t] / (kernels[t]["total_ms"] / 1000.0) / 1e12
+
+    # whole-job aggregate over ranks: max time, summed tokens
+    if world > 1:
+        tt = torch.tensor([total_ms, float(tokens_total), fexec_total], dtype=torch.float64, device=dev)
+        mx = tt.clone()
+        torch.distributed.all_reduce(mx[:1], op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.all_reduce(tt[1:], op=torch.distributed.ReduceOp.SUM)
+        total_ms, tokens_total, fexec_total = float(mx[0]), float(tt[1]), float(tt[2])
+    value = tokens_total / (total_ms / 1000.0)
+
+    # e2e through the host-buffer entry point: H2D of inputs, D2H of logits
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, svl, model, batches, dims, world, dev)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        nl = 8
+        wl_cpu = [{k: v.cpu() for k, v in weights["layers"][l].items()} for l in range(nl)]
+        rest = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in weights.items() if k != "layers"}
+        b_cpu = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in batches[1].items()}
+        tps, secs = cpu_oracle_baseline(dims, wl_cpu, rest, b_cpu, float(b_cpu["budget"][0]), nl)
+        cpu = {"value": tps, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": f"sample 0 of the budget-{float(b_cpu['budget'][0])} batch: token controller, pack, "
+                         f"final norm, LM head whole; decoder layers 0-{nl - 1} timed and scaled x"
+                         f"{dims.n_layers // nl}; fp32 storage, float64 arithmetic; {secs:.1f} s of CPU time"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": workload_config(wl, B),
+            "exec_tflops": fexec_total / (total_ms / 1000.0) / 1e12,
+            "exec_tflops_frac_of_peak": fexec_total / (total_ms / 1000.0) / 1e12 / peak,
+            "per_budget": per_budget, "roofline": roofline, "kernels": kernels,
+            "gpu_launches": int(launches), "gpu_launches_per_step": launches / args.steps,
+            "wall_s_timed": t_wall, "clocks": clk.summary(), "e2e": e2e, "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    model.close()
+
+
+def run_e2e(args, svl, model, batches, dims, world, dev):
+    stream = torch.cuda.current_stream()
+    hosts = []
+    for bt in batches:
+        h = {k: (v.cpu().pin_memory() if isinstance(v, torch.Tensor) else v) for k, v in bt.items()}
+        h["logits"] = torch.empty(bt["B"], dims.vocab, dtype=torch.float32).pin_memory()
+        h["k"] = torch.empty(bt["B"], dtype=torch.int32).pin_memory()
+        hosts.append(h)
+    nv = batches[0]["vis"].shape[0]
+    nt = int(batches[0]["text_ids"].shape[0])
+    B = batches[0]["B"]
+    need = svl.svl_host_workspace_size(model.handle, B, nv, nt)
+    ws = torch.empty(need, dtype=torch.uint8, device=dev)
+
+    def step(i):
+        h = hosts[i % len(hosts)]
+        svl.svl_prefill_from_host(model.handle, B, nv, nt, h["vis"], h["vis_off"], h["text_ids"], h["text_off"],
+                                  h["budget"], h["keep_count"], h["layer_gate"], h["group_gate"], h["logits"],
+                                  h["k"], ws, need, stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for i in range(args.steps):
+        step(i)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b)
+    tokens = sum(int(hosts[i % len(hosts)]["vis"].shape[0] + hosts[i % len(hosts)]["text_ids"].shape[0])
+                 for i in range(args.steps))
+    h0 = hosts[0]
+    h2d = sum(int(h0[k].numel() * h0[k].element_size()) for k in
+              ("vis", "vis_off", "text_ids", "text_off", "budget", "keep_count", "layer_gate", "group_gate"))
+    d2h = int(h0["logits"].numel() * 4 + h0["k"].numel() * 4)
+    if world > 1:
+        t = torch.tensor([ms, float(tokens)], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t[:1], op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.all_reduce(t[1:], op=torch.distributed.ReduceOp.SUM)
+        ms, tokens = float(t[0]), float(t[1])
+    return {"value": tokens / (ms / 1000.0), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "entry_point": "svl_prefill_from_host (pinned host buffers)"}
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -13,8 +13,9 @@
  * Conventions shared by every call below.
  *  - All tensor arguments are DEVICE pointers owned by the caller, unless the
  *    name says host. bf16 tensors are IEEE bfloat16, row-major, contiguous.
- *  - Calls that take a stream are asynchronous on it; the library never
- *    synchronises the stream and never copies device data to the host.
+ *  - Calls that take a stream are asynchronous on it. Apart from
+ *    svl_get_device_status and svl_profile_stop, the library never
+ *    synchronises, and only svl_prefill_from_host copies results to the host.
  *    Counts that depend on data (k, sequence lengths, tile lists) stay on the
  *    device.
  *  - The returned status reports argument and shape errors found on the host;
@@ -189,6 +190,57 @@ svl_status svl_gated_prefill(svl_model* model, int32_t B, int32_t t_cap, void* X
 svl_status svl_flops(const svl_model_desc* desc, int32_t s_text, int32_t s_vis, int32_t n_vis,
                      const uint8_t* layer_gate, const uint8_t* group_gate,
                      double* eq8_flops, double* exec_flops);
+
+/* End to end from HOST buffers: copies the inputs of one batch to the device
+ *  (asynchronously on `stream`; pinned host memory makes the copies
+ *  overlap), runs svl_score_select, svl_pack and svl_gated_prefill (LAST
+ *  logits) and copies the logits [B, V] float32 and k [B] int32 back to the
+ *  host buffers. The caller synchronises `stream` before reading them.
+ *  Host inputs are laid out as the device arguments of (1) and (2):
+ *  h_vis [n_vis_total, C_v] bf16, h_vis_off [B+1], h_text_ids
+ *  [n_text_total], h_text_off [B+1], h_budget [B], h_keep_count [B] or NULL,
+ *  h_layer_gate [B, L], h_group_gate [B, L, G]. `workspace` must hold
+ *  svl_host_workspace_size() bytes for these sizes. */
+svl_status svl_prefill_from_host(svl_model* model, int32_t B, int32_t n_vis_total, int32_t n_text_total,
+                                 const void* h_vis, const int32_t* h_vis_off, const int32_t* h_text_ids,
+                                 const int32_t* h_text_off, const float* h_budget, const int32_t* h_keep_count,
+                                 const uint8_t* h_layer_gate, const uint8_t* h_group_gate,
+                                 float* h_logits, int32_t* h_k,
+                                 void* workspace, size_t workspace_bytes, void* stream);
+
+/* Workspace bytes of svl_prefill_from_host for these sizes. */
+size_t svl_host_workspace_size(const svl_model* model, int32_t B, int64_t n_vis_total, int64_t n_text_total);
+
+/* Kernel timing. While profiling is on, the library records a CUDA event
+ * pair on the launch stream around every kernel it launches, tagged by the
+ * step of the path. svl_profile_stop() waits for the last event, sums the
+ * elapsed times per tag into `out` (at most `cap` entries, *n_out set) and
+ * turns profiling off. */
+typedef struct svl_kernel_time {
+  int32_t tag;       /* SVL_TAG_* */
+  int32_t launches;
+  double total_ms;
+} svl_kernel_time;
+
+#define SVL_TAG_BUDGET_EMBED 0
+#define SVL_TAG_SCORE 1
+#define SVL_TAG_SELECT 2
+#define SVL_TAG_PACK 3
+#define SVL_TAG_PROJECTOR 4
+#define SVL_TAG_SCHEDULE 5
+#define SVL_TAG_RMSNORM 6
+#define SVL_TAG_QKV 7
+#define SVL_TAG_ATTENTION 8
+#define SVL_TAG_OPROJ 9
+#define SVL_TAG_GATEUP 10
+#define SVL_TAG_DOWN 11
+#define SVL_TAG_LMHEAD 12
+#define SVL_TAG_COPY 13
+#define SVL_TAG_COUNT 14
+
+svl_status svl_profile_start(svl_model* model);
+svl_status svl_profile_stop(svl_model* model, svl_kernel_time* out, int32_t cap, int32_t* n_out);
+const char* svl_tag_name(int32_t tag);
 
 /* Reads (and clears) the device status word; synchronises `stream`. */
 svl_status svl_get_device_status(svl_model* model, void* stream, uint32_t* code);

@@ -24,6 +24,11 @@ struct svl_model {
   // B-operand tensor maps of the weights: per layer q, k, v, o, g, u, d
   std::vector<CUtensorMap> tm_layer;
   CUtensorMap tm_ctrl_w1, tm_proj_w1, tm_proj_w2, tm_lm_head;
+  // kernel timing (svl_profile_start / svl_profile_stop)
+  bool prof = false;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
+  std::vector<std::pair<int, size_t>> prof_recs;  // (tag, index of the first event of the pair)
 };
 
 namespace {
@@ -142,6 +147,41 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   return L;
 }
 
+// Device copies of the inputs and intermediate outputs of
+// svl_prefill_from_host; the stage scratch follows at `inner`.
+struct HostLayout {
+  size_t vis, vis_off, text_ids, text_off, text_len, budget, keep, lg, gg;
+  size_t scores, k, kept_idx, kept_off, flags, X, cu, pos, logits, inner, total;
+};
+
+HostLayout host_layout(const svl_model_desc& d, int B, int64_t nv, int64_t nt) {
+  HostLayout L{};
+  Bump b;
+  const int64_t t_cap = std::max<int64_t>(nv + nt, 1);
+  L.vis = b.take(2 * std::max<int64_t>(nv, 1) * d.c_vis);
+  L.vis_off = b.take(4 * (B + 1));
+  L.text_ids = b.take(4 * std::max<int64_t>(nt, 1));
+  L.text_off = b.take(4 * (B + 1));
+  L.text_len = b.take(4 * B);
+  L.budget = b.take(4 * B);
+  L.keep = b.take(4 * B);
+  L.lg = b.take(static_cast<size_t>(B) * d.n_layers);
+  L.gg = b.take(static_cast<size_t>(B) * d.n_layers * d.n_groups);
+  L.scores = b.take(4 * std::max<int64_t>(nv, 1));
+  L.k = b.take(4 * B);
+  L.kept_idx = b.take(4 * std::max<int64_t>(nv, 1));
+  L.kept_off = b.take(4 * (B + 1));
+  L.flags = b.take(4 * B);
+  L.X = b.take(2 * t_cap * d.d_model);
+  L.cu = b.take(4 * (B + 1));
+  L.pos = b.take(4 * t_cap);
+  L.logits = b.take(sizeof(float) * static_cast<size_t>(B) * d.vocab);
+  L.inner = b.off;
+  const size_t a = sel_layout(d, B, nv).total, p = pack_layout(d, nv).total, c = pre_layout(d, B, t_cap).total;
+  L.total = L.inner + std::max(a, std::max(p, c));
+  return L;
+}
+
 template <typename T>
 T* at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
@@ -166,9 +206,35 @@ int gemm_grid(const svl_model* m, int64_t tiles) {
   return static_cast<int>(std::max<int64_t>(g, 1));
 }
 
-svl_status launch(EpiKind kind, const svl_model* m, const GemmParams& p, int64_t tiles, cudaStream_t s) {
+// Counts one kernel launch and, while profiling, brackets it with a pair of
+// events on its stream.
+struct Launch {
+  svl_model* m;
+  cudaStream_t s;
+  size_t first = SIZE_MAX;
+  Launch(svl_model* m_, int tag, cudaStream_t s_) : m(m_), s(s_) {
+    g_launches++;
+    if (!m->prof) return;
+    if (m->ev_used + 2 > m->ev_pool.size()) {
+      for (int i = 0; i < 64; ++i) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return;
+        m->ev_pool.push_back(e);
+      }
+    }
+    first = m->ev_used;
+    m->ev_used += 2;
+    m->prof_recs.emplace_back(tag, first);
+    cudaEventRecord(m->ev_pool[first], s);
+  }
+  ~Launch() {
+    if (first != SIZE_MAX) cudaEventRecord(m->ev_pool[first + 1], s);
+  }
+};
+
+svl_status launch(EpiKind kind, svl_model* m, int tag, const GemmParams& p, int64_t tiles, cudaStream_t s) {
   if (tiles <= 0) return SVL_OK;
-  g_launches++;
+  Launch L(m, tag, s);
   return launch_gemm(kind, p, gemm_grid(m, tiles), s) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
 }
 
@@ -274,6 +340,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
 
 void svl_model_destroy(svl_model* m) {
   if (!m) return;
+  for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
   if (m->d_status) cudaFree(m->d_status);
   if (m->rope_cs) cudaFree(m->rope_cs);
   delete m;
@@ -303,9 +370,11 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
   const svl_model_desc& d = m->d;
   float* e_b = at<float>(ws, L.e_b);
 
-  launch_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.bud_w1),
-                      static_cast<const __nv_bfloat16*>(m->w.bud_w2), d.h_ctrl, B, e_b, s);
-  g_launches++;
+  {
+    Launch L(m, SVL_TAG_BUDGET_EMBED, s);
+    launch_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.bud_w1),
+                        static_cast<const __nv_bfloat16*>(m->w.bud_w2), d.h_ctrl, B, e_b, s);
+  }
 
   if (n_vis_total > 0) {
     GemmParams p = base_params(m);
@@ -324,7 +393,7 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
     p.n_seg = B;
     p.w2 = static_cast<const __nv_bfloat16*>(m->w.ctrl_w2);
     p.c2 = m->w.ctrl_c2;
-    st = launch(EPI_SCORE, m, p, p.grid_m, s);
+    st = launch(EPI_SCORE, m, SVL_TAG_SCORE, p, p.grid_m, s);
     if (st != SVL_OK) return st;
   }
 
@@ -346,10 +415,14 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
   a.k_out = k;
   a.flags = sample_flags;
   a.kept_local = at<int>(ws, L.kept_local);
-  launch_select(a, B, s);
-  g_launches++;
-  launch_compact(B, vis_off, k, a.kept_local, kept_idx, kept_off, at<int>(ws, L.scalars), s);
-  g_launches++;
+  {
+    Launch L1(m, SVL_TAG_SELECT, s);
+    launch_select(a, B, s);
+  }
+  {
+    Launch L2(m, SVL_TAG_SELECT, s);
+    launch_compact(B, vis_off, k, a.kept_local, kept_idx, kept_off, at<int>(ws, L.scalars), s);
+  }
   return last_error();
 }
 
@@ -391,10 +464,14 @@ svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text
   a.stage = d.proj_hidden ? at<__nv_bfloat16>(ws, L.stage) : nullptr;
   a.row_map = d.proj_hidden ? at<int>(ws, L.row_map) : nullptr;
   a.status = m->d_status;
-  launch_pack_offsets(a, s);
-  g_launches++;
-  launch_pack_gather(a, s);
-  g_launches++;
+  {
+    Launch L1(m, SVL_TAG_PACK, s);
+    launch_pack_offsets(a, s);
+  }
+  {
+    Launch L2(m, SVL_TAG_PACK, s);
+    launch_pack_gather(a, s);
+  }
 
   if (d.proj_hidden && n_vis_total > 0) {
     GemmParams p = base_params(m);
@@ -410,7 +487,7 @@ svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text
     p.kgroup = d.c_vis;
     p.out[0] = at<__nv_bfloat16>(ws, L.hp);
     p.ld[0] = d.proj_hidden;
-    st = launch(EPI_GELU, m, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s);
+    st = launch(EPI_GELU, m, SVL_TAG_PROJECTOR, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s);
     if (st != SVL_OK) return st;
 
     GemmParams q = base_params(m);
@@ -427,7 +504,7 @@ svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text
     q.out[0] = X;
     q.ld[0] = d.d_model;
     q.row_map = a.row_map;
-    st = launch(EPI_ROWMAP, m, q, static_cast<int64_t>(q.grid_m) * q.grid_n, s);
+    st = launch(EPI_ROWMAP, m, SVL_TAG_PROJECTOR, q, static_cast<int64_t>(q.grid_m) * q.grid_n, s);
     if (st != SVL_OK) return st;
   }
   return last_error();
@@ -481,8 +558,10 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   sa.attn_cap = L.attn_cap;
   sa.attn_count = counts + 4 * nl;
   sa.status = m->d_status;
-  launch_schedule(sa, s);
-  g_launches++;
+  {
+    Launch L1(m, SVL_TAG_SCHEDULE, s);
+    launch_schedule(sa, s);
+  }
 
   __nv_bfloat16* xn = at<__nv_bfloat16>(ws, L.xn);
   __nv_bfloat16* qb = at<__nv_bfloat16>(ws, L.q);
@@ -520,8 +599,10 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     const CUtensorMap* tm = &m->tm_layer[static_cast<size_t>(l) * 7];
     na.act = sa.act + static_cast<size_t>(l) * B;
     na.gain = static_cast<const __nv_bfloat16*>(lw.attn_norm);
-    launch_rmsnorm(na, s);
-    g_launches++;
+    {
+      Launch L1(m, SVL_TAG_RMSNORM, s);
+      launch_rmsnorm(na, s);
+    }
 
     GemmParams p = base_params(m);
     p.mapA = map_xn;
@@ -543,12 +624,14 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.rope_cs = m->rope_cs;
     p.rope_rows = d.max_seq;
     p.d_head = dh;
-    if ((st = launch(EPI_QKV_ROPE, m, p, L.qkv_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s)) != SVL_OK) return st;
 
     aa.items = sa.attn_items + static_cast<size_t>(l) * L.attn_cap;
     aa.count = counts + 4 * nl + l;
-    launch_attention(aa, s);
-    g_launches++;
+    {
+      Launch L1(m, SVL_TAG_ATTENTION, s);
+      launch_attention(aa, s);
+    }
 
     p = base_params(m);
     p.mapA = map_ao;
@@ -560,11 +643,13 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = hq / d.n_groups;
     p.out[0] = X;
     p.ld[0] = d.d_model;
-    if ((st = launch(EPI_RESID, m, p, L.o_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s)) != SVL_OK) return st;
 
     na.gain = static_cast<const __nv_bfloat16*>(lw.ffn_norm);
-    launch_rmsnorm(na, s);
-    g_launches++;
+    {
+      Launch L1(m, SVL_TAG_RMSNORM, s);
+      launch_rmsnorm(na, s);
+    }
 
     p = base_params(m);
     p.mapA = map_xn;
@@ -578,7 +663,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = d.d_model;
     p.out[0] = hm;
     p.ld[0] = d.d_ffn;
-    if ((st = launch(EPI_SWIGLU, m, p, L.gu_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s)) != SVL_OK) return st;
 
     p = base_params(m);
     p.mapA = map_hm;
@@ -590,7 +675,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = d.d_ffn / d.n_groups;
     p.out[0] = X;
     p.ld[0] = d.d_model;
-    if ((st = launch(EPI_RESID, m, p, L.dn_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s)) != SVL_OK) return st;
   }
 
   // final norm + LM head
@@ -600,8 +685,10 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   if (logits_mode == SVL_LOGITS_LAST) {
     const int n_pad = ((B + 15) / 16) * 16;
     na.Y = at<__nv_bfloat16>(ws, L.yl);
-    launch_final_last_rows(na, n_pad, s);
-    g_launches++;
+    {
+      Launch L1(m, SVL_TAG_RMSNORM, s);
+      launch_final_last_rows(na, n_pad, s);
+    }
     p.mapA = m->tm_lm_head;
     if (!make_map(&p.mapB[0], na.Y, n_pad, d.d_model)) return SVL_ERR_CUDA;
     p.grid_m = (d.vocab + kBM - 1) / kBM;
@@ -613,10 +700,12 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = d.d_model;
     p.out[0] = logits;
     p.ld[0] = d.vocab;
-    if ((st = launch(EPI_LOGITS_T, m, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_LOGITS_T, m, SVL_TAG_LMHEAD, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
   } else {
-    launch_rmsnorm(na, s);
-    g_launches++;
+    {
+      Launch L1(m, SVL_TAG_RMSNORM, s);
+      launch_rmsnorm(na, s);
+    }
     p.mapA = map_xn;
     p.mapB[0] = m->tm_lm_head;
     p.grid_m = (t_cap + kBM - 1) / kBM;
@@ -629,7 +718,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = d.d_model;
     p.out[0] = logits;
     p.ld[0] = d.vocab;
-    if ((st = launch(EPI_F32, m, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_F32, m, SVL_TAG_LMHEAD, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
   }
   return last_error();
 }
@@ -654,6 +743,112 @@ svl_status svl_flops(const svl_model_desc* d, int32_t s_text, int32_t s_vis, int
     *exec = f;
   }
   return SVL_OK;
+}
+
+size_t svl_host_workspace_size(const svl_model* m, int32_t B, int64_t nv, int64_t nt) {
+  if (!m || B <= 0 || nv < 0 || nt < 0) return 0;
+  return host_layout(m->d, B, nv, nt).total;
+}
+
+svl_status svl_prefill_from_host(svl_model* m, int32_t B, int32_t nv, int32_t nt, const void* h_vis,
+                                 const int32_t* h_vis_off, const int32_t* h_text_ids, const int32_t* h_text_off,
+                                 const float* h_budget, const int32_t* h_keep_count, const uint8_t* h_layer_gate,
+                                 const uint8_t* h_group_gate, float* h_logits, int32_t* h_k, void* ws,
+                                 size_t ws_bytes, void* stream) {
+  if (!m || B <= 0 || nv < 0 || nt < 0 || !h_vis_off || !h_text_off || !h_budget || !h_layer_gate ||
+      !h_group_gate || !h_logits || (nv > 0 && !h_vis) || (nt > 0 && !h_text_ids))
+    return SVL_ERR_INVALID_ARG;
+  const HostLayout H = host_layout(m->d, B, nv, nt);
+  svl_status st = check_ws(ws, ws_bytes, H.total);
+  if (st != SVL_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const svl_model_desc& d = m->d;
+  const size_t L = d.n_layers, G = d.n_groups;
+  auto h2d = [&](size_t off, const void* src, size_t bytes) {
+    return bytes == 0 || cudaMemcpyAsync(at<uint8_t>(ws, off), src, bytes, cudaMemcpyHostToDevice, s) == cudaSuccess;
+  };
+  bool ok;
+  {
+    Launch C(m, SVL_TAG_COPY, s);
+    ok = h2d(H.vis, h_vis, 2 * static_cast<size_t>(nv) * d.c_vis) && h2d(H.vis_off, h_vis_off, 4 * (B + 1)) &&
+         h2d(H.text_ids, h_text_ids, 4 * static_cast<size_t>(nt)) && h2d(H.text_off, h_text_off, 4 * (B + 1)) &&
+         h2d(H.budget, h_budget, 4 * B) && h2d(H.lg, h_layer_gate, B * L) && h2d(H.gg, h_group_gate, B * L * G) &&
+         (!h_keep_count || h2d(H.keep, h_keep_count, 4 * B));
+    g_launches--;  // copies are not kernels
+  }
+  if (!ok) return SVL_ERR_CUDA;
+  {
+    Launch L1(m, SVL_TAG_PACK, s);
+    launch_offsets_diff(at<int>(ws, H.text_off), at<int>(ws, H.text_len), B, s);
+  }
+  void* inner = at<uint8_t>(ws, H.inner);
+  const size_t inner_bytes = ws_bytes - H.inner;
+  st = svl_score_select(m, B, nv, at<void>(ws, H.vis), at<int>(ws, H.vis_off), at<int>(ws, H.text_len),
+                        at<float>(ws, H.budget), h_keep_count ? at<int>(ws, H.keep) : nullptr,
+                        at<uint8_t>(ws, H.lg), at<uint8_t>(ws, H.gg), at<float>(ws, H.scores), at<int>(ws, H.k),
+                        at<int>(ws, H.kept_idx), at<int>(ws, H.kept_off), at<uint32_t>(ws, H.flags), inner,
+                        inner_bytes, stream);
+  if (st != SVL_OK) return st;
+  st = svl_pack(m, B, nv, nt, at<void>(ws, H.vis), at<int>(ws, H.vis_off), at<int>(ws, H.kept_idx),
+                at<int>(ws, H.kept_off), at<int>(ws, H.text_ids), at<int>(ws, H.text_off), at<void>(ws, H.X),
+                at<int>(ws, H.cu), at<int>(ws, H.pos), inner, inner_bytes, stream);
+  if (st != SVL_OK) return st;
+  const int t_cap = std::max(nv + nt, 1);
+  st = svl_gated_prefill(m, B, t_cap, at<void>(ws, H.X), at<int>(ws, H.cu), at<int>(ws, H.pos),
+                         at<uint8_t>(ws, H.lg), at<uint8_t>(ws, H.gg), SVL_LOGITS_LAST, at<float>(ws, H.logits),
+                         inner, inner_bytes, stream);
+  if (st != SVL_OK) return st;
+  {
+    Launch C(m, SVL_TAG_COPY, s);
+    g_launches--;
+    ok = cudaMemcpyAsync(h_logits, at<float>(ws, H.logits), sizeof(float) * static_cast<size_t>(B) * d.vocab,
+                         cudaMemcpyDeviceToHost, s) == cudaSuccess &&
+         (!h_k || cudaMemcpyAsync(h_k, at<int>(ws, H.k), 4 * B, cudaMemcpyDeviceToHost, s) == cudaSuccess);
+  }
+  return ok ? SVL_OK : SVL_ERR_CUDA;
+}
+
+svl_status svl_profile_start(svl_model* m) {
+  if (!m) return SVL_ERR_INVALID_ARG;
+  m->prof = true;
+  m->ev_used = 0;
+  m->prof_recs.clear();
+  return SVL_OK;
+}
+
+svl_status svl_profile_stop(svl_model* m, svl_kernel_time* out, int32_t cap, int32_t* n_out) {
+  if (!m || (!out && cap > 0)) return SVL_ERR_INVALID_ARG;
+  m->prof = false;
+  double tot[SVL_TAG_COUNT] = {0};
+  int cnt[SVL_TAG_COUNT] = {0};
+  if (!m->prof_recs.empty()) {
+    if (cudaEventSynchronize(m->ev_pool[m->prof_recs.back().second + 1]) != cudaSuccess) return SVL_ERR_CUDA;
+  }
+  for (const auto& r : m->prof_recs) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, m->ev_pool[r.second], m->ev_pool[r.second + 1]) != cudaSuccess) return SVL_ERR_CUDA;
+    if (r.first >= 0 && r.first < SVL_TAG_COUNT) {
+      tot[r.first] += ms;
+      cnt[r.first] += 1;
+    }
+  }
+  m->prof_recs.clear();
+  m->ev_used = 0;
+  int n = 0;
+  for (int t = 0; t < SVL_TAG_COUNT; ++t) {
+    if (!cnt[t]) continue;
+    if (n < cap) out[n] = svl_kernel_time{t, cnt[t], tot[t]};
+    ++n;
+  }
+  if (n_out) *n_out = std::min(n, cap);
+  return SVL_OK;
+}
+
+const char* svl_tag_name(int32_t tag) {
+  static const char* names[SVL_TAG_COUNT] = {"budget_embed", "score", "select", "pack", "projector",
+                                              "schedule", "rmsnorm", "qkv_gemm", "attention", "o_gemm",
+                                              "gateup_gemm", "down_gemm", "lm_head", "host_copy"};
+  return (tag >= 0 && tag < SVL_TAG_COUNT) ? names[tag] : "unknown";
 }
 
 svl_status svl_get_device_status(svl_model* m, void* stream, uint32_t* code) {

@@ -52,6 +52,7 @@ struct PackArgs {
   uint32_t* status;
 };
 void launch_pack_offsets(const PackArgs& a, cudaStream_t s);
+void launch_offsets_diff(const int* off, int* len, int B, cudaStream_t s);
 void launch_pack_gather(const PackArgs& a, cudaStream_t s);
 
 // ---------------------------------------------------------------- decoder

@@ -66,6 +66,15 @@ __global__ void pack_gather_kernel(PackArgs a) {
   for (int c = lane; c < width / 8; c += 32) dst[c] = bad ? make_uint4(0, 0, 0, 0) : src[c];
 }
 
+__global__ void offsets_diff_kernel(const int* off, int* len, int B) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) len[b] = off[b + 1] - off[b];
+}
+
+void launch_offsets_diff(const int* off, int* len, int B, cudaStream_t s) {
+  offsets_diff_kernel<<<(B + 255) / 256, 256, 0, s>>>(off, len, B);
+}
+
 void launch_pack_offsets(const PackArgs& a, cudaStream_t s) { pack_offsets_kernel<<<1, 32, 0, s>>>(a); }
 
 void launch_pack_gather(const PackArgs& a, cudaStream_t s) {

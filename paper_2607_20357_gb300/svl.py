@@ -24,7 +24,16 @@ SVL_FLAG_OVER_BUDGET = 1
 SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
 
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
-           "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count"]
+           "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
+           "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
+           "svl_tag_name"]
+
+TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
+        "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
+
+
+class KernelTime(ctypes.Structure):
+    _fields_ = [("tag", ctypes.c_int32), ("launches", ctypes.c_int32), ("total_ms", ctypes.c_double)]
 
 
 class ModelDesc(ctypes.Structure):
@@ -73,6 +82,16 @@ def lib():
         L.svl_status_string.restype = ctypes.c_char_p
         L.svl_launch_count.argtypes = []
         L.svl_launch_count.restype = ctypes.c_uint64
+        L.svl_prefill_from_host.argtypes = [vp, i32, i32, i32] + [vp] * 13 + [sz, vp]
+        L.svl_prefill_from_host.restype = ctypes.c_int
+        L.svl_host_workspace_size.argtypes = [vp, i32, i64, i64]
+        L.svl_host_workspace_size.restype = sz
+        L.svl_profile_start.argtypes = [vp]
+        L.svl_profile_start.restype = ctypes.c_int
+        L.svl_profile_stop.argtypes = [vp, ctypes.POINTER(KernelTime), i32, ctypes.POINTER(i32)]
+        L.svl_profile_stop.restype = ctypes.c_int
+        L.svl_tag_name.argtypes = [i32]
+        L.svl_tag_name.restype = ctypes.c_char_p
         _lib = L
     return _lib
 
@@ -160,6 +179,33 @@ def svl_get_device_status(model, stream=None) -> int:
 
 def svl_launch_count() -> int:
     return int(lib().svl_launch_count())
+
+
+def svl_prefill_from_host(model, B, n_vis_total, n_text_total, h_vis, h_vis_off, h_text_ids, h_text_off, h_budget,
+                          h_keep_count, h_layer_gate, h_group_gate, h_logits, h_k, workspace, workspace_bytes,
+                          stream=None):
+    """Host tensors (pinned CPU) in, host logits/k out; async on the stream."""
+    _check("svl_prefill_from_host", lib().svl_prefill_from_host(
+        model, int(B), int(n_vis_total), int(n_text_total), _p(h_vis), _p(h_vis_off), _p(h_text_ids),
+        _p(h_text_off), _p(h_budget), _p(h_keep_count), _p(h_layer_gate), _p(h_group_gate), _p(h_logits),
+        _p(h_k), _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_host_workspace_size(model, B, n_vis_total, n_text_total) -> int:
+    return int(lib().svl_host_workspace_size(model, int(B), int(n_vis_total), int(n_text_total)))
+
+
+def svl_profile_start(model):
+    _check("svl_profile_start", lib().svl_profile_start(model))
+
+
+def svl_profile_stop(model) -> dict:
+    """{tag name: (launches, total ms)} of the kernels since svl_profile_start."""
+    buf = (KernelTime * 32)()
+    n = ctypes.c_int32()
+    _check("svl_profile_stop", lib().svl_profile_stop(model, buf, 32, ctypes.byref(n)))
+    return {lib().svl_tag_name(buf[i].tag).decode(): (int(buf[i].launches), float(buf[i].total_ms))
+            for i in range(n.value)}
 
 
 # --------------------------------------------------------------------------- plumbing

@@ -121,11 +121,18 @@ def _normal(shape, std, g, device, dtype=torch.bfloat16):
     return t.to(dtype)
 
 
-def make_weights(dims: ModelDims, seed: int, device="cpu", std: float = 0.02) -> dict:
+def _tensor_seed(seed: int, layer: int, slot: int) -> int:
+    """Independent stream per tensor, so any subset of layers is reproducible."""
+    return (int(seed) * 1_000_003 + (layer + 1) * 64 + slot) % (1 << 62)
+
+
+def make_weights(dims: ModelDims, seed: int, device="cpu", std: float = 0.02, layers=None) -> dict:
     """All model weights, bf16, ``nn.Linear`` layout, drawn N(0, std).
 
     The token embedding table is drawn N(0, 1) so that text rows enter the
-    residual stream at a scale comparable to projected visual rows.
+    residual stream at a scale comparable to projected visual rows. Each
+    tensor has its own seeded stream (``layers`` limits which decoder layers
+    are drawn; the others are omitted from the list).
 
     Keys: ctrl_w1 [H, C_v], ctrl_w2 [H] and ctrl_c2 (float) for the token
     scorer; bud_w1, bud_w2 [H, H] for the budget MLP; proj_w1 [P_h, C_v],
@@ -133,35 +140,38 @@ def make_weights(dims: ModelDims, seed: int, device="cpu", std: float = 0.02) ->
     wq [A*dh, D], wk/wv [A_kv*dh, D], wo [D, A*dh], wg/wu [D_int, D],
     wd [D, D_int], attn_norm/ffn_norm [D]; final_norm [D]; lm_head [V, D].
     """
-    g = _gen(seed, device)
     D, H = dims.d_model, dims.h_ctrl
+
+    def draw(shape, sd, layer, slot):
+        return _normal(shape, sd, _gen(_tensor_seed(seed, layer, slot), device), device)
+
     w = {
-        "ctrl_w1": _normal((H, dims.c_vis), std, g, device),
-        "ctrl_w2": _normal((H,), std, g, device),
+        "ctrl_w1": draw((H, dims.c_vis), std, -1, 0),
+        "ctrl_w2": draw((H,), std, -1, 1),
         "ctrl_c2": 0.0,
-        "bud_w1": _normal((H, H), std, g, device),
-        "bud_w2": _normal((H, H), std, g, device),
+        "bud_w1": draw((H, H), std, -1, 2),
+        "bud_w2": draw((H, H), std, -1, 3),
     }
     if dims.proj_hidden:
-        w["proj_w1"] = _normal((dims.proj_hidden, dims.c_vis), std, g, device)
-        w["proj_w2"] = _normal((D, dims.proj_hidden), std, g, device)
-    w["embed"] = _normal((dims.vocab, D), 1.0, g, device)
-    layers = []
-    for _ in range(dims.n_layers):
-        layers.append({
-            "wq": _normal((dims.n_heads * dims.d_head, D), std, g, device),
-            "wk": _normal((dims.d_kv, D), std, g, device),
-            "wv": _normal((dims.d_kv, D), std, g, device),
-            "wo": _normal((D, dims.n_heads * dims.d_head), std, g, device),
-            "wg": _normal((dims.d_ffn, D), std, g, device),
-            "wu": _normal((dims.d_ffn, D), std, g, device),
-            "wd": _normal((D, dims.d_ffn), std, g, device),
+        w["proj_w1"] = draw((dims.proj_hidden, dims.c_vis), std, -1, 4)
+        w["proj_w2"] = draw((D, dims.proj_hidden), std, -1, 5)
+    w["embed"] = draw((dims.vocab, D), 1.0, -1, 6)
+    out_layers = []
+    for l in (range(dims.n_layers) if layers is None else layers):
+        out_layers.append({
+            "wq": draw((dims.n_heads * dims.d_head, D), std, l, 0),
+            "wk": draw((dims.d_kv, D), std, l, 1),
+            "wv": draw((dims.d_kv, D), std, l, 2),
+            "wo": draw((D, dims.n_heads * dims.d_head), std, l, 3),
+            "wg": draw((dims.d_ffn, D), std, l, 4),
+            "wu": draw((dims.d_ffn, D), std, l, 5),
+            "wd": draw((D, dims.d_ffn), std, l, 6),
             "attn_norm": torch.ones(D, dtype=torch.bfloat16, device=device),
             "ffn_norm": torch.ones(D, dtype=torch.bfloat16, device=device),
         })
-    w["layers"] = layers
+    w["layers"] = out_layers
     w["final_norm"] = torch.ones(D, dtype=torch.bfloat16, device=device)
-    w["lm_head"] = _normal((dims.vocab, D), std, g, device)
+    w["lm_head"] = draw((dims.vocab, D), std, -1, 7)
     return w
 
 
