@@ -82,7 +82,7 @@ def lib():
         L.svl_status_string.restype = ctypes.c_char_p
         L.svl_launch_count.argtypes = []
         L.svl_launch_count.restype = ctypes.c_uint64
-        L.svl_prefill_from_host.argtypes = [vp, i32, i32, i32] + [vp] * 13 + [sz, vp]
+        L.svl_prefill_from_host.argtypes = [vp, i32, i32, i32] + [vp] * 11 + [sz, vp]
         L.svl_prefill_from_host.restype = ctypes.c_int
         L.svl_host_workspace_size.argtypes = [vp, i32, i64, i64]
         L.svl_host_workspace_size.restype = sz

@@ -59,3 +59,20 @@ def test_host_flops_match_oracle(svl_lib, name):
         n_on = O.effective_groups(lg.numpy(), gg.numpy(), dims.n_prefix).sum(1)
         assert eq8 == pytest.approx(O.prefill_cost_xG(dims, s_text + k, n_on) / dims.n_groups, rel=1e-15)
         assert ex == pytest.approx(O.executed_flops(dims, n_vis, k, s_text, n_on), rel=1e-12)
+
+
+def _declared_param_counts():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    out = {}
+    for m in re.finditer(r"\b(svl_\w+)\s*\(([^;{]*?)\)\s*;", text, re.S):
+        args = m.group(2).strip()
+        out[m.group(1)] = 0 if args in ("", "void") else len(args.split(","))
+    return out
+
+
+def test_binding_argument_counts_match_header(svl_lib):
+    counts = _declared_param_counts()
+    for name in svl.SYMBOLS:
+        fn = getattr(svl_lib, name)
+        assert len(fn.argtypes) == counts[name], (name, len(fn.argtypes), counts[name])
