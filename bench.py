@@ -347,7 +347,7 @@ def run_ours(args, rank, world, local_rank):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        nl = 8
+        nl = 16
         wl_cpu = [{k: v.cpu() for k, v in weights["layers"][l].items()} for l in range(nl)]
         rest = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in weights.items() if k != "layers"}
         b_cpu = {k: (v.cpu() if isinstance(v, torch.Tensor) else v) for k, v in batches[1].items()}
