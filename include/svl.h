@@ -149,6 +149,30 @@ svl_status svl_score_select(svl_model* model, int32_t B, int32_t n_vis_total,
                             uint32_t* sample_flags, void* workspace, size_t workspace_bytes,
                             void* stream);
 
+/* svl_score_select without a workspace argument. The paper has no
+ *  counterpart: this exists for callers that cannot allocate device memory
+ *  for a workspace -- code running during CUDA stream capture (where
+ *  cudaMalloc is not permitted), plugins whose host framework keeps all
+ *  device memory for its own allocator, real-time paths that must not wait
+ *  in an allocator. It allocates nothing; its scratch (budget embeddings and
+ *  per-sample kept lists) lives in one fixed 512 KiB device array inside the
+ *  library, present on every GPU that loads the library until the process
+ *  exits. Limits: B <= 256, n_vis_total <= 65536, h_ctrl <= 256; larger
+ *  calls return SVL_ERR_SHAPE and launch nothing. Outputs and their meaning
+ *  are those of svl_score_select. The first call on a device looks up the
+ *  array's device address (cudaGetSymbolAddress, once per device, with that
+ *  device current and equal to the model's), so make that first call before
+ *  any stream capture. All calls share the one array and it keeps the last
+ *  call's contents; every scratch value a call reads it writes first, so
+ *  nothing needs clearing, but calls that overlap on the GPU (e.g. on two
+ *  streams at once) race on it and must be serialised by the caller. */
+svl_status svl_score_select_noalloc(svl_model* model, int32_t B, int32_t n_vis_total,
+                                    const void* vis_feats, const int32_t* vis_off, const int32_t* text_len,
+                                    const float* budget, const int32_t* keep_count,
+                                    const uint8_t* layer_gate, const uint8_t* group_gate,
+                                    float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off,
+                                    uint32_t* sample_flags, void* stream);
+
 /* (2) Pack (Sec. 3 S = S_text + S_vis; Sec. 3.1 contiguous RoPE).
  *  Sample b's sequence is its kept visual tokens in ascending index order,
  *  projected by the LLaVA MLP W_p2 GELU(W_p1 x) (identity when proj_hidden

@@ -863,3 +863,120 @@ svl_status svl_get_device_status(svl_model* m, void* stream, uint32_t* code) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Token controller without workspace: svl_score_select_noalloc.
+//
+// Some callers cannot hand the library freshly allocated device memory: code
+// that runs while a stream is being captured into a CUDA graph (cudaMalloc is
+// not allowed there), plugins whose host framework has already reserved the
+// device's memory for its own allocator and gives them none, or real-time
+// paths that must not block in the allocator. For them this entry point keeps
+// its scratch -- the budget embeddings e_b and the per-sample kept lists -- in
+// one fixed array in device memory that is part of the library image. Every
+// GPU that loads the library holds the array until the process exits.
+namespace {
+
+constexpr int kNoAllocMaxBatch = 256;     // samples per call
+constexpr int kNoAllocMaxHctrl = 256;     // token-controller hidden width
+constexpr int kNoAllocMaxVis = 65536;     // visual tokens per call (all samples)
+constexpr size_t kNoAllocEbBytes = sizeof(float) * kNoAllocMaxBatch * kNoAllocMaxHctrl;   // 256 KiB
+constexpr size_t kNoAllocListBytes = sizeof(int) * kNoAllocMaxVis;                        // 256 KiB
+constexpr size_t kNoAllocScratchBytes = kNoAllocEbBytes + kNoAllocListBytes;              // 512 KiB
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch array on the current device. In host code
+// the array's name is only a host-side stand-in, so the address is looked up
+// once per device (with that device current) and cached.
+svl_status noalloc_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices) return SVL_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return SVL_ERR_CUDA;
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return SVL_OK;
+}
+
+}  // namespace
+
+extern "C" svl_status svl_score_select_noalloc(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
+                                               const int32_t* vis_off, const int32_t* text_len, const float* budget,
+                                               const int32_t* keep_count, const uint8_t* layer_gate,
+                                               const uint8_t* group_gate, float* scores, int32_t* k,
+                                               int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
+                                               void* stream) {
+  if (!m || B <= 0 || n_vis_total < 0 || !vis_off || !text_len || !budget || !layer_gate || !group_gate ||
+      !scores || !k || !kept_idx || !kept_off)
+    return SVL_ERR_INVALID_ARG;
+  if (n_vis_total > 0 && (!vis_feats || !aligned16(vis_feats))) return SVL_ERR_INVALID_ARG;
+  if (B > kNoAllocMaxBatch || n_vis_total > kNoAllocMaxVis || m->d.h_ctrl > kNoAllocMaxHctrl)
+    return SVL_ERR_SHAPE;  // beyond the fixed scratch array
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev != m->device) return SVL_ERR_INVALID_ARG;
+  void* scratch = nullptr;
+  svl_status st = noalloc_scratch(&scratch);
+  if (st != SVL_OK) return st;
+  float* e_b = static_cast<float*>(scratch);
+  int* kept_local = reinterpret_cast<int*>(static_cast<unsigned char*>(scratch) + kNoAllocEbBytes);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const svl_model_desc& d = m->d;
+
+  // Every scratch element read below is written earlier in the same call
+  // (e_b by the budget MLP, kept_local[vis_off[b] ..] by the select kernel
+  // before compaction reads it), so nothing has to be cleared first.
+  g_launches++;
+  launch_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.bud_w1),
+                      static_cast<const __nv_bfloat16*>(m->w.bud_w2), d.h_ctrl, B, e_b, s);
+  if (n_vis_total > 0) {
+    GemmParams p = base_params(m);
+    if (!make_map(&p.mapA, vis_feats, n_vis_total, d.c_vis)) return SVL_ERR_INVALID_ARG;
+    p.mapB[0] = m->tm_ctrl_w1;
+    p.grid_m = (n_vis_total + kBM - 1) / kBM;
+    p.grid_n = 1;
+    p.bn = d.h_ctrl;
+    p.m_limit = n_vis_total;
+    p.n_limit = d.h_ctrl;
+    p.K = d.c_vis;
+    p.kgroup = d.c_vis;
+    p.out[0] = scores;
+    p.e_b = e_b;
+    p.seg_off = vis_off;
+    p.n_seg = B;
+    p.w2 = static_cast<const __nv_bfloat16*>(m->w.ctrl_w2);
+    p.c2 = m->w.ctrl_c2;
+    g_launches++;
+    if (launch_gemm(EPI_SCORE, p, gemm_grid(m, p.grid_m), s) != cudaSuccess) return SVL_ERR_CUDA;
+  }
+  SelectArgs a;
+  a.scores = scores;
+  a.vis_off = vis_off;
+  a.text_len = text_len;
+  a.budget = budget;
+  a.keep_count = keep_count;
+  a.layer_gate = layer_gate;
+  a.group_gate = group_gate;
+  a.L = d.n_layers;
+  a.G = d.n_groups;
+  a.P = d.n_prefix;
+  a.D = d.d_model;
+  a.Dkv = static_cast<long long>(d.n_kv_heads) * (d.d_model / d.n_heads);
+  a.Di = d.d_ffn;
+  a.V = d.vocab;
+  a.k_out = k;
+  a.flags = sample_flags;
+  a.kept_local = kept_local;
+  g_launches++;
+  launch_select(a, B, s);
+  g_launches++;
+  launch_compact(B, vis_off, k, kept_local, kept_idx, kept_off, nullptr, s);
+  return last_error();
+}

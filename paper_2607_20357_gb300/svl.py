@@ -26,7 +26,7 @@ SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
-           "svl_tag_name"]
+           "svl_tag_name", "svl_score_select_noalloc"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
@@ -92,6 +92,8 @@ def lib():
         L.svl_profile_stop.restype = ctypes.c_int
         L.svl_tag_name.argtypes = [i32]
         L.svl_tag_name.restype = ctypes.c_char_p
+        L.svl_score_select_noalloc.argtypes = [vp, i32, i32] + [vp] * 13
+        L.svl_score_select_noalloc.restype = ctypes.c_int
         _lib = L
     return _lib
 
@@ -143,6 +145,16 @@ def svl_score_select(model, B, n_vis_total, vis_feats, vis_off, text_len, budget
         model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
         _p(layer_gate), _p(group_gate), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags),
         _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_score_select_noalloc(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
+                             group_gate, scores, k, kept_idx, kept_off, sample_flags, stream=None):
+    """svl_score_select for callers that cannot allocate a workspace: the
+    library's fixed device scratch array is used instead (see svl.h)."""
+    _check("svl_score_select_noalloc", lib().svl_score_select_noalloc(
+        model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
+        _p(layer_gate), _p(group_gate), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags),
+        _stream(stream)))
 
 
 def svl_pack(model, B, n_vis_total, n_text_total, vis_feats, vis_off, kept_idx, kept_off, text_ids, text_off,
