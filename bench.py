@@ -49,6 +49,9 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="decoder layers (default: all 32). Fewer layers only for small profiler captures; "
+                         "such a line is not the benchmark value")
     return ap.parse_args()
 
 
@@ -240,6 +243,8 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     wl = synth.WORKLOADS[WORKLOAD]
+    if args.layers:
+        wl = synth.dataclasses.replace(wl, dims=synth.reduced(wl.dims, n_layers=args.layers))
     dims = wl.dims
     B = wl.batch
     pk = peaks()
@@ -362,7 +367,7 @@ def run_ours(args, rank, world, local_rank):
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": workload_config(wl, B),
+            "config": dict(workload_config(wl, B), **({"profiling_only_layers": args.layers} if args.layers else {})),
             "exec_tflops": fexec_total / (total_ms / 1000.0) / 1e12,
             "exec_tflops_frac_of_peak": fexec_total / (total_ms / 1000.0) / 1e12 / peak,
             "per_budget": per_budget, "roofline": roofline, "kernels": kernels,
