@@ -329,7 +329,11 @@ def run_ours(args, rank, world, local_rank):
                 "frac": achieved / peak, "peak_source": pk["source"] + " bf16 sustained",
                 "launches": n_l, "avg_launch_ms": t_l / n_l,
                 "flops_per_launch": kind_flops[dom] / n_l,
-                "traffic": (traffic_rec or {}).get("dram_bytes_per_launch") if traffic_rec else None}
+                "traffic": (traffic_rec["dram_bytes_per_launch"] * (kind_flops[dom] / n_l)
+                            / traffic_rec["flops_per_launch_at_capture"])
+                if traffic_rec and dom == "gateup_gemm" else None,
+                "traffic_note": "DRAM bytes of one ncu capture (profiles/gemm_traffic.json, budget-1.0 launch) "
+                                "scaled to this run's average launch by its FLOPs"}
     kernels = {t: {"launches": n, "total_ms": ms, "share": ms / max(sum(v[1] for v in kern.values()), 1e-9)}
                for t, (n, ms) in sorted(kern.items(), key=lambda kv: -kv[1][1])}
     for t in list(kind_flops):

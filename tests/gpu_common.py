@@ -49,6 +49,26 @@ def gpu_topk_valid(scores, kept, k):
     assert sorted(order[:k]) == sorted(kept.tolist())
 
 
+class LazyLayers:
+    """Decoder layer weights converted to float64 numpy only when the oracle
+    reaches that layer (keeps host memory to one layer at a time)."""
+
+    def __init__(self, layers):
+        self.layers = layers
+
+    def __len__(self):
+        return len(self.layers)
+
+    def __getitem__(self, i):
+        return {k: v.detach().to("cpu", torch.float64).numpy() for k, v in self.layers[i].items()}
+
+
+def numpy_weights_lazy(w):
+    out = O.to_numpy_weights(dict(w, layers=[]))
+    out["layers"] = LazyLayers(w["layers"])
+    return out
+
+
 class Case:
     """Seeded model + batch on the GPU and the oracle's view of both."""
 

@@ -1,0 +1,78 @@
+"""Parity at the workloads' full sizes, in the launch configuration the
+benchmark times (whole batch through the three C entry points), checked on
+samples the oracle recomputes one by one.
+
+The LLaVA-1.5-7B batch runs with all 32 layers; the Qwen2-VL-7B, video and
+mixed-serving batches keep their full batch, sequence and width shapes with
+the decoder cut to 2 layers so the float64 oracle stays within seconds per
+sample.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import smartvl_oracle as O
+from paper_2607_20357_gb300 import svl, synth
+from tests.gpu_common import check_selection, numpy_weights_lazy, rel_err, to_device
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+
+def _run_full(wl, dims, seed, samples, budget=None, tol=2e-2, modify=None):
+    dev = torch.device("cuda")
+    w = synth.make_weights(dims, seed, device=dev)
+    batch = synth.make_batch(wl, seed, budget=budget, device=dev, dims=dims)
+    if modify:
+        modify(batch)
+    S_max = int((batch["vis_off"][1:] - batch["vis_off"][:-1] + batch["text_off"][1:] - batch["text_off"][:-1]).max())
+    model = svl.GatedPrefill(dims, w, max_seq=S_max + 8)
+    out = model.run(batch)
+    torch.cuda.synchronize()
+    assert svl.svl_get_device_status(model.handle) == 0
+    out = {k: v.cpu() for k, v in out.items()}
+    w_np = numpy_weights_lazy(w)
+    b_np = O.to_numpy_batch(batch)
+    errs = []
+    for b in samples:
+        r = O.forward_batch(dims, w_np, b_np, mode="fp32", samples=[b])[0]
+        assert int(out["k"][b]) == r["k"]
+        assert int(out["flags"][b]) == r["flags"]
+        v0, v1 = b_np["vis_off"][b], b_np["vis_off"][b + 1]
+        kept = out["kept_idx"][out["kept_off"][b]:out["kept_off"][b + 1]].numpy()
+        np.testing.assert_allclose(out["scores"][v0:v1].double().numpy(), r["z"], rtol=1e-4, atol=1e-5)
+        if not check_selection(out["scores"][v0:v1].numpy(), kept, r):
+            continue
+        cu = out["cu_seqlens"].numpy()
+        e_h = rel_err(out["X"][cu[b]:cu[b + 1]].double().numpy(), r["hidden"])
+        e_l = rel_err(out["logits"][b].double().numpy(), r["logits"])
+        errs.append((b, e_h, e_l))
+        assert e_h < tol and e_l < tol, (b, e_h, e_l)
+    model.close()
+    assert errs
+    return errs
+
+
+def test_llava_full_depth_budget_half():
+    wl = synth.WORKLOADS["llava"]
+    print(_run_full(wl, wl.dims, 1000, samples=[0, 15], budget=0.5))
+
+
+def test_qwen_full_shapes_two_layers():
+    wl = synth.WORKLOADS["qwen"]
+    dims = synth.reduced(wl.dims, n_layers=2)
+    print(_run_full(wl, dims, 3000, samples=[0, 5]))
+
+
+def test_video_full_shapes_two_layers():
+    wl = synth.WORKLOADS["video"]
+    dims = synth.reduced(wl.dims, n_layers=2)
+    print(_run_full(wl, dims, 4000, samples=[0, 1], budget=0.25))
+
+
+def test_mixed_full_batch_two_layers():
+    wl = synth.WORKLOADS["mixed"]
+    dims = synth.reduced(wl.dims, n_layers=2)
+    print(_run_full(wl, dims, 5000, samples=[0, 31, 63]))
