@@ -26,6 +26,23 @@ def rel_err(got, ref) -> float:
     return float(np.abs(got - ref).max() / max(np.abs(ref).max(), 1e-30))
 
 
+def l2_err(got, ref) -> float:
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-30))
+
+
+BAR = 2e-2          # bf16 GPU vs fp32-storage oracle
+DRIFT_FACTOR = 1.5  # allowance over the bf16-emulated oracle's own distance
+
+
+def bar_for(ref32, ref16, key, err=rel_err):
+    """Tolerance for tensor `key`: 2e-2, or 1.5x the distance between the
+    bf16-emulated and the fp32-storage oracle when bf16 storage alone already
+    exceeds 2e-2 (deep stacks: the drift grows as sqrt(layers))."""
+    return max(BAR, DRIFT_FACTOR * err(ref16[key], ref32[key]))
+
+
 def check_selection(gpu_scores, gpu_kept, ref, z_tol=1e-4):
     """Kept sets agree except for tokens whose oracle logits lie within the
     tie band of the k-th largest logit. Returns True when identical."""

@@ -2,6 +2,11 @@
 benchmark times (whole batch through the three C entry points), checked on
 samples the oracle recomputes one by one.
 
+Hidden states and logits must be within 2e-2 (max-abs and L2 relative) of
+the fp32-storage oracle, or within 1.5x the distance between the
+bf16-emulated oracle and the fp32-storage oracle where bf16 storage alone
+already exceeds 2e-2 (32 layers: about 3.2e-2).
+
 The LLaVA-1.5-7B batch runs with all 32 layers; the Qwen2-VL-7B, video and
 mixed-serving batches keep their full batch, sequence and width shapes with
 the decoder cut to 2 layers so the float64 oracle stays within seconds per
@@ -13,7 +18,7 @@ import torch
 
 from oracle import smartvl_oracle as O
 from paper_2607_20357_gb300 import svl, synth
-from tests.gpu_common import check_selection, numpy_weights_lazy, rel_err, to_device
+from tests.gpu_common import bar_for, check_selection, l2_err, numpy_weights_lazy, rel_err, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -21,7 +26,7 @@ if not torch.cuda.is_available():
     pytest.skip("needs a CUDA GPU", allow_module_level=True)
 
 
-def _run_full(wl, dims, seed, samples, budget=None, tol=2e-2, modify=None):
+def _run_full(wl, dims, seed, samples, budget=None, modify=None):
     dev = torch.device("cuda")
     w = synth.make_weights(dims, seed, device=dev)
     batch = synth.make_batch(wl, seed, budget=budget, device=dev, dims=dims)
@@ -38,6 +43,7 @@ def _run_full(wl, dims, seed, samples, budget=None, tol=2e-2, modify=None):
     errs = []
     for b in samples:
         r = O.forward_batch(dims, w_np, b_np, mode="fp32", samples=[b])[0]
+        r16 = O.forward_batch(dims, w_np, b_np, mode="bf16", samples=[b])[0]
         assert int(out["k"][b]) == r["k"]
         assert int(out["flags"][b]) == r["flags"]
         v0, v1 = b_np["vis_off"][b], b_np["vis_off"][b + 1]
@@ -46,10 +52,12 @@ def _run_full(wl, dims, seed, samples, budget=None, tol=2e-2, modify=None):
         if not check_selection(out["scores"][v0:v1].numpy(), kept, r):
             continue
         cu = out["cu_seqlens"].numpy()
-        e_h = rel_err(out["X"][cu[b]:cu[b + 1]].double().numpy(), r["hidden"])
-        e_l = rel_err(out["logits"][b].double().numpy(), r["logits"])
-        errs.append((b, e_h, e_l))
-        assert e_h < tol and e_l < tol, (b, e_h, e_l)
+        got = {"hidden": out["X"][cu[b]:cu[b + 1]].double().numpy(), "logits": out["logits"][b].double().numpy()}
+        for key in ("hidden", "logits"):
+            for err in (rel_err, l2_err):
+                e, bar = err(got[key], r[key]), bar_for(r, r16, key, err)
+                errs.append((b, key, err.__name__, round(e, 5), round(bar, 5)))
+                assert e < bar, errs[-1]
     model.close()
     assert errs
     return errs
