@@ -91,23 +91,15 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __syncthreads();
   const int nseg = s_nseg;
   const int hq = (a.A / G) * a.dh, hk = (a.Akv / G) * a.dh;
-  // Rows of the layer in 128-row tiles; with fewer than four waves of
-  // 256-column tiles, halve the column width so the last wave is not mostly
-  // idle (tiles still hold whole heads: d_head divides 128).
-  int m_tiles = 0;
-  for (int s = 0; s < nseg; ++s) m_tiles += (seg[s].y - seg[s].x + kBM_SCHED - 1) / kBM_SCHED;
-  const int waves4 = 4 * max(a.num_sms, 1);
 
   // ---- QKV (N-sparse over active groups' Q, K, V columns)
   int off = 0;
-  const int n_on_max = __popc(nseg ? seg[0].z : 0);  // estimate from the first segment
-  const int qkv_step = (m_tiles * ((n_on_max * (hq + 2 * hk) + 255) / 256) < waves4) ? 128 : 256;
   for (int s = 0; s < nseg; ++s) {
     const int4 sg = seg[s];
     if (tid == 0) {
-      int c = build_runs(nt, 0, sg.z, G, hq, qkv_step, 0);
-      c = build_runs(nt, c, sg.z, G, hk, qkv_step, 1);
-      c = build_runs(nt, c, sg.z, G, hk, qkv_step, 2);
+      int c = build_runs(nt, 0, sg.z, G, hq, 256, 0);
+      c = build_runs(nt, c, sg.z, G, hk, 256, 1);
+      c = build_runs(nt, c, sg.z, G, hk, 256, 2);
       s_nnt = c;
     }
     __syncthreads();
@@ -119,8 +111,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
 
   // ---- O projection (K-sparse: kmask = segment mask), all D columns
   off = 0;
-  const int od_step = (m_tiles * ((a.D + 255) / 256) < waves4) ? 128 : 256;
-  if (tid == 0) s_nnt = build_runs(nt, 0, 1, 1, a.D, od_step, 0);
+  if (tid == 0) s_nnt = build_runs(nt, 0, 1, 1, a.D, 256, 0);
   __syncthreads();
   for (int s = 0; s < nseg; ++s) {
     const int4 sg = seg[s];

@@ -58,7 +58,6 @@ void launch_pack_gather(const PackArgs& a, cudaStream_t s);
 // ---------------------------------------------------------------- decoder
 struct ScheduleArgs {
   int B, L, G, P;
-  int num_sms;              // tiles per wave of the persistent GEMM
   int A, Akv, dh, D, Di;
   const int* cu_seqlens;
   const uint8_t* layer_gate;
