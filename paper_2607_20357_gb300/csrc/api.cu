@@ -121,8 +121,9 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   L.n_pad = ((B + 15) / 16) * 16;
   L.mt_max = static_cast<int>(t_cap / 128 + B + 1);
   const int qkv_nt = static_cast<int>((hq / 256 + G + 1) + 2 * (dkv / 256 + G + 1));
-  L.qkv_cap = L.mt_max * qkv_nt;
-  L.o_cap = L.mt_max * ((d.d_model + 255) / 256);
+  // + 256: room for the split tail (at most half a wave of extra tiles)
+  L.qkv_cap = L.mt_max * qkv_nt + 256;
+  L.o_cap = L.mt_max * ((d.d_model + 255) / 256) + 256;
   L.dn_cap = L.o_cap;
   L.gu_cap = L.mt_max * (d.d_ffn / 128 + G + 1);
   L.attn_cap = static_cast<int>(d.n_heads * (t_cap / kAttnQ + B + 1));
@@ -532,6 +533,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   sa.L = nl;
   sa.G = d.n_groups;
   sa.P = d.n_prefix;
+  sa.num_sms = m->num_sms;
   sa.A = d.n_heads;
   sa.Akv = d.n_kv_heads;
   sa.dh = dh;

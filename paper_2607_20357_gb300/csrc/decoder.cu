@@ -59,6 +59,27 @@ __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const
   }
 }
 
+// The persistent GEMM runs tiles in waves of num_sms. When the last wave is
+// at most half full, each of its tiles is cut into two half-width tiles
+// (which then still fit in one wave and finish in about half the time).
+// `head` > 0: halves must hold whole heads of that width (RoPE epilogue).
+// Runs on one thread after the list is complete; returns the new count.
+__device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head) {
+  const int r = count % num_sms;
+  if (r == 0 || 2 * r > num_sms) return count;
+  int added = 0;
+  for (int i = count - r; i < count; ++i) {
+    const int4 t = tiles[i];
+    const int nc = t.w & 0xFFFF;
+    const int half = nc / 2;
+    if (nc < 64 || (half & 15) || (head > 0 && half % head) || count + added >= cap) continue;
+    tiles[i] = make_int4(t.x, t.y, t.z, (t.w & ~0xFFFF) | half);
+    tiles[count + added] = make_int4(t.x, t.y, t.z + half, (t.w & ~0xFFFF) | (nc - half));
+    ++added;
+  }
+  return count + added;
+}
+
 __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __shared__ NTile nt[kMaxNT];
   __shared__ int s_nseg, s_nnt;
@@ -107,7 +128,10 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
     __syncthreads();
   }
-  if (tid == 0) a.qkv_count[l] = min(off, a.qkv_cap);
+  __syncthreads();
+  if (tid == 0)
+    a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, min(off, a.qkv_cap), a.qkv_cap,
+                                a.num_sms, a.dh);
 
   // ---- O projection (K-sparse: kmask = segment mask), all D columns
   off = 0;
@@ -118,7 +142,9 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     emit_tiles(a.o_tiles + static_cast<size_t>(l) * a.o_cap, off, a.o_cap, sg.x, sg.y, nt, s_nnt, sg.z, a.status);
     off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
   }
-  if (tid == 0) a.o_count[l] = min(off, a.o_cap);
+  __syncthreads();
+  if (tid == 0)
+    a.o_count[l] = split_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms, 0);
   // ---- down projection: same tiles shape as O
   off = 0;
   for (int s = 0; s < nseg; ++s) {
@@ -126,7 +152,10 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     emit_tiles(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, off, a.dn_cap, sg.x, sg.y, nt, s_nnt, sg.z, a.status);
     off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
   }
-  if (tid == 0) a.dn_count[l] = min(off, a.dn_cap);
+  __syncthreads();
+  if (tid == 0)
+    a.dn_count[l] = split_tail(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, min(off, a.dn_cap), a.dn_cap,
+                               a.num_sms, 0);
   __syncthreads();
 
   // ---- gate/up (N-sparse over active FFN channels, 128 per tile)

@@ -213,17 +213,38 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
   } else if constexpr (KIND == EPI_RESID) {
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
     const size_t ld = static_cast<size_t>(p.ld[0]);
+    __nv_bfloat16* orow = out + static_cast<size_t>(row) * ld + ti.n0;
+    // residual chunks double-buffered in registers: the load of chunk c+32
+    // is in flight while chunk c is added and stored
+    uint4 xa[4], xb[4];
+    if (rv) {
+      const uint4* s0 = reinterpret_cast<const uint4*>(orow);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) xa[i] = (i * 8 < ti.ncols) ? s0[i] : make_uint4(0, 0, 0, 0);
+    }
     for (int c = 0; c < ti.ncols; c += 32) {
+      const int n = min(32, ti.ncols - c);
+      if (rv && c + 32 < ti.ncols) {
+        const uint4* s1 = reinterpret_cast<const uint4*>(orow + c + 32);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) xb[i] = (c + 32 + i * 8 < ti.ncols) ? s1[i] : make_uint4(0, 0, 0, 0);
+      }
       tmem_ld32(taddr + c, v);
       if (rv) {
-        const int n = min(32, ti.ncols - c);
-        __nv_bfloat16* o = out + static_cast<size_t>(row) * ld + ti.n0 + c;
-        float x[32];
-        load_bf16(o, x, n);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] += x[j];
-        store_bf16(o, v, n);
+        for (int i = 0; i < 4; ++i) {
+          const uint32_t w[4] = {xa[i].x, xa[i].y, xa[i].z, xa[i].w};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float2 f = unpack_bf16x2(w[q]);
+            v[8 * i + 2 * q] += f.x;
+            v[8 * i + 2 * q + 1] += f.y;
+          }
+        }
+        store_bf16(orow + c, v, n);
       }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) xa[i] = xb[i];
     }
   } else if constexpr (KIND == EPI_SWIGLU) {
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
@@ -314,6 +335,16 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
     if (!ti.valid) continue;
     const int acc = it & 1;
     const uint32_t aph = (it >> 1) & 1;
+    if constexpr (KIND == EPI_RESID) {
+      // pull this row's residual segment toward L2 while the main loop runs
+      const int prow = ti.m0 + q * 32 + lane;
+      if (prow < ti.m_end) {
+        const char* base = reinterpret_cast<const char*>(
+            reinterpret_cast<const __nv_bfloat16*>(p.out[0]) + static_cast<size_t>(prow) * p.ld[0] + ti.n0);
+        for (int off = 0; off < ti.ncols * 2; off += 128)
+          asm volatile("prefetch.global.L2 [%0];" ::"l"(base + off));
+      }
+    }
     const bool ok = mbar_wait(&tfull[acc], aph, abort);
     __syncwarp();
     if (!__all_sync(0xffffffffu, ok)) {

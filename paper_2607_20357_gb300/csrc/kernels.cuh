@@ -58,6 +58,7 @@ void launch_pack_gather(const PackArgs& a, cudaStream_t s);
 // ---------------------------------------------------------------- decoder
 struct ScheduleArgs {
   int B, L, G, P;
+  int num_sms;              // CTAs of the persistent GEMM (one wave of tiles)
   int A, Akv, dh, D, Di;
   const int* cu_seqlens;
   const uint8_t* layer_gate;
