@@ -50,12 +50,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 2-D bf16 tensor map, K-major rows of `cols` elements, boxes of 64 x 128
 // with 128-byte swizzle (the layout the tcgen05 descriptors expect).
-bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols) {
+bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows = 128) {
   auto fn = encode_fn();
-  if (!fn || !ptr || rows == 0 || cols == 0 || (reinterpret_cast<uintptr_t>(ptr) & 15)) return false;
+  if (!fn || !ptr || rows == 0 || cols == 0 || (reinterpret_cast<uintptr_t>(ptr) & 15) || ((cols * 2) & 15))
+    return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), 128};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK), box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -75,7 +76,7 @@ struct PackLayout {
   size_t scalars, stage, hp, row_map, total;
 };
 struct PreLayout {
-  int64_t t_cap;
+  int64_t t_cap, t_pad;
   int n_pad, mt_max, qkv_cap, o_cap, gu_cap, dn_cap, attn_cap;
   size_t xn, q, k, v, ao, hmid, yl, act, seg, qkv, o, gu, dn, attn, counts, total;
 };
@@ -118,6 +119,7 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   const int64_t hq = static_cast<int64_t>(d.n_heads) * dh;
   const int G = d.n_groups;
   L.t_cap = t_cap;
+  L.t_pad = (t_cap + 7) & ~int64_t(7);
   L.n_pad = ((B + 15) / 16) * 16;
   L.mt_max = static_cast<int>(t_cap / 128 + B + 1);
   const int qkv_nt = static_cast<int>((hq / 256 + G + 1) + 2 * (dkv / 256 + G + 1));
@@ -131,7 +133,7 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   L.xn = b.take(2 * t_cap * d.d_model);
   L.q = b.take(2 * t_cap * hq);
   L.k = b.take(2 * t_cap * dkv);
-  L.v = b.take(2 * t_cap * dkv);
+  L.v = b.take(2 * L.t_pad * dkv);  // V^T [dkv, t_pad]
   L.ao = b.take(2 * t_cap * hq);
   L.hmid = b.take(2 * t_cap * d.d_ffn);
   L.yl = b.take(2 * static_cast<size_t>(L.n_pad) * d.d_model);
@@ -585,16 +587,23 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   na.Y = xn;
   na.cu_seqlens = cu_seqlens;
 
-  AttnArgs aa;
-  aa.Q = qb;
-  aa.K = kb;
-  aa.V = vb;
-  aa.O = ao;
+  // V^T is read in 128-key tiles that may run past the rows written in this
+  // call; zero it once so those (masked) keys hold finite values
+  if (cudaMemsetAsync(vb, 0, sizeof(__nv_bfloat16) * static_cast<size_t>(L.t_pad) * dkv, s) != cudaSuccess)
+    return SVL_ERR_CUDA;
+  AttnTcArgs aa;
+  std::memset(&aa, 0, sizeof(aa));
+  if (!make_map(&aa.mapQ, qb, t_cap, hq) || !make_map(&aa.mapK, kb, t_cap, dkv) ||
+      !make_map(&aa.mapVt, vb, dkv, L.t_pad, static_cast<uint32_t>(dh)))
+    return SVL_ERR_CUDA;
   aa.cap = L.attn_cap;
   aa.A = d.n_heads;
   aa.Akv = d.n_kv_heads;
   aa.dh = dh;
   aa.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(dh)));
+  aa.O = ao;
+  aa.ldo = hq;
+  aa.status = m->d_status;
 
   for (int l = 0; l < nl; ++l) {
     const svl_layer_weights& lw = m->layers[l];
@@ -621,7 +630,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.out[2] = vb;
     p.ld[0] = hq;
     p.ld[1] = dkv;
-    p.ld[2] = dkv;
+    p.ld[2] = static_cast<int>(L.t_pad);
     p.pos = pos;
     p.rope_cs = m->rope_cs;
     p.rope_rows = d.max_seq;
@@ -632,7 +641,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     aa.count = counts + 4 * nl + l;
     {
       Launch L1(m, SVL_TAG_ATTENTION, s);
-      launch_attention(aa, s);
+      if (launch_attention_tc(aa, gemm_grid(m, L.attn_cap), s) != cudaSuccess) return SVL_ERR_CUDA;
     }
 
     p = base_params(m);

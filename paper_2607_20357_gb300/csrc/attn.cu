@@ -1,232 +1,332 @@
-// Variable-length causal attention over active heads only (Sec. 3.2: a gated
-// group's heads are never computed). One CTA per work item (sample, head,
-// block of 64 queries); keys run from the sample's first row up to the last
-// query of the block. GQA: query head h reads KV head h / (A / A_kv).
+// Variable-length causal attention over active heads only (Sec. 3.2: the
+// heads of a gated-off group are never computed), on tcgen05 tensor cores.
 //
-// Online softmax (running max and sum per row, output rescaled per key tile)
-// with bf16 m16n8k16 tensor-core MMAs; K/V tiles of 64 keys are double
-// buffered with cp.async; shared-memory rows are XOR-swizzled in 16-byte
-// chunks so that ldmatrix is conflict-free.
+// Persistent kernel, one CTA per SM, work items (sample, active head, block
+// of 128 queries) from the device schedule. Per item and per tile of 128 keys:
+//   S = Q K^T          tcgen05.mma M=128 N=128 K=d_head, into one of two TMEM
+//                      S buffers (S(j+1) is computed while row j's softmax runs)
+//   softmax            four warps, one query row per thread: running max and
+//                      sum, P = exp2(S*scale - max) rounded to bf16 and written
+//                      to shared memory in the 128-byte-swizzled K-major layout
+//   O_tile = P V       tcgen05.mma M=128 N=d_head K=128 into a TMEM buffer;
+//                      the thread folds it into its fp32 output row in
+//                      registers: O = O*exp2(m_old - m_new) + O_tile
+// V arrives transposed (V^T, keys contiguous) so that both MMA operands are
+// K-major. Key tiles start at the sample's first row rounded down to a
+// multiple of 8 (TMA needs a 16-byte aligned innermost coordinate); keys of
+// the neighbouring sample that this pulls in are masked, like every key after
+// the query (causal) or past the block's last query.
+//
+// Warp 0: TMA producer (Q once per item, K and V^T double buffered).
+// Warp 1: TMEM allocation and the MMA-issuing thread.
+// Warps 2-5: softmax and output. Every wait is bounded.
 #include "kernels.cuh"
 
 namespace svl {
 
-constexpr int kAttnThreads = 128;  // 4 warps x 16 query rows
-constexpr int kKT = 64;            // keys per tile
-
-SVL_DEVINL void cp_async16(uint32_t dst, const void* src, bool valid) {
-  const int n = valid ? 16 : 0;
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n) : "memory");
-}
-SVL_DEVINL void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-SVL_DEVINL void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-SVL_DEVINL void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-SVL_DEVINL void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-SVL_DEVINL void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
-// Byte offset of (row, 16-byte chunk) in a tile with DH bf16 per row.
-template <int DH>
-SVL_DEVINL uint32_t swz(int row, int chunk) {
-  return static_cast<uint32_t>(row * DH * 2 + ((chunk ^ (row & 7)) << 4));
-}
-
-// Loads `rows` rows (row0.. of a [*, ld] bf16 matrix, column offset col0) into
-// a 64 x DH tile; rows at or beyond `row_end` are zero-filled.
-template <int DH>
-SVL_DEVINL void load_tile(uint32_t sbase, const __nv_bfloat16* g, size_t ld, int row0, int row_end, int col0) {
-  constexpr int CH = DH / 8;  // 16-byte chunks per row
-  for (int i = threadIdx.x; i < 64 * CH; i += kAttnThreads) {
-    const int r = i / CH, c = i % CH;
-    const int gr = row0 + r;
-    const bool ok = gr < row_end;
-    const __nv_bfloat16* src = g + static_cast<size_t>(ok ? gr : row0) * ld + col0 + c * 8;
-    cp_async16(sbase + swz<DH>(r, c), src, ok);
-  }
-}
+constexpr int kAttnThreads = 192;
+constexpr int kKeyTile = 128;
 
 template <int DH>
-__global__ void __launch_bounds__(kAttnThreads) attn_kernel(AttnArgs a) {
-  extern __shared__ __align__(128) uint8_t smem[];
-  const int n_items = min(*a.count, a.cap);
-  if (static_cast<int>(blockIdx.x) >= n_items) return;
-  const int4 it = a.items[blockIdx.x];
-  const int q0 = it.x, q_end = it.y, r0 = it.z, h = it.w;
-  const int kvh = h / (a.A / a.Akv);
-  const size_t ldq = static_cast<size_t>(a.A) * DH, ldk = static_cast<size_t>(a.Akv) * DH;
-  constexpr int TILE = 64 * DH * 2;
-  const uint32_t sQ = smem_u32(smem);
-  const uint32_t sK0 = sQ + TILE, sV0 = sQ + 3 * TILE;  // K: 2 buffers, V: 2 buffers, TILE apart
+struct AttnSmem {
+  static constexpr int kQ = 128 * DH * 2;          // Q: DH/64 atoms of 128 rows x 128 B
+  static constexpr int kK = kKeyTile * DH * 2;     // K stage
+  static constexpr int kV = DH * kKeyTile * 2;     // V^T stage: 2 atoms of DH rows x 128 B
+  static constexpr int kP = 128 * kKeyTile * 2;    // P buffer: 2 atoms of 128 rows x 128 B
+  static constexpr int q = 0;
+  static constexpr int k0 = kQ;
+  static constexpr int v0 = k0 + 2 * kK;
+  static constexpr int p0 = v0 + 2 * kV;
+  static constexpr int bars = p0 + 2 * kP;
+  static constexpr int total = bars + 256 + 1024;  // + barriers + alignment slack
+};
+
+struct AttnBars {
+  uint64_t q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], p_full, o_full[2];
+};
+
+SVL_DEVINL void attn_abort(volatile int* abort, uint32_t* status) {
+  *abort = 1;
+  report(status, SVL_DEV_TIMEOUT);
+}
+
+SVL_DEVINL int n_key_tiles(const int4& it) {
+  const int key_base = it.z & ~7;
+  return (it.y - key_base + kKeyTile - 1) / kKeyTile;
+}
+
+SVL_DEVINL float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// TMEM columns: S buffers 0 and 128, P V buffers 256 and 384.
+template <int DH>
+__global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_constant__ AttnTcArgs a) {
+  using L = AttnSmem<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  AttnBars* bar = reinterpret_cast<AttnBars*>(sm + L::bars);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 1);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int kv_end = q_end;
-  const int n_tiles = (kv_end - r0 + kKT - 1) / kKT;
+  const int n_items = min(*a.count, a.cap);
 
-  load_tile<DH>(sQ, a.Q, ldq, q0, q_end, h * DH);
-  load_tile<DH>(sK0, a.K, ldk, r0, kv_end, kvh * DH);
-  load_tile<DH>(sV0, a.V, ldk, r0, kv_end, kvh * DH);
-  cp_async_commit();
-
-  // Q fragments of this warp's 16 rows
-  uint32_t qf[DH / 16][4];
-  float o[DH / 8][4];
-#pragma unroll
-  for (int i = 0; i < DH / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  float m_run[2] = {-INFINITY, -INFINITY}, l_run[2] = {0.f, 0.f};
-  const int g = lane >> 2, tq = lane & 3;
-  const int qrow0 = q0 + warp * 16 + g;  // global query rows g and g + 8
-
-  for (int j = 0; j < n_tiles; ++j) {
-    const int buf = j & 1;
-    if (j + 1 < n_tiles) {
-      const int nb = buf ^ 1;
-      load_tile<DH>(sK0 + nb * TILE, a.K, ldk, r0 + (j + 1) * kKT, kv_end, kvh * DH);
-      load_tile<DH>(sV0 + nb * TILE, a.V, ldk, r0 + (j + 1) * kKT, kv_end, kvh * DH);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
+  if (threadIdx.x == 0) {
+    mbar_init(&bar->q_full, 1);
+    mbar_init(&bar->q_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bar->k_full[i], 1);
+      mbar_init(&bar->k_empty[i], 1);
+      mbar_init(&bar->v_full[i], 1);
+      mbar_init(&bar->v_empty[i], 1);
+      mbar_init(&bar->s_full[i], 1);
+      mbar_init(&bar->o_full[i], 1);
     }
-    __syncthreads();
-    if (j == 0) {
+    mbar_init(&bar->p_full, 128);
+    *abort = 0;
+    fence_barrier_init();
+    fence_proxy_async();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int g = 0, li = 0;
+      bool ok = true;
+      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x, ++li) {
+        const int4 it = a.items[i];
+        const int h = it.w, kvh = h / (a.A / a.Akv), key_base = it.z & ~7, nt = n_key_tiles(it);
+        if (!mbar_wait(&bar->q_empty, (li & 1) ^ 1, abort)) { ok = false; break; }
+        mbar_arrive_expect_tx(&bar->q_full, L::kQ);
+        for (int at = 0; at < DH / 64; ++at)
+          tma_load_2d(sm + L::q + at * 128 * 128, &a.mapQ, &bar->q_full, h * DH + at * 64, it.x);
+        for (int j = 0; j < nt; ++j, ++g) {
+          const int s = g & 1;
+          const uint32_t ph = ((g >> 1) & 1) ^ 1;
+          const int key0 = key_base + j * kKeyTile;
+          if (!mbar_wait(&bar->k_empty[s], ph, abort)) { ok = false; break; }
+          mbar_arrive_expect_tx(&bar->k_full[s], L::kK);
+          for (int at = 0; at < DH / 64; ++at)
+            tma_load_2d(sm + L::k0 + s * L::kK + at * kKeyTile * 128, &a.mapK, &bar->k_full[s], kvh * DH + at * 64,
+                        key0);
+          if (!mbar_wait(&bar->v_empty[s], ph, abort)) { ok = false; break; }
+          mbar_arrive_expect_tx(&bar->v_full[s], L::kV);
+          for (int at = 0; at < 2; ++at)
+            tma_load_2d(sm + L::v0 + s * L::kV + at * DH * 128, &a.mapVt, &bar->v_full[s], key0 + at * 64, kvh * DH);
+        }
+      }
+      if (!ok) attn_abort(abort, a.status);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16_f32(128, kKeyTile), id_o = idesc_bf16_f32(128, DH);
+      const uint32_t sq = smem_u32(sm + L::q);
+      int g = 0, li = 0;
+      bool ok = true;
+      // S(gg) = Q K(gg)^T into S buffer gg&1; frees the K stage when done
+      auto issue_s = [&](int gg, bool last_of_item) -> bool {
+        const int s = gg & 1;
+        if (!mbar_wait(&bar->k_full[s], (gg >> 1) & 1, abort)) return false;
+        tc_fence_after();
+        const uint32_t sk = smem_u32(sm + L::k0 + s * L::kK);
 #pragma unroll
-      for (int kk = 0; kk < DH / 16; ++kk) {
-        const int row = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-        const int chunk = kk * 2 + (lane >> 4);
-        ldsm_x4(sQ + swz<DH>(row, chunk), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * (128 * 128) + (kk & 3) * 32;
+          const uint32_t offk = (kk >> 2) * (kKeyTile * 128) + (kk & 3) * 32;
+          tc_mma_bf16(tmem + s * 128, smem_desc_sw128(sq + off), smem_desc_sw128(sk + offk), id_s, kk > 0);
+        }
+        tc_commit(&bar->s_full[s]);
+        tc_commit(&bar->k_empty[s]);
+        if (last_of_item) tc_commit(&bar->q_empty);  // Q may be replaced once these finish
+        return true;
+      };
+      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x, ++li) {
+        const int nt = n_key_tiles(a.items[i]);
+        if (!mbar_wait(&bar->q_full, li & 1, abort)) { ok = false; break; }
+        tc_fence_after();
+        ok = issue_s(g, nt == 1) && (nt < 2 || issue_s(g + 1, nt == 2));
+        for (int j = 0; j < nt && ok; ++j) {
+          const int gj = g + j, s = gj & 1;
+          if (!mbar_wait(&bar->p_full, gj & 1, abort) || !mbar_wait(&bar->v_full[s], (gj >> 1) & 1, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sp = smem_u32(sm + L::p0 + s * L::kP);
+          const uint32_t sv = smem_u32(sm + L::v0 + s * L::kV);
+#pragma unroll
+          for (int kk = 0; kk < kKeyTile / 16; ++kk) {
+            const uint32_t offp = (kk >> 2) * (128 * 128) + (kk & 3) * 32;
+            const uint32_t offv = (kk >> 2) * (DH * 128) + (kk & 3) * 32;
+            tc_mma_bf16(tmem + 256 + s * 128, smem_desc_sw128(sp + offp), smem_desc_sw128(sv + offv), id_o, kk > 0);
+          }
+          tc_commit(&bar->o_full[s]);
+          tc_commit(&bar->v_empty[s]);
+          if (j + 2 < nt) ok = issue_s(gj + 2, j + 2 == nt - 1);
+        }
+        g += nt;
+      }
+      if (!ok) attn_abort(abort, a.status);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax + output
+    const int q = warp & 3;
+    const int row = q * 32 + lane;  // query row within the block = TMEM lane
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const float sc = a.scale_log2;
+    int g = 0;
+    bool ok = true;
+    for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
+      const int4 it = a.items[i];
+      const int qg = it.x + row;  // global query row
+      const int key_base = it.z & ~7, nt = n_key_tiles(it);
+      float o[DH];
+#pragma unroll
+      for (int d = 0; d < DH; ++d) o[d] = 0.f;
+      float m_run = -INFINITY, l_run = 0.f;
+      float cr0 = 0.f, cr1 = 0.f;  // correction factors of the (even, odd) tiles whose P V is pending
+
+      // O = O * corr(t) + (P V)(t), once the MMA for tile t has finished
+      auto fold = [&](int t) -> bool {
+        const int s = t & 1;
+        const bool got = mbar_wait(&bar->o_full[s], (t >> 1) & 1, abort);
+        __syncwarp();
+        if (!__all_sync(0xffffffffu, got)) return false;
+        tc_fence_after();
+        const float c = ((t - g) & 1) ? cr1 : cr0;
+        float v[32];
+#pragma unroll
+        for (int cc = 0; cc < DH; cc += 32) {
+          tmem_ld32(tmem + 256 + s * 128 + lane_off + cc, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[cc + e] = fmaf(o[cc + e], c, v[e]);
+        }
+        tc_fence_before();
+        return true;
+      };
+
+      for (int j = 0; j < nt; ++j) {
+        const int gj = g + j, s = gj & 1;
+        if (j >= 2 && !fold(gj - 2)) { ok = false; break; }
+        const bool got = mbar_wait(&bar->s_full[s], (gj >> 1) & 1, abort);
+        __syncwarp();
+        if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t ts = tmem + s * 128 + lane_off;
+        const int kbase = key_base + j * kKeyTile;
+        // keys kbase + [lo, hi) are valid for this row; a tile wholly inside
+        // the sample and before the block's first query needs no mask
+        const bool full = kbase >= it.z && kbase + kKeyTile - 1 <= it.x;
+        const int lo = full ? 0 : max(it.z - kbase, 0);
+        // (a row that precedes the whole tile has no valid key: empty range)
+        const int hi = full ? kKeyTile : max(min(min(qg + 1, it.y) - kbase, kKeyTile), lo);
+        float v[32];
+        float mx = -INFINITY;
+        for (int c = 0; c < kKeyTile; c += 32) {
+          tmem_ld32(ts + c, v);
+          if (full) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e) mx = fmaxf(mx, v[e]);
+          } else {
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              if (static_cast<unsigned>(c + e - lo) < static_cast<unsigned>(hi - lo)) mx = fmaxf(mx, v[e]);
+          }
+        }
+        const float m_new = fmaxf(m_run, mx * sc);
+        const float mref = (m_new == -INFINITY) ? 0.f : m_new;
+        const float corr = (m_run == -INFINITY) ? 0.f : ex2(m_run - mref);
+        m_run = m_new;
+        if (j & 1) cr1 = corr; else cr0 = corr;
+        uint8_t* prow = sm + L::p0 + s * L::kP + row * 128;
+        float rs = 0.f;
+        for (int c = 0; c < kKeyTile; c += 32) {
+          tmem_ld32(ts + c, v);
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 32; e += 2) {
+            float x0 = fmaf(v[e], sc, -mref), x1 = fmaf(v[e + 1], sc, -mref);
+            if (!full) {
+              if (static_cast<unsigned>(c + e - lo) >= static_cast<unsigned>(hi - lo)) x0 = -INFINITY;
+              if (static_cast<unsigned>(c + e + 1 - lo) >= static_cast<unsigned>(hi - lo)) x1 = -INFINITY;
+            }
+            const float p0 = ex2(x0), p1 = ex2(x1);
+            rs += p0 + p1;
+            pk[e >> 1] = pack_bf16x2(p0, p1);
+          }
+          // keys c..c+31: atom c/64, 16-byte chunks (c%64)/8 .. +3, 128-byte swizzle
+          const int atom = c >> 6, ch0 = (c & 63) >> 3;
+          uint8_t* base = prow + atom * (128 * 128);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int ch = (ch0 + u) ^ (row & 7);
+            *reinterpret_cast<uint4*>(base + (ch << 4)) =
+                make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+          }
+        }
+        l_run = l_run * corr + rs;
+        fence_proxy_async();  // P written by threads, read by the tensor core
+        tc_fence_before();
+        mbar_arrive(&bar->p_full);
+      }
+      if (ok && nt >= 2) ok = fold(g + nt - 2);
+      if (ok) ok = fold(g + nt - 1);
+      g += nt;
+      if (!ok) break;
+      if (qg < it.y) {
+        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+        uint4* dst = reinterpret_cast<uint4*>(a.O + static_cast<size_t>(qg) * a.ldo + static_cast<size_t>(it.w) * DH);
+#pragma unroll
+        for (int d = 0; d < DH; d += 8)
+          dst[d / 8] = make_uint4(pack_bf16x2(o[d] * inv, o[d + 1] * inv), pack_bf16x2(o[d + 2] * inv, o[d + 3] * inv),
+                                  pack_bf16x2(o[d + 4] * inv, o[d + 5] * inv), pack_bf16x2(o[d + 6] * inv, o[d + 7] * inv));
       }
     }
-    const uint32_t sK = sK0 + buf * TILE, sV = sV0 + buf * TILE;
-
-    // S = Q K^T for 64 keys: 8 n-blocks of 8 keys
-    float s[8][4];
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) s[nb][0] = s[nb][1] = s[nb][2] = s[nb][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < DH / 16; ++kk) {
-#pragma unroll
-      for (int nb2 = 0; nb2 < 4; ++nb2) {  // two n-blocks per ldmatrix.x4
-        const int key = nb2 * 16 + (lane & 7) + (lane >> 4) * 8;
-        const int chunk = kk * 2 + ((lane >> 3) & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(sK + swz<DH>(key, chunk), b0, b1, b2, b3);
-        mma16816(s[2 * nb2], qf[kk], b0, b1);
-        mma16816(s[2 * nb2 + 1], qf[kk], b2, b3);
-      }
-    }
-    // causal mask and scale (log2 domain)
-    const int key_base = r0 + j * kKT;
-    float mx[2] = {m_run[0], m_run[1]};
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = key_base + nb * 8 + tq * 2 + (e & 1);
-        const int qr = qrow0 + (e >> 1) * 8;
-        float v = s[nb][e] * a.scale_log2;
-        if (key > qr || key >= kv_end) v = -INFINITY;
-        s[nb][e] = v;
-        mx[e >> 1] = fmaxf(mx[e >> 1], v);
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
-    }
-    float corr[2], rs[2] = {0.f, 0.f};
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      corr[r] = (m_run[r] == -INFINITY) ? 0.f : exp2f(m_run[r] - mx[r]);
-      m_run[r] = mx[r];
-    }
-    const float mref0 = mx[0] == -INFINITY ? 0.f : mx[0];
-    const float mref1 = mx[1] == -INFINITY ? 0.f : mx[1];
-    uint32_t pf[4][4];  // P as A fragments: 4 k-steps of 16 keys
-#pragma unroll
-    for (int nb = 0; nb < 8; ++nb) {
-      const float p0 = exp2f(s[nb][0] - mref0), p1 = exp2f(s[nb][1] - mref0);
-      const float p2 = exp2f(s[nb][2] - mref1), p3 = exp2f(s[nb][3] - mref1);
-      rs[0] += p0 + p1;
-      rs[1] += p2 + p3;
-      pf[nb >> 1][(nb & 1) * 2 + 0] = pack_bf16x2(p0, p1);
-      pf[nb >> 1][(nb & 1) * 2 + 1] = pack_bf16x2(p2, p3);
-    }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 1);
-      rs[r] += __shfl_xor_sync(0xffffffffu, rs[r], 2);
-      l_run[r] = l_run[r] * corr[r] + rs[r];
-    }
-#pragma unroll
-    for (int i = 0; i < DH / 8; ++i) {
-      o[i][0] *= corr[0];
-      o[i][1] *= corr[0];
-      o[i][2] *= corr[1];
-      o[i][3] *= corr[1];
-    }
-    // O += P V: k = 64 keys (4 steps), n = DH dims (DH/8 blocks)
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-#pragma unroll
-      for (int nb2 = 0; nb2 < DH / 16; ++nb2) {
-        const int key = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-        const int chunk = nb2 * 2 + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(sV + swz<DH>(key, chunk), b0, b1, b2, b3);
-        mma16816(o[2 * nb2], pf[kk], b0, b1);
-        mma16816(o[2 * nb2 + 1], pf[kk], b2, b3);
-      }
-    }
-    __syncthreads();
+    if (!ok) attn_abort(abort, a.status);
   }
 
-  // normalise and store rows < q_end
-  const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;
-  const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
-  __nv_bfloat16* out = a.O + static_cast<size_t>(h) * DH;
-#pragma unroll
-  for (int nb = 0; nb < DH / 8; ++nb) {
-    const int col = nb * 8 + tq * 2;
-    if (qrow0 < q_end)
-      *reinterpret_cast<uint32_t*>(out + static_cast<size_t>(qrow0) * ldq + col) =
-          pack_bf16x2(o[nb][0] * inv0, o[nb][1] * inv0);
-    if (qrow0 + 8 < q_end)
-      *reinterpret_cast<uint32_t*>(out + static_cast<size_t>(qrow0 + 8) * ldq + col) =
-          pack_bf16x2(o[nb][2] * inv1, o[nb][3] * inv1);
+  __syncwarp();
+  if (*abort) {
+    long long t0 = clock64();
+    while (clock64() - t0 < 20000000LL) {
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
   }
 }
 
 template <int DH>
-static void launch_dh(const AttnArgs& a, cudaStream_t s) {
-  constexpr int smem = 5 * 64 * DH * 2;
+static cudaError_t launch_dh(const AttnTcArgs& a, int grid, cudaStream_t s) {
   static bool configured = false;
   if (!configured) {
-    cudaFuncSetAttribute(attn_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         AttnSmem<DH>::total);
+    if (e != cudaSuccess) return e;
     configured = true;
   }
-  if (a.cap > 0) attn_kernel<DH><<<a.cap, kAttnThreads, smem, s>>>(a);
+  attn_tc_kernel<DH><<<grid, kAttnThreads, AttnSmem<DH>::total, s>>>(a);
+  return cudaGetLastError();
 }
 
-void launch_attention(const AttnArgs& a, cudaStream_t s) {
-  if (a.dh == 128) launch_dh<128>(a, s);
-  else launch_dh<64>(a, s);
+cudaError_t launch_attention_tc(const AttnTcArgs& a, int grid, cudaStream_t s) {
+  if (a.cap <= 0) return cudaSuccess;
+  return a.dh == 128 ? launch_dh<128>(a, grid, s) : launch_dh<64>(a, grid, s);
 }
 
 }  // namespace svl

@@ -205,9 +205,15 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
         }
       }
     } else {
+      // V is stored transposed, V^T[column][row], so that attention reads
+      // keys contiguously (ld = padded row count)
       for (int c = 0; c < ti.ncols; c += 32) {
         tmem_ld32(taddr + c, v);
-        if (rv) store_bf16(out + static_cast<size_t>(row) * ld + ti.n0 + c, v, min(32, ti.ncols - c));
+        if (rv) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (c + j < ti.ncols) out[static_cast<size_t>(ti.n0 + c + j) * ld + row] = __float2bfloat16_rn(v[j]);
+        }
       }
     }
   } else if constexpr (KIND == EPI_RESID) {

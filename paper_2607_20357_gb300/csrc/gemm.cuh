@@ -23,7 +23,7 @@ constexpr int kTmemCols = 512;     // two accumulators (epilogue overlaps the ne
 constexpr int kGemmSmem = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 
 enum EpiKind : int {
-  EPI_QKV_ROPE = 0,  // mat 0/1: RoPE then bf16 store to Q/K; mat 2: bf16 store to V
+  EPI_QKV_ROPE = 0,  // mat 0/1: RoPE then bf16 store to Q/K; mat 2: bf16 store to V^T (transposed)
   EPI_RESID = 1,     // out[r, n] = bf16(out[r, n] + acc)
   EPI_SWIGLU = 2,    // out[r, n0 + c] = bf16(SiLU(acc[c]) * acc[128 + c])
   EPI_GELU = 3,      // out[r, n] = bf16(GELU(acc))

@@ -6,7 +6,7 @@
 namespace svl {
 
 constexpr int kSelectThreads = 512;
-constexpr int kAttnQ = 64;        // query rows per attention work item
+constexpr int kAttnQ = 128;       // query rows per attention work item
 constexpr int kNBand = 8;         // n-tiles per raster band in the tile lists
 constexpr int kBM_SCHED = 128;    // tile rows (the GEMM's M)
 
@@ -89,18 +89,20 @@ void launch_rmsnorm(const NormArgs& a, cudaStream_t s);
 // Final norm of each sample's last row into Y[b] (rows B..n_pad-1 zeroed).
 void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s);
 
-struct AttnArgs {
-  const __nv_bfloat16* Q;   // [T, A*dh]
-  const __nv_bfloat16* K;   // [T, Akv*dh]
-  const __nv_bfloat16* V;
-  __nv_bfloat16* O;         // [T, A*dh]
+struct AttnTcArgs {
+  CUtensorMap mapQ;         // Q   [T_cap, A*dh]      boxes 64 x 128
+  CUtensorMap mapK;         // K   [T_cap, A_kv*dh]   boxes 64 x 128
+  CUtensorMap mapVt;        // V^T [A_kv*dh, T_pad]   boxes 64 x dh
   const int4* items;        // {q0, q_end, r0, head}
   const int* count;
   int cap;
   int A, Akv, dh;
   float scale_log2;         // log2(e) / sqrt(dh)
+  __nv_bfloat16* O;         // [T_cap, A*dh]
+  int ldo;
+  uint32_t* status;
 };
-void launch_attention(const AttnArgs& a, cudaStream_t s);
+cudaError_t launch_attention_tc(const AttnTcArgs& a, int grid, cudaStream_t s);
 
 // RoPE table: cs[p * half + i] = (cos, sin)(p * theta^(-2i/dh)), double precision.
 void launch_rope_table(float2* cs, int max_seq, int dh, double theta, cudaStream_t s);
