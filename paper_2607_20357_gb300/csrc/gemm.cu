@@ -55,9 +55,26 @@ SVL_DEVINL TileInfo get_tile(const GemmParams& p, int t) {
   return ti;
 }
 
-SVL_DEVINL bool kblock_on(int kb, int kmask, int kgb) {
-  return kmask == 0 || ((kmask >> (kb / kgb)) & 1);
-}
+// Walks the K blocks of a tile, skipping the blocks of gated-off groups
+// (kmask bit j clear: K blocks [j*kgb, (j+1)*kgb) are not visited). The group
+// index is kept incrementally: no division in the issue loops.
+struct KWalk {
+  int kb, grp, kin;
+  const int nkb, kgb, kmask;
+  SVL_DEVINL KWalk(int nkb_, int kgb_, int kmask_) : kb(-1), grp(0), kin(-1), nkb(nkb_), kgb(kgb_), kmask(kmask_) {}
+  // advances to the next active K block; false when the tile is done
+  SVL_DEVINL bool next() {
+    while (true) {
+      ++kb;
+      if (kb >= nkb) return false;
+      if (++kin == kgb) {
+        kin = 0;
+        ++grp;
+      }
+      if (kmask == 0 || ((kmask >> grp) & 1)) return true;
+    }
+  }
+};
 
 SVL_DEVINL void set_abort(volatile int* abort, uint32_t* status) {
   *abort = 1;
@@ -79,8 +96,9 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
     const CUtensorMap* mb1 = p.b_split ? &p.mapB[1] : &p.mapB[ti.mat];
     const int y1 = p.b_split ? ti.n0 : ti.n0 + kBHalf;
     const uint32_t bytes = kABytes + halves * kBHalfBytes;
-    for (int kb = 0; kb < nkb; ++kb) {
-      if (!kblock_on(kb, ti.kmask, kgb)) continue;
+    KWalk w(nkb, kgb, ti.kmask);
+    while (w.next()) {
+      const int kb = w.kb;
       if (!mbar_wait(&empty[s], ph ^ 1, abort)) {
         set_abort(abort, p.status);
         return;
@@ -120,8 +138,8 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
     const uint32_t idesc = idesc_bf16_f32(kBM, n);
     const uint32_t d = tmem + acc * kAccCols;
     uint32_t accumulate = 0;
-    for (int kb = 0; kb < nkb; ++kb) {
-      if (!kblock_on(kb, ti.kmask, kgb)) continue;
+    KWalk w(nkb, kgb, ti.kmask);
+    while (w.next()) {
       if (!mbar_wait(&full[s], ph, abort)) {
         set_abort(abort, p.status);
         return;
