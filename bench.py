@@ -49,6 +49,7 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-hbm-sweep", action="store_true")
     ap.add_argument("--layers", type=int, default=0,
                     help="decoder layers (default: all 32). Fewer layers only for small profiler captures; "
                          "such a line is not the benchmark value")
@@ -282,6 +283,7 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
         t_wall = time.perf_counter() - t_wall0
     kern = svl.svl_profile_stop(model.handle)
+    per_launch = svl.svl_profile_launches(model.handle)
     launches = svl.svl_launch_count() - launches0
     if world > 1:
         torch.distributed.barrier()
@@ -310,6 +312,17 @@ def run_ours(args, rank, world, local_rank):
         fexec_total += fex * nsteps
         for kk, v in per_kind_flops(dims, k, st, lg.numpy(), gg.numpy()).items():
             kind_flops[kk] = kind_flops.get(kk, 0.0) + v * nsteps
+
+    # device time per tag and budget (every step launches the same kernels)
+    per_step = len(per_launch) // max(args.steps, 1)
+    for p in per_budget:
+        j = [q["budget"] for q in per_budget].index(p["budget"])
+        agg = {}
+        steps_j = list(range(j, args.steps, len(batches)))
+        for i in steps_j:
+            for tag, ms in per_launch[i * per_step:(i + 1) * per_step]:
+                agg[tag] = agg.get(tag, 0.0) + ms / len(steps_j)
+        p["kernel_ms"] = {t: round(v, 4) for t, v in sorted(agg.items(), key=lambda kv: -kv[1])}
 
     # linear-in-FLOPs check: t(b)/t(1) / (F(b)/F(1)) - 1
     full = [p for p in per_budget if abs(p["budget"] - 1.0) < 1e-6]
@@ -349,6 +362,10 @@ def run_ours(args, rank, world, local_rank):
         total_ms, tokens_total, fexec_total = float(mx[0]), float(tt[1]), float(tt[2])
     value = tokens_total / (total_ms / 1000.0)
 
+    hbm = None
+    if rank == 0 and not args.no_hbm_sweep:
+        hbm = run_hbm_sweep(svl, model, wl, dev, pk)
+
     # e2e through the host-buffer entry point: H2D of inputs, D2H of logits
     e2e = None
     if not args.no_e2e:
@@ -377,9 +394,53 @@ def run_ours(args, rank, world, local_rank):
             "per_budget": per_budget, "roofline": roofline, "kernels": kernels,
             "gpu_launches": int(launches), "gpu_launches_per_step": launches / args.steps,
             "wall_s_timed": t_wall, "clocks": clk.summary(), "e2e": e2e, "cpu_baseline": cpu,
+            "hbm_kernels_sweep": hbm,
         }
         print(json.dumps(line), flush=True)
     model.close()
+
+
+def run_hbm_sweep(svl, model, wl, dev, pk, reps=5):
+    """Token controller and pack alone at 1x, 4x and 16x the benchmark batch
+    (budget 0.5): achieved bandwidth of the HBM-bound kernels from their
+    algorithmic bytes and CUDA-event times."""
+    d = wl.dims
+    out = []
+    for mult in (1, 4, 16):
+        B = wl.batch * mult
+        bt = synth.make_batch(wl, SEED + 7 + mult, budget=0.5, batch=B, device=dev)
+        o = model.alloc_outputs(bt)
+        for _ in range(2):
+            model.run(bt, out=o, stages=("select", "pack"))
+        torch.cuda.synchronize()
+        svl.svl_profile_start(model.handle)
+        for _ in range(reps):
+            model.run(bt, out=o, stages=("select", "pack"))
+        kern = svl.svl_profile_stop(model.handle)
+        nv = int(bt["vis"].shape[0])
+        nt = int(bt["text_ids"].shape[0])
+        k = int(o["k"].sum())
+        rows = {
+            # visual features read + logits written
+            "score": (2 * nv * d.c_vis + 4 * nv, kern.get("score")),
+            # logits read + kept indices written
+            "select": (4 * nv + 4 * k + 4 * B, kern.get("select")),
+            # kept features gathered to the projector staging rows, text embedding rows copied
+            "pack": (2 * (2 * k * d.c_vis) + 2 * (2 * nt * d.d_model) + 4 * nt + 8 * (nv + nt), kern.get("pack")),
+        }
+        line = {"batch": B, "visual_tokens": nv, "kept": k}
+        for name, (nbytes, km) in rows.items():
+            if km is None:
+                continue
+            ms = km[1] / reps
+            gbs = nbytes / (ms / 1000.0) / 1e9
+            line[name] = {"ms": round(ms, 4), "bytes": nbytes, "gb_s": round(gbs, 1),
+                          "frac_of_measured_hbm": round(gbs / pk["hbm_gbs"], 3),
+                          "launches": km[0] // reps}
+        out.append(line)
+        del bt, o
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_e2e(args, svl, model, batches, dims, world, dev):

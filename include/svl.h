@@ -63,7 +63,7 @@ typedef enum svl_status {
  * Supported: D = A * d_head with d_head in {64, 128}; A % G == 0 and
  * A_kv % G == 0 (each group owns whole KV heads); (D_int / G) % 64 == 0;
  * (A / G) * d_head % 64 == 0; D, C_v, proj_hidden multiples of 64;
- * H in {16, 32, ..., 256}; proj_hidden == 0 requires C_v == D. */
+ * H in {16, 32, ..., 128}; proj_hidden == 0 requires C_v == D. */
 typedef struct svl_model_desc {
   int32_t n_layers;     /* L */
   int32_t d_model;      /* D */
@@ -264,6 +264,10 @@ typedef struct svl_kernel_time {
 
 svl_status svl_profile_start(svl_model* model);
 svl_status svl_profile_stop(svl_model* model, svl_kernel_time* out, int32_t cap, int32_t* n_out);
+/* The individual launches of the last profiling window (after
+ * svl_profile_stop), in launch order: tag and elapsed milliseconds of each.
+ * Writes at most `cap` entries and sets *n_out to the number written. */
+svl_status svl_profile_launches(svl_model* model, int32_t* tags, float* ms, int32_t cap, int32_t* n_out);
 const char* svl_tag_name(int32_t tag);
 
 /* Reads (and clears) the device status word; synchronises `stream`. */

@@ -29,6 +29,7 @@ struct svl_model {
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   std::vector<std::pair<int, size_t>> prof_recs;  // (tag, index of the first event of the pair)
+  std::vector<std::pair<int, float>> prof_last;   // per-launch times of the last window
 };
 
 namespace {
@@ -279,7 +280,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   if ((d.d_ffn / G) % 64 || d.d_ffn % G) return SVL_ERR_UNSUPPORTED;
   if (((d.n_heads / G) * dh) % 64) return SVL_ERR_UNSUPPORTED;
   if (d.d_model % 64 || d.c_vis % 64 || d.proj_hidden % 64) return SVL_ERR_UNSUPPORTED;
-  if (d.h_ctrl % 16 || d.h_ctrl > 256) return SVL_ERR_UNSUPPORTED;
+  if (d.h_ctrl % 16 || d.h_ctrl > 128) return SVL_ERR_UNSUPPORTED;
   if (d.proj_hidden == 0 && d.c_vis != d.d_model) return SVL_ERR_UNSUPPORTED;
   // Eq. 8 times G must stay exact in double precision at the longest sequence
   {
@@ -832,12 +833,14 @@ svl_status svl_profile_stop(svl_model* m, svl_kernel_time* out, int32_t cap, int
   m->prof = false;
   double tot[SVL_TAG_COUNT] = {0};
   int cnt[SVL_TAG_COUNT] = {0};
+  m->prof_last.clear();
   if (!m->prof_recs.empty()) {
     if (cudaEventSynchronize(m->ev_pool[m->prof_recs.back().second + 1]) != cudaSuccess) return SVL_ERR_CUDA;
   }
   for (const auto& r : m->prof_recs) {
     float ms = 0.f;
     if (cudaEventElapsedTime(&ms, m->ev_pool[r.second], m->ev_pool[r.second + 1]) != cudaSuccess) return SVL_ERR_CUDA;
+    m->prof_last.emplace_back(r.first, ms);
     if (r.first >= 0 && r.first < SVL_TAG_COUNT) {
       tot[r.first] += ms;
       cnt[r.first] += 1;
@@ -852,6 +855,17 @@ svl_status svl_profile_stop(svl_model* m, svl_kernel_time* out, int32_t cap, int
     ++n;
   }
   if (n_out) *n_out = std::min(n, cap);
+  return SVL_OK;
+}
+
+svl_status svl_profile_launches(svl_model* m, int32_t* tags, float* ms, int32_t cap, int32_t* n_out) {
+  if (!m || cap < 0 || (cap > 0 && (!tags || !ms))) return SVL_ERR_INVALID_ARG;
+  const int n = std::min<int>(cap, static_cast<int>(m->prof_last.size()));
+  for (int i = 0; i < n; ++i) {
+    tags[i] = m->prof_last[i].first;
+    ms[i] = m->prof_last[i].second;
+  }
+  if (n_out) *n_out = n;
   return SVL_OK;
 }
 

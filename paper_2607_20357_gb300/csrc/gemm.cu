@@ -81,7 +81,22 @@ SVL_DEVINL void set_abort(volatile int* abort, uint32_t* status) {
   report(status, SVL_DEV_TIMEOUT);
 }
 
+// Stage geometry per epilogue: the token-score GEMM (N = H <= 128) needs one
+// B box per stage, so its 32 KB stages fit six deep in the same shared memory
+// and keep more of the streamed features in flight.
+template <int KIND>
+struct StageCfg {
+  static constexpr int stages = kStages;
+  static constexpr int bytes = kStageBytes;
+};
+template <>
+struct StageCfg<EPI_SCORE> {
+  static constexpr int stages = 6;
+  static constexpr int bytes = kABytes + kBHalfBytes;
+};
+
 // ------------------------------------------------------------------ producer
+template <int NST, int SBYTES>
 SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* full,
                               uint64_t* empty, volatile int* abort) {
   const int ntiles = num_tiles(p);
@@ -103,13 +118,13 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
         set_abort(abort, p.status);
         return;
       }
-      uint8_t* sa = stages + s * kStageBytes;
+      uint8_t* sa = stages + s * SBYTES;
       uint8_t* sb = sa + kABytes;
       mbar_arrive_expect_tx(&full[s], bytes);
       tma_load_2d(sa, &p.mapA, &full[s], kb * kBK, ti.m0);
       tma_load_2d(sb, mb0, &full[s], kb * kBK, ti.n0);
       if (halves == 2) tma_load_2d(sb + kBHalfBytes, mb1, &full[s], kb * kBK, y1);
-      if (++s == kStages) {
+      if (++s == NST) {
         s = 0;
         ph ^= 1;
       }
@@ -118,6 +133,7 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
 }
 
 // ------------------------------------------------------------------ MMA issuer
+template <int NST, int SBYTES>
 SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, uint64_t* empty,
                          uint64_t* tfull, uint64_t* tempty, uint32_t tmem, volatile int* abort) {
   const int ntiles = num_tiles(p);
@@ -145,7 +161,7 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
         return;
       }
       tc_fence_after();
-      const uint32_t a0 = smem_u32(stages + s * kStageBytes);
+      const uint32_t a0 = smem_u32(stages + s * SBYTES);
       const uint32_t b0 = a0 + kABytes;
 #pragma unroll
       for (int k = 0; k < kBK / 16; ++k) {
@@ -154,7 +170,7 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
         accumulate = 1;
       }
       tc_commit(&empty[s]);
-      if (++s == kStages) {
+      if (++s == NST) {
         s = 0;
         ph ^= 1;
       }
@@ -321,15 +337,22 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
       }
     }
   } else if constexpr (KIND == EPI_SCORE) {
-    int b = 0;
-    if (rv) {
-      int lo = 0, hi = p.n_seg;  // find b with seg_off[b] <= row < seg_off[b+1]
+    // sample of this row: lane 0 searches for the warp's first row, then each
+    // lane walks forward (32 consecutive tokens span few samples)
+    const int lane = threadIdx.x & 31;
+    const int r_first = row - lane;
+    int b0 = 0;
+    if (lane == 0) {
+      int lo = 0, hi = p.n_seg;  // seg_off[lo] <= r_first < seg_off[lo + 1]
       while (hi - lo > 1) {
-        int mid = (lo + hi) >> 1;
-        if (p.seg_off[mid] <= row) lo = mid; else hi = mid;
+        const int mid = (lo + hi) >> 1;
+        if (p.seg_off[mid] <= r_first) lo = mid; else hi = mid;
       }
-      b = lo;
+      b0 = lo;
     }
+    int b = __shfl_sync(0xffffffffu, b0, 0);
+    if (rv)
+      while (b + 1 < p.n_seg && p.seg_off[b + 1] <= row) ++b;
     const int H = ti.ncols;
     const float* eb = p.e_b + static_cast<size_t>(b) * H;
     float z = 0.f;
@@ -389,19 +412,20 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
 // ------------------------------------------------------------------ kernel
 template <int KIND>
 __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
+  constexpr int NST = StageCfg<KIND>::stages, SBYTES = StageCfg<KIND>::bytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* stages = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(stages + kStages * kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(stages + NST * SBYTES);
   uint64_t* full = bars;
-  uint64_t* empty = bars + kStages;
-  uint64_t* tfull = bars + 2 * kStages;
-  uint64_t* tempty = bars + 2 * kStages + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kStages + 4);
+  uint64_t* empty = bars + NST;
+  uint64_t* tfull = bars + 2 * NST;
+  uint64_t* tempty = bars + 2 * NST + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * NST + 4);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kStages; ++i) {
+    for (int i = 0; i < NST; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
@@ -425,9 +449,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    if (lane == 0) producer_loop(p, stages, full, empty, abort);
+    if (lane == 0) producer_loop<NST, SBYTES>(p, stages, full, empty, abort);
   } else if (warp == 1) {
-    if (lane == 0) mma_loop(p, stages, full, empty, tfull, tempty, tmem, abort);
+    if (lane == 0) mma_loop<NST, SBYTES>(p, stages, full, empty, tfull, tempty, tmem, abort);
   } else {
     epilogue_loop<KIND>(p, tfull, tempty, tmem, abort);
   }
@@ -450,13 +474,15 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
 
 template <int KIND>
 static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t stream) {
+  constexpr int smem = StageCfg<KIND>::stages * StageCfg<KIND>::bytes + 1024 + 256;
+  static_assert(smem <= 232448, "shared memory per CTA");
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGemmSmem);
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  gemm_kernel<KIND><<<grid, kGemmThreads, kGemmSmem, stream>>>(p);
+  gemm_kernel<KIND><<<grid, kGemmThreads, smem, stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
   __shared__ int warp_sums[32];
   __shared__ int best_k;
   __shared__ int s_prefix_cnt[2];
-  __shared__ long long n_on_sum;
+  __shared__ long long n_on_sum;  // updated with 64-bit atomics
 
   const int b = blockIdx.x, tid = threadIdx.x;
   const int v0 = a.vis_off[b], v1 = a.vis_off[b + 1];
@@ -85,17 +85,19 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
 
   // ---- k from the budget (Eq. 8, exact integers scaled by G)
   if (tid == 0) {
-    long long s = 0;
-    for (int l = 0; l < a.L; ++l) {
-      int on = 0;
-      for (int j = 0; j < a.G; ++j) {
-        const bool e = (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * a.G + j]);
-        on += e ? 1 : 0;
-      }
-      s += on;
-    }
-    n_on_sum = s;
+    n_on_sum = 0;
     best_k = -1;
+  }
+  __syncthreads();
+  {
+    int on = 0;  // active (layer, group) pairs of this sample
+    for (int idx = tid; idx < a.L * a.G; idx += blockDim.x) {
+      const int l = idx / a.G;
+      on += ((l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[b * a.L * a.G + idx])) ? 1 : 0;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) on += __shfl_xor_sync(0xffffffffu, on, o);
+    if ((tid & 31) == 0 && on) atomicAdd(reinterpret_cast<unsigned long long*>(&n_on_sum), static_cast<unsigned long long>(on));
   }
   __syncthreads();
   int k;
@@ -149,14 +151,39 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
       if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 0xFF], 1);
     }
     __syncthreads();
-    if (tid == 0) {
-      int above = 0, d = 255;
-      for (; d > 0; --d) {
-        if (above + hist[d] >= remaining) break;
-        above += hist[d];
+    if (tid < 32) {
+      // warp 0: counts above each digit (suffix sums from 255 down), then the
+      // largest digit d whose keys with digit >= d reach `remaining`
+      int cnt[8], sum = 0;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        cnt[u] = hist[255 - (tid * 8 + u)];  // lane t holds digits 255-8t .. 248-8t
+        sum += cnt[u];
       }
-      s_prefix_cnt[0] = d;
-      s_prefix_cnt[1] = remaining - above;
+      int incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (tid >= o) incl += y;
+      }
+      int above = incl - sum;  // keys with a digit above this lane's first digit
+      int found = -1, found_above = 0;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (found < 0 && above + cnt[u] >= remaining) {
+          found = 255 - (tid * 8 + u);
+          found_above = above;
+        }
+        above += cnt[u];
+      }
+      const unsigned ballot = __ballot_sync(0xffffffffu, found >= 0);
+      const int first = ballot ? __ffs(ballot) - 1 : 31;
+      const int d = __shfl_sync(0xffffffffu, found, first);
+      const int ab = __shfl_sync(0xffffffffu, found_above, first);
+      if (tid == 0) {
+        s_prefix_cnt[0] = d < 0 ? 0 : d;
+        s_prefix_cnt[1] = remaining - (d < 0 ? 0 : ab);
+      }
     }
     __syncthreads();
     prefix |= static_cast<uint32_t>(s_prefix_cnt[0]) << shift;
@@ -191,17 +218,21 @@ __global__ void compact_kernel(int B, const int* __restrict__ vis_off, const int
                                int* __restrict__ kept_off, int* __restrict__ kept_total) {
   __shared__ int off;
   const int b = blockIdx.x;
+  if (threadIdx.x == 0) off = 0;
+  __syncthreads();
+  int part = 0;  // k of the samples before b, summed by all threads
+  for (int i = threadIdx.x; i < b; i += blockDim.x) part += k[i];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+  if ((threadIdx.x & 31) == 0 && part) atomicAdd(&off, part);
+  __syncthreads();
   if (threadIdx.x == 0) {
-    int s = 0;
-    for (int i = 0; i < b; ++i) s += k[i];
-    off = s;
-    kept_off[b] = s;
+    kept_off[b] = off;
     if (b == B - 1) {
-      kept_off[B] = s + k[b];
-      if (kept_total) *kept_total = s + k[b];
+      kept_off[B] = off + k[b];
+      if (kept_total) *kept_total = off + k[b];
     }
   }
-  __syncthreads();
   const int kb = k[b];
   const int* src = kept_local + vis_off[b];
   for (int i = threadIdx.x; i < kb; i += blockDim.x) kept_idx[off + i] = src[i];

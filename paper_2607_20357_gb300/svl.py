@@ -26,7 +26,7 @@ SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
-           "svl_tag_name", "svl_score_select_noalloc"]
+           "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
@@ -94,6 +94,9 @@ def lib():
         L.svl_tag_name.restype = ctypes.c_char_p
         L.svl_score_select_noalloc.argtypes = [vp, i32, i32] + [vp] * 13
         L.svl_score_select_noalloc.restype = ctypes.c_int
+        L.svl_profile_launches.argtypes = [vp, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_float), i32,
+                                           ctypes.POINTER(i32)]
+        L.svl_profile_launches.restype = ctypes.c_int
         _lib = L
     return _lib
 
@@ -209,6 +212,15 @@ def svl_host_workspace_size(model, B, n_vis_total, n_text_total) -> int:
 
 def svl_profile_start(model):
     _check("svl_profile_start", lib().svl_profile_start(model))
+
+
+def svl_profile_launches(model, cap=1 << 16):
+    """[(tag name, ms)] of every launch of the last profiling window."""
+    tags = (ctypes.c_int32 * cap)()
+    ms = (ctypes.c_float * cap)()
+    n = ctypes.c_int32()
+    _check("svl_profile_launches", lib().svl_profile_launches(model, tags, ms, cap, ctypes.byref(n)))
+    return [(TAGS[tags[i]] if 0 <= tags[i] < len(TAGS) else str(tags[i]), float(ms[i])) for i in range(n.value)]
 
 
 def svl_profile_stop(model) -> dict:
