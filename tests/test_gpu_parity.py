@@ -160,3 +160,14 @@ def test_logits_all_rows_tiny():
     T = int(out["cu_seqlens"][-1])
     assert rel_err(out["logits"][:T].double().numpy(), want) < 2e-2
     case.close()
+
+
+def test_split_tail_llava_one_layer_full_batch():
+    """B = 16 LLaVA rows at b = 0.5 give the O and down projections four full
+    waves plus a tail that the schedule splits along K; every sample must
+    still match."""
+    dims = synth.reduced(LLAVA.dims, n_layers=1)
+    case = Case(dims, LLAVA, seed=12, batch=16, budget=0.5)
+    errs = _compare_end_to_end(case, case.run())
+    assert len(errs) >= 14
+    case.close()
