@@ -236,8 +236,10 @@ svl_status svl_prefill_from_host(svl_model* model, int32_t B, int32_t n_vis_tota
 size_t svl_host_workspace_size(const svl_model* model, int32_t B, int64_t n_vis_total, int64_t n_text_total);
 
 /* Kernel timing. While profiling is on, the library records a CUDA event
- * pair on the launch stream around every kernel it launches, tagged by the
- * step of the path. svl_profile_stop() waits for the last event, sums the
+ * pair on the launch stream around every kernel it launches whose tag bit is
+ * set in `tag_mask`, tagged by the step of the path (events between kernels
+ * keep a kernel from starting before its predecessor finishes, so record
+ * only what is needed while timing end to end). svl_profile_stop() waits for the last event, sums the
  * elapsed times per tag into `out` (at most `cap` entries, *n_out set) and
  * turns profiling off. */
 typedef struct svl_kernel_time {
@@ -262,7 +264,7 @@ typedef struct svl_kernel_time {
 #define SVL_TAG_COPY 13
 #define SVL_TAG_COUNT 14
 
-svl_status svl_profile_start(svl_model* model);
+svl_status svl_profile_start(svl_model* model, uint32_t tag_mask); /* bit t: record SVL_TAG t */
 svl_status svl_profile_stop(svl_model* model, svl_kernel_time* out, int32_t cap, int32_t* n_out);
 /* The individual launches of the last profiling window (after
  * svl_profile_stop), in launch order: tag and elapsed milliseconds of each.

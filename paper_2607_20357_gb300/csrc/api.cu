@@ -26,6 +26,7 @@ struct svl_model {
   CUtensorMap tm_ctrl_w1, tm_proj_w1, tm_proj_w2, tm_lm_head;
   // kernel timing (svl_profile_start / svl_profile_stop)
   bool prof = false;
+  uint32_t prof_mask = 0;
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   std::vector<std::pair<int, size_t>> prof_recs;  // (tag, index of the first event of the pair)
@@ -218,7 +219,7 @@ struct Launch {
   size_t first = SIZE_MAX;
   Launch(svl_model* m_, int tag, cudaStream_t s_) : m(m_), s(s_) {
     g_launches++;
-    if (!m->prof) return;
+    if (!m->prof || !((m->prof_mask >> tag) & 1u)) return;
     if (m->ev_used + 2 > m->ev_pool.size()) {
       for (int i = 0; i < 64; ++i) {
         cudaEvent_t e;
@@ -820,9 +821,10 @@ svl_status svl_prefill_from_host(svl_model* m, int32_t B, int32_t nv, int32_t nt
   return ok ? SVL_OK : SVL_ERR_CUDA;
 }
 
-svl_status svl_profile_start(svl_model* m) {
+svl_status svl_profile_start(svl_model* m, uint32_t tag_mask) {
   if (!m) return SVL_ERR_INVALID_ARG;
   m->prof = true;
+  m->prof_mask = tag_mask;
   m->ev_used = 0;
   m->prof_recs.clear();
   return SVL_OK;

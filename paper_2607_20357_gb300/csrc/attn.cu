@@ -72,7 +72,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_items = min(*a.count, a.cap);
 
   if (threadIdx.x == 0) {
     mbar_init(&bar->q_full, 1);
@@ -98,6 +97,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
+  const int n_items = min(*a.count, a.cap);
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -320,8 +322,7 @@ static cudaError_t launch_dh(const AttnTcArgs& a, int grid, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  attn_tc_kernel<DH><<<grid, kAttnThreads, AttnSmem<DH>::total, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(attn_tc_kernel<DH>, grid, kAttnThreads, AttnSmem<DH>::total, s, a);
 }
 
 cudaError_t launch_attention_tc(const AttnTcArgs& a, int grid, cudaStream_t s) {

@@ -84,6 +84,8 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __shared__ NTile nt[kMaxNT];
   __shared__ int s_nseg, s_nnt;
   __shared__ int s_heads[256];
+  pdl_trigger();
+  pdl_wait();
   const int l = blockIdx.x, tid = threadIdx.x;
   const int B = a.B, G = a.G;
   int4* seg = a.seg + static_cast<size_t>(l) * B;
@@ -211,7 +213,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   if (tid == 0) a.attn_count[l] = min(off, a.attn_cap);
 }
 
-void launch_schedule(const ScheduleArgs& a, cudaStream_t s) { schedule_kernel<<<a.L, 256, 0, s>>>(a); }
+void launch_schedule(const ScheduleArgs& a, cudaStream_t s) { launch_pdl(schedule_kernel, a.L, 256, 0, s, a); }
 
 // ---------------------------------------------------------------- RMSNorm
 SVL_DEVINL int find_sample(const int* cu, int B, int r) {
@@ -256,6 +258,8 @@ SVL_DEVINL void norm_row(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bf
 }
 
 __global__ void rmsnorm_kernel(NormArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + warp;
   const int T = a.cu_seqlens[a.B];
@@ -265,6 +269,8 @@ __global__ void rmsnorm_kernel(NormArgs a) {
 }
 
 __global__ void final_rows_kernel(NormArgs a, int n_pad) {
+  pdl_trigger();
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b = blockIdx.x * (blockDim.x >> 5) + warp;
   if (b >= n_pad) return;
@@ -279,11 +285,11 @@ __global__ void final_rows_kernel(NormArgs a, int n_pad) {
 
 void launch_rmsnorm(const NormArgs& a, cudaStream_t s) {
   const int grid = (a.t_cap + 7) / 8;
-  if (grid > 0) rmsnorm_kernel<<<grid, 256, 0, s>>>(a);
+  if (grid > 0) launch_pdl(rmsnorm_kernel, grid, 256, 0, s, a);
 }
 
 void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s) {
-  final_rows_kernel<<<(n_pad + 7) / 8, 256, 0, s>>>(a, n_pad);
+  launch_pdl(final_rows_kernel, (n_pad + 7) / 8, 256, 0, s, a, n_pad);
 }
 
 __global__ void rope_table_kernel(float2* cs, int max_seq, int dh, double theta) {

@@ -447,6 +447,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // set-up above touches no global data; from here on the predecessor's
+  // outputs are read
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) producer_loop<NST, SBYTES>(p, stages, full, empty, abort);
@@ -482,8 +486,7 @@ static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t strea
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  gemm_kernel<KIND><<<grid, kGemmThreads, smem, stream>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(gemm_kernel<KIND>, grid, kGemmThreads, smem, stream, p);
 }
 
 cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream) {

@@ -7,6 +7,8 @@
 namespace svl {
 
 __global__ void pack_offsets_kernel(PackArgs a) {
+  pdl_trigger();
+  pdl_wait();
   if (threadIdx.x != 0) return;
   int t = 0;
   a.cu_seqlens[0] = 0;
@@ -25,6 +27,8 @@ __global__ void pack_offsets_kernel(PackArgs a) {
 
 // One warp per output row.
 __global__ void pack_gather_kernel(PackArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int r = blockIdx.x * (blockDim.x >> 5) + warp;
   const int T = *a.t_total;
@@ -67,20 +71,22 @@ __global__ void pack_gather_kernel(PackArgs a) {
 }
 
 __global__ void offsets_diff_kernel(const int* off, int* len, int B) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < B) len[b] = off[b + 1] - off[b];
 }
 
 void launch_offsets_diff(const int* off, int* len, int B, cudaStream_t s) {
-  offsets_diff_kernel<<<(B + 255) / 256, 256, 0, s>>>(off, len, B);
+  launch_pdl(offsets_diff_kernel, (B + 255) / 256, 256, 0, s, off, len, B);
 }
 
-void launch_pack_offsets(const PackArgs& a, cudaStream_t s) { pack_offsets_kernel<<<1, 32, 0, s>>>(a); }
+void launch_pack_offsets(const PackArgs& a, cudaStream_t s) { launch_pdl(pack_offsets_kernel, 1, 32, 0, s, a); }
 
 void launch_pack_gather(const PackArgs& a, cudaStream_t s) {
   const int rows_per_block = 8;
   const int grid = (a.t_cap + rows_per_block - 1) / rows_per_block;
-  if (grid > 0) pack_gather_kernel<<<grid, rows_per_block * 32, 0, s>>>(a);
+  if (grid > 0) launch_pdl(pack_gather_kernel, grid, rows_per_block * 32, 0, s, a);
 }
 
 }  // namespace svl

@@ -11,6 +11,8 @@ __global__ void budget_embed_kernel(const float* __restrict__ budget, const __nv
                                     const __nv_bfloat16* __restrict__ w2, int H, float* __restrict__ e_b) {
   __shared__ double pe[256];
   __shared__ double hid[256];
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x, i = threadIdx.x;
   const double bv = static_cast<double>(budget[b]);
   if (i < H) {
@@ -77,6 +79,8 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
   __shared__ int best_k;
   __shared__ int s_prefix_cnt[2];
   __shared__ long long n_on_sum;  // updated with 64-bit atomics
+  pdl_trigger();
+  pdl_wait();
 
   const int b = blockIdx.x, tid = threadIdx.x;
   const int v0 = a.vis_off[b], v1 = a.vis_off[b + 1];
@@ -217,6 +221,8 @@ __global__ void compact_kernel(int B, const int* __restrict__ vis_off, const int
                                const int* __restrict__ kept_local, int* __restrict__ kept_idx,
                                int* __restrict__ kept_off, int* __restrict__ kept_total) {
   __shared__ int off;
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   if (threadIdx.x == 0) off = 0;
   __syncthreads();
@@ -240,16 +246,16 @@ __global__ void compact_kernel(int B, const int* __restrict__ vis_off, const int
 
 void launch_budget_embed(const float* budget, const __nv_bfloat16* w1, const __nv_bfloat16* w2, int H, int B,
                          float* e_b, cudaStream_t s) {
-  budget_embed_kernel<<<B, 256, 0, s>>>(budget, w1, w2, H, e_b);
+  launch_pdl(budget_embed_kernel, B, 256, 0, s, budget, w1, w2, H, e_b);
 }
 
 void launch_select(const SelectArgs& a, int B, cudaStream_t s) {
-  select_kernel<<<B, kSelectThreads, 0, s>>>(a);
+  launch_pdl(select_kernel, B, kSelectThreads, 0, s, a);
 }
 
 void launch_compact(int B, const int* vis_off, const int* k, const int* kept_local, int* kept_idx, int* kept_off,
                     int* kept_total, cudaStream_t s) {
-  compact_kernel<<<B, 256, 0, s>>>(B, vis_off, k, kept_local, kept_idx, kept_off, kept_total);
+  launch_pdl(compact_kernel, B, 256, 0, s, B, vis_off, k, kept_local, kept_idx, kept_off, kept_total);
 }
 
 }  // namespace svl

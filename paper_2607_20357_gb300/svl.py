@@ -86,7 +86,7 @@ def lib():
         L.svl_prefill_from_host.restype = ctypes.c_int
         L.svl_host_workspace_size.argtypes = [vp, i32, i64, i64]
         L.svl_host_workspace_size.restype = sz
-        L.svl_profile_start.argtypes = [vp]
+        L.svl_profile_start.argtypes = [vp, ctypes.c_uint32]
         L.svl_profile_start.restype = ctypes.c_int
         L.svl_profile_stop.argtypes = [vp, ctypes.POINTER(KernelTime), i32, ctypes.POINTER(i32)]
         L.svl_profile_stop.restype = ctypes.c_int
@@ -210,8 +210,11 @@ def svl_host_workspace_size(model, B, n_vis_total, n_text_total) -> int:
     return int(lib().svl_host_workspace_size(model, int(B), int(n_vis_total), int(n_text_total)))
 
 
-def svl_profile_start(model):
-    _check("svl_profile_start", lib().svl_profile_start(model))
+def svl_profile_start(model, tags=None):
+    """Records events around the kernels whose tag names are in `tags`
+    (default: every kernel)."""
+    mask = 0xFFFFFFFF if tags is None else sum(1 << TAGS.index(t) for t in tags)
+    _check("svl_profile_start", lib().svl_profile_start(model, ctypes.c_uint32(mask)))
 
 
 def svl_profile_launches(model, cap=1 << 16):
