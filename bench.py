@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-hbm-sweep", action="store_true")
+    ap.add_argument("--hbm-only", type=str, default="",
+                    help="comma-separated batch multipliers: run only the token-controller/pack sweep "
+                         "(for small profiler captures)")
     ap.add_argument("--layers", type=int, default=0,
                     help="decoder layers (default: all 32). Fewer layers only for small profiler captures; "
                          "such a line is not the benchmark value")
@@ -253,6 +256,11 @@ def run_ours(args, rank, world, local_rank):
     weights = synth.make_weights(dims, SEED, device=dev)
     max_seq = wl.n_vis[1] + wl.s_text[1] + 64
     model = svl.GatedPrefill(dims, weights, max_seq=max_seq)
+    if args.hbm_only:
+        mults = tuple(int(x) for x in args.hbm_only.split(","))
+        print(json.dumps({"hbm_kernels_sweep": run_hbm_sweep(svl, model, wl, dev, pk, mults=mults)}), flush=True)
+        model.close()
+        return
     seed = SEED + 17 * rank
     batches = [synth.make_batch(wl, seed, budget=b, device=dev) for b in wl.budgets]
     outs = [model.alloc_outputs(bt) for bt in batches]
@@ -411,13 +419,13 @@ def run_ours(args, rank, world, local_rank):
     model.close()
 
 
-def run_hbm_sweep(svl, model, wl, dev, pk, reps=5):
+def run_hbm_sweep(svl, model, wl, dev, pk, reps=5, mults=(1, 4, 16)):
     """Token controller and pack alone at 1x, 4x and 16x the benchmark batch
     (budget 0.5): achieved bandwidth of the HBM-bound kernels from their
     algorithmic bytes and CUDA-event times."""
     d = wl.dims
     out = []
-    for mult in (1, 4, 16):
+    for mult in mults:
         B = wl.batch * mult
         bt = synth.make_batch(wl, SEED + 7 + mult, budget=0.5, batch=B, device=dev)
         o = model.alloc_outputs(bt)

@@ -125,6 +125,14 @@ void svl_model_destroy(svl_model* model);
 size_t svl_workspace_size(const svl_model* model, int32_t max_batch, int64_t max_vis_total,
                           int64_t max_text_total);
 
+#define SVL_STAGE_SELECT 1u  /* svl_score_select */
+#define SVL_STAGE_PACK 2u    /* svl_pack */
+#define SVL_STAGE_PREFILL 4u /* svl_gated_prefill */
+/* Workspace bytes for only the stages in `stages` (a caller that only runs
+ * the token controller needs far less than svl_workspace_size()). */
+size_t svl_workspace_size_for(const svl_model* model, uint32_t stages, int32_t max_batch, int64_t max_vis_total,
+                              int64_t max_text_total);
+
 /* (1) Token controller (Sec. 3.1; Sec. 3.3 "Inference"; Eq. 5; Eq. 8).
  *  Scores every visual token, z_i = w2 . SiLU(W1 x_i + e_b) + c2, with the
  *  budget embedding e_b = W_b2 SiLU(W_b1 PE(b)); derives k_b as the largest
@@ -271,6 +279,14 @@ svl_status svl_profile_stop(svl_model* model, svl_kernel_time* out, int32_t cap,
  * Writes at most `cap` entries and sets *n_out to the number written. */
 svl_status svl_profile_launches(svl_model* model, int32_t* tags, float* ms, int32_t cap, int32_t* n_out);
 const char* svl_tag_name(int32_t tag);
+
+/* Self-test of the device-side time-out path (the paper has no
+ * counterpart): launches one CTA that waits on a shared-memory barrier that
+ * nothing ever arrives on, giving up after `wait_cycles` SM clock cycles the
+ * way every wait in the library does, so SVL_DEV_TIMEOUT is set in the
+ * status word and the kernel returns normally. `wait_cycles` is clamped to
+ * [1000, 1e9]. Asynchronous on `stream`. */
+svl_status svl_selftest_wait_timeout(svl_model* model, uint64_t wait_cycles, void* stream);
 
 /* Reads (and clears) the device status word; synchronises `stream`. */
 svl_status svl_get_device_status(svl_model* model, void* stream, uint32_t* code);

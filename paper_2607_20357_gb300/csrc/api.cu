@@ -351,12 +351,20 @@ void svl_model_destroy(svl_model* m) {
   delete m;
 }
 
-size_t svl_workspace_size(const svl_model* m, int32_t max_batch, int64_t max_vis_total, int64_t max_text_total) {
+size_t svl_workspace_size_for(const svl_model* m, uint32_t stages, int32_t max_batch, int64_t max_vis_total,
+                              int64_t max_text_total) {
   if (!m || max_batch <= 0 || max_vis_total < 0 || max_text_total < 0) return 0;
-  const size_t a = sel_layout(m->d, max_batch, max_vis_total).total;
-  const size_t b = pack_layout(m->d, max_vis_total).total;
-  const size_t c = pre_layout(m->d, max_batch, max_vis_total + max_text_total).total;
-  return std::max(a, std::max(b, c));
+  size_t need = 0;
+  if (stages & SVL_STAGE_SELECT) need = std::max(need, sel_layout(m->d, max_batch, max_vis_total).total);
+  if (stages & SVL_STAGE_PACK) need = std::max(need, pack_layout(m->d, max_vis_total).total);
+  if (stages & SVL_STAGE_PREFILL)
+    need = std::max(need, pre_layout(m->d, max_batch, max_vis_total + max_text_total).total);
+  return need;
+}
+
+size_t svl_workspace_size(const svl_model* m, int32_t max_batch, int64_t max_vis_total, int64_t max_text_total) {
+  return svl_workspace_size_for(m, SVL_STAGE_SELECT | SVL_STAGE_PACK | SVL_STAGE_PREFILL, max_batch, max_vis_total,
+                                max_text_total);
 }
 
 svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
@@ -876,6 +884,16 @@ const char* svl_tag_name(int32_t tag) {
                                               "schedule", "rmsnorm", "qkv_gemm", "attention", "o_gemm",
                                               "gateup_gemm", "down_gemm", "lm_head", "host_copy"};
   return (tag >= 0 && tag < SVL_TAG_COUNT) ? names[tag] : "unknown";
+}
+
+svl_status svl_selftest_wait_timeout(svl_model* m, uint64_t wait_cycles, void* stream) {
+  if (!m) return SVL_ERR_INVALID_ARG;
+  const long long c = static_cast<long long>(std::min<uint64_t>(std::max<uint64_t>(wait_cycles, 1000), 1000000000));
+  {
+    Launch L1(m, SVL_TAG_SCHEDULE, static_cast<cudaStream_t>(stream));
+    launch_selftest_wait(m->d_status, c, static_cast<cudaStream_t>(stream));
+  }
+  return last_error();
 }
 
 svl_status svl_get_device_status(svl_model* m, void* stream, uint32_t* code) {

@@ -98,14 +98,14 @@ SVL_DEVINL bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase with the given parity to complete. Gives up when
-// `*abort` becomes non-zero or after kWaitCycles; returns false then.
-SVL_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+// `*abort` becomes non-zero or after `limit` cycles; returns false then.
+SVL_DEVINL bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, long long limit = kWaitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   }
 }
 

@@ -292,6 +292,22 @@ void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s) {
   launch_pdl(final_rows_kernel, (n_pad + 7) / 8, 256, 0, s, a, n_pad);
 }
 
+__global__ void selftest_wait_kernel(uint32_t* status, long long cycles) {
+  __shared__ uint64_t bar;
+  __shared__ int abort;
+  if (threadIdx.x == 0) {
+    abort = 0;
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !mbar_wait(&bar, 0, &abort, cycles)) report(status, SVL_DEV_TIMEOUT);
+}
+
+void launch_selftest_wait(uint32_t* status, long long cycles, cudaStream_t s) {
+  selftest_wait_kernel<<<1, 32, 0, s>>>(status, cycles);
+}
+
 __global__ void rope_table_kernel(float2* cs, int max_seq, int dh, double theta) {
   const int half = dh / 2;
   const long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;

@@ -26,7 +26,8 @@ SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
-           "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches"]
+           "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches", "svl_selftest_wait_timeout",
+           "svl_workspace_size_for"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
@@ -97,6 +98,10 @@ def lib():
         L.svl_profile_launches.argtypes = [vp, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_float), i32,
                                            ctypes.POINTER(i32)]
         L.svl_profile_launches.restype = ctypes.c_int
+        L.svl_selftest_wait_timeout.argtypes = [vp, ctypes.c_uint64, vp]
+        L.svl_selftest_wait_timeout.restype = ctypes.c_int
+        L.svl_workspace_size_for.argtypes = [vp, ctypes.c_uint32, i32, i64, i64]
+        L.svl_workspace_size_for.restype = sz
         _lib = L
     return _lib
 
@@ -139,6 +144,15 @@ def svl_model_destroy(model):
 
 def svl_workspace_size(model, max_batch, max_vis_total, max_text_total) -> int:
     return int(lib().svl_workspace_size(model, int(max_batch), int(max_vis_total), int(max_text_total)))
+
+
+STAGE_BITS = {"select": 1, "pack": 2, "prefill": 4}
+
+
+def svl_workspace_size_for(model, stages, max_batch, max_vis_total, max_text_total) -> int:
+    mask = sum(STAGE_BITS[s] for s in stages)
+    return int(lib().svl_workspace_size_for(model, ctypes.c_uint32(mask), int(max_batch), int(max_vis_total),
+                                            int(max_text_total)))
 
 
 def svl_score_select(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
@@ -184,6 +198,11 @@ def svl_flops(desc: ModelDesc, s_text, s_vis, n_vis, layer_gate=None, group_gate
     _check("svl_flops", lib().svl_flops(ctypes.byref(desc), int(s_text), int(s_vis), int(n_vis), lg, gg,
                                         ctypes.byref(eq8), ctypes.byref(ex)))
     return eq8.value, ex.value
+
+
+def svl_selftest_wait_timeout(model, wait_cycles=100000, stream=None):
+    _check("svl_selftest_wait_timeout", lib().svl_selftest_wait_timeout(model, ctypes.c_uint64(int(wait_cycles)),
+                                                                        _stream(stream)))
 
 
 def svl_get_device_status(model, stream=None) -> int:
@@ -280,8 +299,8 @@ class GatedPrefill:
         except Exception:
             pass
 
-    def workspace(self, B, n_vis, n_text, device="cuda"):
-        need = svl_workspace_size(self.handle, B, n_vis, n_text)
+    def workspace(self, B, n_vis, n_text, device="cuda", stages=("select", "pack", "prefill")):
+        need = svl_workspace_size_for(self.handle, stages, B, n_vis, n_text)
         if self._ws is None or self._ws.numel() < need:
             self._ws = torch.empty(need, dtype=torch.uint8, device=device)
         return self._ws, self._ws.numel()
@@ -314,7 +333,7 @@ class GatedPrefill:
         nv = batch["vis"].shape[0]
         nt = int(batch["text_ids"].shape[0])
         out = out or self.alloc_outputs(batch, logits_mode)
-        ws, wsb = self.workspace(B, nv, nt, batch["vis"].device)
+        ws, wsb = self.workspace(B, nv, nt, batch["vis"].device, stages)
         if "select" in stages:
             svl_score_select(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"], batch["budget"],
                              batch["keep_count"], batch["layer_gate"], batch["group_gate"], out["scores"], out["k"],
