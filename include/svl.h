@@ -94,9 +94,9 @@ typedef struct svl_layer_weights {
   const void* ffn_norm;   /* [D] */
 } svl_layer_weights;
 
-/* All weights: device bf16 unless noted. The model keeps these pointers (it
- * does not copy them): the caller keeps the memory alive until
- * svl_model_destroy(). */
+/* All weights: device bf16 unless noted, 16-byte aligned. The model keeps
+ * these pointers (it does not copy them): the caller keeps the memory alive
+ * until svl_model_destroy(). */
 typedef struct svl_weights {
   const void* ctrl_w1;    /* [H, C_v]  token scorer, first layer */
   const void* ctrl_w2;    /* [H]       token scorer, output weights */

@@ -294,6 +294,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
       !w->layers)
     return SVL_ERR_INVALID_ARG;
   if (d.proj_hidden && (!w->proj_w1 || !w->proj_w2)) return SVL_ERR_INVALID_ARG;
+  if (!aligned16(w->ctrl_w2) || !aligned16(w->embed)) return SVL_ERR_INVALID_ARG;  // read as 16-byte vectors
   if (!encode_fn()) return SVL_ERR_CUDA;
 
   svl_model* m = new svl_model();

@@ -1,58 +1,68 @@
 // Variable-length causal attention over active heads only (Sec. 3.2: the
 // heads of a gated-off group are never computed), on tcgen05 tensor cores.
 //
-// Persistent kernel, one CTA per SM, work items (sample, active head, block
-// of 128 queries) from the device schedule. Per item and per tile of 128 keys:
-//   S = Q K^T          tcgen05.mma M=128 N=128 K=d_head, into one of two TMEM
-//                      S buffers (S(j+1) is computed while row j's softmax runs)
-//   softmax            four warps, one query row per thread: running max and
-//                      sum, P = exp2(S*scale - max) rounded to bf16 and written
-//                      to shared memory in the 128-byte-swizzled K-major layout
-//   O_tile = P V       tcgen05.mma M=128 N=d_head K=128 into a TMEM buffer;
-//                      the thread folds it into its fp32 output row in
-//                      registers: O = O*exp2(m_old - m_new) + O_tile
-// V arrives transposed (V^T, keys contiguous) so that both MMA operands are
-// K-major. Key tiles start at the sample's first row rounded down to a
-// multiple of 8 (TMA needs a 16-byte aligned innermost coordinate); keys of
-// the neighbouring sample that this pulls in are masked, like every key after
-// the query (causal) or past the block's last query.
+// Persistent kernel, one CTA per SM. A work item from the device schedule is
+// (sample, active head, up to 256 consecutive queries); its first 128 queries
+// are block A, the rest block B. Each block owns a Q buffer, an S and an O
+// accumulator in TMEM, a P buffer in shared memory and four softmax warps.
+// Both blocks walk the same key tiles, so every K and V^T tile is loaded once
+// for 256 queries. Per tile of 128 keys and block:
+//   S = Q K^T      tcgen05.mma M=128 N=128 K=d_head into the block's S columns
+//   softmax        one query row per thread: row max, P = exp2(S*scale - m)
+//                  rounded to bf16 and written to shared memory in the
+//                  128-byte-swizzled K-major layout, row sum
+//   O += P V       tcgen05.mma M=128 N=d_head K=128 into the block's O columns
+// The running max m is only moved when a tile's max exceeds it by more than
+// 2^8 (then O and the row sum are rescaled in place); otherwise P is formed
+// against the stale max, its entries stay below 256 and O needs no per-tile
+// correction. O / rowsum is written out once per item.
 //
-// Warp 0: TMA producer (Q once per item, K and V^T double buffered).
-// Warp 1: TMEM allocation and the MMA-issuing thread.
-// Warps 2-5: softmax and output. Every wait is bounded.
+// The MMA thread works in rounds: in round j, for each block whose softmax of
+// tile j-1 is done, it issues S of tile j and P V of tile j-1, so one block's
+// softmax overlaps the other block's products. V arrives transposed (V^T,
+// keys contiguous) so that both operands are K-major; K and V^T tiles share a
+// ring of shared-memory stages that the producer fills in the order the MMA
+// thread consumes them. Key tiles start at the sample's first row rounded down
+// to a multiple of 8 (TMA needs a 16-byte aligned innermost coordinate); keys
+// of the neighbouring sample that this pulls in are masked, like every key
+// after the query (causal) or past the sample's end.
+//
+// Warp 0: TMA producer. Warp 1: TMEM allocation and the MMA-issuing thread.
+// Warps 2-5: block A softmax and output; warps 6-9: block B.
+// Every barrier completes at most once ahead of its waiter; every wait is
+// bounded.
 #include "kernels.cuh"
 
 namespace svl {
 
-constexpr int kAttnThreads = 192;
+constexpr int kAttnThreads = 320;
 constexpr int kKeyTile = 128;
+constexpr int kRing = 3;
+constexpr float kRescaleLog2 = 8.f;  // move the running max when it grows by more than 2^8
+static_assert(kAttnQ == 256, "an attention item is two blocks of 128 queries");
 
 template <int DH>
 struct AttnSmem {
-  static constexpr int kQ = 128 * DH * 2;          // Q: DH/64 atoms of 128 rows x 128 B
-  static constexpr int kK = kKeyTile * DH * 2;     // K stage
-  static constexpr int kV = DH * kKeyTile * 2;     // V^T stage: 2 atoms of DH rows x 128 B
-  static constexpr int kP = 128 * kKeyTile * 2;    // P buffer: 2 atoms of 128 rows x 128 B
-  static constexpr int q = 0;
-  static constexpr int k0 = kQ;
-  static constexpr int v0 = k0 + 2 * kK;
-  static constexpr int p0 = v0 + 2 * kV;
-  static constexpr int bars = p0 + 2 * kP;
+  static constexpr int kAtom = 128 * 128;     // 128 rows x 128 B
+  static constexpr int kQ = 128 * DH * 2;     // Q tile: DH/64 atoms
+  static constexpr int kStage = 128 * DH * 2; // K tile (DH/64 atoms of 128 keys) or V^T tile (2 x DH rows x 128 B)
+  static constexpr int kVAtom = DH * 128;     // V^T: DH rows x 64 keys
+  static constexpr int kP = 128 * kKeyTile * 2;
+  static constexpr int q0 = 0;
+  static constexpr int p0 = q0 + 2 * kQ;
+  static constexpr int r0 = p0 + 2 * kP;
+  static constexpr int bars = r0 + kRing * kStage;
   static constexpr int total = bars + 256 + 1024;  // + barriers + alignment slack
 };
+static_assert(AttnSmem<128>::total <= 232448, "attention shared memory");
 
 struct AttnBars {
-  uint64_t q_full, q_empty, k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2], p_full, o_full[2];
+  uint64_t q_full[2], q_empty[2], r_full[kRing], r_empty[kRing], s_full[2], p_full[2], pv_done[2];
 };
 
 SVL_DEVINL void attn_abort(volatile int* abort, uint32_t* status) {
   *abort = 1;
   report(status, SVL_DEV_TIMEOUT);
-}
-
-SVL_DEVINL int n_key_tiles(const int4& it) {
-  const int key_base = it.z & ~7;
-  return (it.y - key_base + kKeyTile - 1) / kKeyTile;
 }
 
 SVL_DEVINL float ex2(float x) {
@@ -61,7 +71,99 @@ SVL_DEVINL float ex2(float x) {
   return y;
 }
 
-// TMEM columns: S buffers 0 and 128, P V buffers 256 and 384.
+SVL_DEVINL float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// Two fp32 lanes in one 64-bit register: (a*b + c) and (a + b) per lane.
+SVL_DEVINL uint64_t f2(float lo, float hi) {
+  return (static_cast<uint64_t>(__float_as_uint(hi)) << 32) | __float_as_uint(lo);
+}
+SVL_DEVINL uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+SVL_DEVINL uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+SVL_DEVINL float lo2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v)); }
+SVL_DEVINL float hi2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
+
+// Tile counts of an item {q0, q_end, r0, head}: block A is queries
+// [q0, min(q0 + 128, q_end)), block B the rest (possibly empty). Key tiles
+// start at r0 rounded down to 8; a block needs the tiles up to its last query.
+struct ItemTiles {
+  int na, nb, n;
+};
+SVL_DEVINL ItemTiles item_tiles(const int4& it) {
+  const int key_base = it.z & ~7;
+  const int a_end = min(it.x + 128, it.y);
+  ItemTiles t;
+  t.na = (a_end - key_base + kKeyTile - 1) / kKeyTile;
+  t.nb = it.y > a_end ? (it.y - key_base + kKeyTile - 1) / kKeyTile : 0;
+  t.n = max(t.na, t.nb);
+  return t;
+}
+
+// Ring positions of an item's 2n tiles relative to its first: K(0), then per
+// round j = 1..n: K(j) (while j < n) and V(j-1).
+SVL_DEVINL int pos_k(int j) { return j == 0 ? 0 : 2 * j - 1; }
+SVL_DEVINL int pos_v(int m, int n) { return m + 1 < n ? 2 * m + 2 : 2 * m + 1; }
+
+// Row max of 64 scores, masked to [lo, lo + span) unless `full`.
+SVL_DEVINL float row_max64(const uint32_t* sv, int base, bool full, int lo, unsigned span, float m) {
+  float m0 = m, m1 = -INFINITY;
+  if (full) {
+#pragma unroll
+    for (int e = 0; e < 64; e += 4) {
+      m0 = max3(m0, __uint_as_float(sv[e]), __uint_as_float(sv[e + 1]));
+      m1 = max3(m1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
+    }
+  } else {
+#pragma unroll
+    for (int e = 0; e < 64; e += 2) {
+      const float a = static_cast<unsigned>(base + e - lo) < span ? __uint_as_float(sv[e]) : -INFINITY;
+      const float b = static_cast<unsigned>(base + e + 1 - lo) < span ? __uint_as_float(sv[e + 1]) : -INFINITY;
+      if (e & 2) m1 = max3(m1, a, b); else m0 = max3(m0, a, b);
+    }
+  }
+  return fmaxf(m0, m1);
+}
+
+// P = exp2(S*scale - m) for 64 keys, rounded to bf16 into this row of the
+// swizzled P atom; returns the row sum of the unrounded values.
+SVL_DEVINL float exp_store64(const uint32_t* sv, int base, bool full, int lo, unsigned span, uint64_t sc2,
+                             uint64_t nm2, uint8_t* patom_row, int row) {
+  uint64_t acc0 = 0, acc1 = 0;
+#pragma unroll
+  for (int c8 = 0; c8 < 8; ++c8) {
+    uint32_t pk[4];
+#pragma unroll
+    for (int e2 = 0; e2 < 4; ++e2) {
+      const int e = 8 * c8 + 2 * e2;
+      const uint64_t xv = fma2(f2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), sc2, nm2);
+      float x0 = lo2(xv), x1 = hi2(xv);
+      if (!full) {
+        if (static_cast<unsigned>(base + e - lo) >= span) x0 = -INFINITY;
+        if (static_cast<unsigned>(base + e + 1 - lo) >= span) x1 = -INFINITY;
+      }
+      const float p0 = ex2(x0), p1 = ex2(x1);
+      if (e2 & 1) acc1 = add2(acc1, f2(p0, p1)); else acc0 = add2(acc0, f2(p0, p1));
+      pk[e2] = pack_bf16x2(p0, p1);
+    }
+    // keys base + 8*c8 .. +7: 16-byte chunk c8 of the row, 128-byte swizzle
+    *reinterpret_cast<uint4*>(patom_row + ((c8 ^ (row & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+  }
+  const uint64_t acc = add2(acc0, acc1);
+  return lo2(acc) + hi2(acc);
+}
+
+// TMEM columns: block x holds S at 256*x and O at 256*x + 128.
 template <int DH>
 __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_constant__ AttnTcArgs a) {
   using L = AttnSmem<DH>;
@@ -74,17 +176,17 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    mbar_init(&bar->q_full, 1);
-    mbar_init(&bar->q_empty, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&bar->k_full[i], 1);
-      mbar_init(&bar->k_empty[i], 1);
-      mbar_init(&bar->v_full[i], 1);
-      mbar_init(&bar->v_empty[i], 1);
+      mbar_init(&bar->q_full[i], 1);
+      mbar_init(&bar->q_empty[i], 1);
       mbar_init(&bar->s_full[i], 1);
-      mbar_init(&bar->o_full[i], 1);
+      mbar_init(&bar->p_full[i], 128);
+      mbar_init(&bar->pv_done[i], 1);
     }
-    mbar_init(&bar->p_full, 128);
+    for (int i = 0; i < kRing; ++i) {
+      mbar_init(&bar->r_full[i], 1);
+      mbar_init(&bar->r_empty[i], 1);
+    }
     *abort = 0;
     fence_barrier_init();
     fence_proxy_async();
@@ -100,33 +202,51 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
   pdl_trigger();
   pdl_wait();
   const int n_items = min(*a.count, a.cap);
+  const int group = a.A / a.Akv;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      int g = 0, li = 0;
+      int base = 0, nq[2] = {0, 0};
       bool ok = true;
-      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x, ++li) {
-        const int4 it = a.items[i];
-        const int h = it.w, kvh = h / (a.A / a.Akv), key_base = it.z & ~7, nt = n_key_tiles(it);
-        if (!mbar_wait(&bar->q_empty, (li & 1) ^ 1, abort)) { ok = false; break; }
-        mbar_arrive_expect_tx(&bar->q_full, L::kQ);
+      int4 it = blockIdx.x < n_items ? a.items[blockIdx.x] : make_int4(0, 0, 0, 0);
+      auto load_q = [&](int x, const int4& cur) -> bool {
+        if (!mbar_wait(&bar->q_empty[x], (nq[x] & 1) ^ 1, abort)) return false;
+        ++nq[x];
+        mbar_arrive_expect_tx(&bar->q_full[x], L::kQ);
         for (int at = 0; at < DH / 64; ++at)
-          tma_load_2d(sm + L::q + at * 128 * 128, &a.mapQ, &bar->q_full, h * DH + at * 64, it.x);
-        for (int j = 0; j < nt; ++j, ++g) {
-          const int s = g & 1;
-          const uint32_t ph = ((g >> 1) & 1) ^ 1;
-          const int key0 = key_base + j * kKeyTile;
-          if (!mbar_wait(&bar->k_empty[s], ph, abort)) { ok = false; break; }
-          mbar_arrive_expect_tx(&bar->k_full[s], L::kK);
-          for (int at = 0; at < DH / 64; ++at)
-            tma_load_2d(sm + L::k0 + s * L::kK + at * kKeyTile * 128, &a.mapK, &bar->k_full[s], kvh * DH + at * 64,
-                        key0);
-          if (!mbar_wait(&bar->v_empty[s], ph, abort)) { ok = false; break; }
-          mbar_arrive_expect_tx(&bar->v_full[s], L::kV);
-          for (int at = 0; at < 2; ++at)
-            tma_load_2d(sm + L::v0 + s * L::kV + at * DH * 128, &a.mapVt, &bar->v_full[s], key0 + at * 64, kvh * DH);
+          tma_load_2d(sm + L::q0 + x * L::kQ + at * L::kAtom, &a.mapQ, &bar->q_full[x], cur.w * DH + at * 64,
+                      cur.x + 128 * x);
+        return true;
+      };
+      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
+        const int4 cur = it;
+        if (i + gridDim.x < n_items) it = a.items[i + gridDim.x];  // next item, loaded early
+        const ItemTiles nt = item_tiles(cur);
+        const int kvh = cur.w / group, key_base = cur.z & ~7;
+        ok = load_q(0, cur);
+        // block B's Q after the first two key tiles: its buffer frees only
+        // when the previous item's last S of block B is done
+        const int p_qb = min(1, 2 * nt.n - 1);
+        for (int p = 0; p < 2 * nt.n && ok; ++p) {
+          // position p of this item: K(j) or V(m), see pos_k / pos_v
+          const bool is_k = p == 0 || (p & 1 && p < 2 * nt.n - 1);
+          const int tile = is_k ? (p + 1) >> 1 : (p == 2 * nt.n - 1 ? nt.n - 1 : (p >> 1) - 1);
+          const int g = base + p, st = g % kRing;
+          if (!mbar_wait(&bar->r_empty[st], ((g / kRing) & 1) ^ 1, abort)) { ok = false; break; }
+          mbar_arrive_expect_tx(&bar->r_full[st], L::kStage);
+          uint8_t* dst = sm + L::r0 + st * L::kStage;
+          const int key0 = key_base + tile * kKeyTile;
+          if (is_k) {
+            for (int at = 0; at < DH / 64; ++at)
+              tma_load_2d(dst + at * L::kAtom, &a.mapK, &bar->r_full[st], kvh * DH + at * 64, key0);
+          } else {
+            for (int h2 = 0; h2 < 2; ++h2)
+              tma_load_2d(dst + h2 * L::kVAtom, &a.mapVt, &bar->r_full[st], key0 + 64 * h2, kvh * DH);
+          }
+          if (p == p_qb && nt.nb > 0) ok = load_q(1, cur);
         }
+        base += 2 * nt.n;
       }
       if (!ok) attn_abort(abort, a.status);
     }
@@ -134,167 +254,197 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       const uint32_t id_s = idesc_bf16_f32(128, kKeyTile), id_o = idesc_bf16_f32(128, DH);
-      const uint32_t sq = smem_u32(sm + L::q);
-      int g = 0, li = 0;
+      int base = 0, nq[2] = {0, 0}, np[2] = {0, 0};
       bool ok = true;
-      // S(gg) = Q K(gg)^T into S buffer gg&1; frees the K stage when done
-      auto issue_s = [&](int gg, bool last_of_item) -> bool {
-        const int s = gg & 1;
-        if (!mbar_wait(&bar->k_full[s], (gg >> 1) & 1, abort)) return false;
+      auto ring_wait = [&](int g) -> bool {
+        if (!mbar_wait(&bar->r_full[g % kRing], (g / kRing) & 1, abort)) return false;
         tc_fence_after();
-        const uint32_t sk = smem_u32(sm + L::k0 + s * L::kK);
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * (128 * 128) + (kk & 3) * 32;
-          const uint32_t offk = (kk >> 2) * (kKeyTile * 128) + (kk & 3) * 32;
-          tc_mma_bf16(tmem + s * 128, smem_desc_sw128(sq + off), smem_desc_sw128(sk + offk), id_s, kk > 0);
-        }
-        tc_commit(&bar->s_full[s]);
-        tc_commit(&bar->k_empty[s]);
-        if (last_of_item) tc_commit(&bar->q_empty);  // Q may be replaced once these finish
         return true;
       };
-      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x, ++li) {
-        const int nt = n_key_tiles(a.items[i]);
-        if (!mbar_wait(&bar->q_full, li & 1, abort)) { ok = false; break; }
-        tc_fence_after();
-        ok = issue_s(g, nt == 1) && (nt < 2 || issue_s(g + 1, nt == 2));
-        for (int j = 0; j < nt && ok; ++j) {
-          const int gj = g + j, s = gj & 1;
-          if (!mbar_wait(&bar->p_full, gj & 1, abort) || !mbar_wait(&bar->v_full[s], (gj >> 1) & 1, abort)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t sp = smem_u32(sm + L::p0 + s * L::kP);
-          const uint32_t sv = smem_u32(sm + L::v0 + s * L::kV);
+      auto mma_s = [&](int x, int g) {
+        // descriptors advance by (byte offset >> 4) in their start-address field
+        const uint64_t dq = smem_desc_sw128(smem_u32(sm + L::q0 + x * L::kQ));
+        const uint64_t dk = smem_desc_sw128(smem_u32(sm + L::r0 + (g % kRing) * L::kStage));
 #pragma unroll
-          for (int kk = 0; kk < kKeyTile / 16; ++kk) {
-            const uint32_t offp = (kk >> 2) * (128 * 128) + (kk & 3) * 32;
-            const uint32_t offv = (kk >> 2) * (DH * 128) + (kk & 3) * 32;
-            tc_mma_bf16(tmem + 256 + s * 128, smem_desc_sw128(sp + offp), smem_desc_sw128(sv + offv), id_o, kk > 0);
-          }
-          tc_commit(&bar->o_full[s]);
-          tc_commit(&bar->v_empty[s]);
-          if (j + 2 < nt) ok = issue_s(gj + 2, j + 2 == nt - 1);
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint32_t off = ((kk >> 2) * L::kAtom + (kk & 3) * 32) >> 4;
+          tc_mma_bf16(tmem + 256 * x, dq + off, dk + off, id_s, kk > 0);
         }
-        g += nt;
+        tc_commit(&bar->s_full[x]);
+      };
+      auto mma_pv = [&](int x, int g, bool acc) {
+        const uint64_t dp = smem_desc_sw128(smem_u32(sm + L::p0 + x * L::kP));
+        const uint64_t dv = smem_desc_sw128(smem_u32(sm + L::r0 + (g % kRing) * L::kStage));
+#pragma unroll
+        for (int kk = 0; kk < kKeyTile / 16; ++kk) {
+          const uint32_t offp = ((kk >> 2) * L::kAtom + (kk & 3) * 32) >> 4;
+          const uint32_t offv = ((kk >> 2) * L::kVAtom + (kk & 3) * 32) >> 4;
+          tc_mma_bf16(tmem + 256 * x + 128, dp + offp, dv + offv, id_o, (acc || kk > 0) ? 1u : 0u);
+        }
+        tc_commit(&bar->pv_done[x]);
+      };
+      int4 it = blockIdx.x < n_items ? a.items[blockIdx.x] : make_int4(0, 0, 0, 0);
+      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
+        const ItemTiles nt = item_tiles(it);
+        if (i + gridDim.x < n_items) it = a.items[i + gridDim.x];  // next item, loaded early
+        const int ntx[2] = {nt.na, nt.nb};
+        // round 0: S of tile 0 for both blocks
+        ok = ring_wait(base + pos_k(0));
+#pragma unroll
+        for (int x = 0; x < 2; ++x) {
+          if (ok && ntx[x] > 0) {
+            ok = mbar_wait(&bar->q_full[x], nq[x] & 1, abort);
+            if (ok) {
+              tc_fence_after();
+              mma_s(x, base + pos_k(0));
+              if (ntx[x] == 1) tc_commit(&bar->q_empty[x]);
+              ++nq[x];
+            }
+          }
+        }
+        if (!ok) break;
+        tc_commit(&bar->r_empty[(base + pos_k(0)) % kRing]);
+        // rounds 1..n: S of tile j and P V of tile j-1
+        for (int j = 1; j <= nt.n && ok; ++j) {
+          const int gk = base + pos_k(j), gv = base + pos_v(j - 1, nt.n);
+          bool k_ready = false, v_ready = false;
+#pragma unroll
+          for (int x = 0; x < 2; ++x) {
+            if (ok && j - 1 < ntx[x]) {
+              ok = mbar_wait(&bar->p_full[x], np[x] & 1, abort);
+              ++np[x];
+              if (ok) tc_fence_after();
+              if (ok && j < ntx[x]) {
+                if (!k_ready) ok = k_ready = ring_wait(gk);
+                if (ok) {
+                  mma_s(x, gk);
+                  if (j == ntx[x] - 1) tc_commit(&bar->q_empty[x]);
+                }
+              }
+              if (ok && !v_ready) ok = v_ready = ring_wait(gv);
+              if (ok) mma_pv(x, gv, j > 1);
+            }
+          }
+          if (!ok) break;
+          if (j < nt.n) tc_commit(&bar->r_empty[gk % kRing]);
+          tc_commit(&bar->r_empty[gv % kRing]);
+        }
+        base += 2 * nt.n;
       }
       if (!ok) attn_abort(abort, a.status);
     }
   } else {
     // ------------------------------------------------------------ softmax + output
-    const int q = warp & 3;
+    const int x = (warp - 2) >> 2;  // block: 0 = A, 1 = B
+    const int q = warp & 3;         // TMEM lane quarter this warp may access
     const int row = q * 32 + lane;  // query row within the block = TMEM lane
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const uint32_t t_s = tmem + 256 * x + lane_off, t_o = tmem + 256 * x + 128 + lane_off;
+    uint8_t* prow = sm + L::p0 + x * L::kP + row * 128;
     const float sc = a.scale_log2;
-    int g = 0;
+    const uint64_t sc2 = f2(sc, sc);
+    int t = 0;  // tiles of this block so far (barrier phases)
     bool ok = true;
+    auto wait_all = [&](uint64_t* b, uint32_t parity) -> bool {
+      const bool got = mbar_wait(b, parity, abort);
+      __syncwarp();
+      return __all_sync(0xffffffffu, got);
+    };
     for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
-      const int4 it = a.items[i];
-      const int qg = it.x + row;  // global query row
-      const int key_base = it.z & ~7, nt = n_key_tiles(it);
-      float o[DH];
-#pragma unroll
-      for (int d = 0; d < DH; ++d) o[d] = 0.f;
+      const int4 cur = a.items[i];
+      const ItemTiles ntt = item_tiles(cur);
+      const int nt = x == 0 ? ntt.na : ntt.nb;
+      if (nt == 0) continue;
+      const int qb0 = cur.x + 128 * x;  // first query of this block
+      const int qg = qb0 + row;         // global query row
+      const int key_base = cur.z & ~7;
       float m_run = -INFINITY, l_run = 0.f;
-      float cr0 = 0.f, cr1 = 0.f;  // correction factors of the (even, odd) tiles whose P V is pending
-
-      // O = O * corr(t) + (P V)(t), once the MMA for tile t has finished
-      auto fold = [&](int t) -> bool {
-        const int s = t & 1;
-        const bool got = mbar_wait(&bar->o_full[s], (t >> 1) & 1, abort);
-        __syncwarp();
-        if (!__all_sync(0xffffffffu, got)) return false;
+      for (int j = 0; j < nt; ++j, ++t) {
+        if (!wait_all(&bar->s_full[x], t & 1)) { ok = false; break; }
         tc_fence_after();
-        const float c = ((t - g) & 1) ? cr1 : cr0;
-        float v[32];
-#pragma unroll
-        for (int cc = 0; cc < DH; cc += 32) {
-          tmem_ld32(tmem + 256 + s * 128 + lane_off + cc, v);
-#pragma unroll
-          for (int e = 0; e < 32; ++e) o[cc + e] = fmaf(o[cc + e], c, v[e]);
-        }
-        tc_fence_before();
-        return true;
-      };
-
-      for (int j = 0; j < nt; ++j) {
-        const int gj = g + j, s = gj & 1;
-        if (j >= 2 && !fold(gj - 2)) { ok = false; break; }
-        const bool got = mbar_wait(&bar->s_full[s], (gj >> 1) & 1, abort);
-        __syncwarp();
-        if (!__all_sync(0xffffffffu, got)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t ts = tmem + s * 128 + lane_off;
-        const int kbase = key_base + j * kKeyTile;
         // keys kbase + [lo, hi) are valid for this row; a tile wholly inside
         // the sample and before the block's first query needs no mask
-        const bool full = kbase >= it.z && kbase + kKeyTile - 1 <= it.x;
-        const int lo = full ? 0 : max(it.z - kbase, 0);
+        const int kbase = key_base + j * kKeyTile;
+        const bool full = kbase >= cur.z && kbase + kKeyTile - 1 <= qb0;
+        const int lo = full ? 0 : max(cur.z - kbase, 0);
         // (a row that precedes the whole tile has no valid key: empty range)
-        const int hi = full ? kKeyTile : max(min(min(qg + 1, it.y) - kbase, kKeyTile), lo);
-        float v[32];
-        float mx = -INFINITY;
-        for (int c = 0; c < kKeyTile; c += 32) {
-          tmem_ld32(ts + c, v);
-          if (full) {
-#pragma unroll
-            for (int e = 0; e < 32; ++e) mx = fmaxf(mx, v[e]);
-          } else {
-#pragma unroll
-            for (int e = 0; e < 32; ++e)
-              if (static_cast<unsigned>(c + e - lo) < static_cast<unsigned>(hi - lo)) mx = fmaxf(mx, v[e]);
-          }
-        }
-        const float m_new = fmaxf(m_run, mx * sc);
-        const float mref = (m_new == -INFINITY) ? 0.f : m_new;
-        const float corr = (m_run == -INFINITY) ? 0.f : ex2(m_run - mref);
-        m_run = m_new;
-        if (j & 1) cr1 = corr; else cr0 = corr;
-        uint8_t* prow = sm + L::p0 + s * L::kP + row * 128;
-        float rs = 0.f;
-        for (int c = 0; c < kKeyTile; c += 32) {
-          tmem_ld32(ts + c, v);
-          uint32_t pk[16];
-#pragma unroll
-          for (int e = 0; e < 32; e += 2) {
-            float x0 = fmaf(v[e], sc, -mref), x1 = fmaf(v[e + 1], sc, -mref);
-            if (!full) {
-              if (static_cast<unsigned>(c + e - lo) >= static_cast<unsigned>(hi - lo)) x0 = -INFINITY;
-              if (static_cast<unsigned>(c + e + 1 - lo) >= static_cast<unsigned>(hi - lo)) x1 = -INFINITY;
+        const int hi = full ? kKeyTile : max(min(min(qg + 1, cur.y) - kbase, kKeyTile), lo);
+        const unsigned span = static_cast<unsigned>(hi - lo);
+        // row max over both halves of the tile; the second half stays in
+        // registers, the first is read again for the exponentials
+        uint32_t sv[64];
+        tmem_ld32_async(t_s, sv);
+        tmem_ld32_async(t_s + 32, sv + 32);
+        tmem_ld_wait32(sv);
+        tmem_ld_wait32(sv + 32);
+        float mx = row_max64(sv, 0, full, lo, span, -INFINITY);
+        tmem_ld32_async(t_s + 64, sv);
+        tmem_ld32_async(t_s + 96, sv + 32);
+        tmem_ld_wait32(sv);
+        tmem_ld_wait32(sv + 32);
+        mx = row_max64(sv, 64, full, lo, span, mx);
+        const float m_tile = mx * sc;
+        if (j == 0) {
+          m_run = m_tile;
+        } else {
+          // P V of the previous tile must be done: it reads the P buffer and
+          // accumulates into O
+          if (!wait_all(&bar->pv_done[x], (t - 1) & 1)) { ok = false; break; }
+          tc_fence_after();
+          const bool need = m_tile > m_run + kRescaleLog2;
+          if (__any_sync(0xffffffffu, need)) {
+            const float corr = need ? ex2(m_run - m_tile) : 1.f;
+            if (need) {
+              l_run *= corr;
+              m_run = m_tile;
             }
-            const float p0 = ex2(x0), p1 = ex2(x1);
-            rs += p0 + p1;
-            pk[e >> 1] = pack_bf16x2(p0, p1);
-          }
-          // keys c..c+31: atom c/64, 16-byte chunks (c%64)/8 .. +3, 128-byte swizzle
-          const int atom = c >> 6, ch0 = (c & 63) >> 3;
-          uint8_t* base = prow + atom * (128 * 128);
+#pragma unroll 1
+            for (int cc = 0; cc < DH; cc += 32) {
+              uint32_t ov[32];
+              tmem_ld32_async(t_o + cc, ov);
+              tmem_ld_wait32(ov);
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const int ch = (ch0 + u) ^ (row & 7);
-            *reinterpret_cast<uint4*>(base + (ch << 4)) =
-                make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+              for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
+              tmem_st32(t_o + cc, ov);
+            }
+            tmem_st_wait();
           }
         }
-        l_run = l_run * corr + rs;
+        const float mref = (m_run == -INFINITY) ? 0.f : m_run;
+        const uint64_t nm2 = f2(-mref, -mref);
+        float rs = exp_store64(sv, 64, full, lo, span, sc2, nm2, prow + L::kAtom, row);
+        tmem_ld32_async(t_s, sv);
+        tmem_ld32_async(t_s + 32, sv + 32);
+        tmem_ld_wait32(sv);
+        tmem_ld_wait32(sv + 32);
+        rs += exp_store64(sv, 0, full, lo, span, sc2, nm2, prow, row);
+        l_run += rs;
         fence_proxy_async();  // P written by threads, read by the tensor core
         tc_fence_before();
-        mbar_arrive(&bar->p_full);
+        mbar_arrive(&bar->p_full[x]);
       }
-      if (ok && nt >= 2) ok = fold(g + nt - 2);
-      if (ok) ok = fold(g + nt - 1);
-      g += nt;
       if (!ok) break;
-      if (qg < it.y) {
-        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-        uint4* dst = reinterpret_cast<uint4*>(a.O + static_cast<size_t>(qg) * a.ldo + static_cast<size_t>(it.w) * DH);
+      // block done: O of the last P V, divided by the row sum
+      if (!wait_all(&bar->pv_done[x], (t - 1) & 1)) { ok = false; break; }
+      tc_fence_after();
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+      uint4* dst = reinterpret_cast<uint4*>(a.O + static_cast<size_t>(qg) * a.ldo + static_cast<size_t>(cur.w) * DH);
+#pragma unroll 1
+      for (int cc = 0; cc < DH; cc += 32) {
+        uint32_t ov[32];
+        tmem_ld32_async(t_o + cc, ov);
+        tmem_ld_wait32(ov);
+        if (qg < cur.y) {
 #pragma unroll
-        for (int d = 0; d < DH; d += 8)
-          dst[d / 8] = make_uint4(pack_bf16x2(o[d] * inv, o[d + 1] * inv), pack_bf16x2(o[d + 2] * inv, o[d + 3] * inv),
-                                  pack_bf16x2(o[d + 4] * inv, o[d + 5] * inv), pack_bf16x2(o[d + 6] * inv, o[d + 7] * inv));
+          for (int d = 0; d < 32; d += 8)
+            dst[(cc + d) / 8] = make_uint4(
+                pack_bf16x2(__uint_as_float(ov[d]) * inv, __uint_as_float(ov[d + 1]) * inv),
+                pack_bf16x2(__uint_as_float(ov[d + 2]) * inv, __uint_as_float(ov[d + 3]) * inv),
+                pack_bf16x2(__uint_as_float(ov[d + 4]) * inv, __uint_as_float(ov[d + 5]) * inv),
+                pack_bf16x2(__uint_as_float(ov[d + 6]) * inv, __uint_as_float(ov[d + 7]) * inv));
+        }
       }
+      tc_fence_before();  // O read before the next item's first P V overwrites it
     }
     if (!ok) attn_abort(abort, a.status);
   }

@@ -10,7 +10,7 @@
 //    consecutive active groups), gate/up tiles only active FFN channels;
 //    O and down tiles carry the mask so their K loop visits only active
 //    groups' rows of W_O / W_down;
-//  * attention items are (sample, active head, 64-query block).
+//  * attention items are (sample, active head, block of kAttnQ queries).
 #include "kernels.cuh"
 
 namespace svl {
@@ -172,7 +172,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   }
   if (tid == 0) a.gu_count[l] = min(off, a.gu_cap);
 
-  // ---- attention items: per active sample, 64-query blocks (latest first), active heads
+  // ---- attention items: per active sample, blocks of kAttnQ queries (latest first), active heads
   off = 0;
   int4* items = a.attn_items + static_cast<size_t>(l) * a.attn_cap;
   const int hpg = a.A / G;

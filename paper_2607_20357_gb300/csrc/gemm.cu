@@ -354,13 +354,26 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
     if (rv)
       while (b + 1 < p.n_seg && p.seg_off[b + 1] <= row) ++b;
     const int H = ti.ncols;
-    const float* eb = p.e_b + static_cast<size_t>(b) * H;
+    const float4* eb = reinterpret_cast<const float4*>(p.e_b + static_cast<size_t>(b) * H);
+    const uint4* w2v = reinterpret_cast<const uint4*>(p.w2);
     float z = 0.f;
     for (int c = 0; c < H; c += 32) {
       tmem_ld32(taddr + c, v);
+      // 32 hidden units: e_b as 8 float4, w2 as 4 x 8 bf16 (H is a multiple of 16)
+      const int n = min(32, H - c);
 #pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (c + j < H) z += __bfloat162float(p.w2[c + j]) * silu_f(v[j] + eb[c + j]);
+      for (int q = 0; q < 4; ++q) {
+        if (q * 8 >= n) break;
+        const uint4 wq = w2v[(c >> 3) + q];
+        const float4 e0 = eb[(c >> 2) + 2 * q], e1 = eb[(c >> 2) + 2 * q + 1];
+        const float2 w0 = unpack_bf16x2(wq.x), w1 = unpack_bf16x2(wq.y), w2_ = unpack_bf16x2(wq.z),
+                     w3 = unpack_bf16x2(wq.w);
+        const int j = 8 * q;
+        z += w0.x * silu_f(v[j] + e0.x) + w0.y * silu_f(v[j + 1] + e0.y);
+        z += w1.x * silu_f(v[j + 2] + e0.z) + w1.y * silu_f(v[j + 3] + e0.w);
+        z += w2_.x * silu_f(v[j + 4] + e1.x) + w2_.y * silu_f(v[j + 5] + e1.y);
+        z += w3.x * silu_f(v[j + 6] + e1.z) + w3.y * silu_f(v[j + 7] + e1.w);
+      }
     }
     if (rv) {
       z += p.c2;
