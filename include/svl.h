@@ -62,7 +62,8 @@ typedef enum svl_status {
  * vision feature width; H the token-controller hidden width.
  * Supported: D = A * d_head with d_head in {64, 128}; A % G == 0 and
  * A_kv % G == 0 (each group owns whole KV heads); (D_int / G) % 64 == 0;
- * (A / G) * d_head % 64 == 0; D, C_v, proj_hidden multiples of 64;
+ * (A / G) * d_head % 64 == 0; D a multiple of 128; C_v, proj_hidden
+ * multiples of 64;
  * H in {16, 32, ..., 128}; proj_hidden == 0 requires C_v == D. */
 typedef struct svl_model_desc {
   int32_t n_layers;     /* L */
@@ -96,7 +97,10 @@ typedef struct svl_layer_weights {
 
 /* All weights: device bf16 unless noted, 16-byte aligned. The model keeps
  * these pointers (it does not copy them): the caller keeps the memory alive
- * until svl_model_destroy(). */
+ * until svl_model_destroy(). One exception: RMSNorm is computed inside the
+ * GEMMs that follow it, so a layer whose attn_norm (ffn_norm) gains are not
+ * all exactly 1 gets model-owned copies of W_q, W_k, W_v (W_g, W_u) with the
+ * gains folded into their columns, made once by svl_model_create. */
 typedef struct svl_weights {
   const void* ctrl_w1;    /* [H, C_v]  token scorer, first layer */
   const void* ctrl_w2;    /* [H]       token scorer, output weights */

@@ -23,6 +23,9 @@ struct svl_model {
   float2* rope_cs = nullptr;
   // B-operand tensor maps of the weights: per layer q, k, v, o, g, u, d
   std::vector<CUtensorMap> tm_layer;
+  // norm gains folded into the projections after them (allocated only for
+  // layers whose gains are not all ones): per layer q, k, v, g, u or nullptr
+  std::vector<void*> folded;
   CUtensorMap tm_ctrl_w1, tm_proj_w1, tm_proj_w2, tm_lm_head;
   // kernel timing (svl_profile_start / svl_profile_stop)
   bool prof = false;
@@ -80,7 +83,8 @@ struct PackLayout {
 struct PreLayout {
   int64_t t_cap, t_pad;
   int n_pad, mt_max, qkv_cap, o_cap, gu_cap, dn_cap, attn_cap;
-  size_t xn, q, k, v, ao, hmid, yl, act, seg, qkv, o, gu, dn, attn, counts, total;
+  int ss_slots;
+  size_t xn, q, k, v, ao, hmid, yl, ss_a, ss_b, act, seg, qkv, o, gu, dn, attn, counts, total;
 };
 
 struct Bump {
@@ -139,6 +143,11 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   L.ao = b.take(2 * t_cap * hq);
   L.hmid = b.take(2 * t_cap * d.d_ffn);
   L.yl = b.take(2 * static_cast<size_t>(L.n_pad) * d.d_model);
+  // partial sums of squares of the residual stream, [D/128][t_pad] each: A
+  // feeds the attention input norm, B the MLP input norm
+  L.ss_slots = d.d_model / 128;
+  L.ss_a = b.take(sizeof(float) * L.ss_slots * L.t_pad);
+  L.ss_b = b.take(sizeof(float) * L.ss_slots * L.t_pad);
   const size_t nl = d.n_layers;
   L.act = b.take(nl * B);
   L.seg = b.take(sizeof(int4) * nl * B);
@@ -280,7 +289,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   if (G > 8 || d.n_heads % G || d.n_kv_heads % G || d.n_heads % d.n_kv_heads) return SVL_ERR_UNSUPPORTED;
   if ((d.d_ffn / G) % 64 || d.d_ffn % G) return SVL_ERR_UNSUPPORTED;
   if (((d.n_heads / G) * dh) % 64) return SVL_ERR_UNSUPPORTED;
-  if (d.d_model % 64 || d.c_vis % 64 || d.proj_hidden % 64) return SVL_ERR_UNSUPPORTED;
+  if (d.d_model % 128 || d.c_vis % 64 || d.proj_hidden % 64) return SVL_ERR_UNSUPPORTED;
   if (d.h_ctrl % 16 || d.h_ctrl > 128) return SVL_ERR_UNSUPPORTED;
   if (d.proj_hidden == 0 && d.c_vis != d.d_model) return SVL_ERR_UNSUPPORTED;
   // Eq. 8 times G must stay exact in double precision at the longest sequence
@@ -306,13 +315,57 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
   const int64_t dkv = static_cast<int64_t>(d.n_kv_heads) * dh, hq = static_cast<int64_t>(d.n_heads) * dh;
   bool ok = true;
+  for (int l = 0; l < d.n_layers && ok; ++l) {
+    const svl_layer_weights& lw = m->layers[l];
+    ok = lw.wq && lw.wk && lw.wv && lw.wo && lw.wg && lw.wu && lw.wd && lw.attn_norm && lw.ffn_norm;
+  }
+  if (!ok) {
+    delete m;
+    return SVL_ERR_INVALID_ARG;
+  }
+  // RMSNorm runs fused into the GEMMs after it (x / rms(x) scales the
+  // accumulator rows), so each norm gain is folded into the columns of the
+  // projections it feeds: W' = W diag(gain). Layers whose gains are exactly 1
+  // keep the caller's weights.
+  {
+    int* flags = nullptr;
+    std::vector<int> host(2 * static_cast<size_t>(d.n_layers), 1);
+    ok = cudaMalloc(&flags, sizeof(int) * host.size()) == cudaSuccess &&
+         cudaMemcpy(flags, host.data(), sizeof(int) * host.size(), cudaMemcpyHostToDevice) == cudaSuccess;
+    for (int l = 0; l < d.n_layers && ok; ++l) {
+      ok = gain_is_one(static_cast<const __nv_bfloat16*>(m->layers[l].attn_norm), d.d_model, flags + 2 * l, 0) ==
+               cudaSuccess &&
+           gain_is_one(static_cast<const __nv_bfloat16*>(m->layers[l].ffn_norm), d.d_model, flags + 2 * l + 1, 0) ==
+               cudaSuccess;
+    }
+    ok = ok && cudaMemcpy(host.data(), flags, sizeof(int) * host.size(), cudaMemcpyDeviceToHost) == cudaSuccess;
+    if (flags) cudaFree(flags);
+    m->folded.assign(static_cast<size_t>(d.n_layers) * 5, nullptr);
+    for (int l = 0; l < d.n_layers && ok; ++l) {
+      svl_layer_weights& lw = m->layers[l];
+      const void** src[5] = {&lw.wq, &lw.wk, &lw.wv, &lw.wg, &lw.wu};
+      const int64_t rows[5] = {hq, dkv, dkv, d.d_ffn, d.d_ffn};
+      for (int i = 0; i < 5 && ok; ++i) {
+        const bool attn = i < 3;
+        if (host[2 * l + (attn ? 0 : 1)]) continue;
+        const void* gain = attn ? lw.attn_norm : lw.ffn_norm;
+        void* dst = nullptr;
+        ok = cudaMalloc(&dst, 2 * static_cast<size_t>(rows[i]) * d.d_model) == cudaSuccess;
+        if (!ok) break;
+        m->folded[static_cast<size_t>(l) * 5 + i] = dst;
+        ok = fold_gain(static_cast<const __nv_bfloat16*>(*src[i]), static_cast<const __nv_bfloat16*>(gain),
+                       static_cast<__nv_bfloat16*>(dst), rows[i], d.d_model, 0) == cudaSuccess;
+        *src[i] = dst;
+      }
+    }
+    if (!ok || cudaDeviceSynchronize() != cudaSuccess) {
+      svl_model_destroy(m);
+      return SVL_ERR_CUDA;
+    }
+  }
   m->tm_layer.resize(static_cast<size_t>(d.n_layers) * 7);
   for (int l = 0; l < d.n_layers && ok; ++l) {
     const svl_layer_weights& lw = m->layers[l];
-    if (!lw.wq || !lw.wk || !lw.wv || !lw.wo || !lw.wg || !lw.wu || !lw.wd || !lw.attn_norm || !lw.ffn_norm) {
-      ok = false;
-      break;
-    }
     CUtensorMap* t = &m->tm_layer[static_cast<size_t>(l) * 7];
     ok = make_map(t + 0, lw.wq, hq, d.d_model) && make_map(t + 1, lw.wk, dkv, d.d_model) &&
          make_map(t + 2, lw.wv, dkv, d.d_model) && make_map(t + 3, lw.wo, d.d_model, hq) &&
@@ -325,7 +378,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
     ok = make_map(&m->tm_proj_w1, w->proj_w1, d.proj_hidden, d.c_vis) &&
          make_map(&m->tm_proj_w2, w->proj_w2, d.d_model, d.proj_hidden);
   if (!ok) {
-    delete m;
+    svl_model_destroy(m);
     return SVL_ERR_INVALID_ARG;
   }
   if (cudaMalloc(&m->d_status, sizeof(uint32_t)) != cudaSuccess ||
@@ -349,6 +402,8 @@ void svl_model_destroy(svl_model* m) {
   for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
   if (m->d_status) cudaFree(m->d_status);
   if (m->rope_cs) cudaFree(m->rope_cs);
+  for (void* f : m->folded)
+    if (f) cudaFree(f);
   delete m;
 }
 
@@ -584,10 +639,22 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   __nv_bfloat16* vb = at<__nv_bfloat16>(ws, L.v);
   __nv_bfloat16* ao = at<__nv_bfloat16>(ws, L.ao);
   __nv_bfloat16* hm = at<__nv_bfloat16>(ws, L.hmid);
-  CUtensorMap map_xn, map_ao, map_hm;
-  if (!make_map(&map_xn, xn, t_cap, d.d_model) || !make_map(&map_ao, ao, t_cap, hq) ||
-      !make_map(&map_hm, hm, t_cap, d.d_ffn))
+  CUtensorMap map_x, map_xn, map_ao, map_hm;
+  if (!make_map(&map_x, X, t_cap, d.d_model) || !make_map(&map_xn, xn, t_cap, d.d_model) ||
+      !make_map(&map_ao, ao, t_cap, hq) || !make_map(&map_hm, hm, t_cap, d.d_ffn))
     return SVL_ERR_CUDA;
+  // fused RMSNorm: per-row partial sums of squares of X (see GemmParams)
+  float* ss_a = at<float>(ws, L.ss_a);
+  float* ss_b = at<float>(ws, L.ss_b);
+  const int ss_ld = static_cast<int>(L.t_pad);
+  auto set_norm = [&](GemmParams& p, const float* in, float* out) {
+    p.ss_in = in;
+    p.ss_out = out;
+    p.ss_ld = ss_ld;
+    p.ss_slots = L.ss_slots;
+    p.ss_inv_d = 1.f / static_cast<float>(d.d_model);
+    p.ss_eps = d.rms_eps;
+  };
 
   NormArgs na;
   na.t_cap = t_cap;
@@ -616,18 +683,19 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   aa.ldo = hq;
   aa.status = m->d_status;
 
-  for (int l = 0; l < nl; ++l) {
-    const svl_layer_weights& lw = m->layers[l];
-    const CUtensorMap* tm = &m->tm_layer[static_cast<size_t>(l) * 7];
-    na.act = sa.act + static_cast<size_t>(l) * B;
-    na.gain = static_cast<const __nv_bfloat16*>(lw.attn_norm);
-    {
-      Launch L1(m, SVL_TAG_RMSNORM, s);
-      launch_rmsnorm(na, s);
-    }
+  {
+    Launch L1(m, SVL_TAG_RMSNORM, s);
+    launch_norm_init(static_cast<const __nv_bfloat16*>(X), cu_seqlens, B, static_cast<int>(t_cap), d.d_model, ss_a,
+                     ss_ld, L.ss_slots, s);
+  }
 
+  for (int l = 0; l < nl; ++l) {
+    const CUtensorMap* tm = &m->tm_layer[static_cast<size_t>(l) * 7];
+
+    // attention input norm fused into the QKV GEMM (gain folded into W_qkv)
     GemmParams p = base_params(m);
-    p.mapA = map_xn;
+    set_norm(p, ss_a, nullptr);
+    p.mapA = map_x;
     p.mapB[0] = tm[0];
     p.mapB[1] = tm[1];
     p.mapB[2] = tm[2];
@@ -665,16 +733,13 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = hq / d.n_groups;
     p.out[0] = X;
     p.ld[0] = d.d_model;
+    set_norm(p, nullptr, ss_b);  // sums of squares of the updated rows for the MLP norm
     if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s)) != SVL_OK) return st;
 
-    na.gain = static_cast<const __nv_bfloat16*>(lw.ffn_norm);
-    {
-      Launch L1(m, SVL_TAG_RMSNORM, s);
-      launch_rmsnorm(na, s);
-    }
-
+    // MLP input norm fused into the gate/up GEMM (gain folded into W_g, W_u)
     p = base_params(m);
-    p.mapA = map_xn;
+    set_norm(p, ss_b, nullptr);
+    p.mapA = map_x;
     p.mapB[0] = tm[4];
     p.mapB[1] = tm[5];
     p.b_split = 1;
@@ -697,6 +762,7 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = d.d_ffn / d.n_groups;
     p.out[0] = X;
     p.ld[0] = d.d_model;
+    set_norm(p, nullptr, ss_a);  // for the next layer's attention norm
     if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s)) != SVL_OK) return st;
   }
 

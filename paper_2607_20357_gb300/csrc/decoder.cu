@@ -62,7 +62,8 @@ __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const
 // The persistent GEMM runs tiles in waves of num_sms. When the last wave is
 // at most half full, each of its tiles is cut into two half-width tiles
 // (which then still fit in one wave and finish in about half the time).
-// `head` > 0: halves must hold whole heads of that width (RoPE epilogue).
+// `head` > 0: halves must be multiples of that width (whole heads for the
+// RoPE epilogue; 128-column norm slots for the residual epilogue).
 // Runs on one thread after the list is complete; returns the new count.
 __device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head) {
   const int r = count % num_sms;
@@ -146,7 +147,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   }
   __syncthreads();
   if (tid == 0)
-    a.o_count[l] = split_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms, 0);
+    a.o_count[l] = split_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms, 128);
   // ---- down projection: same tiles shape as O
   off = 0;
   for (int s = 0; s < nseg; ++s) {
@@ -157,7 +158,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __syncthreads();
   if (tid == 0)
     a.dn_count[l] = split_tail(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, min(off, a.dn_cap), a.dn_cap,
-                               a.num_sms, 0);
+                               a.num_sms, 128);
   __syncthreads();
 
   // ---- gate/up (N-sparse over active FFN channels, 128 per tile)
@@ -281,6 +282,64 @@ __global__ void final_rows_kernel(NormArgs a, int n_pad) {
     return;
   }
   norm_row(a.X + static_cast<size_t>(r1 - 1) * a.D, a.gain, y, a.D, a.eps, lane);
+}
+
+// Sum of squares of every packed row of X into slot 0 of ss ([slots][ss_ld]),
+// the other slots zeroed: the first layer's fused RMSNorm reads these.
+__global__ void norm_init_kernel(const __nv_bfloat16* X, const int* cu_seqlens, int B, int t_cap, int D, float* ss,
+                                 int ss_ld, int slots) {
+  pdl_trigger();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * (blockDim.x >> 5) + warp;
+  if (r >= cu_seqlens[B] || r >= t_cap) return;
+  const uint4* xv = reinterpret_cast<const uint4*>(X + static_cast<size_t>(r) * D);
+  float acc = 0.f;
+  for (int c = lane; c < D / 8; c += 32) {
+    const uint4 u = xv[c];
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = unpack_bf16x2(w[i]);
+      acc = fmaf(f.x, f.x, fmaf(f.y, f.y, acc));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  for (int i = lane; i < slots; i += 32) ss[static_cast<size_t>(i) * ss_ld + r] = i == 0 ? acc : 0.f;
+}
+
+void launch_norm_init(const __nv_bfloat16* X, const int* cu_seqlens, int B, int t_cap, int D, float* ss, int ss_ld,
+                      int slots, cudaStream_t s) {
+  const int grid = (t_cap + 7) / 8;
+  if (grid > 0) launch_pdl(norm_init_kernel, grid, 256, 0, s, X, cu_seqlens, B, t_cap, D, ss, ss_ld, slots);
+}
+
+// W'[r][c] = W[r][c] * g[c] (a norm gain folded into the projection after it)
+__global__ void fold_gain_kernel(const __nv_bfloat16* W, const __nv_bfloat16* g, __nv_bfloat16* out, int64_t rows,
+                                 int cols) {
+  const int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  if (i >= rows * cols) return;
+  const int c = static_cast<int>(i % cols);
+  out[i] = __float2bfloat16_rn(__bfloat162float(W[i]) * __bfloat162float(g[c]));
+}
+
+// flag = 0 unless every gain is exactly 1
+__global__ void gain_is_one_kernel(const __nv_bfloat16* g, int n, int* flag) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+    if (__bfloat162float(g[i]) != 1.f) *flag = 0;
+}
+
+cudaError_t fold_gain(const __nv_bfloat16* W, const __nv_bfloat16* g, __nv_bfloat16* out, int64_t rows, int cols,
+                      cudaStream_t s) {
+  const int64_t n = rows * cols;
+  fold_gain_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(W, g, out, rows, cols);
+  return cudaGetLastError();
+}
+
+cudaError_t gain_is_one(const __nv_bfloat16* g, int n, int* flag, cudaStream_t s) {
+  gain_is_one_kernel<<<(n + 255) / 256, 256, 0, s>>>(g, n, flag);
+  return cudaGetLastError();
 }
 
 void launch_rmsnorm(const NormArgs& a, cudaStream_t s) {

@@ -204,6 +204,33 @@ SVL_DEVINL void load_bf16(const __nv_bfloat16* src, float* v, int n) {
   }
 }
 
+// 1 / rms of this row of the residual stream, from its partial sums of squares
+SVL_DEVINL float row_rms_scale(const GemmParams& p, int row) {
+  float s = 0.f;
+  for (int i = 0; i < p.ss_slots; ++i) s += p.ss_in[static_cast<size_t>(i) * p.ss_ld + row];
+  return rsqrtf(s * p.ss_inv_d + p.ss_eps);
+}
+
+// store_bf16 that also returns the sum of squares of the rounded values
+SVL_DEVINL float store_bf16_ss(__nv_bfloat16* dst, const float* v, int n /*16 or 32*/) {
+  uint4* d = reinterpret_cast<uint4*>(dst);
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (i * 8 < n) {
+      uint32_t w[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        w[q] = pack_bf16x2(v[8 * i + 2 * q], v[8 * i + 2 * q + 1]);
+        const float2 f = unpack_bf16x2(w[q]);
+        ss = fmaf(f.x, f.x, fmaf(f.y, f.y, ss));
+      }
+      d[i] = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+  }
+  return ss;
+}
+
 template <int KIND>
 SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, bool rv,
                               uint32_t taddr) {
@@ -211,6 +238,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
   if constexpr (KIND == EPI_QKV_ROPE) {
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[ti.mat]);
     const size_t ld = static_cast<size_t>(p.ld[ti.mat]);
+    const float rs = (p.ss_in && rv) ? row_rms_scale(p, row) : 1.f;
     if (ti.mat < 2) {
       const int dh = p.d_head, half = dh / 2;
       int prow = rv ? p.pos[row] : 0;
@@ -228,7 +256,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
               const float2 c = cs[i0 + j];
-              const float x1 = v[j], x2 = w[j];
+              const float x1 = v[j] * rs, x2 = w[j] * rs;
               v[j] = x1 * c.x - x2 * c.y;
               w[j] = x2 * c.x + x1 * c.y;
             }
@@ -246,7 +274,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
         if (rv) {
 #pragma unroll
           for (int j = 0; j < 32; ++j)
-            if (c + j < ti.ncols) out[static_cast<size_t>(ti.n0 + c + j) * ld + row] = __float2bfloat16_rn(v[j]);
+            if (c + j < ti.ncols) out[static_cast<size_t>(ti.n0 + c + j) * ld + row] = __float2bfloat16_rn(v[j] * rs);
         }
       }
     }
@@ -257,6 +285,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
     // residual chunks double-buffered in registers: the load of chunk c+32
     // is in flight while chunk c is added and stored
     uint4 xa[4], xb[4];
+    float hss = 0.f;
     if (rv) {
       const uint4* s0 = reinterpret_cast<const uint4*>(orow);
 #pragma unroll
@@ -281,7 +310,16 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
             v[8 * i + 2 * q + 1] += f.y;
           }
         }
-        store_bf16(orow + c, v, n);
+        if (p.ss_out) {
+          hss += store_bf16_ss(orow + c, v, n);
+          // one partial per 128 columns of the residual stream
+          if (((c + 32) & 127) == 0 || c + 32 >= ti.ncols) {
+            p.ss_out[static_cast<size_t>((ti.n0 + c) >> 7) * p.ss_ld + row] = hss;
+            hss = 0.f;
+          }
+        } else {
+          store_bf16(orow + c, v, n);
+        }
       }
 #pragma unroll
       for (int i = 0; i < 4; ++i) xa[i] = xb[i];
@@ -290,12 +328,13 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
     const size_t ld = static_cast<size_t>(p.ld[0]);
     float u[32];
+    const float rs = (p.ss_in && rv) ? row_rms_scale(p, row) : 1.f;
     for (int c = 0; c < ti.ncols; c += 32) {
       tmem_ld32(taddr + c, v);
       tmem_ld32(taddr + kBHalf + c, u);
       if (rv) {
 #pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * u[j];
+        for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j] * rs) * (u[j] * rs);
         store_bf16(out + static_cast<size_t>(row) * ld + ti.n0 + c, v, min(32, ti.ncols - c));
       }
     }

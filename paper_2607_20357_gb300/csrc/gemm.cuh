@@ -68,6 +68,15 @@ struct GemmParams {
   int n_seg;
   const __nv_bfloat16* w2;
   float c2;
+  // RMSNorm fused into the GEMMs around it: per-row partial sums of squares
+  // of the residual stream, one slot per 128 columns ([slot][row], ss_ld
+  // floats apart). The residual epilogue writes the slots of the columns it
+  // stores (ss_out); the QKV and gate/up epilogues sum a row's ss_slots slots
+  // and scale its accumulator by 1/sqrt(sum/D + eps) (ss_in).
+  const float* ss_in;
+  float* ss_out;
+  int ss_ld, ss_slots;
+  float ss_inv_d, ss_eps;
   uint32_t* status;
 };
 

@@ -86,6 +86,14 @@ struct NormArgs {
 };
 void launch_rmsnorm(const NormArgs& a, cudaStream_t s);
 
+// Fused-RMSNorm support: sums of squares of the packed rows (slot 0), norm
+// gains folded into a projection's columns, and a check for unit gains.
+void launch_norm_init(const __nv_bfloat16* X, const int* cu_seqlens, int B, int t_cap, int D, float* ss, int ss_ld,
+                      int slots, cudaStream_t s);
+cudaError_t fold_gain(const __nv_bfloat16* W, const __nv_bfloat16* g, __nv_bfloat16* out, int64_t rows, int cols,
+                      cudaStream_t s);
+cudaError_t gain_is_one(const __nv_bfloat16* g, int n, int* flag, cudaStream_t s);
+
 // Final norm of each sample's last row into Y[b] (rows B..n_pad-1 zeroed).
 void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s);
 

@@ -12,7 +12,7 @@ import torch
 
 from oracle import smartvl_oracle as O
 from paper_2607_20357_gb300 import svl, synth
-from tests.gpu_common import Case, bar_for, check_selection, gpu_topk_valid, l2_err, rel_err
+from tests.gpu_common import Case, bar_for, check_selection, gpu_topk_valid, l2_err, rel_err, to_device
 
 pytestmark = pytest.mark.gpu
 
@@ -170,4 +170,23 @@ def test_split_tail_llava_one_layer_full_batch():
     case = Case(dims, LLAVA, seed=12, batch=16, budget=0.5)
     errs = _compare_end_to_end(case, case.run())
     assert len(errs) >= 14
+    case.close()
+
+
+def test_norm_gains_folded_tiny():
+    """Non-unit RMSNorm gains: the norm runs inside the GEMM epilogues and the
+    library folds each gain into the columns of the projections it feeds."""
+    case = Case(TINY.dims, TINY, seed=9)
+    case.model.close()
+    g = torch.Generator().manual_seed(99)
+    w = synth.make_weights(TINY.dims, 9)
+    for lw in w["layers"]:
+        for key in ("attn_norm", "ffn_norm"):
+            lw[key] = (0.5 + torch.rand(TINY.dims.d_model, generator=g)).to(torch.bfloat16)
+    case.w_np = O.to_numpy_weights(w)
+    case.w = to_device(w)
+    case.model = svl.GatedPrefill(TINY.dims, case.w, max_seq=8192)
+    errs = _compare_end_to_end(case, case.run())
+    e_h, e_l, e_h16, e_l16 = errs[0]
+    assert e_h16 < 1e-2 and e_l16 < 1e-2, errs
     case.close()
