@@ -83,8 +83,9 @@ struct PackLayout {
 struct PreLayout {
   int64_t t_cap, t_pad;
   int n_pad, mt_max, qkv_cap, o_cap, gu_cap, dn_cap, attn_cap;
-  int ss_slots;
-  size_t xn, q, k, v, ao, hmid, yl, ss_a, ss_b, act, seg, qkv, o, gu, dn, attn, counts, total;
+  int ss_slots, ks_units;
+  size_t xn, q, k, v, ao, hmid, yl, ss_a, ss_b, ks_part, ks_ticket, ks_info, act, seg, qkv, o, gu, dn, attn, counts,
+      total;
 };
 
 struct Bump {
@@ -148,7 +149,13 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   L.ss_slots = d.d_model / 128;
   L.ss_a = b.take(sizeof(float) * L.ss_slots * L.t_pad);
   L.ss_b = b.take(sizeof(float) * L.ss_slots * L.t_pad);
+  // K-split tail of the residual GEMMs: at most 8 shares per tail tile and
+  // 256 shares in all, fp32 128 x 256 each
+  L.ks_units = static_cast<int>(std::min<int64_t>(256, 8LL * L.mt_max * ((d.d_model + 255) / 256)));
+  L.ks_part = b.take(sizeof(float) * static_cast<size_t>(L.ks_units) * kBM * 256);
   const size_t nl = d.n_layers;
+  L.ks_ticket = b.take(sizeof(int) * L.ks_units * 2 * nl);  // per layer and residual GEMM
+  L.ks_info = b.take(sizeof(int) * 8 * nl);
   L.act = b.take(nl * B);
   L.seg = b.take(sizeof(int4) * nl * B);
   L.qkv = b.take(sizeof(int4) * nl * L.qkv_cap);
@@ -627,7 +634,11 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   sa.attn_items = at<int4>(ws, L.attn);
   sa.attn_cap = L.attn_cap;
   sa.attn_count = counts + 4 * nl;
+  sa.ks_info = at<int>(ws, L.ks_info);
+  sa.ks_units = L.ks_units;
   sa.status = m->d_status;
+  int* ks_ticket = at<int>(ws, L.ks_ticket);
+  if (cudaMemsetAsync(ks_ticket, 0, sizeof(int) * L.ks_units * 2 * nl, s) != cudaSuccess) return SVL_ERR_CUDA;
   {
     Launch L1(m, SVL_TAG_SCHEDULE, s);
     launch_schedule(sa, s);
@@ -733,6 +744,9 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = hq / d.n_groups;
     p.out[0] = X;
     p.ld[0] = d.d_model;
+    p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8;
+    p.ks_part = at<float>(ws, L.ks_part);
+    p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
     set_norm(p, nullptr, ss_b);  // sums of squares of the updated rows for the MLP norm
     if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s)) != SVL_OK) return st;
 
@@ -762,6 +776,9 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     p.kgroup = d.d_ffn / d.n_groups;
     p.out[0] = X;
     p.ld[0] = d.d_model;
+    p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8 + 4;
+    p.ks_part = at<float>(ws, L.ks_part);
+    p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;
     set_norm(p, nullptr, ss_a);  // for the next layer's attention norm
     if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s)) != SVL_OK) return st;
   }

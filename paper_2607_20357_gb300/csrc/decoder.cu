@@ -62,8 +62,7 @@ __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const
 // The persistent GEMM runs tiles in waves of num_sms. When the last wave is
 // at most half full, each of its tiles is cut into two half-width tiles
 // (which then still fit in one wave and finish in about half the time).
-// `head` > 0: halves must be multiples of that width (whole heads for the
-// RoPE epilogue; 128-column norm slots for the residual epilogue).
+// `head` > 0: halves must hold whole heads of that width (RoPE epilogue).
 // Runs on one thread after the list is complete; returns the new count.
 __device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head) {
   const int r = count % num_sms;
@@ -79,6 +78,30 @@ __device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head
     ++added;
   }
   return count + added;
+}
+
+// Residual GEMMs (O, down) cut the tiles of a last wave that is at most half
+// full along K instead: each of the r tail tiles is repeated s times (s =
+// num_sms / r, at most 8, within the list capacity and the partial buffer),
+// the copies compute shares of the tile's K blocks side by side in that wave
+// and the last to finish sums them. Full-width tiles keep the tensor core's
+// widest MMAs. Writes {first copy index, r, s} to info; returns the count.
+__device__ int split_k_tail(int4* tiles, int count, int cap, int num_sms, int units, int* info) {
+  info[0] = count;
+  info[1] = 0;
+  info[2] = 1;
+  const int r = count % num_sms;
+  if (r == 0 || 2 * r > num_sms) return count;
+  int sp = min(min(num_sms / r, 8), units / r);
+  sp = min(sp, 1 + (cap - count) / r);
+  if (sp < 2) return count;
+  const int first = count - r;
+  for (int part = 1; part < sp; ++part)
+    for (int i = 0; i < r; ++i) tiles[count + (part - 1) * r + i] = tiles[first + i];
+  info[0] = first;
+  info[1] = r;
+  info[2] = sp;
+  return count + r * (sp - 1);
 }
 
 __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
@@ -147,7 +170,8 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   }
   __syncthreads();
   if (tid == 0)
-    a.o_count[l] = split_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms, 128);
+    a.o_count[l] = split_k_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms,
+                                a.ks_units, a.ks_info + static_cast<size_t>(l) * 8);
   // ---- down projection: same tiles shape as O
   off = 0;
   for (int s = 0; s < nseg; ++s) {
@@ -157,8 +181,8 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   }
   __syncthreads();
   if (tid == 0)
-    a.dn_count[l] = split_tail(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, min(off, a.dn_cap), a.dn_cap,
-                               a.num_sms, 128);
+    a.dn_count[l] = split_k_tail(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, min(off, a.dn_cap), a.dn_cap,
+                                 a.num_sms, a.ks_units, a.ks_info + static_cast<size_t>(l) * 8 + 4);
   __syncthreads();
 
   // ---- gate/up (N-sparse over active FFN channels, 128 per tile)

@@ -18,6 +18,7 @@ namespace svl {
 
 struct TileInfo {
   int m0, m_end, n0, ncols, mat, kmask;
+  int part, nsplit, slot;  // K-split share (nsplit == 1: the whole tile)
   bool valid;
 };
 
@@ -52,7 +53,26 @@ SVL_DEVINL TileInfo get_tile(const GemmParams& p, int t) {
     ti.kmask = 0;
     ti.valid = ti.m0 < mlim && ti.ncols > 0;
   }
+  ti.part = 0;
+  ti.nsplit = 1;
+  ti.slot = 0;
+  if (p.ks_info && t >= p.ks_info[0]) {
+    const int r = p.ks_info[1], sp = p.ks_info[2];
+    if (r > 0 && sp > 1) {
+      const int u = t - p.ks_info[0];
+      ti.slot = u % r;
+      ti.part = u / r;
+      ti.nsplit = sp;
+    }
+  }
   return ti;
+}
+
+// Share [i0, i1) of the tile's active K blocks (all of them unless K-split).
+SVL_DEVINL void k_share(const TileInfo& ti, int nkb, int kgb, int& i0, int& i1) {
+  const int n = ti.kmask ? __popc(ti.kmask) * kgb : nkb;
+  i0 = (n * ti.part) / ti.nsplit;
+  i1 = (n * (ti.part + 1)) / ti.nsplit;
 }
 
 // Walks the K blocks of a tile, skipping the blocks of gated-off groups
@@ -112,7 +132,11 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
     const int y1 = p.b_split ? ti.n0 : ti.n0 + kBHalf;
     const uint32_t bytes = kABytes + halves * kBHalfBytes;
     KWalk w(nkb, kgb, ti.kmask);
-    while (w.next()) {
+    int i0, i1;
+    k_share(ti, nkb, kgb, i0, i1);
+    for (int i = 0; i < i0; ++i) w.next();
+    for (int i = i0; i < i1; ++i) {
+      w.next();
       const int kb = w.kb;
       if (!mbar_wait(&empty[s], ph ^ 1, abort)) {
         set_abort(abort, p.status);
@@ -154,8 +178,9 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
     const uint32_t idesc = idesc_bf16_f32(kBM, n);
     const uint32_t d = tmem + acc * kAccCols;
     uint32_t accumulate = 0;
-    KWalk w(nkb, kgb, ti.kmask);
-    while (w.next()) {
+    int i0, i1;
+    k_share(ti, nkb, kgb, i0, i1);
+    for (int i = i0; i < i1; ++i) {
       if (!mbar_wait(&full[s], ph, abort)) {
         set_abort(abort, p.status);
         return;
@@ -422,9 +447,119 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
   }
 }
 
+// Rendezvous of the four epilogue warps around a K-split ticket.
+struct KsSync {
+  uint64_t* gather;  // 128 arrivals: every row of this share is stored
+  uint64_t* done;    // 1 arrival: every share of the tile is stored (*flag = 1) or a wait gave up (0)
+  volatile int* flag;
+  uint32_t phase;
+};
+
+SVL_DEVINL int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Residual epilogue of one K-split share. The share's accumulator goes to
+// ks_part; once every share of the tile is stored (the shares run side by
+// side in the last wave of the persistent grid, whose CTAs are all resident),
+// this CTA sums all shares in order for its 1/nsplit of the tile's rows, adds
+// them to the residual rows and writes their norm partial sums. Every wait is
+// bounded; returns false on a time-out.
+SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, uint32_t taddr, bool empty, KsSync& ks,
+                            volatile int* abort) {
+  const size_t unit = static_cast<size_t>(ti.slot) * ti.nsplit;
+  float* mine = p.ks_part + ((unit + ti.part) * kBM + lrow) * kAccCols;
+  float v[32];
+  for (int c = 0; c < ti.ncols; c += 32) {
+    if (!empty) {
+      tmem_ld32(taddr + c, v);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = 0.f;
+    }
+    float4* d = reinterpret_cast<float4*>(mine + c);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+  }
+  __threadfence();
+  mbar_arrive(ks.gather);
+  if (threadIdx.x == 2 * 32) {
+    int all = 0;
+    if (mbar_wait(ks.gather, ks.phase, abort)) {
+      int* ticket = p.ks_ticket + ti.slot;
+      atomicAdd(ticket, 1);
+      const long long t0 = clock64();
+      while (true) {
+        if (ld_acquire(ticket) >= ti.nsplit) {
+          all = 1;
+          break;
+        }
+        if (*abort || clock64() - t0 > kWaitCycles) break;
+      }
+    }
+    *ks.flag = all;
+    mbar_arrive(ks.done);
+  }
+  const bool got = mbar_wait(ks.done, ks.phase, abort);
+  ks.phase ^= 1;
+  __syncwarp();
+  if (!__all_sync(0xffffffffu, got) || !*ks.flag) return false;
+  // this share's rows [r0, r1) of the tile; one work item = (row, 128 columns)
+  const int r0 = (kBM * ti.part) / ti.nsplit, r1 = (kBM * (ti.part + 1)) / ti.nsplit;
+  const int nsl = (ti.ncols + 127) / 128;
+  const int items = (r1 - r0) * nsl;
+  const int et = threadIdx.x - 2 * 32;  // 0..127
+  const float* base = p.ks_part + unit * kBM * kAccCols;
+  for (int w = et; w < items; w += 4 * 32) {
+    const int lr = r0 + w / nsl, sl = w % nsl;
+    const int row = ti.m0 + lr;
+    if (row >= ti.m_end) continue;
+    __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out[0]) + static_cast<size_t>(row) * p.ld[0] + ti.n0;
+    float hss = 0.f;
+    for (int c = sl * 128; c < min(ti.ncols, sl * 128 + 128); c += 32) {
+      const int n = min(32, ti.ncols - c);
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = 0.f;
+      for (int q = 0; q < ti.nsplit; ++q) {
+        const float4* src = reinterpret_cast<const float4*>(base + (static_cast<size_t>(q) * kBM + lr) * kAccCols + c);
+        float4 f[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) f[i] = __ldcg(src + i);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          v[4 * i] += f[i].x;
+          v[4 * i + 1] += f[i].y;
+          v[4 * i + 2] += f[i].z;
+          v[4 * i + 3] += f[i].w;
+        }
+      }
+      const uint4* xs = reinterpret_cast<const uint4*>(orow + c);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (i * 8 < n) {
+          const uint4 x = xs[i];
+          const uint32_t wd[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float2 f = unpack_bf16x2(wd[k]);
+            v[8 * i + 2 * k] += f.x;
+            v[8 * i + 2 * k + 1] += f.y;
+          }
+        }
+      }
+      if (p.ss_out) hss += store_bf16_ss(orow + c, v, n);
+      else store_bf16(orow + c, v, n);
+    }
+    if (p.ss_out) p.ss_out[static_cast<size_t>((ti.n0 >> 7) + sl) * p.ss_ld + row] = hss;
+  }
+  return true;
+}
+
 template <int KIND>
 SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem,
-                              volatile int* abort) {
+                              volatile int* abort, KsSync& ks) {
   const int ntiles = num_tiles(p);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;  // TMEM lane quarter this warp may access
@@ -454,7 +589,20 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
     const int row = ti.m0 + q * 32 + lane;
     const bool rv = row < ti.m_end;
     const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
-    epilogue_tile<KIND>(p, ti, row, rv, taddr);
+    if constexpr (KIND == EPI_RESID) {
+      if (ti.nsplit > 1) {
+        int i0, i1;
+        k_share(ti, p.K / kBK, p.kgroup / kBK, i0, i1);
+        if (!ksplit_tile(p, ti, q * 32 + lane, taddr, i0 == i1, ks, abort)) {
+          set_abort(abort, p.status);
+          return;
+        }
+      } else {
+        epilogue_tile<KIND>(p, ti, row, rv, taddr);
+      }
+    } else {
+      epilogue_tile<KIND>(p, ti, row, rv, taddr);
+    }
     tc_fence_before();
     mbar_arrive(&tempty[acc]);
     ++it;
@@ -474,6 +622,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   uint64_t* tempty = bars + 2 * NST + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * NST + 4);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  KsSync ks{bars + 2 * NST + 5, bars + 2 * NST + 6, reinterpret_cast<volatile int*>(bars + 2 * NST + 7), 0};
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -485,6 +634,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
       mbar_init(&tfull[i], 1);
       mbar_init(&tempty[i], 4 * 32);
     }
+    mbar_init(ks.gather, 4 * 32);
+    mbar_init(ks.done, 1);
     *abort = 0;
     fence_barrier_init();
     fence_proxy_async();
@@ -509,7 +660,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   } else if (warp == 1) {
     if (lane == 0) mma_loop<NST, SBYTES>(p, stages, full, empty, tfull, tempty, tmem, abort);
   } else {
-    epilogue_loop<KIND>(p, tfull, tempty, tmem, abort);
+    epilogue_loop<KIND>(p, tfull, tempty, tmem, abort, ks);
   }
 
   __syncwarp();

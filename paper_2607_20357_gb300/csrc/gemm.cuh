@@ -77,6 +77,15 @@ struct GemmParams {
   float* ss_out;
   int ss_ld, ss_slots;
   float ss_inv_d, ss_eps;
+  // K-split tail (residual GEMMs): from tile index ks_info[0] on, the list
+  // holds the ks_info[1] tail tiles repeated ks_info[2] times; copy `part`
+  // of tail tile `slot` computes that share of the tile's active K blocks and
+  // stores it to ks_part, counts itself in ks_ticket[slot] and, once all
+  // shares are in, reduces its own slice of the tile's rows. Tickets start
+  // at zero (a separate array per launch).
+  const int* ks_info;  // [3] on the device, or nullptr
+  float* ks_part;      // [tail tiles * parts][128][256]
+  int* ks_ticket;      // [tail tiles]
   uint32_t* status;
 };
 

@@ -71,6 +71,8 @@ struct ScheduleArgs {
   int4* gu_tiles; int gu_cap; int* gu_count;
   int4* dn_tiles; int dn_cap; int* dn_count;
   int4* attn_items; int attn_cap; int* attn_count;
+  int* ks_info;             // [L][2][4]: K-split tail of the O (0) and down (1) lists, see GemmParams
+  int ks_units;             // most tail shares the partial buffer holds
   uint32_t* status;
 };
 void launch_schedule(const ScheduleArgs& a, cudaStream_t s);

@@ -164,8 +164,10 @@ def test_logits_all_rows_tiny():
 
 def test_split_tail_llava_one_layer_full_batch():
     """B = 16 LLaVA rows at b = 0.5 give the O and down projections four full
-    waves plus a tail that the schedule splits along K; every sample must
-    still match."""
+    waves plus a tail of 48 tiles that the schedule cuts into three K shares
+    each (the last share to finish sums them); every sample must still match.
+    The tiny cases cut their single O tile into eight shares, four of them
+    empty."""
     dims = synth.reduced(LLAVA.dims, n_layers=1)
     case = Case(dims, LLAVA, seed=12, batch=16, budget=0.5)
     errs = _compare_end_to_end(case, case.run())
