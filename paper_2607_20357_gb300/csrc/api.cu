@@ -379,7 +379,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
          make_map(t + 4, lw.wg, d.d_ffn, d.d_model) && make_map(t + 5, lw.wu, d.d_ffn, d.d_model) &&
          make_map(t + 6, lw.wd, d.d_model, d.d_ffn);
   }
-  ok = ok && make_map(&m->tm_ctrl_w1, w->ctrl_w1, d.h_ctrl, d.c_vis) &&
+  ok = ok && make_map(&m->tm_ctrl_w1, w->ctrl_w1, d.h_ctrl, d.c_vis, static_cast<uint32_t>(d.h_ctrl)) &&
        make_map(&m->tm_lm_head, w->lm_head, d.vocab, d.d_model);
   if (ok && d.proj_hidden)
     ok = make_map(&m->tm_proj_w1, w->proj_w1, d.proj_hidden, d.c_vis) &&
@@ -469,7 +469,8 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
     p.n_seg = B;
     p.w2 = static_cast<const __nv_bfloat16*>(m->w.ctrl_w2);
     p.c2 = m->w.ctrl_c2;
-    st = launch(EPI_SCORE, m, SVL_TAG_SCORE, p, p.grid_m, s);
+    p.b_box_rows = d.h_ctrl;
+    st = launch(d.h_ctrl <= 64 ? EPI_SCORE : EPI_SCORE_WIDE, m, SVL_TAG_SCORE, p, p.grid_m, s);
     if (st != SVL_OK) return st;
   }
 
@@ -1082,8 +1083,10 @@ extern "C" svl_status svl_score_select_noalloc(svl_model* m, int32_t B, int32_t 
     p.n_seg = B;
     p.w2 = static_cast<const __nv_bfloat16*>(m->w.ctrl_w2);
     p.c2 = m->w.ctrl_c2;
+    p.b_box_rows = d.h_ctrl;
     g_launches++;
-    if (launch_gemm(EPI_SCORE, p, gemm_grid(m, p.grid_m), s) != cudaSuccess) return SVL_ERR_CUDA;
+    if (launch_gemm(d.h_ctrl <= 64 ? EPI_SCORE : EPI_SCORE_WIDE, p, gemm_grid(m, p.grid_m), s) != cudaSuccess)
+      return SVL_ERR_CUDA;
   }
   SelectArgs a;
   a.scores = scores;

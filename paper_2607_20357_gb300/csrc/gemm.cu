@@ -101,9 +101,9 @@ SVL_DEVINL void set_abort(volatile int* abort, uint32_t* status) {
   report(status, SVL_DEV_TIMEOUT);
 }
 
-// Stage geometry per epilogue: the token-score GEMM (N = H <= 128) needs one
-// B box per stage, so its 32 KB stages fit six deep in the same shared memory
-// and keep more of the streamed features in flight.
+// Stage geometry per epilogue: the token-score GEMM streams the features
+// once and reads a B box of only H rows per stage (H <= 64: 24 KB stages,
+// nine deep; H <= 128: 32 KB, six deep), keeping more feature bytes in flight.
 template <int KIND>
 struct StageCfg {
   static constexpr int stages = kStages;
@@ -111,6 +111,11 @@ struct StageCfg {
 };
 template <>
 struct StageCfg<EPI_SCORE> {
+  static constexpr int stages = 9;
+  static constexpr int bytes = kABytes + kBHalfBytes / 2;
+};
+template <>
+struct StageCfg<EPI_SCORE_WIDE> {
   static constexpr int stages = 6;
   static constexpr int bytes = kABytes + kBHalfBytes;
 };
@@ -130,7 +135,7 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
     const CUtensorMap* mb0 = p.b_split ? &p.mapB[0] : &p.mapB[ti.mat];
     const CUtensorMap* mb1 = p.b_split ? &p.mapB[1] : &p.mapB[ti.mat];
     const int y1 = p.b_split ? ti.n0 : ti.n0 + kBHalf;
-    const uint32_t bytes = kABytes + halves * kBHalfBytes;
+    const uint32_t bytes = kABytes + halves * (p.b_box_rows ? p.b_box_rows * 128 : kBHalfBytes);
     KWalk w(nkb, kgb, ti.kmask);
     int i0, i1;
     k_share(ti, nkb, kgb, i0, i1);
@@ -400,7 +405,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
           if (c + j < ti.ncols) o[j] = v[j];
       }
     }
-  } else if constexpr (KIND == EPI_SCORE) {
+  } else if constexpr (KIND == EPI_SCORE || KIND == EPI_SCORE_WIDE) {
     // sample of this row: lane 0 searches for the warp's first row, then each
     // lane walks forward (32 consecutive tokens span few samples)
     const int lane = threadIdx.x & 31;
@@ -702,6 +707,7 @@ cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_
     case EPI_LOGITS_T: return launch_kind<EPI_LOGITS_T>(p, grid, stream);
     case EPI_F32: return launch_kind<EPI_F32>(p, grid, stream);
     case EPI_SCORE: return launch_kind<EPI_SCORE>(p, grid, stream);
+    case EPI_SCORE_WIDE: return launch_kind<EPI_SCORE_WIDE>(p, grid, stream);
     default: return cudaErrorInvalidValue;
   }
 }

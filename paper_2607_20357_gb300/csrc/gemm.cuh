@@ -30,7 +30,8 @@ enum EpiKind : int {
   EPI_ROWMAP = 4,    // out[row_map[r], n] = bf16(acc)
   EPI_LOGITS_T = 5,  // out[n, r] = acc (fp32): swapped LM head, r = vocab id, n = sample
   EPI_F32 = 6,       // out[r, n] = acc (fp32)
-  EPI_SCORE = 7,     // z[r] = sum_h w2[h] SiLU(acc[h] + e_b[sample(r), h]) + c2
+  EPI_SCORE = 7,     // z[r] = sum_h w2[h] SiLU(acc[h] + e_b[sample(r), h]) + c2, H <= 64
+  EPI_SCORE_WIDE = 8,  // the same for 64 < H <= 128 (larger B boxes, fewer stages)
   EPI_COUNT = 8
 };
 
@@ -55,6 +56,7 @@ struct GemmParams {
   int K;       // multiple of 64
   int kgroup;  // K elements per gate group (kmask), multiple of 64
   int b_split; // 1: B rows 0-127 from mapB[0], rows 128-255 from mapB[1] (gate | up)
+  int b_box_rows;  // rows of one B box when mapB has boxes of fewer than 128 rows (0: 128)
   // epilogue operands
   void* out[3];
   int ld[3];

@@ -192,3 +192,24 @@ def test_norm_gains_folded_tiny():
     e_h, e_l, e_h16, e_l16 = errs[0]
     assert e_h16 < 1e-2 and e_l16 < 1e-2, errs
     case.close()
+
+
+def test_select_wide_scorer_h128():
+    """A token-controller hidden width of 128 takes the wide score GEMM
+    (32 KB stages); scores, k and the kept set must still match."""
+    dims = synth.reduced(TINY.dims, h_ctrl=128)
+    case = Case(dims, TINY, seed=13)
+    out = case.model.run(case.b, stages=("select",))
+    torch.cuda.synchronize()
+    assert svl.svl_get_device_status(case.model.handle) == 0
+    out = {k: v.cpu() for k, v in out.items()}
+    v0, v1 = case.b_np["vis_off"][0], case.b_np["vis_off"][1]
+    t_len = case.b_np["text_off"][1] - case.b_np["text_off"][0]
+    z, k, fl, kept = O.score_select_sample(dims, case.w_np, case.b_np["vis"][v0:v1], float(case.b_np["budget"][0]),
+                                           t_len, case.b_np["layer_gate"][0], case.b_np["group_gate"][0],
+                                           int(case.b_np["keep_count"][0]))
+    np.testing.assert_allclose(out["scores"][v0:v1].double().numpy(), z, rtol=1e-4, atol=1e-5)
+    assert int(out["k"][0]) == k
+    gk = out["kept_idx"][out["kept_off"][0]:out["kept_off"][1]].numpy()
+    check_selection(out["scores"][v0:v1].numpy(), gk, {"k": k, "kept": kept, "z": z})
+    case.close()
