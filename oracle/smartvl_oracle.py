@@ -32,6 +32,11 @@ What each function follows:
   the layer through its residual connection. Gated-off parts contribute zero
   (masked-dense definition).
 * ``forward_sample`` / ``forward_batch`` -- the whole path, sample by sample.
+* ``paper_rule_sample`` -- Sec. 3.1 and Sec. 3.3 "Inference", the paper's own
+  rule: tokens with sigma(z) > 0.5 survive, gates are the compute
+  controller's logits thresholded at 0, and for b < 1 the budget projection
+  first drops the lowest-confidence tokens, then (only when no visual token
+  fits) head groups, lowest gate logit first.
 
 Pins (checked by ``tests/test_oracle_pins.py``, all CPU): brute-force subset
 selection, closed-form budget inversion, an operation counter against Eq. 8,
@@ -47,6 +52,7 @@ import numpy as np
 from scipy.special import erf
 
 OVER_BUDGET = 1  # sample flag: even zero visual tokens exceed the budget
+GROUPS_DROPPED = 2  # sample flag (paper rule): the projection turned head groups off
 
 
 # ----------------------------------------------------------------------------
@@ -156,6 +162,54 @@ def budget_keep_count(dims, budget: float, n_vis: int, s_text: int, groups_on, k
         if float(prefill_cost_xG(dims, s_text + k, groups_on)) <= limit:
             return k, 0
     return 0, OVER_BUDGET
+
+
+def paper_rule_counts(dims, budget: float, n_vis: int, s_text: int, z, gate_logits, keep_count: int = -1):
+    """The paper's inference rule for one sample (Sec. 3.1, Sec. 3.3).
+
+    Token mask: sigma(z_i) > 0.5, i.e. z_i > 0 (no Gumbel noise at inference).
+    Gates: group j of layer l runs if l < P (prefix layers) or its compute
+    controller logit is > 0 (sigma > 0.5). Budget projection against
+    b * C_full (Eq. 2 with Eq. 8): first discard the lowest-confidence visual
+    tokens, k = min(#{z > 0}, the largest k within the budget for these
+    gates); when even k = 0 exceeds the budget, turn active groups of layers
+    l >= P off in increasing order of their logit (equal logits: lower
+    (l, j) first) until the cost fits, the fewest groups that make it fit
+    (k stays 0: tokens went first). If the prefix layers alone exceed it, every
+    other group is off and the sample is flagged OVER_BUDGET.
+
+    Returns (k, flags, gates[L, G] as 0/1 ints).
+    """
+    L, G, P = dims.n_layers, dims.n_groups, dims.n_prefix
+    logits = np.asarray(gate_logits, dtype=np.float64).reshape(L, G)
+    gates = np.zeros((L, G), dtype=np.int64)
+    for l in range(L):
+        for j in range(G):
+            gates[l, j] = 1 if (l < P or logits[l, j] > 0) else 0
+    n_pos = int(np.sum(np.asarray(z, dtype=np.float64) > 0))
+    if keep_count >= 0:
+        return min(int(keep_count), int(n_vis)), 0, gates
+    k, flags = budget_keep_count(dims, budget, n_vis, s_text, gates.sum(axis=1))
+    if flags == 0:
+        return min(k, n_pos), 0, gates
+    # no visual token fits: head groups go, lowest logit first
+    c_full = prefill_cost_xG(dims, int(n_vis) + int(s_text), [G] * L)
+    limit = float(np.float32(budget)) * float(c_full)
+    order = sorted(((logits[l, j], l * G + j) for l in range(P, L) for j in range(G) if gates[l, j]))
+    for _, idx in order:
+        gates[idx // G, idx % G] = 0
+        if float(prefill_cost_xG(dims, int(s_text), gates.sum(axis=1))) <= limit:
+            return 0, GROUPS_DROPPED, gates
+    return 0, OVER_BUDGET | (GROUPS_DROPPED if order else 0), gates
+
+
+def paper_rule_sample(dims, weights, x, budget, s_text, gate_logits, keep_count=-1):
+    """Token controller under the paper's rule: logits, k, flags, kept indices
+    and the projected gates [L, G]."""
+    e_b = budget_embedding(float(np.float32(budget)), weights["bud_w1"], weights["bud_w2"])
+    z = token_logits(x, e_b, weights["ctrl_w1"], weights["ctrl_w2"], weights["ctrl_c2"])
+    k, flags, gates = paper_rule_counts(dims, budget, x.shape[0], s_text, z, gate_logits, keep_count)
+    return z, k, flags, select_kept(z, k), gates
 
 
 def select_kept(z: np.ndarray, k: int) -> np.ndarray:

@@ -394,3 +394,88 @@ def test_eq8_accepts_fixed_width_integers():
     assert a == O.prefill_cost_xG(dims, 4672, [4] * 32)
     assert O.budget_keep_count(dims, 0.25, np.int32(4608), np.int32(64), [4] * 32) == \
         O.budget_keep_count(dims, 0.25, 4608, 64, [4] * 32)
+
+
+# ----------------------------------------------------------------------------
+# the paper's own inference rule (Sec. 3.1, Sec. 3.3 "Inference")
+# ----------------------------------------------------------------------------
+def _limit(dims, budget, n_vis, s_text):
+    return float(np.float32(budget)) * float(O.prefill_cost_xG(dims, n_vis + s_text, [dims.n_groups] * dims.n_layers))
+
+
+def test_paper_rule_keeps_exactly_positive_logits_when_budget_is_loose():
+    """b = 1 and every gate logit positive: the kept set is {i : sigma(z_i) > 0.5}."""
+    dims = synth.WORKLOADS["tiny"].dims
+    rng = np.random.default_rng(3)
+    for n in (0, 1, 7, 64):
+        z = rng.normal(size=n)
+        logits = np.abs(rng.normal(size=(dims.n_layers, dims.n_groups))) + 0.1
+        k, flags, gates = O.paper_rule_counts(dims, 1.0, n, 16, z, logits)
+        assert flags == 0 and gates.all()
+        assert k == int(np.sum(1.0 / (1.0 + np.exp(-z)) > 0.5))
+        np.testing.assert_array_equal(O.select_kept(z, k), np.flatnonzero(z > 0))
+
+
+def test_paper_rule_gate_threshold_is_strict():
+    """sigma(0) = 0.5 is not > 0.5: a zero logit switches its group off; prefix layers always run."""
+    dims = synth.reduced(synth.WORKLOADS["tiny"].dims, n_layers=3, n_prefix=1)
+    logits = np.array([[-5.0, -1.0, 0.0, 2.0], [0.0, 1e-6, -1e-6, 3.0], [7.0, 0.0, 0.0, 0.0]])
+    _, _, gates = O.paper_rule_counts(dims, 1.0, 4, 8, np.ones(4), logits)
+    np.testing.assert_array_equal(gates, [[1, 1, 1, 1], [0, 1, 0, 1], [1, 0, 0, 0]])
+
+
+def test_paper_rule_budget_caps_the_threshold_count():
+    """When fewer tokens fit than pass the threshold, the lowest-confidence
+    ones go first: k is the budget count for the controller's gates."""
+    dims = synth.WORKLOADS["tiny"].dims
+    z = np.linspace(-1.0, 3.0, 64)  # 48 positive logits
+    logits = np.ones((dims.n_layers, dims.n_groups))
+    logits[1, 2] = -1.0
+    for b in (0.4, 0.6, 0.8):
+        k, flags, gates = O.paper_rule_counts(dims, b, 64, 16, z, logits)
+        kb, fb = O.budget_keep_count(dims, b, 64, 16, gates.sum(axis=1))
+        assert fb == 0 and flags == 0 and k == min(kb, 48)
+        assert O.prefill_cost_xG(dims, 16 + k, gates.sum(axis=1)) <= _limit(dims, b, 64, 16)
+    k, _, _ = O.paper_rule_counts(dims, 0.4, 64, 16, z, logits)
+    assert k < 48  # the budget binds at b = 0.4
+
+
+def test_paper_rule_fallback_drops_fewest_groups_lowest_logit_first():
+    """Text alone over budget: tokens all go, then the d lowest-logit active
+    non-prefix groups, with d the smallest count that fits."""
+    dims = synth.reduced(synth.WORKLOADS["tiny"].dims, n_layers=4, n_prefix=1)
+    rng = np.random.default_rng(11)
+    logits = rng.normal(size=(4, 4))
+    logits[1, 0] = -0.5  # off by the threshold already
+    hit = 0
+    for b in np.linspace(0.05, 0.5, 19):
+        k, flags, gates = O.paper_rule_counts(dims, float(b), 32, 48, rng.normal(size=32), logits)
+        start = np.array([[1] * 4] + [[1 if v > 0 else 0 for v in row] for row in logits[1:]])
+        limit = _limit(dims, b, 32, 48)
+        if O.prefill_cost_xG(dims, 48, start.sum(axis=1)) <= limit:
+            assert not (flags & O.GROUPS_DROPPED) and (gates == start).all()
+            continue
+        hit += 1
+        assert k == 0 and (flags & O.GROUPS_DROPPED)
+        assert gates[0].all()  # the prefix layer
+        dropped = [(logits[l, j], l * 4 + j) for l in range(1, 4) for j in range(4) if start[l, j] and not gates[l, j]]
+        kept = [(logits[l, j], l * 4 + j) for l in range(1, 4) for j in range(4) if gates[l, j]]
+        assert not (gates & ~start.astype(bool)).any()
+        if kept and dropped:
+            assert max(dropped) < min(kept)  # lowest logits first
+        if not (flags & O.OVER_BUDGET):
+            assert O.prefill_cost_xG(dims, 48, gates.sum(axis=1)) <= limit
+            # one group fewer dropped (the highest-logit dropped one back on) no longer fits
+            g2 = gates.copy()
+            _, idx = max(dropped)
+            g2[idx // 4, idx % 4] = 1
+            assert O.prefill_cost_xG(dims, 48, g2.sum(axis=1)) > limit
+    assert hit >= 5
+
+
+def test_paper_rule_over_budget_when_prefix_alone_exceeds():
+    dims = synth.reduced(synth.WORKLOADS["tiny"].dims, n_layers=3, n_prefix=1)
+    logits = np.ones((3, 4))
+    k, flags, gates = O.paper_rule_counts(dims, 0.01, 16, 64, np.ones(16), logits)
+    assert k == 0 and flags == (O.OVER_BUDGET | O.GROUPS_DROPPED)
+    np.testing.assert_array_equal(gates, [[1, 1, 1, 1], [0, 0, 0, 0], [0, 0, 0, 0]])
