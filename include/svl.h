@@ -56,6 +56,7 @@ typedef enum svl_status {
 
 /* Per-sample flag bits written by svl_score_select. */
 #define SVL_FLAG_OVER_BUDGET 0x1u /* even zero visual tokens exceed b * C_full */
+#define SVL_FLAG_GROUPS_DROPPED 0x2u /* paper rule: the budget projection switched head groups off */
 
 /* Model dimensions.  Notation of Sec. 3: L layers, width D, A heads, FFN
  * width D_int, vocabulary V, G head groups, P prefix layers; C_v is the
@@ -160,6 +161,36 @@ svl_status svl_score_select(svl_model* model, int32_t B, int32_t n_vis_total,
                             float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off,
                             uint32_t* sample_flags, void* workspace, size_t workspace_bytes,
                             void* stream);
+
+/* The paper's own inference rule for the token controller (Sec. 3.1 and
+ * Sec. 3.3 "Inference"), with the LLM-side gates given as the compute
+ * controller's pre-threshold logits instead of 0/1 masks:
+ *   - a visual token survives if sigma(z_i) > 0.5, i.e. z_i > 0;
+ *   - group j of layer l runs if l < P or gate_logits[b, l, j] > 0;
+ *   - budget projection against b * C_full (Eq. 2, Eq. 8): the kept count is
+ *     k = min(#{z_i > 0}, the largest count within the budget for these
+ *     gates), the lowest logits going first (ties: lower index);
+ *   - if even k = 0 exceeds the budget, the fewest active groups of layers
+ *     l >= P that bring the text-only cost within it are switched off, in
+ *     increasing order of their logit (equal logits: lower l * G + j first);
+ *     sample_flags gets SVL_FLAG_GROUPS_DROPPED, and also
+ *     SVL_FLAG_OVER_BUDGET if the prefix layers alone exceed the budget
+ *     (every other group is then off).
+ * keep_count >= 0 overrides k as in svl_score_select (no projection).
+ * Arguments as svl_score_select, except:
+ *   gate_logits     [B, L, G] float32, device
+ *   layer_gate_out  [B, L] uint8, device: 1 where any group of the layer runs
+ *   group_gate_out  [B, L, G] uint8, device: the projected gates
+ * The two gate outputs are what svl_gated_prefill takes. The comparison
+ * z_i > 0 is made on the float32 logits written to `scores`. Workspace:
+ * svl_workspace_size_for(..., SVL_STAGE_SELECT, ...). Errors: as
+ * svl_score_select. */
+svl_status svl_score_select_paper(svl_model* model, int32_t B, int32_t n_vis_total, const void* vis_feats,
+                                  const int32_t* vis_off, const int32_t* text_len, const float* budget,
+                                  const int32_t* keep_count, const float* gate_logits, float* scores,
+                                  int32_t* k, int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
+                                  uint8_t* layer_gate_out, uint8_t* group_gate_out, void* workspace,
+                                  size_t workspace_bytes, void* stream);
 
 /* svl_score_select without a workspace argument. The paper has no
  *  counterpart: this exists for callers that cannot allocate device memory

@@ -430,14 +430,19 @@ size_t svl_workspace_size(const svl_model* m, int32_t max_batch, int64_t max_vis
                                 max_text_total);
 }
 
-svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
-                            const int32_t* vis_off, const int32_t* text_len, const float* budget,
-                            const int32_t* keep_count, const uint8_t* layer_gate, const uint8_t* group_gate,
-                            float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
-                            void* ws, size_t ws_bytes, void* stream) {
-  if (!m || B <= 0 || n_vis_total < 0 || !vis_off || !text_len || !budget || !layer_gate || !group_gate ||
-      !scores || !k || !kept_idx || !kept_off)
+namespace {
+// Token controller: scores, k and the kept lists. Gates are given
+// (layer_gate, group_gate) or, under the paper's rule, derived from the
+// compute controller's logits and projected (gate_logits, *_out).
+svl_status score_select_impl(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
+                             const int32_t* vis_off, const int32_t* text_len, const float* budget,
+                             const int32_t* keep_count, const uint8_t* layer_gate, const uint8_t* group_gate,
+                             const float* gate_logits, uint8_t* layer_gate_out, uint8_t* group_gate_out,
+                             float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off,
+                             uint32_t* sample_flags, void* ws, size_t ws_bytes, void* stream) {
+  if (!m || B <= 0 || n_vis_total < 0 || !vis_off || !text_len || !budget || !scores || !k || !kept_idx || !kept_off)
     return SVL_ERR_INVALID_ARG;
+  if (gate_logits ? (!layer_gate_out || !group_gate_out) : (!layer_gate || !group_gate)) return SVL_ERR_INVALID_ARG;
   if (n_vis_total > 0 && (!vis_feats || !aligned16(vis_feats))) return SVL_ERR_INVALID_ARG;
   const SelLayout L = sel_layout(m->d, B, n_vis_total);
   svl_status st = check_ws(ws, ws_bytes, L.total);
@@ -475,6 +480,7 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
   }
 
   SelectArgs a;
+  std::memset(&a, 0, sizeof(a));
   a.scores = scores;
   a.vis_off = vis_off;
   a.text_len = text_len;
@@ -492,6 +498,9 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
   a.k_out = k;
   a.flags = sample_flags;
   a.kept_local = at<int>(ws, L.kept_local);
+  a.gate_logits = gate_logits;
+  a.layer_gate_out = layer_gate_out;
+  a.group_gate_out = group_gate_out;
   {
     Launch L1(m, SVL_TAG_SELECT, s);
     launch_select(a, B, s);
@@ -501,6 +510,30 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
     launch_compact(B, vis_off, k, a.kept_local, kept_idx, kept_off, at<int>(ws, L.scalars), s);
   }
   return last_error();
+}
+}  // namespace
+
+svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
+                            const int32_t* vis_off, const int32_t* text_len, const float* budget,
+                            const int32_t* keep_count, const uint8_t* layer_gate, const uint8_t* group_gate,
+                            float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
+                            void* ws, size_t ws_bytes, void* stream) {
+  if (!layer_gate || !group_gate) return SVL_ERR_INVALID_ARG;
+  return score_select_impl(m, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
+                           group_gate, nullptr, nullptr, nullptr, scores, k, kept_idx, kept_off, sample_flags, ws,
+                           ws_bytes, stream);
+}
+
+svl_status svl_score_select_paper(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
+                                  const int32_t* vis_off, const int32_t* text_len, const float* budget,
+                                  const int32_t* keep_count, const float* gate_logits, float* scores, int32_t* k,
+                                  int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
+                                  uint8_t* layer_gate_out, uint8_t* group_gate_out, void* ws, size_t ws_bytes,
+                                  void* stream) {
+  if (!gate_logits) return SVL_ERR_INVALID_ARG;
+  return score_select_impl(m, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, nullptr, nullptr,
+                           gate_logits, layer_gate_out, group_gate_out, scores, k, kept_idx, kept_off, sample_flags,
+                           ws, ws_bytes, stream);
 }
 
 svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text_total, const void* vis_feats,
@@ -1089,6 +1122,7 @@ extern "C" svl_status svl_score_select_noalloc(svl_model* m, int32_t B, int32_t 
       return SVL_ERR_CUDA;
   }
   SelectArgs a;
+  std::memset(&a, 0, sizeof(a));
   a.scores = scores;
   a.vis_off = vis_off;
   a.text_len = text_len;

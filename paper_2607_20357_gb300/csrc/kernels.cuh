@@ -23,6 +23,12 @@ struct SelectArgs {
   int* k_out;
   uint32_t* flags;
   int* kept_local;
+  // the paper's own rule (Sec. 3.1, 3.3): gates from compute-controller
+  // logits (> 0), k = min(#{z > 0}, budget count), group fallback; nullptr:
+  // gates given, k = budget count
+  const float* gate_logits;  // [B, L, G]
+  uint8_t* layer_gate_out;   // [B, L] projected gates (paper rule)
+  uint8_t* group_gate_out;   // [B, L, G]
 };
 
 void launch_budget_embed(const float* budget, const __nv_bfloat16* w1, const __nv_bfloat16* w2, int H, int B,

@@ -73,12 +73,20 @@ SVL_DEVINL int block_exclusive_scan(int v, int* total, int* warp_sums) {
 // One block per sample: k from the budget (largest k with Eq. 8 cost within
 // b * C_full), then the k largest logits (ties: lower index), written in
 // ascending index order to kept_local[vis_off[b] ...].
+//
+// Under the paper's own rule (a.gate_logits set; Sec. 3.1 and Sec. 3.3
+// "Inference") the gates are the compute controller's logits > 0 (prefix
+// layers always on), k is capped by the number of logits z > 0 (sigma > 0.5),
+// and when no visual token fits the budget, the fewest active groups of layers
+// l >= P that make it fit are switched off, lowest logit first (equal logits:
+// lower (l, j) first); the projected gates are written out.
 __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
   __shared__ int hist[256];
   __shared__ int warp_sums[32];
   __shared__ int best_k;
   __shared__ int s_prefix_cnt[2];
   __shared__ long long n_on_sum;  // updated with 64-bit atomics
+  __shared__ int n_pos, keep_groups;
   pdl_trigger();
   pdl_wait();
 
@@ -91,17 +99,29 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
   if (tid == 0) {
     n_on_sum = 0;
     best_k = -1;
+    n_pos = 0;
+    keep_groups = -1;
   }
   __syncthreads();
+  const float* gl = a.gate_logits ? a.gate_logits + static_cast<size_t>(b) * a.L * a.G : nullptr;
+  auto active = [&](int idx) -> bool {
+    const int l = idx / a.G;
+    if (l < a.P) return true;
+    return gl ? gl[idx] > 0.f : (a.layer_gate[b * a.L + l] && a.group_gate[b * a.L * a.G + idx]);
+  };
   {
     int on = 0;  // active (layer, group) pairs of this sample
-    for (int idx = tid; idx < a.L * a.G; idx += blockDim.x) {
-      const int l = idx / a.G;
-      on += ((l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[b * a.L * a.G + idx])) ? 1 : 0;
-    }
+    for (int idx = tid; idx < a.L * a.G; idx += blockDim.x) on += active(idx) ? 1 : 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) on += __shfl_xor_sync(0xffffffffu, on, o);
     if ((tid & 31) == 0 && on) atomicAdd(reinterpret_cast<unsigned long long*>(&n_on_sum), static_cast<unsigned long long>(on));
+    if (gl) {
+      int pos = 0;  // logits z > 0, i.e. sigma(z) > 0.5
+      for (int i = tid; i < n; i += blockDim.x) pos += a.scores[v0 + i] > 0.f ? 1 : 0;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) pos += __shfl_xor_sync(0xffffffffu, pos, o);
+      if ((tid & 31) == 0 && pos) atomicAdd(&n_pos, pos);
+    }
   }
   __syncthreads();
   int k;
@@ -124,11 +144,49 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
     // cost grows with k, so the feasible set is a prefix: take the max
     if (mine >= 0) atomicMax(&best_k, static_cast<int>(mine));
     __syncthreads();
-    if (best_k < 0) {
+    if (best_k >= 0) {
+      k = gl ? min(best_k, n_pos) : best_k;
+    } else if (!gl) {
       k = 0;
       flags |= SVL_FLAG_OVER_BUDGET;
     } else {
-      k = best_k;
+      // paper rule: no visual token fits, so head groups go. The most groups
+      // that still fit with the text alone (prefix groups cannot go):
+      k = 0;
+      const long long n_min = static_cast<long long>(min(a.P, a.L)) * G;
+      const long long per = lin * s_text + 4 * D * s_text * s_text, lm = G * 2 * D * V * s_text;
+      for (long long nk = n_min + tid; nk < n_on_sum; nk += blockDim.x)
+        if (static_cast<double>(nk * per + lm) <= limit) atomicMax(&keep_groups, static_cast<int>(nk));
+      __syncthreads();
+      if (n_on_sum > n_min) flags |= SVL_FLAG_GROUPS_DROPPED;
+      const bool over = keep_groups < 0;  // even the prefix layers alone exceed the budget
+      if (over) flags |= SVL_FLAG_OVER_BUDGET;
+      __syncthreads();
+      if (over && tid == 0) keep_groups = static_cast<int>(n_min);
+    }
+  }
+  if (gl) {
+    // projected gates: the (n_on - keep_groups) lowest-logit active groups
+    // of layers >= P are off (none unless the fallback ran)
+    __syncthreads();
+    const int drop = keep_groups < 0 ? 0 : static_cast<int>(n_on_sum) - keep_groups;
+    uint8_t* go = a.group_gate_out + static_cast<size_t>(b) * a.L * a.G;
+    for (int idx = tid; idx < a.L * a.G; idx += blockDim.x) {
+      bool on = active(idx);
+      if (on && drop > 0 && idx >= a.P * a.G) {
+        const float v = gl[idx];
+        int rank = 0;
+        for (int j = a.P * a.G; j < a.L * a.G; ++j)
+          if (active(j) && (gl[j] < v || (gl[j] == v && j < idx))) ++rank;
+        on = rank >= drop;
+      }
+      go[idx] = on ? 1 : 0;
+    }
+    __syncthreads();
+    for (int l = tid; l < a.L; l += blockDim.x) {
+      int any = 0;
+      for (int j = 0; j < a.G; ++j) any |= go[l * a.G + j];
+      a.layer_gate_out[static_cast<size_t>(b) * a.L + l] = any ? 1 : 0;
     }
   }
   if (tid == 0) {

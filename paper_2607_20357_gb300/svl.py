@@ -21,13 +21,14 @@ _lib = None
 SVL_LOGITS_LAST = 0
 SVL_LOGITS_ALL = 1
 SVL_FLAG_OVER_BUDGET = 1
+SVL_FLAG_GROUPS_DROPPED = 2
 SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
 
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
            "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches", "svl_selftest_wait_timeout",
-           "svl_workspace_size_for"]
+           "svl_workspace_size_for", "svl_score_select_paper"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
@@ -93,6 +94,8 @@ def lib():
         L.svl_profile_stop.restype = ctypes.c_int
         L.svl_tag_name.argtypes = [i32]
         L.svl_tag_name.restype = ctypes.c_char_p
+        L.svl_score_select_paper.argtypes = [vp, i32, i32] + [vp] * 14 + [sz, vp]
+        L.svl_score_select_paper.restype = ctypes.c_int
         L.svl_score_select_noalloc.argtypes = [vp, i32, i32] + [vp] * 13
         L.svl_score_select_noalloc.restype = ctypes.c_int
         L.svl_profile_launches.argtypes = [vp, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_float), i32,
@@ -162,6 +165,17 @@ def svl_score_select(model, B, n_vis_total, vis_feats, vis_off, text_len, budget
         model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
         _p(layer_gate), _p(group_gate), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags),
         _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_score_select_paper(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, gate_logits,
+                           scores, k, kept_idx, kept_off, sample_flags, layer_gate_out, group_gate_out, workspace,
+                           workspace_bytes, stream=None):
+    """The paper's own inference rule (sigma(z) > 0.5 tokens, gates from the
+    compute controller's logits, budget projection): see svl.h."""
+    _check("svl_score_select_paper", lib().svl_score_select_paper(
+        model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
+        _p(gate_logits), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags), _p(layer_gate_out),
+        _p(group_gate_out), _p(workspace), int(workspace_bytes), _stream(stream)))
 
 
 def svl_score_select_noalloc(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
@@ -325,16 +339,31 @@ class GatedPrefill:
             "logits": torch.empty((B if logits_mode == SVL_LOGITS_LAST else max(t_cap, 1)), d.vocab,
                                   dtype=torch.float32, device=dev),
             "text_len": (batch["text_off"][1:] - batch["text_off"][:-1]).to(torch.int32).contiguous(),
+            # projected gates of the paper's rule (rule="paper")
+            "layer_gate": torch.empty(B, d.n_layers, dtype=torch.uint8, device=dev),
+            "group_gate": torch.empty(B, d.n_layers, d.n_groups, dtype=torch.uint8, device=dev),
         }
 
     def run(self, batch: dict, out: Optional[dict] = None, logits_mode: int = SVL_LOGITS_LAST, stream=None,
-            stages=("select", "pack", "prefill")):
+            stages=("select", "pack", "prefill"), rule: str = "budget"):
+        """rule="budget": k from the budget for the given gates (the hot path);
+        rule="paper": the paper's own inference rule from batch["gate_logits"]
+        ([B, L, G] compute-controller logits), whose projected gates (in
+        out["layer_gate"], out["group_gate"]) then drive the prefill."""
         B = batch["B"]
         nv = batch["vis"].shape[0]
         nt = int(batch["text_ids"].shape[0])
         out = out or self.alloc_outputs(batch, logits_mode)
         ws, wsb = self.workspace(B, nv, nt, batch["vis"].device, stages)
-        if "select" in stages:
+        if rule not in ("budget", "paper"):
+            raise ValueError(f"unknown rule {rule!r}")
+        gates = (out["layer_gate"], out["group_gate"]) if rule == "paper" else (batch["layer_gate"], batch["group_gate"])
+        if "select" in stages and rule == "paper":
+            svl_score_select_paper(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"],
+                                   batch["budget"], batch["keep_count"], batch["gate_logits"], out["scores"],
+                                   out["k"], out["kept_idx"], out["kept_off"], out["flags"], out["layer_gate"],
+                                   out["group_gate"], ws, wsb, stream)
+        elif "select" in stages:
             svl_score_select(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"], batch["budget"],
                              batch["keep_count"], batch["layer_gate"], batch["group_gate"], out["scores"], out["k"],
                              out["kept_idx"], out["kept_off"], out["flags"], ws, wsb, stream)
@@ -343,5 +372,5 @@ class GatedPrefill:
                      batch["text_ids"], batch["text_off"], out["X"], out["cu_seqlens"], out["pos"], ws, wsb, stream)
         if "prefill" in stages:
             svl_gated_prefill(self.handle, B, max(nv + nt, 1), out["X"], out["cu_seqlens"], out["pos"],
-                              batch["layer_gate"], batch["group_gate"], logits_mode, out["logits"], ws, wsb, stream)
+                              gates[0], gates[1], logits_mode, out["logits"], ws, wsb, stream)
         return out
