@@ -32,6 +32,11 @@ What each function follows:
   the layer through its residual connection. Gated-off parts contribute zero
   (masked-dense definition).
 * ``forward_sample`` / ``forward_batch`` -- the whole path, sample by sample.
+* ``survival_rate`` / ``controller_gate_logits`` / ``forward_controlled`` --
+  Sec. 3.2 LLM-side compute controller: the budget token (Eq. 5 encoding,
+  its own MLP to D) appended after the text, P prefix layers at full
+  capacity, kappa = sum sigma(z_i) / N, the fused state h + MLP_kappa(PE(kappa))
+  (Eq. 7), a linear gate head thresholded at 0, the remaining layers gated.
 * ``paper_rule_sample`` -- Sec. 3.1 and Sec. 3.3 "Inference", the paper's own
   rule: tokens with sigma(z) > 0.5 survive, gates are the compute
   controller's logits thresholded at 0, and for b < 1 the budget projection
@@ -210,6 +215,88 @@ def paper_rule_sample(dims, weights, x, budget, s_text, gate_logits, keep_count=
     z = token_logits(x, e_b, weights["ctrl_w1"], weights["ctrl_w2"], weights["ctrl_c2"])
     k, flags, gates = paper_rule_counts(dims, budget, x.shape[0], s_text, z, gate_logits, keep_count)
     return z, k, flags, select_kept(z, k), gates
+
+
+def project_gates(dims, budget: float, n_vis: int, s_text: int, k: int, gates, logits):
+    """Budget projection on head groups alone, for a token count already
+    committed (the compute controller decides after the prefix layers have
+    run on the kept tokens, Sec. 3.2): while Eq. 8 at S = S_text + k exceeds
+    b * C_full, the active group of layers l >= P with the lowest logit goes
+    (equal logits: lower l * G + j first). Returns (gates, flags)."""
+    L, G, P = dims.n_layers, dims.n_groups, dims.n_prefix
+    gates = np.array(gates, dtype=np.int64).reshape(L, G)
+    logits = np.asarray(logits, dtype=np.float64).reshape(L, G)
+    limit = float(np.float32(budget)) * float(prefill_cost_xG(dims, int(n_vis) + int(s_text), [G] * L))
+    S = int(s_text) + int(k)
+    if float(prefill_cost_xG(dims, S, gates.sum(axis=1))) <= limit:
+        return gates, 0
+    order = sorted(((logits[l, j], l * G + j) for l in range(P, L) for j in range(G) if gates[l, j]))
+    for _, idx in order:
+        gates[idx // G, idx % G] = 0
+        if float(prefill_cost_xG(dims, S, gates.sum(axis=1))) <= limit:
+            return gates, GROUPS_DROPPED
+    return gates, OVER_BUDGET | (GROUPS_DROPPED if order else 0)
+
+
+def survival_rate(z) -> float:
+    """kappa = sum_i sigma(z_i) / N, the soft fraction of surviving visual
+    tokens that conditions the compute controller (Sec. 3.2); 0 for N = 0."""
+    z = np.asarray(z, dtype=np.float64)
+    return float(np.sum(1.0 / (1.0 + np.exp(-z))) / len(z)) if len(z) else 0.0
+
+
+def controller_gate_logits(dims, weights, h_prefix, kappa: float) -> np.ndarray:
+    """Eq. 7 and the gate head: h~ = h_b^(P) + MLP_kappa(PE(kappa)), then
+    W_h h~ + c_h reshaped to [L - P, G] (rows = layers P .. L-1)."""
+    h = np.asarray(h_prefix, dtype=np.float64) + budget_embedding(kappa, weights["kap_w1"], weights["kap_w2"])
+    n = (dims.n_layers - dims.n_prefix) * dims.n_groups
+    out = weights["gate_w"][:n] @ h + weights["gate_c"][:n]
+    return out.reshape(dims.n_layers - dims.n_prefix, dims.n_groups)
+
+
+def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_count=-1, gates_override=None,
+                       project=True):
+    """The inference path with the compute controller in the loop (Sec. 3.2,
+    Sec. 3.3): tokens with z > 0 survive (keep_count >= 0 overrides), the
+    sequence is [kept visual][text][budget token] with positions 0..S, the
+    prefix layers run at full capacity, the gate head reads the budget
+    token's state, the remaining layers run under its gates (thresholded at
+    0, then projected onto the budget for b < 1 unless ``project`` is False),
+    and the logits come from the last row -- the budget token, which the
+    answer follows. ``gates_override`` ([L, G]) replaces the controller's
+    decision (to replay another implementation's gates).
+    """
+    store = make_store(mode)
+    L, G, P = dims.n_layers, dims.n_groups, dims.n_prefix
+    e_b = budget_embedding(float(np.float32(budget)), weights["bud_w1"], weights["bud_w2"])
+    z = token_logits(x, e_b, weights["ctrl_w1"], weights["ctrl_w2"], weights["ctrl_c2"])
+    kappa = survival_rate(z)
+    k = min(int(keep_count), x.shape[0]) if keep_count >= 0 else int(np.sum(z > 0))
+    kept = select_kept(z, k)
+    X, pos = pack_sample(dims, weights, x, kept, text_ids, store)
+    tok = store(budget_embedding(float(np.float32(budget)), weights["llm_bud_w1"], weights["llm_bud_w2"]))
+    X = np.concatenate([X, tok[None, :]], axis=0)
+    pos = np.concatenate([pos, [len(pos)]])
+    on = np.ones(G, dtype=np.int64)
+    for l in range(P):
+        X = decoder_layer(X, pos, weights["layers"][l], on, dims, store)
+    gate_logits = controller_gate_logits(dims, weights, X[-1], kappa)
+    full_logits = np.zeros((L, G))
+    full_logits[P:] = gate_logits
+    gates = np.ones((L, G), dtype=np.int64)
+    gates[P:] = (gate_logits > 0).astype(np.int64)
+    flags = 0
+    if gates_override is not None:
+        gates = np.array(gates_override, dtype=np.int64).reshape(L, G)
+    elif project and float(np.float32(budget)) < 1.0:
+        gates, flags = project_gates(dims, budget, x.shape[0], len(text_ids), k, gates, full_logits)
+    for l in range(P, L):
+        if gates[l].any():
+            X = decoder_layer(X, pos, weights["layers"][l], gates[l], dims, store)
+    y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
+    logits = make_store("fp64" if mode == "fp64" else "fp32")(weights["lm_head"] @ y)
+    return {"z": z, "kappa": kappa, "k": k, "kept": kept, "gate_logits": gate_logits, "gates": gates,
+            "flags": flags, "hidden": X, "logits": logits}
 
 
 def select_kept(z: np.ndarray, k: int) -> np.ndarray:

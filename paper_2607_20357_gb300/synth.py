@@ -138,7 +138,9 @@ def make_weights(dims: ModelDims, seed: int, device="cpu", std: float = 0.02, la
     scorer; bud_w1, bud_w2 [H, H] for the budget MLP; proj_w1 [P_h, C_v],
     proj_w2 [D, P_h] when a projector exists; embed [V, D]; per layer
     wq [A*dh, D], wk/wv [A_kv*dh, D], wo [D, A*dh], wg/wu [D_int, D],
-    wd [D, D_int], attn_norm/ffn_norm [D]; final_norm [D]; lm_head [V, D].
+    wd [D, D_int], attn_norm/ffn_norm [D]; final_norm [D]; lm_head [V, D];
+    compute controller llm_bud_w1, kap_w1 [H, H], llm_bud_w2, kap_w2 [D, H],
+    gate_w [(L-P)*G, D] (bf16) and gate_c [(L-P)*G] (float32).
     """
     D, H = dims.d_model, dims.h_ctrl
 
@@ -172,6 +174,20 @@ def make_weights(dims: ModelDims, seed: int, device="cpu", std: float = 0.02, la
     w["layers"] = out_layers
     w["final_norm"] = torch.ones(D, dtype=torch.bfloat16, device=device)
     w["lm_head"] = draw((dims.vocab, D), std, -1, 7)
+    # LLM-side compute controller (Sec. 3.2): budget-token MLP H -> H -> D,
+    # token-count MLP H -> H -> D, linear gate head over (L - P) x G groups.
+    # Scales give the budget token a residual-stream-sized embedding and gate
+    # logits of order one; the gate biases are drawn around +0.3 (the paper
+    # initialises them positively).
+    n_gate = max(dims.n_layers - dims.n_prefix, 0) * dims.n_groups
+    cs = 1.0 / math.sqrt(H)
+    w["llm_bud_w1"] = draw((H, H), cs, -1, 8)
+    w["llm_bud_w2"] = draw((D, H), cs, -1, 9)
+    w["kap_w1"] = draw((H, H), cs, -1, 10)
+    w["kap_w2"] = draw((D, H), cs, -1, 11)
+    w["gate_w"] = draw((max(n_gate, 1), D), 1.0 / math.sqrt(D), -1, 12)
+    gc = _gen(_tensor_seed(seed, -1, 13), device)
+    w["gate_c"] = (0.3 + torch.randn(max(n_gate, 1), generator=gc, dtype=torch.float32, device=device))
     return w
 
 

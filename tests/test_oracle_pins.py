@@ -479,3 +479,88 @@ def test_paper_rule_over_budget_when_prefix_alone_exceeds():
     k, flags, gates = O.paper_rule_counts(dims, 0.01, 16, 64, np.ones(16), logits)
     assert k == 0 and flags == (O.OVER_BUDGET | O.GROUPS_DROPPED)
     np.testing.assert_array_equal(gates, [[1, 1, 1, 1], [0, 0, 0, 0], [0, 0, 0, 0]])
+
+
+# ----------------------------------------------------------------------------
+# the LLM-side compute controller (Sec. 3.2, Eq. 7)
+# ----------------------------------------------------------------------------
+def test_survival_rate_closed_form():
+    assert O.survival_rate([]) == 0.0
+    assert O.survival_rate([0.0, 0.0, 0.0]) == 0.5
+    assert abs(O.survival_rate([50.0, -50.0]) - 0.5) < 1e-15
+    z = np.random.default_rng(4).normal(size=333) * 3
+    assert abs(O.survival_rate(z) - torch.sigmoid(torch.tensor(z)).mean().item()) < 1e-14
+
+
+def test_controller_gate_logits_match_library_layers():
+    """W_h (h + W_k2 SiLU(W_k1 PE(kappa))) + c_h, written with torch.nn.functional."""
+    dims = synth.reduced(SMALL, n_prefix=1)
+    w = np_weights(dims)
+    rng = np.random.default_rng(5)
+    h = rng.normal(size=dims.d_model)
+    for kappa in (0.0, 0.37, 1.0):
+        half = dims.h_ctrl // 2
+        om = 10000.0 ** (-2.0 * torch.arange(half, dtype=torch.float64) / dims.h_ctrl)
+        pe = torch.cat([torch.sin(1000.0 * kappa * om), torch.cos(1000.0 * kappa * om)])
+        t = lambda a: torch.as_tensor(a, dtype=torch.float64)
+        e = torch.nn.functional.linear(torch.nn.functional.silu(torch.nn.functional.linear(pe, t(w["kap_w1"]))),
+                                       t(w["kap_w2"]))
+        want = torch.nn.functional.linear(t(h) + e, t(w["gate_w"]), t(w["gate_c"]))
+        got = O.controller_gate_logits(dims, w, h, kappa)
+        assert got.shape == (dims.n_layers - 1, dims.n_groups)
+        np.testing.assert_allclose(got.reshape(-1), want.numpy(), rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("dims", [SMALL, SMALL_ID])
+def test_controlled_all_prefix_equals_dense_with_budget_token(dims):
+    """With every layer a prefix layer nothing is gated: the forward is the
+    dense transformer over [kept visual][text][budget token], positions 0..S."""
+    dims = synth.reduced(dims, n_prefix=dims.n_layers)
+    w = np_weights(dims)
+    x, ids = _sample(dims)
+    out = O.forward_controlled(dims, w, x, ids, 0.7, mode="fp64", keep_count=x.shape[0])
+    tok = O.budget_embedding(float(np.float32(0.7)), w["llm_bud_w1"], w["llm_bud_w2"])
+    X0 = np.concatenate([_packed_rows(dims, w, x, np.arange(x.shape[0]), ids), tok[None, :]], 0)
+    hid, logits = dense_forward(X0, w["layers"], w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(out["hidden"], hid, rtol=1e-10, atol=1e-10)
+    np.testing.assert_allclose(out["logits"], logits, rtol=1e-10, atol=1e-10)
+
+
+def test_controlled_gates_threshold_and_token_rule():
+    """Unprojected: tokens are exactly those with z > 0, gates of layers >= P
+    are exactly the gate logits > 0, prefix layers always run."""
+    dims = synth.reduced(SMALL, n_layers=4, n_prefix=1)
+    w = np_weights(dims, seed=8)
+    x, ids = _sample(dims, seed=2)
+    out = O.forward_controlled(dims, w, x, ids, 0.5, project=False)
+    np.testing.assert_array_equal(out["kept"], np.flatnonzero(out["z"] > 0))
+    assert out["gates"][0].all()
+    np.testing.assert_array_equal(out["gates"][1:], (out["gate_logits"] > 0).astype(np.int64))
+    assert abs(out["kappa"] - O.survival_rate(out["z"])) == 0.0
+
+
+def test_project_gates_fewest_lowest_logit_groups():
+    dims = synth.reduced(synth.WORKLOADS["tiny"].dims, n_layers=4, n_prefix=1)
+    rng = np.random.default_rng(12)
+    logits = rng.normal(size=(4, 4))
+    start = np.ones((4, 4), dtype=np.int64)
+    hits = 0
+    for b in np.linspace(0.1, 0.9, 17):
+        gates, flags = O.project_gates(dims, float(b), 64, 16, 40, start, logits)
+        limit = _limit(dims, b, 64, 16)
+        if O.prefill_cost_xG(dims, 56, start.sum(axis=1)) <= limit:
+            assert flags == 0 and (gates == start).all()
+            continue
+        hits += 1
+        assert gates[0].all() and (flags & O.GROUPS_DROPPED)
+        off = [(logits[l, j], l * 4 + j) for l in range(1, 4) for j in range(4) if not gates[l, j]]
+        on = [(logits[l, j], l * 4 + j) for l in range(1, 4) for j in range(4) if gates[l, j]]
+        if off and on:
+            assert max(off) < min(on)
+        if not (flags & O.OVER_BUDGET):
+            assert O.prefill_cost_xG(dims, 56, gates.sum(axis=1)) <= limit
+            g2 = gates.copy()
+            _, idx = max(off)
+            g2[idx // 4, idx % 4] = 1
+            assert O.prefill_cost_xG(dims, 56, g2.sum(axis=1)) > limit
+    assert hits >= 4
