@@ -114,6 +114,14 @@ typedef struct svl_weights {
   const void* final_norm; /* [D] */
   const void* lm_head;    /* [V, D] */
   const svl_layer_weights* layers; /* HOST array of n_layers entries */
+  /* LLM-side compute controller (Sec. 3.2), used only by
+   * svl_pack_controlled / svl_controlled_prefill; may be NULL otherwise. */
+  const void* llm_bud_w1; /* [H, H]  budget-token MLP: e = W2 SiLU(W1 PE(b)), Eq. 5 encoding */
+  const void* llm_bud_w2; /* [D, H] */
+  const void* kap_w1;     /* [H, H]  token-count MLP of Eq. 7: W2 SiLU(W1 PE(kappa)) */
+  const void* kap_w2;     /* [D, H] */
+  const void* gate_w;     /* [(L - P) * G, D] gate head W_h (rows: layer P.., group) */
+  const float* gate_c;    /* [(L - P) * G] gate head bias c_h, float32 */
 } svl_weights;
 
 typedef struct svl_model svl_model;
@@ -189,8 +197,54 @@ svl_status svl_score_select_paper(svl_model* model, int32_t B, int32_t n_vis_tot
                                   const int32_t* vis_off, const int32_t* text_len, const float* budget,
                                   const int32_t* keep_count, const float* gate_logits, float* scores,
                                   int32_t* k, int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
-                                  uint8_t* layer_gate_out, uint8_t* group_gate_out, void* workspace,
-                                  size_t workspace_bytes, void* stream);
+                                  uint8_t* layer_gate_out, uint8_t* group_gate_out, float* kappa_out,
+                                  void* workspace, size_t workspace_bytes, void* stream);
+/* With gate_logits == NULL the gates are not known yet (the compute
+ * controller decides them after the prefix layers, svl_controlled_prefill):
+ * k = #{z_i > 0} (keep_count >= 0 overrides), no budget projection here, the
+ * gate outputs may be NULL and are not written. kappa_out [B] (device, or
+ * NULL) receives the token survival rate kappa = sum_i sigma(z_i) / N_b of
+ * Sec. 3.2 (0 for N_b = 0), in both modes. */
+
+/* Packs like svl_pack and appends to each sample its budget token (Sec. 3.2:
+ * e_b = MLP_LLM(PE(b)) with the Eq. 5 encoding, weights llm_bud_w1/w2) as its
+ * last row, position S_b. X, pos: room for n_vis_total + n_text_total + B
+ * rows. Errors: as svl_pack; SVL_ERR_UNSUPPORTED without the controller
+ * weights. */
+svl_status svl_pack_controlled(svl_model* model, int32_t B, int32_t n_vis_total, int32_t n_text_total,
+                               const void* vis_feats, const int32_t* vis_off, const int32_t* kept_idx,
+                               const int32_t* kept_off, const int32_t* text_ids, const int32_t* text_off,
+                               const float* budget, void* X, int32_t* cu_seqlens, int32_t* pos, void* workspace,
+                               size_t workspace_bytes, void* stream);
+
+/* The gated prefill with the LLM-side compute controller in the loop
+ * (Sec. 3.2, Eq. 7): over a batch packed by svl_pack_controlled, the P
+ * prefix layers run at full capacity; then, per sample, the budget token's
+ * state h plus W_k2 SiLU(W_k1 PE(kappa)) feeds the linear gate head, group j
+ * of layer l >= P runs if its logit is > 0, and with `project` != 0 and
+ * b < 1 the fewest active groups (lowest logit first; equal logits: lower
+ * l * G + j first) are switched off until Eq. 8 at S = S_text + k fits
+ * b * C_full (Sec. 3.3; the token count is already committed). The device
+ * schedule of the remaining layers is rebuilt from these gates with no host
+ * round trip, and the logits come from each sample's last row (the budget
+ * token, which the answer follows).
+ *   budget, kappa   [B] float32, device (kappa from svl_score_select_paper)
+ *   k, text_len     [B] int32, device: kept visual tokens, text tokens
+ *   vis_off         [B+1] int32, device: visual tokens per sample (C_full)
+ *   layer_gate_out  [B, L], group_gate_out [B, L, G] uint8, device: the
+ *                   gates used (prefix layers on)
+ *   gate_logits_out [B, L - P, G] float32, device, or NULL
+ *   sample_flags    [B] uint32, device, or NULL: SVL_FLAG_GROUPS_DROPPED /
+ *                   SVL_FLAG_OVER_BUDGET or-ed in by the projection
+ * Other arguments as svl_gated_prefill (t_cap counts the budget-token rows).
+ * Errors: as svl_gated_prefill; SVL_ERR_UNSUPPORTED without the controller
+ * weights. */
+svl_status svl_controlled_prefill(svl_model* model, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                                  const int32_t* pos, const float* budget, const float* kappa, const int32_t* k,
+                                  const int32_t* vis_off, const int32_t* text_len, int32_t project,
+                                  int32_t logits_mode, float* logits, uint8_t* layer_gate_out,
+                                  uint8_t* group_gate_out, float* gate_logits_out, uint32_t* sample_flags,
+                                  void* workspace, size_t workspace_bytes, void* stream);
 
 /* svl_score_select without a workspace argument. The paper has no
  *  counterpart: this exists for callers that cannot allocate device memory

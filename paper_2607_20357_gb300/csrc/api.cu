@@ -78,7 +78,7 @@ struct SelLayout {
   size_t e_b, scalars, kept_local, total;
 };
 struct PackLayout {
-  size_t scalars, stage, hp, row_map, total;
+  size_t scalars, stage, hp, row_map, tok, total;
 };
 struct PreLayout {
   int64_t t_cap, t_pad;
@@ -107,10 +107,11 @@ SelLayout sel_layout(const svl_model_desc& d, int B, int64_t nv) {
   return L;
 }
 
-PackLayout pack_layout(const svl_model_desc& d, int64_t nv) {
+PackLayout pack_layout(const svl_model_desc& d, int B, int64_t nv) {
   PackLayout L{};
   Bump b;
   L.scalars = b.take(64);
+  L.tok = b.take(2 * static_cast<size_t>(B) * d.d_model);  // budget-token rows (compute controller)
   if (d.proj_hidden) {
     L.stage = b.take(2 * nv * d.c_vis);
     L.hp = b.take(2 * nv * d.proj_hidden);
@@ -198,7 +199,7 @@ HostLayout host_layout(const svl_model_desc& d, int B, int64_t nv, int64_t nt) {
   L.pos = b.take(4 * t_cap);
   L.logits = b.take(sizeof(float) * static_cast<size_t>(B) * d.vocab);
   L.inner = b.off;
-  const size_t a = sel_layout(d, B, nv).total, p = pack_layout(d, nv).total, c = pre_layout(d, B, t_cap).total;
+  const size_t a = sel_layout(d, B, nv).total, p = pack_layout(d, B, nv).total, c = pre_layout(d, B, t_cap).total;
   L.total = L.inner + std::max(a, std::max(p, c));
   return L;
 }
@@ -419,9 +420,9 @@ size_t svl_workspace_size_for(const svl_model* m, uint32_t stages, int32_t max_b
   if (!m || max_batch <= 0 || max_vis_total < 0 || max_text_total < 0) return 0;
   size_t need = 0;
   if (stages & SVL_STAGE_SELECT) need = std::max(need, sel_layout(m->d, max_batch, max_vis_total).total);
-  if (stages & SVL_STAGE_PACK) need = std::max(need, pack_layout(m->d, max_vis_total).total);
+  if (stages & SVL_STAGE_PACK) need = std::max(need, pack_layout(m->d, max_batch, max_vis_total).total);
   if (stages & SVL_STAGE_PREFILL)
-    need = std::max(need, pre_layout(m->d, max_batch, max_vis_total + max_text_total).total);
+    need = std::max(need, pre_layout(m->d, max_batch, max_vis_total + max_text_total + max_batch).total);
   return need;
 }
 
@@ -437,12 +438,15 @@ namespace {
 svl_status score_select_impl(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
                              const int32_t* vis_off, const int32_t* text_len, const float* budget,
                              const int32_t* keep_count, const uint8_t* layer_gate, const uint8_t* group_gate,
-                             const float* gate_logits, uint8_t* layer_gate_out, uint8_t* group_gate_out,
-                             float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off,
+                             int rule, const float* gate_logits, uint8_t* layer_gate_out, uint8_t* group_gate_out,
+                             float* kappa_out, float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off,
                              uint32_t* sample_flags, void* ws, size_t ws_bytes, void* stream) {
+  // rule 0: budget count for given gates; 1: paper rule with gate logits;
+  // 2: paper rule, gates decided later (threshold only)
   if (!m || B <= 0 || n_vis_total < 0 || !vis_off || !text_len || !budget || !scores || !k || !kept_idx || !kept_off)
     return SVL_ERR_INVALID_ARG;
-  if (gate_logits ? (!layer_gate_out || !group_gate_out) : (!layer_gate || !group_gate)) return SVL_ERR_INVALID_ARG;
+  if (rule == 0 && (!layer_gate || !group_gate)) return SVL_ERR_INVALID_ARG;
+  if (rule == 1 && (!gate_logits || !layer_gate_out || !group_gate_out)) return SVL_ERR_INVALID_ARG;
   if (n_vis_total > 0 && (!vis_feats || !aligned16(vis_feats))) return SVL_ERR_INVALID_ARG;
   const SelLayout L = sel_layout(m->d, B, n_vis_total);
   svl_status st = check_ws(ws, ws_bytes, L.total);
@@ -498,9 +502,11 @@ svl_status score_select_impl(svl_model* m, int32_t B, int32_t n_vis_total, const
   a.k_out = k;
   a.flags = sample_flags;
   a.kept_local = at<int>(ws, L.kept_local);
-  a.gate_logits = gate_logits;
+  a.gate_logits = rule == 1 ? gate_logits : nullptr;
   a.layer_gate_out = layer_gate_out;
   a.group_gate_out = group_gate_out;
+  a.threshold_only = rule == 2 ? 1 : 0;
+  a.kappa = kappa_out;
   {
     Launch L1(m, SVL_TAG_SELECT, s);
     launch_select(a, B, s);
@@ -518,42 +524,51 @@ svl_status svl_score_select(svl_model* m, int32_t B, int32_t n_vis_total, const 
                             const int32_t* keep_count, const uint8_t* layer_gate, const uint8_t* group_gate,
                             float* scores, int32_t* k, int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
                             void* ws, size_t ws_bytes, void* stream) {
-  if (!layer_gate || !group_gate) return SVL_ERR_INVALID_ARG;
   return score_select_impl(m, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
-                           group_gate, nullptr, nullptr, nullptr, scores, k, kept_idx, kept_off, sample_flags, ws,
-                           ws_bytes, stream);
+                           group_gate, 0, nullptr, nullptr, nullptr, nullptr, scores, k, kept_idx, kept_off,
+                           sample_flags, ws, ws_bytes, stream);
 }
 
 svl_status svl_score_select_paper(svl_model* m, int32_t B, int32_t n_vis_total, const void* vis_feats,
                                   const int32_t* vis_off, const int32_t* text_len, const float* budget,
                                   const int32_t* keep_count, const float* gate_logits, float* scores, int32_t* k,
                                   int32_t* kept_idx, int32_t* kept_off, uint32_t* sample_flags,
-                                  uint8_t* layer_gate_out, uint8_t* group_gate_out, void* ws, size_t ws_bytes,
-                                  void* stream) {
-  if (!gate_logits) return SVL_ERR_INVALID_ARG;
+                                  uint8_t* layer_gate_out, uint8_t* group_gate_out, float* kappa_out, void* ws,
+                                  size_t ws_bytes, void* stream) {
   return score_select_impl(m, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, nullptr, nullptr,
-                           gate_logits, layer_gate_out, group_gate_out, scores, k, kept_idx, kept_off, sample_flags,
-                           ws, ws_bytes, stream);
+                           gate_logits ? 1 : 2, gate_logits, layer_gate_out, group_gate_out, kappa_out, scores, k,
+                           kept_idx, kept_off, sample_flags, ws, ws_bytes, stream);
 }
 
-svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text_total, const void* vis_feats,
-                    const int32_t* vis_off, const int32_t* kept_idx, const int32_t* kept_off,
-                    const int32_t* text_ids, const int32_t* text_off, void* X, int32_t* cu_seqlens, int32_t* pos,
-                    void* ws, size_t ws_bytes, void* stream) {
+namespace {
+// Packs kept visual rows and text rows; with `budget` (compute controller,
+// Sec. 3.2) each sample also gets its budget token as its last row.
+svl_status pack_impl(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text_total, const void* vis_feats,
+                     const int32_t* vis_off, const int32_t* kept_idx, const int32_t* kept_off,
+                     const int32_t* text_ids, const int32_t* text_off, const float* budget, void* X,
+                     int32_t* cu_seqlens, int32_t* pos, void* ws, size_t ws_bytes, void* stream) {
   if (!m || B <= 0 || n_vis_total < 0 || n_text_total < 0 || !vis_off || !kept_idx || !kept_off || !text_off ||
       !X || !cu_seqlens || !pos)
     return SVL_ERR_INVALID_ARG;
   if ((n_text_total > 0 && !text_ids) || (n_vis_total > 0 && !vis_feats)) return SVL_ERR_INVALID_ARG;
   if (!aligned16(X) || (vis_feats && !aligned16(vis_feats))) return SVL_ERR_INVALID_ARG;
-  const PackLayout L = pack_layout(m->d, n_vis_total);
+  const PackLayout L = pack_layout(m->d, B, n_vis_total);
   svl_status st = check_ws(ws, ws_bytes, L.total);
   if (st != SVL_OK) return st;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const svl_model_desc& d = m->d;
-  const int64_t t_cap = static_cast<int64_t>(n_vis_total) + n_text_total;
+  const int64_t t_cap = static_cast<int64_t>(n_vis_total) + n_text_total + (budget ? B : 0);
   if (t_cap > INT32_MAX / 2) return SVL_ERR_SHAPE;
 
   PackArgs a;
+  std::memset(&a, 0, sizeof(a));
+  if (budget) {
+    __nv_bfloat16* tok = at<__nv_bfloat16>(ws, L.tok);
+    a.tok_rows = tok;
+    Launch L0(m, SVL_TAG_PACK, s);
+    launch_llm_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.llm_bud_w1),
+                            static_cast<const __nv_bfloat16*>(m->w.llm_bud_w2), d.h_ctrl, d.d_model, B, tok, s);
+  }
   a.B = B;
   a.D = d.d_model;
   a.c_vis = d.c_vis;
@@ -619,10 +634,35 @@ svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text
   }
   return last_error();
 }
+}  // namespace
 
-svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
-                             const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
-                             int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream) {
+svl_status svl_pack(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text_total, const void* vis_feats,
+                    const int32_t* vis_off, const int32_t* kept_idx, const int32_t* kept_off,
+                    const int32_t* text_ids, const int32_t* text_off, void* X, int32_t* cu_seqlens, int32_t* pos,
+                    void* ws, size_t ws_bytes, void* stream) {
+  return pack_impl(m, B, n_vis_total, n_text_total, vis_feats, vis_off, kept_idx, kept_off, text_ids, text_off,
+                   nullptr, X, cu_seqlens, pos, ws, ws_bytes, stream);
+}
+
+svl_status svl_pack_controlled(svl_model* m, int32_t B, int32_t n_vis_total, int32_t n_text_total,
+                               const void* vis_feats, const int32_t* vis_off, const int32_t* kept_idx,
+                               const int32_t* kept_off, const int32_t* text_ids, const int32_t* text_off,
+                               const float* budget, void* X, int32_t* cu_seqlens, int32_t* pos, void* ws,
+                               size_t ws_bytes, void* stream) {
+  if (!m || !budget) return SVL_ERR_INVALID_ARG;
+  if (!m->w.llm_bud_w1 || !m->w.llm_bud_w2) return SVL_ERR_UNSUPPORTED;
+  return pack_impl(m, B, n_vis_total, n_text_total, vis_feats, vis_off, kept_idx, kept_off, text_ids, text_off,
+                   budget, X, cu_seqlens, pos, ws, ws_bytes, stream);
+}
+
+namespace {
+// The gated decoder forward. With `ctl` (compute controller, Sec. 3.2) the
+// gate arrays are outputs: they start all on, the controller kernel writes
+// them after the prefix layers, and the device schedule is built again.
+svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                        const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
+                        int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream,
+                        const CtlArgs* ctl) {
   if (!m || B <= 0 || t_cap <= 0 || !X || !cu_seqlens || !pos || !layer_gate || !group_gate || !logits)
     return SVL_ERR_INVALID_ARG;
   if (logits_mode != SVL_LOGITS_LAST && logits_mode != SVL_LOGITS_ALL) return SVL_ERR_INVALID_ARG;
@@ -671,6 +711,13 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
   sa.ks_info = at<int>(ws, L.ks_info);
   sa.ks_units = L.ks_units;
   sa.status = m->d_status;
+  if (ctl) {
+    // controller path: every group on until the controller has decided
+    if (cudaMemsetAsync(const_cast<uint8_t*>(layer_gate), 1, static_cast<size_t>(B) * nl, s) != cudaSuccess ||
+        cudaMemsetAsync(const_cast<uint8_t*>(group_gate), 1, static_cast<size_t>(B) * nl * d.n_groups, s) !=
+            cudaSuccess)
+      return SVL_ERR_CUDA;
+  }
   int* ks_ticket = at<int>(ws, L.ks_ticket);
   if (cudaMemsetAsync(ks_ticket, 0, sizeof(int) * L.ks_units * 2 * nl, s) != cudaSuccess) return SVL_ERR_CUDA;
   {
@@ -736,6 +783,23 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
 
   for (int l = 0; l < nl; ++l) {
     const CUtensorMap* tm = &m->tm_layer[static_cast<size_t>(l) * 7];
+    if (ctl && l == std::min(d.n_prefix, nl)) {
+      // the budget token's state after the prefix layers decides the gates
+      // of the remaining layers; their tile lists are rebuilt on the device
+      CtlArgs c = *ctl;
+      c.X = static_cast<const __nv_bfloat16*>(X);
+      c.cu_seqlens = cu_seqlens;
+      c.layer_gate = const_cast<uint8_t*>(layer_gate);
+      c.group_gate = const_cast<uint8_t*>(group_gate);
+      {
+        Launch L1(m, SVL_TAG_SCHEDULE, s);
+        launch_controller(c, s);
+      }
+      {
+        Launch L1(m, SVL_TAG_SCHEDULE, s);
+        launch_schedule(sa, s);
+      }
+    }
 
     // attention input norm fused into the QKV GEMM (gain folded into W_qkv)
     GemmParams p = base_params(m);
@@ -860,6 +924,51 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
     if ((st = launch(EPI_F32, m, SVL_TAG_LMHEAD, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
   }
   return last_error();
+}
+}  // namespace
+
+svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                             const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
+                             int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream) {
+  return prefill_impl(m, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, logits_mode, logits, ws, ws_bytes,
+                      stream, nullptr);
+}
+
+svl_status svl_controlled_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                                  const int32_t* pos, const float* budget, const float* kappa, const int32_t* k,
+                                  const int32_t* vis_off, const int32_t* text_len, int32_t project,
+                                  int32_t logits_mode, float* logits, uint8_t* layer_gate_out,
+                                  uint8_t* group_gate_out, float* gate_logits_out, uint32_t* sample_flags, void* ws,
+                                  size_t ws_bytes, void* stream) {
+  if (!m || !budget || !kappa || !k || !vis_off || !text_len || !layer_gate_out || !group_gate_out)
+    return SVL_ERR_INVALID_ARG;
+  const svl_model_desc& d = m->d;
+  if (!m->w.kap_w1 || !m->w.kap_w2 || !m->w.gate_w || !m->w.gate_c) return SVL_ERR_UNSUPPORTED;
+  CtlArgs c;
+  std::memset(&c, 0, sizeof(c));
+  c.B = B;
+  c.L = d.n_layers;
+  c.G = d.n_groups;
+  c.P = d.n_prefix;
+  c.D = d.d_model;
+  c.H = d.h_ctrl;
+  c.Dkv = static_cast<long long>(d.n_kv_heads) * (d.d_model / d.n_heads);
+  c.Di = d.d_ffn;
+  c.V = d.vocab;
+  c.project = project ? 1 : 0;
+  c.kappa = kappa;
+  c.budget = budget;
+  c.k = k;
+  c.vis_off = vis_off;
+  c.text_len = text_len;
+  c.kap_w1 = static_cast<const __nv_bfloat16*>(m->w.kap_w1);
+  c.kap_w2 = static_cast<const __nv_bfloat16*>(m->w.kap_w2);
+  c.gate_w = static_cast<const __nv_bfloat16*>(m->w.gate_w);
+  c.gate_c = m->w.gate_c;
+  c.gate_logits = gate_logits_out;
+  c.flags = sample_flags;
+  return prefill_impl(m, B, t_cap, X, cu_seqlens, pos, layer_gate_out, group_gate_out, logits_mode, logits, ws,
+                      ws_bytes, stream, &c);
 }
 
 svl_status svl_flops(const svl_model_desc* d, int32_t s_text, int32_t s_vis, int32_t n_vis, const uint8_t* lg,

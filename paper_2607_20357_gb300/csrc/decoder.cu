@@ -240,6 +240,125 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
 
 void launch_schedule(const ScheduleArgs& a, cudaStream_t s) { launch_pdl(schedule_kernel, a.L, 256, 0, s, a); }
 
+// LLM-side compute controller (Sec. 3.2), one block per sample:
+//   h~ = h_b^(P) + W_k2 SiLU(W_k1 PE(kappa))          (Eq. 7; h_b^(P) = the budget
+//                                                     token's row after P layers)
+//   logit[l - P][j] = W_h[(l - P) G + j] . h~ + c_h    (gate head)
+//   group (l, j) runs if l < P or logit > 0 (sigma > 0.5; no noise at inference)
+// With `project` and b < 1, the token count being committed, the fewest
+// active groups of layers >= P are switched off, lowest logit first (equal
+// logits: lower l * G + j first), until Eq. 8 at S = S_text + k is within
+// b * C_full (Sec. 3.3 "Inference").
+constexpr int kCtlThreads = 256;
+__global__ void __launch_bounds__(kCtlThreads) controller_kernel(CtlArgs a) {
+  extern __shared__ float ctl_smem[];
+  float* ht = ctl_smem;           // [D] fused state
+  float* lg = ctl_smem + a.D;     // [(L - P) * G] gate logits
+  __shared__ double pe[256], hid[256];
+  __shared__ int keep_groups;
+  __shared__ long long n_on_sh;
+  pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int L = a.L, G = a.G, P = min(a.P, a.L), H = a.H, D = a.D;
+  const int ng = (L - P) * G;
+  const int row = a.cu_seqlens[b + 1] - 1;
+  // e_kappa = W_k2 SiLU(W_k1 PE(kappa)), PE as Eq. 5
+  if (tid < H) {
+    const int half = H / 2, f = tid < half ? tid : tid - half;
+    const double arg = 1000.0 * static_cast<double>(a.kappa[b]) * pow(10000.0, -2.0 * f / H);
+    pe[tid] = tid < half ? sin(arg) : cos(arg);
+  }
+  if (tid == 0) {
+    keep_groups = -1;
+    n_on_sh = 0;
+  }
+  __syncthreads();
+  if (tid < H) {
+    double s = 0.0;
+    for (int j = 0; j < H; ++j) s += static_cast<double>(__bfloat162float(a.kap_w1[tid * H + j])) * pe[j];
+    hid[tid] = s / (1.0 + exp(-s));
+  }
+  __syncthreads();
+  for (int d = tid; d < D; d += blockDim.x) {
+    double s = row >= 0 ? static_cast<double>(__bfloat162float(a.X[static_cast<size_t>(row) * D + d])) : 0.0;
+    for (int j = 0; j < H; ++j) s += static_cast<double>(__bfloat162float(a.kap_w2[static_cast<size_t>(d) * H + j])) * hid[j];
+    ht[d] = static_cast<float>(s);
+  }
+  __syncthreads();
+  // gate head: one warp per logit, lanes along D
+  for (int o = warp; o < ng; o += blockDim.x / 32) {
+    const __nv_bfloat16* wr = a.gate_w + static_cast<size_t>(o) * D;
+    float acc = 0.f;
+    for (int d = lane; d < D; d += 32) acc = fmaf(__bfloat162float(wr[d]), ht[d], acc);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+    if (lane == 0) {
+      lg[o] = acc + a.gate_c[o];
+      if (a.gate_logits) a.gate_logits[static_cast<size_t>(b) * ng + o] = lg[o];
+    }
+  }
+  __syncthreads();
+  // raw gates and their count (prefix groups always on)
+  int on = 0;
+  for (int idx = tid; idx < L * G; idx += blockDim.x) on += (idx < P * G || lg[idx - P * G] > 0.f) ? 1 : 0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) on += __shfl_xor_sync(0xffffffffu, on, off);
+  if (lane == 0 && on) atomicAdd(reinterpret_cast<unsigned long long*>(&n_on_sh), static_cast<unsigned long long>(on));
+  __syncthreads();
+  uint32_t flags = 0;
+  int drop = 0;
+  if (a.project && a.budget[b] < 1.0f) {
+    const long long D64 = D, Dkv = a.Dkv, Di = a.Di, V = a.V, G64 = G, L64 = L;
+    const long long lin = 4 * D64 * D64 + 4 * D64 * Dkv + 6 * D64 * Di;
+    const long long nv = a.vis_off[b + 1] - a.vis_off[b], st = a.text_len[b];
+    const long long S_full = nv + st, S = st + a.k[b];
+    const long long c_full = G64 * L64 * (lin * S_full + 4 * D64 * S_full * S_full) + G64 * 2 * D64 * V * S_full;
+    const double limit = static_cast<double>(a.budget[b]) * static_cast<double>(c_full);
+    const long long per = lin * S + 4 * D64 * S * S, lm = G64 * 2 * D64 * V * S;
+    const long long n_on = n_on_sh, n_min = static_cast<long long>(P) * G;
+    if (static_cast<double>(n_on * per + lm) > limit) {
+      for (long long nk = n_min + tid; nk < n_on; nk += blockDim.x)
+        if (static_cast<double>(nk * per + lm) <= limit) atomicMax(&keep_groups, static_cast<int>(nk));
+      __syncthreads();
+      if (n_on > n_min) flags |= SVL_FLAG_GROUPS_DROPPED;
+      if (keep_groups < 0) flags |= SVL_FLAG_OVER_BUDGET;
+      drop = static_cast<int>(n_on - (keep_groups < 0 ? n_min : keep_groups));
+    }
+  }
+  uint8_t* go = a.group_gate + static_cast<size_t>(b) * L * G;
+  for (int idx = tid; idx < L * G; idx += blockDim.x) {
+    bool active = idx < P * G || lg[idx - P * G] > 0.f;
+    if (active && drop > 0 && idx >= P * G) {
+      const float v = lg[idx - P * G];
+      int rank = 0;
+      for (int j = P * G; j < L * G; ++j) {
+        const float w = lg[j - P * G];
+        if (w > 0.f && (w < v || (w == v && j < idx))) ++rank;
+      }
+      active = rank >= drop;
+    }
+    go[idx] = active ? 1 : 0;
+  }
+  __syncthreads();
+  for (int l = tid; l < L; l += blockDim.x) {
+    int any = 0;
+    for (int j = 0; j < G; ++j) any |= go[l * G + j];
+    a.layer_gate[static_cast<size_t>(b) * L + l] = any ? 1 : 0;
+  }
+  if (tid == 0 && a.flags) a.flags[b] |= flags;
+}
+
+void launch_controller(const CtlArgs& a, cudaStream_t s) {
+  const size_t smem = sizeof(float) * (static_cast<size_t>(a.D) + static_cast<size_t>(a.L - min(a.P, a.L)) * a.G);
+  static bool configured = false;
+  if (!configured && smem > 48 * 1024) {
+    cudaFuncSetAttribute(controller_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 160 * 1024);
+    configured = true;
+  }
+  launch_pdl(controller_kernel, a.B, kCtlThreads, smem, s, a);
+}
+
 // ---------------------------------------------------------------- RMSNorm
 SVL_DEVINL int find_sample(const int* cu, int B, int r) {
   int lo = 0, hi = B;

@@ -29,6 +29,8 @@ struct SelectArgs {
   const float* gate_logits;  // [B, L, G]
   uint8_t* layer_gate_out;   // [B, L] projected gates (paper rule)
   uint8_t* group_gate_out;   // [B, L, G]
+  int threshold_only;        // paper rule, gates decided later: k = #{z > 0}
+  float* kappa;              // [B] sum sigma(z) / N, or nullptr
 };
 
 void launch_budget_embed(const float* budget, const __nv_bfloat16* w1, const __nv_bfloat16* w2, int H, int B,
@@ -55,8 +57,12 @@ struct PackArgs {
   int use_projector;       // 1: visual rows go to the staging buffer
   __nv_bfloat16* stage;    // [kept_total, c_vis]
   int* row_map;            // [kept_total] -> row of X
+  const __nv_bfloat16* tok_rows;  // [B, D] budget-token rows appended after the text, or nullptr
   uint32_t* status;
 };
+// e^LLM_b = W2 SiLU(W1 PE(b)) (Sec. 3.2: the Eq. 5 encoding, its own MLP to D), bf16 rows.
+void launch_llm_budget_embed(const float* budget, const __nv_bfloat16* w1, const __nv_bfloat16* w2, int H, int D,
+                             int B, __nv_bfloat16* out, cudaStream_t s);
 void launch_pack_offsets(const PackArgs& a, cudaStream_t s);
 void launch_offsets_diff(const int* off, int* len, int B, cudaStream_t s);
 void launch_pack_gather(const PackArgs& a, cudaStream_t s);
@@ -82,6 +88,32 @@ struct ScheduleArgs {
   uint32_t* status;
 };
 void launch_schedule(const ScheduleArgs& a, cudaStream_t s);
+
+// LLM-side compute controller (Sec. 3.2, Eq. 7), one block per sample: the
+// budget token's state after the prefix layers plus MLP_kappa(PE(kappa)),
+// the linear gate head, gates = logit > 0 for layers >= P, and (project) the
+// group-only budget projection at S = S_text + k.
+struct CtlArgs {
+  int B, L, G, P, D, H;
+  long long Dkv, Di, V;
+  int project;
+  const __nv_bfloat16* X;
+  const int* cu_seqlens;
+  const float* kappa;
+  const float* budget;
+  const int* k;
+  const int* vis_off;
+  const int* text_len;
+  const __nv_bfloat16* kap_w1;
+  const __nv_bfloat16* kap_w2;
+  const __nv_bfloat16* gate_w;
+  const float* gate_c;
+  float* gate_logits;   // [B, L - P, G] or nullptr
+  uint8_t* layer_gate;  // [B, L]
+  uint8_t* group_gate;  // [B, L, G]
+  uint32_t* flags;      // [B] or nullptr
+};
+void launch_controller(const CtlArgs& a, cudaStream_t s);
 
 struct NormArgs {
   int t_cap, D, B;

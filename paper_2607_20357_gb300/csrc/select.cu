@@ -87,6 +87,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
   __shared__ int s_prefix_cnt[2];
   __shared__ long long n_on_sum;  // updated with 64-bit atomics
   __shared__ int n_pos, keep_groups;
+  __shared__ double kappa_sum;
   pdl_trigger();
   pdl_wait();
 
@@ -101,6 +102,7 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
     best_k = -1;
     n_pos = 0;
     keep_groups = -1;
+    kappa_sum = 0.0;
   }
   __syncthreads();
   const float* gl = a.gate_logits ? a.gate_logits + static_cast<size_t>(b) * a.L * a.G : nullptr;
@@ -110,25 +112,39 @@ __global__ void __launch_bounds__(kSelectThreads) select_kernel(SelectArgs a) {
     return gl ? gl[idx] > 0.f : (a.layer_gate[b * a.L + l] && a.group_gate[b * a.L * a.G + idx]);
   };
   {
-    int on = 0;  // active (layer, group) pairs of this sample
-    for (int idx = tid; idx < a.L * a.G; idx += blockDim.x) on += active(idx) ? 1 : 0;
+    // active (layer, group) pairs of this sample; not needed (and no gates
+    // given) when the gates are decided later
+    int on = 0;
+    if (!a.threshold_only)
+      for (int idx = tid; idx < a.L * a.G; idx += blockDim.x) on += active(idx) ? 1 : 0;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) on += __shfl_xor_sync(0xffffffffu, on, o);
     if ((tid & 31) == 0 && on) atomicAdd(reinterpret_cast<unsigned long long*>(&n_on_sum), static_cast<unsigned long long>(on));
-    if (gl) {
+    if (gl || a.threshold_only) {
       int pos = 0;  // logits z > 0, i.e. sigma(z) > 0.5
       for (int i = tid; i < n; i += blockDim.x) pos += a.scores[v0 + i] > 0.f ? 1 : 0;
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) pos += __shfl_xor_sync(0xffffffffu, pos, o);
       if ((tid & 31) == 0 && pos) atomicAdd(&n_pos, pos);
     }
+    if (a.kappa) {
+      // survival rate kappa = sum sigma(z_i) / N that conditions the compute controller (Sec. 3.2)
+      double sg = 0.0;
+      for (int i = tid; i < n; i += blockDim.x) sg += 1.0 / (1.0 + exp(-static_cast<double>(a.scores[v0 + i])));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sg += __shfl_xor_sync(0xffffffffu, sg, o);
+      if ((tid & 31) == 0) atomicAdd(&kappa_sum, sg);
+    }
   }
   __syncthreads();
   int k;
   uint32_t flags = 0;
   const int kc = a.keep_count ? a.keep_count[b] : -1;
+  if (tid == 0 && a.kappa) a.kappa[b] = n > 0 ? static_cast<float>(kappa_sum / n) : 0.f;
   if (kc >= 0) {
     k = min(kc, n);
+  } else if (a.threshold_only) {
+    k = n_pos;  // the compute controller decides the gates later
   } else {
     const long long D = a.D, Dkv = a.Dkv, Di = a.Di, V = a.V, G = a.G, L = a.L;
     const long long lin = 4 * D * D + 4 * D * Dkv + 6 * D * Di;

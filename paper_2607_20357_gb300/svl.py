@@ -28,7 +28,7 @@ SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_s
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
            "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches", "svl_selftest_wait_timeout",
-           "svl_workspace_size_for", "svl_score_select_paper"]
+           "svl_workspace_size_for", "svl_score_select_paper", "svl_pack_controlled", "svl_controlled_prefill"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
@@ -52,7 +52,9 @@ class Weights(ctypes.Structure):
     _fields_ = [("ctrl_w1", ctypes.c_void_p), ("ctrl_w2", ctypes.c_void_p), ("ctrl_c2", ctypes.c_float),
                 ("bud_w1", ctypes.c_void_p), ("bud_w2", ctypes.c_void_p), ("proj_w1", ctypes.c_void_p),
                 ("proj_w2", ctypes.c_void_p), ("embed", ctypes.c_void_p), ("final_norm", ctypes.c_void_p),
-                ("lm_head", ctypes.c_void_p), ("layers", ctypes.POINTER(LayerWeights))]
+                ("lm_head", ctypes.c_void_p), ("layers", ctypes.POINTER(LayerWeights)),
+                ("llm_bud_w1", ctypes.c_void_p), ("llm_bud_w2", ctypes.c_void_p), ("kap_w1", ctypes.c_void_p),
+                ("kap_w2", ctypes.c_void_p), ("gate_w", ctypes.c_void_p), ("gate_c", ctypes.c_void_p)]
 
 
 def lib():
@@ -94,8 +96,12 @@ def lib():
         L.svl_profile_stop.restype = ctypes.c_int
         L.svl_tag_name.argtypes = [i32]
         L.svl_tag_name.restype = ctypes.c_char_p
-        L.svl_score_select_paper.argtypes = [vp, i32, i32] + [vp] * 14 + [sz, vp]
+        L.svl_score_select_paper.argtypes = [vp, i32, i32] + [vp] * 15 + [sz, vp]
         L.svl_score_select_paper.restype = ctypes.c_int
+        L.svl_pack_controlled.argtypes = [vp, i32, i32, i32] + [vp] * 11 + [sz, vp]
+        L.svl_pack_controlled.restype = ctypes.c_int
+        L.svl_controlled_prefill.argtypes = [vp, i32, i32] + [vp] * 8 + [i32, i32] + [vp] * 6 + [sz, vp]
+        L.svl_controlled_prefill.restype = ctypes.c_int
         L.svl_score_select_noalloc.argtypes = [vp, i32, i32] + [vp] * 13
         L.svl_score_select_noalloc.restype = ctypes.c_int
         L.svl_profile_launches.argtypes = [vp, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_float), i32,
@@ -168,14 +174,31 @@ def svl_score_select(model, B, n_vis_total, vis_feats, vis_off, text_len, budget
 
 
 def svl_score_select_paper(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, gate_logits,
-                           scores, k, kept_idx, kept_off, sample_flags, layer_gate_out, group_gate_out, workspace,
-                           workspace_bytes, stream=None):
+                           scores, k, kept_idx, kept_off, sample_flags, layer_gate_out, group_gate_out, kappa_out,
+                           workspace, workspace_bytes, stream=None):
     """The paper's own inference rule (sigma(z) > 0.5 tokens, gates from the
-    compute controller's logits, budget projection): see svl.h."""
+    compute controller's logits or decided later, budget projection): see svl.h."""
     _check("svl_score_select_paper", lib().svl_score_select_paper(
         model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
         _p(gate_logits), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags), _p(layer_gate_out),
-        _p(group_gate_out), _p(workspace), int(workspace_bytes), _stream(stream)))
+        _p(group_gate_out), _p(kappa_out), _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_pack_controlled(model, B, n_vis_total, n_text_total, vis_feats, vis_off, kept_idx, kept_off, text_ids,
+                        text_off, budget, X, cu_seqlens, pos, workspace, workspace_bytes, stream=None):
+    _check("svl_pack_controlled", lib().svl_pack_controlled(
+        model, int(B), int(n_vis_total), int(n_text_total), _p(vis_feats), _p(vis_off), _p(kept_idx),
+        _p(kept_off), _p(text_ids), _p(text_off), _p(budget), _p(X), _p(cu_seqlens), _p(pos), _p(workspace),
+        int(workspace_bytes), _stream(stream)))
+
+
+def svl_controlled_prefill(model, B, t_cap, X, cu_seqlens, pos, budget, kappa, k, vis_off, text_len, project,
+                           logits_mode, logits, layer_gate_out, group_gate_out, gate_logits_out, sample_flags,
+                           workspace, workspace_bytes, stream=None):
+    _check("svl_controlled_prefill", lib().svl_controlled_prefill(
+        model, int(B), int(t_cap), _p(X), _p(cu_seqlens), _p(pos), _p(budget), _p(kappa), _p(k), _p(vis_off),
+        _p(text_len), int(project), int(logits_mode), _p(logits), _p(layer_gate_out), _p(group_gate_out),
+        _p(gate_logits_out), _p(sample_flags), _p(workspace), int(workspace_bytes), _stream(stream)))
 
 
 def svl_score_select_noalloc(model, B, n_vis_total, vis_feats, vis_off, text_len, budget, keep_count, layer_gate,
@@ -297,7 +320,8 @@ class GatedPrefill:
         self._wts = Weights(weights["ctrl_w1"].data_ptr(), weights["ctrl_w2"].data_ptr(), float(weights["ctrl_c2"]),
                             weights["bud_w1"].data_ptr(), weights["bud_w2"].data_ptr(), opt("proj_w1"),
                             opt("proj_w2"), weights["embed"].data_ptr(), weights["final_norm"].data_ptr(),
-                            weights["lm_head"].data_ptr(), lw)
+                            weights["lm_head"].data_ptr(), lw, opt("llm_bud_w1"), opt("llm_bud_w2"), opt("kap_w1"),
+                            opt("kap_w2"), opt("gate_w"), opt("gate_c"))
         self.handle = svl_model_create(self.desc, self._wts)
         self._ws = None
         self._ws_key = None
@@ -325,7 +349,7 @@ class GatedPrefill:
         nv = batch["vis"].shape[0]
         nt = int(batch["text_ids"].shape[0])
         dev = batch["vis"].device
-        t_cap = nv + nt
+        t_cap = nv + nt + B  # room for one budget-token row per sample (rule="controller")
         i32 = dict(dtype=torch.int32, device=dev)
         return {
             "scores": torch.empty(max(nv, 1), dtype=torch.float32, device=dev),
@@ -339,30 +363,56 @@ class GatedPrefill:
             "logits": torch.empty((B if logits_mode == SVL_LOGITS_LAST else max(t_cap, 1)), d.vocab,
                                   dtype=torch.float32, device=dev),
             "text_len": (batch["text_off"][1:] - batch["text_off"][:-1]).to(torch.int32).contiguous(),
-            # projected gates of the paper's rule (rule="paper")
+            # projected gates of the paper's rule (rule="paper") or the controller's (rule="controller")
             "layer_gate": torch.empty(B, d.n_layers, dtype=torch.uint8, device=dev),
             "group_gate": torch.empty(B, d.n_layers, d.n_groups, dtype=torch.uint8, device=dev),
+            "kappa": torch.empty(B, dtype=torch.float32, device=dev),
+            "gate_logits": torch.empty(B, max(d.n_layers - d.n_prefix, 1), d.n_groups, dtype=torch.float32,
+                                       device=dev),
         }
+
+    def _run_controlled(self, batch, out, logits_mode, stream, stages, ws, wsb, nv, nt):
+        B = batch["B"]
+        if "select" in stages:
+            svl_score_select_paper(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"],
+                                   batch["budget"], batch["keep_count"], None, out["scores"], out["k"],
+                                   out["kept_idx"], out["kept_off"], out["flags"], None, None, out["kappa"], ws, wsb,
+                                   stream)
+        if "pack" in stages:
+            svl_pack_controlled(self.handle, B, nv, nt, batch["vis"], batch["vis_off"], out["kept_idx"],
+                                out["kept_off"], batch["text_ids"], batch["text_off"], batch["budget"], out["X"],
+                                out["cu_seqlens"], out["pos"], ws, wsb, stream)
+        if "prefill" in stages:
+            svl_controlled_prefill(self.handle, B, nv + nt + B, out["X"], out["cu_seqlens"], out["pos"],
+                                   batch["budget"], out["kappa"], out["k"], batch["vis_off"], out["text_len"], 1,
+                                   logits_mode, out["logits"], out["layer_gate"], out["group_gate"],
+                                   out["gate_logits"], out["flags"], ws, wsb, stream)
+        return out
 
     def run(self, batch: dict, out: Optional[dict] = None, logits_mode: int = SVL_LOGITS_LAST, stream=None,
             stages=("select", "pack", "prefill"), rule: str = "budget"):
         """rule="budget": k from the budget for the given gates (the hot path);
         rule="paper": the paper's own inference rule from batch["gate_logits"]
         ([B, L, G] compute-controller logits), whose projected gates (in
-        out["layer_gate"], out["group_gate"]) then drive the prefill."""
+        out["layer_gate"], out["group_gate"]) then drive the prefill;
+        rule="controller": tokens with z > 0, the budget token appended, and
+        the compute controller deciding the gates on the device after the
+        prefix layers (out["kappa"], out["gate_logits"], out gates)."""
         B = batch["B"]
         nv = batch["vis"].shape[0]
         nt = int(batch["text_ids"].shape[0])
         out = out or self.alloc_outputs(batch, logits_mode)
         ws, wsb = self.workspace(B, nv, nt, batch["vis"].device, stages)
-        if rule not in ("budget", "paper"):
+        if rule not in ("budget", "paper", "controller"):
             raise ValueError(f"unknown rule {rule!r}")
+        if rule == "controller":
+            return self._run_controlled(batch, out, logits_mode, stream, stages, ws, wsb, nv, nt)
         gates = (out["layer_gate"], out["group_gate"]) if rule == "paper" else (batch["layer_gate"], batch["group_gate"])
         if "select" in stages and rule == "paper":
             svl_score_select_paper(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"],
                                    batch["budget"], batch["keep_count"], batch["gate_logits"], out["scores"],
                                    out["k"], out["kept_idx"], out["kept_off"], out["flags"], out["layer_gate"],
-                                   out["group_gate"], ws, wsb, stream)
+                                   out["group_gate"], out["kappa"], ws, wsb, stream)
         elif "select" in stages:
             svl_score_select(self.handle, B, nv, batch["vis"], batch["vis_off"], out["text_len"], batch["budget"],
                              batch["keep_count"], batch["layer_gate"], batch["group_gate"], out["scores"], out["k"],
