@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--hbm-only", type=str, default="",
                     help="comma-separated batch multipliers: run only the token-controller/pack sweep "
                          "(for small profiler captures)")
+    ap.add_argument("--workload", default=WORKLOAD, choices=["llava", "llava13b"],
+                    help="llava (the benchmark line) or llava13b (the same batch on LLaVA-1.5-13B shapes)")
     ap.add_argument("--layers", type=int, default=0,
                     help="decoder layers (default: all 32). Fewer layers only for small profiler captures; "
                          "such a line is not the benchmark value")
@@ -69,15 +71,23 @@ def peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
 
+def weight_count(d):
+    dh = d.d_model // d.n_heads
+    per = d.d_model * (d.n_heads * dh * 2 + 2 * d.n_kv_heads * dh) + 3 * d.d_model * d.d_ffn
+    return d.n_layers * per + 2 * d.vocab * d.d_model
+
+
 def workload_config(wl, batch):
     d = wl.dims
+    name = "LLaVA-1.5-7B" if wl.name == "llava" else "LLaVA-1.5-13B"
     return {
-        "workload": "LLaVA-1.5-7B-shaped gated prefill: B=16, 576 visual (C_v 1024, MLP projector) + 64 text "
-                    "tokens, 32 layers d4096 h32 ffn11008 V32000, G=4 head groups, budgets 0.25/0.5/0.75/1.0",
+        "workload": f"{name}-shaped gated prefill: B={batch}, 576 visual (C_v 1024, MLP projector) + 64 text "
+                    f"tokens, {d.n_layers} layers d{d.d_model} h{d.n_heads} ffn{d.d_ffn} V{d.vocab}, "
+                    f"G={d.n_groups} head groups, {d.n_prefix} prefix layers, budgets 0.25/0.5/0.75/1.0",
         "batch": batch, "n_vis": wl.n_vis[0], "s_text": wl.s_text[0], "budgets": list(wl.budgets),
         "layers": d.n_layers, "d_model": d.d_model, "heads": d.n_heads, "d_ffn": d.d_ffn, "vocab": d.vocab,
         "groups": d.n_groups, "gates": wl.gates,
-        "l2": "not flushed: each step streams 13 GB of weights through the 129 MB L2",
+        "l2": f"not flushed: each step streams {2 * weight_count(d) / 1e9:.0f} GB of weights through the 129 MB L2",
         "parallelism": "replicas (independent batches per GPU, no collective)",
     }
 
@@ -207,7 +217,7 @@ def run_reference(args, rank, world):
     0-1 of 32 timed and scaled to the full depth."""
     if rank != 0:
         return
-    wl = synth.WORKLOADS[WORKLOAD]
+    wl = synth.WORKLOADS[args.workload]
     dims = wl.dims
     nl = 2
     w = synth.make_weights(dims, SEED, device="cpu", layers=range(nl))
@@ -246,7 +256,7 @@ def run_ours(args, rank, world, local_rank):
     from paper_2607_20357_gb300 import svl
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    wl = synth.WORKLOADS[WORKLOAD]
+    wl = synth.WORKLOADS[args.workload]
     if args.layers:
         wl = synth.dataclasses.replace(wl, dims=synth.reduced(wl.dims, n_layers=args.layers))
     dims = wl.dims

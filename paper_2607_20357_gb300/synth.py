@@ -67,6 +67,10 @@ LLAVA7B = dict(n_layers=32, d_model=4096, n_heads=32, n_kv_heads=32, d_ffn=11008
                vocab=32000, n_groups=4, n_prefix=0, c_vis=1024, h_ctrl=64,
                proj_hidden=4096, rms_eps=1e-5, rope_theta=1e4)
 
+LLAVA13B = dict(n_layers=40, d_model=5120, n_heads=40, n_kv_heads=40, d_ffn=13824,
+                vocab=32000, n_groups=4, n_prefix=20, c_vis=1024, h_ctrl=64,
+                proj_hidden=5120, rms_eps=1e-5, rope_theta=1e4)
+
 WORKLOADS = {
     # 64 visual tokens of dim 256, 16 text ids, MLP 256->64->1 scorer, keep 32,
     # 2-layer d=256 decoder, 4 heads, head gates Bernoulli(0.75).
@@ -95,6 +99,12 @@ WORKLOADS = {
         "video", ModelDims(**LLAVA7B),
         batch=2, n_vis=(4608, 4608), s_text=(64, 64), budgets=(0.1, 0.25, 0.5),
         gates="all_on", features="video"),
+    # LLaVA-1.5-13B (Sec. 4.4: 40 language layers, a fixed 20-layer prefix):
+    # the LLaVA batch on the larger backbone.
+    "llava13b": Workload(
+        "llava13b", ModelDims(**LLAVA13B),
+        batch=16, n_vis=(576, 576), s_text=(64, 64), budgets=(0.25, 0.5, 0.75, 1.0),
+        gates="all_on", features="lowrank_clusters"),
     # Serving mix: 64 samples, text 16..256, budgets U[0.1,1], budget-scaled gates.
     "mixed": Workload(
         "mixed", ModelDims(**LLAVA7B),

@@ -9,8 +9,8 @@ already exceeds 2e-2 (32 layers: about 3.2e-2).
 
 The LLaVA-1.5-7B batch runs with all 32 layers; the Qwen2-VL-7B, video and
 mixed-serving batches keep their full batch, sequence and width shapes with
-the decoder cut to 2 layers so the float64 oracle stays within seconds per
-sample.
+the decoder cut to 2 layers (LLaVA-1.5-13B: 3 layers, one of them a prefix
+layer) so the float64 oracle stays within seconds per sample.
 """
 import numpy as np
 import pytest
@@ -84,3 +84,18 @@ def test_mixed_full_batch_two_layers():
     wl = synth.WORKLOADS["mixed"]
     dims = synth.reduced(wl.dims, n_layers=2)
     print(_run_full(wl, dims, 5000, samples=[0, 31, 63]))
+
+
+def test_llava13b_full_shapes_three_layers_with_prefix():
+    """LLaVA-1.5-13B widths (d 5120, 40 heads, FFN 13824) on the full batch,
+    the decoder cut to 3 layers of which 1 is a prefix layer (the model has a
+    20-layer prefix over 40 layers), with budget-scaled head gates on the
+    others."""
+    wl = synth.WORKLOADS["llava13b"]
+    dims = synth.reduced(wl.dims, n_layers=3, n_prefix=1)
+
+    def gate(batch):
+        g = torch.Generator().manual_seed(13)
+        batch["group_gate"].copy_((torch.rand(batch["group_gate"].shape, generator=g) < 0.7).to(torch.uint8))
+
+    print(_run_full(wl, dims, 1300, samples=[0, 9], budget=0.5, modify=gate))
