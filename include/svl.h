@@ -246,6 +246,40 @@ svl_status svl_controlled_prefill(svl_model* model, int32_t B, int32_t t_cap, vo
                                   uint8_t* group_gate_out, float* gate_logits_out, uint32_t* sample_flags,
                                   void* workspace, size_t workspace_bytes, void* stream);
 
+/* ------------------------------------------------------------------------
+ * Gated decode with a KV cache (the paper leaves decode open, Sec. 5). Each
+ * sample keeps its prefill gates: a gated-off head group has no cached keys
+ * or values and no compute, a skipped layer is bypassed.
+ *
+ * The cache is caller-owned device memory, 16-byte aligned:
+ *   K then V, each [L][B][max_len][A_kv * d_head] bf16; position p of
+ *   sample b at row p. max_len <= the model's max_seq (RoPE table).
+ * svl_kv_cache_size: its bytes (0 on bad arguments). */
+size_t svl_kv_cache_size(const svl_model* model, int32_t B, int32_t max_len);
+
+/* svl_gated_prefill that also stores every layer's keys and values of the
+ * prompt into the cache and writes cache_len[B] (device int32) = the prompt
+ * length S_b of each sample. Errors: as svl_gated_prefill; prompt rows past
+ * max_len are not stored. */
+svl_status svl_gated_prefill_kv(svl_model* model, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                                const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
+                                int32_t logits_mode, float* logits, void* kv_cache, int32_t max_len,
+                                int32_t* cache_len, void* workspace, size_t workspace_bytes, void* stream);
+
+/* One decode step: token tokens[b] (device int32 [B]) is fed to sample b at
+ * position cache_len[b]; its keys and values are appended to the cache, it
+ * attends to positions 0..cache_len[b] under the sample's gates
+ * (layer_gate [B, L], group_gate [B, L, G] as for the prefill), logits[B, V]
+ * (float32) are those of the new position, next_token[B] (device int32, or
+ * NULL) the largest logit (equal logits: lower id), and cache_len[b] is
+ * advanced by one. Workspace: svl_decode_workspace_size(model, B) bytes.
+ * A fed id outside [0, V) or a full cache sets SVL_DEV_BAD_INDEX (the id is
+ * read as 0; a full cache skips the sample's attention). */
+size_t svl_decode_workspace_size(const svl_model* model, int32_t B);
+svl_status svl_decode_step(svl_model* model, int32_t B, const int32_t* tokens, void* kv_cache, int32_t max_len,
+                           int32_t* cache_len, const uint8_t* layer_gate, const uint8_t* group_gate, float* logits,
+                           int32_t* next_token, void* workspace, size_t workspace_bytes, void* stream);
+
 /* svl_score_select without a workspace argument. The paper has no
  *  counterpart: this exists for callers that cannot allocate device memory
  *  for a workspace -- code running during CUDA stream capture (where

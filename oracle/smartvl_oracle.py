@@ -37,6 +37,10 @@ What each function follows:
   its own MLP to D) appended after the text, P prefix layers at full
   capacity, kappa = sum sigma(z_i) / N, the fused state h + MLP_kappa(PE(kappa))
   (Eq. 7), a linear gate head thresholded at 0, the remaining layers gated.
+* ``decode_reference`` -- gated decode, which the paper leaves open (Sec. 5),
+  written without a cache: after feeding tokens t_1..t_n, the logits are
+  those of the forward over [kept visual][text][t_1..t_n] under the prompt's
+  gates, the kept visual tokens fixed by the prompt's own selection.
 * ``paper_rule_sample`` -- Sec. 3.1 and Sec. 3.3 "Inference", the paper's own
   rule: tokens with sigma(z) > 0.5 survive, gates are the compute
   controller's logits thresholded at 0, and for b < 1 the budget projection
@@ -423,6 +427,19 @@ def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
     y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
     logits = make_store("fp64" if mode == "fp64" else "fp32")(weights["lm_head"] @ y)
     return {"z": z, "k": k, "flags": flags, "kept": kept, "hidden": X, "logits": logits}
+
+
+def decode_reference(dims, weights, x, text_ids, budget, layer_gate, group_gate, fed, keep_count=-1, mode="fp32"):
+    """Prompt forward, then one forward per fed token over the extended
+    sequence (the definition a KV cache must reproduce). Returns the prompt's
+    result and the list of per-step results (``logits`` of the new position,
+    ``hidden`` of all rows)."""
+    first = forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate, keep_count, mode)
+    steps = []
+    for n in range(1, len(fed) + 1):
+        ids = np.concatenate([np.asarray(text_ids), np.asarray(fed[:n])])
+        steps.append(forward_sample(dims, weights, x, ids, budget, layer_gate, group_gate, first["k"], mode))
+    return first, steps
 
 
 def forward_batch(dims, weights, batch, mode="fp32", n_layers=None, samples=None):

@@ -656,13 +656,27 @@ svl_status svl_pack_controlled(svl_model* m, int32_t B, int32_t n_vis_total, int
 }
 
 namespace {
+// KV cache of a prefill (store each layer's K, V) or a decode step (one new
+// row per sample: embedding of the fed token, attention against the cache,
+// greedy next token).
+struct StepCtx {
+  __nv_bfloat16* kv;  // [2][L][B][max_len][dkv]
+  int max_len;
+  int decode;
+  int* cache_len;        // [B] decode: positions so far (advanced by one)
+  const int* tokens;     // [B] decode: fed token ids
+  int* next_token;       // [B] decode: greedy next token, or nullptr
+};
+
 // The gated decoder forward. With `ctl` (compute controller, Sec. 3.2) the
 // gate arrays are outputs: they start all on, the controller kernel writes
 // them after the prefix layers, and the device schedule is built again.
+// With `kvx` the keys and values go to the cache (prefill) or the step is a
+// decode step over one row per sample.
 svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
                         const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
                         int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream,
-                        const CtlArgs* ctl) {
+                        const CtlArgs* ctl, const StepCtx* kvx = nullptr) {
   if (!m || B <= 0 || t_cap <= 0 || !X || !cu_seqlens || !pos || !layer_gate || !group_gate || !logits)
     return SVL_ERR_INVALID_ARG;
   if (logits_mode != SVL_LOGITS_LAST && logits_mode != SVL_LOGITS_ALL) return SVL_ERR_INVALID_ARG;
@@ -676,6 +690,13 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   const int hq = d.n_heads * dh, dkv = d.n_kv_heads * dh;
   const int nl = d.n_layers;
   int* counts = at<int>(ws, L.counts);
+  if (kvx && kvx->decode) {
+    // the step's rows: embeddings of the fed tokens at their cache positions
+    Launch L0(m, SVL_TAG_PACK, s);
+    launch_decode_prep(B, d.d_model, d.vocab, kvx->tokens, kvx->cache_len, kvx->max_len,
+                       static_cast<const __nv_bfloat16*>(m->w.embed), static_cast<__nv_bfloat16*>(X),
+                       const_cast<int32_t*>(cu_seqlens), const_cast<int32_t*>(pos), m->d_status, s);
+  }
 
   ScheduleArgs sa;
   sa.B = B;
@@ -825,9 +846,53 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.d_head = dh;
     if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s)) != SVL_OK) return st;
 
-    aa.items = sa.attn_items + static_cast<size_t>(l) * L.attn_cap;
-    aa.count = counts + 4 * nl + l;
-    {
+    const size_t layer_kv = static_cast<size_t>(B) * (kvx ? kvx->max_len : 0) * dkv;
+    if (kvx && kvx->decode) {
+      DecAttnArgs da;
+      std::memset(&da, 0, sizeof(da));
+      da.B = B;
+      da.A = d.n_heads;
+      da.Akv = d.n_kv_heads;
+      da.dh = dh;
+      da.dkv = dkv;
+      da.G = d.n_groups;
+      da.L = nl;
+      da.P = d.n_prefix;
+      da.l = l;
+      da.max_len = kvx->max_len;
+      da.t_pad = static_cast<int>(L.t_pad);
+      da.ldq = hq;
+      da.ldo = hq;
+      da.scale = static_cast<float>(1.0 / std::sqrt(static_cast<double>(dh)));
+      da.cache_len = kvx->cache_len;
+      da.layer_gate = layer_gate;
+      da.group_gate = group_gate;
+      da.q = qb;
+      da.k = kb;
+      da.vt = vb;
+      da.k_cache = kvx->kv + static_cast<size_t>(l) * layer_kv;
+      da.v_cache = kvx->kv + static_cast<size_t>(nl + l) * layer_kv;
+      da.out = ao;
+      Launch L1(m, SVL_TAG_ATTENTION, s);
+      launch_decode_attn(da, s);
+    } else {
+      if (kvx) {
+        KvArgs ka;
+        ka.B = B;
+        ka.dkv = dkv;
+        ka.max_len = kvx->max_len;
+        ka.t_pad = static_cast<int>(L.t_pad);
+        ka.cu_seqlens = cu_seqlens;
+        ka.pos = pos;
+        ka.k = kb;
+        ka.vt = vb;
+        ka.k_cache = kvx->kv + static_cast<size_t>(l) * layer_kv;
+        ka.v_cache = kvx->kv + static_cast<size_t>(nl + l) * layer_kv;
+        Launch L1(m, SVL_TAG_COPY, s);
+        launch_kv_store(ka, t_cap, s);
+      }
+      aa.items = sa.attn_items + static_cast<size_t>(l) * L.attn_cap;
+      aa.count = counts + 4 * nl + l;
       Launch L1(m, SVL_TAG_ATTENTION, s);
       if (launch_attention_tc(aa, gemm_grid(m, L.attn_cap), s) != cudaSuccess) return SVL_ERR_CUDA;
     }
@@ -923,6 +988,13 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ld[0] = d.vocab;
     if ((st = launch(EPI_F32, m, SVL_TAG_LMHEAD, p, static_cast<int64_t>(p.grid_m) * p.grid_n, s)) != SVL_OK) return st;
   }
+  if (kvx && kvx->decode) {
+    Launch L1(m, SVL_TAG_LMHEAD, s);
+    launch_decode_finish(B, d.vocab, logits, kvx->next_token, kvx->cache_len, s);
+  } else if (kvx && kvx->cache_len) {
+    launch_offsets_diff(cu_seqlens, kvx->cache_len, B, s);  // cache length = prompt length
+    g_launches++;
+  }
   return last_error();
 }
 }  // namespace
@@ -969,6 +1041,48 @@ svl_status svl_controlled_prefill(svl_model* m, int32_t B, int32_t t_cap, void* 
   c.flags = sample_flags;
   return prefill_impl(m, B, t_cap, X, cu_seqlens, pos, layer_gate_out, group_gate_out, logits_mode, logits, ws,
                       ws_bytes, stream, &c);
+}
+
+size_t svl_kv_cache_size(const svl_model* m, int32_t B, int32_t max_len) {
+  if (!m || B <= 0 || max_len <= 0) return 0;
+  const size_t dkv = static_cast<size_t>(m->d.n_kv_heads) * (m->d.d_model / m->d.n_heads);
+  return 2 * sizeof(__nv_bfloat16) * static_cast<size_t>(m->d.n_layers) * B * max_len * dkv;
+}
+
+svl_status svl_gated_prefill_kv(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
+                                const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
+                                int32_t logits_mode, float* logits, void* kv_cache, int32_t max_len,
+                                int32_t* cache_len, void* ws, size_t ws_bytes, void* stream) {
+  if (!m || !kv_cache || !cache_len || max_len <= 0 || max_len > m->d.max_seq || !aligned16(kv_cache))
+    return SVL_ERR_INVALID_ARG;
+  StepCtx kx{static_cast<__nv_bfloat16*>(kv_cache), max_len, 0, cache_len, nullptr, nullptr};
+  return prefill_impl(m, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, logits_mode, logits, ws, ws_bytes,
+                      stream, nullptr, &kx);
+}
+
+size_t svl_decode_workspace_size(const svl_model* m, int32_t B) {
+  if (!m || B <= 0) return 0;
+  const size_t head = align256(2 * static_cast<size_t>(B) * m->d.d_model) + align256(4 * (B + 1)) + align256(4 * B);
+  return head + pre_layout(m->d, B, B).total;
+}
+
+svl_status svl_decode_step(svl_model* m, int32_t B, const int32_t* tokens, void* kv_cache, int32_t max_len,
+                           int32_t* cache_len, const uint8_t* layer_gate, const uint8_t* group_gate, float* logits,
+                           int32_t* next_token, void* ws, size_t ws_bytes, void* stream) {
+  if (!m || B <= 0 || !tokens || !kv_cache || max_len <= 0 || max_len > m->d.max_seq || !cache_len ||
+      !layer_gate || !group_gate || !logits || !aligned16(kv_cache) || !ws)
+    return SVL_ERR_INVALID_ARG;
+  if (ws_bytes < svl_decode_workspace_size(m, B)) return SVL_ERR_WORKSPACE;
+  // the step's rows, cu_seqlens and positions live at the head of the workspace
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  const size_t xb = align256(2 * static_cast<size_t>(B) * m->d.d_model), cb = align256(4 * (B + 1)),
+               pb = align256(4 * B);
+  void* X = base;
+  int32_t* cu = reinterpret_cast<int32_t*>(base + xb);
+  int32_t* pos = reinterpret_cast<int32_t*>(base + xb + cb);
+  StepCtx kx{static_cast<__nv_bfloat16*>(kv_cache), max_len, 1, cache_len, tokens, next_token};
+  return prefill_impl(m, B, B, X, cu, pos, layer_gate, group_gate, SVL_LOGITS_LAST, logits, base + xb + cb + pb,
+                      ws_bytes - (xb + cb + pb), stream, nullptr, &kx);
 }
 
 svl_status svl_flops(const svl_model_desc* d, int32_t s_text, int32_t s_vis, int32_t n_vis, const uint8_t* lg,

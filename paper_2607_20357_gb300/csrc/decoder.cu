@@ -360,14 +360,6 @@ void launch_controller(const CtlArgs& a, cudaStream_t s) {
 }
 
 // ---------------------------------------------------------------- RMSNorm
-SVL_DEVINL int find_sample(const int* cu, int B, int r) {
-  int lo = 0, hi = B;
-  while (hi - lo > 1) {
-    const int mid = (lo + hi) >> 1;
-    if (cu[mid] <= r) lo = mid; else hi = mid;
-  }
-  return lo;
-}
 
 SVL_DEVINL void norm_row(const __nv_bfloat16* x, const __nv_bfloat16* g, __nv_bfloat16* y, int D, float eps,
                          int lane) {

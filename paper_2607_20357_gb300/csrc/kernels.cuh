@@ -67,6 +67,47 @@ void launch_pack_offsets(const PackArgs& a, cudaStream_t s);
 void launch_offsets_diff(const int* off, int* len, int B, cudaStream_t s);
 void launch_pack_gather(const PackArgs& a, cudaStream_t s);
 
+// Sample b of the packed row r: cu[b] <= r < cu[b+1].
+SVL_DEVINL int find_sample(const int* cu, int B, int r) {
+  int lo = 0, hi = B;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (cu[mid] <= r) lo = mid; else hi = mid;
+  }
+  return lo;
+}
+
+// ---------------------------------------------------------------- decode
+// Cache of one layer: [B][max_len][dkv] bf16 for K and for V.
+struct KvArgs {
+  int B, dkv, max_len, t_pad;
+  const int* cu_seqlens;
+  const int* pos;
+  const __nv_bfloat16* k;   // [t_cap, dkv]
+  const __nv_bfloat16* vt;  // [dkv, t_pad]
+  __nv_bfloat16* k_cache;
+  __nv_bfloat16* v_cache;
+};
+void launch_kv_store(const KvArgs& a, int t_cap, cudaStream_t s);
+void launch_decode_prep(int B, int D, int V, const int* tokens, const int* cache_len, int max_len,
+                        const __nv_bfloat16* embed, __nv_bfloat16* X, int* cu_seqlens, int* pos, uint32_t* status,
+                        cudaStream_t s);
+struct DecAttnArgs {
+  int B, A, Akv, dh, dkv, G, L, P, l, max_len, t_pad, ldq, ldo;
+  float scale;
+  const int* cache_len;
+  const uint8_t* layer_gate;
+  const uint8_t* group_gate;
+  const __nv_bfloat16* q;   // [B, A*dh]
+  const __nv_bfloat16* k;   // [B, dkv] the new tokens' keys
+  const __nv_bfloat16* vt;  // [dkv, t_pad] their values, transposed
+  __nv_bfloat16* k_cache;   // this layer's [B][max_len][dkv]
+  __nv_bfloat16* v_cache;
+  __nv_bfloat16* out;       // [B, A*dh]
+};
+void launch_decode_attn(const DecAttnArgs& a, cudaStream_t s);
+void launch_decode_finish(int B, int V, const float* logits, int* next_token, int* cache_len, cudaStream_t s);
+
 // ---------------------------------------------------------------- decoder
 struct ScheduleArgs {
   int B, L, G, P;

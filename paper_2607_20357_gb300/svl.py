@@ -28,7 +28,8 @@ SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_s
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
            "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches", "svl_selftest_wait_timeout",
-           "svl_workspace_size_for", "svl_score_select_paper", "svl_pack_controlled", "svl_controlled_prefill"]
+           "svl_workspace_size_for", "svl_score_select_paper", "svl_pack_controlled", "svl_controlled_prefill",
+           "svl_kv_cache_size", "svl_gated_prefill_kv", "svl_decode_workspace_size", "svl_decode_step"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
@@ -102,6 +103,14 @@ def lib():
         L.svl_pack_controlled.restype = ctypes.c_int
         L.svl_controlled_prefill.argtypes = [vp, i32, i32] + [vp] * 8 + [i32, i32] + [vp] * 6 + [sz, vp]
         L.svl_controlled_prefill.restype = ctypes.c_int
+        L.svl_kv_cache_size.argtypes = [vp, i32, i32]
+        L.svl_kv_cache_size.restype = sz
+        L.svl_gated_prefill_kv.argtypes = [vp, i32, i32, vp, vp, vp, vp, vp, i32, vp, vp, i32, vp, vp, sz, vp]
+        L.svl_gated_prefill_kv.restype = ctypes.c_int
+        L.svl_decode_workspace_size.argtypes = [vp, i32]
+        L.svl_decode_workspace_size.restype = sz
+        L.svl_decode_step.argtypes = [vp, i32, vp, vp, i32] + [vp] * 6 + [sz, vp]
+        L.svl_decode_step.restype = ctypes.c_int
         L.svl_score_select_noalloc.argtypes = [vp, i32, i32] + [vp] * 13
         L.svl_score_select_noalloc.restype = ctypes.c_int
         L.svl_profile_launches.argtypes = [vp, ctypes.POINTER(i32), ctypes.POINTER(ctypes.c_float), i32,
@@ -182,6 +191,29 @@ def svl_score_select_paper(model, B, n_vis_total, vis_feats, vis_off, text_len, 
         model, int(B), int(n_vis_total), _p(vis_feats), _p(vis_off), _p(text_len), _p(budget), _p(keep_count),
         _p(gate_logits), _p(scores), _p(k), _p(kept_idx), _p(kept_off), _p(sample_flags), _p(layer_gate_out),
         _p(group_gate_out), _p(kappa_out), _p(workspace), int(workspace_bytes), _stream(stream)))
+
+
+def svl_kv_cache_size(model, B, max_len) -> int:
+    return int(lib().svl_kv_cache_size(model, int(B), int(max_len)))
+
+
+def svl_gated_prefill_kv(model, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, logits_mode, logits,
+                         kv_cache, max_len, cache_len, workspace, workspace_bytes, stream=None):
+    _check("svl_gated_prefill_kv", lib().svl_gated_prefill_kv(
+        model, int(B), int(t_cap), _p(X), _p(cu_seqlens), _p(pos), _p(layer_gate), _p(group_gate),
+        int(logits_mode), _p(logits), _p(kv_cache), int(max_len), _p(cache_len), _p(workspace),
+        int(workspace_bytes), _stream(stream)))
+
+
+def svl_decode_workspace_size(model, B) -> int:
+    return int(lib().svl_decode_workspace_size(model, int(B)))
+
+
+def svl_decode_step(model, B, tokens, kv_cache, max_len, cache_len, layer_gate, group_gate, logits, next_token,
+                    workspace, workspace_bytes, stream=None):
+    _check("svl_decode_step", lib().svl_decode_step(
+        model, int(B), _p(tokens), _p(kv_cache), int(max_len), _p(cache_len), _p(layer_gate), _p(group_gate),
+        _p(logits), _p(next_token), _p(workspace), int(workspace_bytes), _stream(stream)))
 
 
 def svl_pack_controlled(model, B, n_vis_total, n_text_total, vis_feats, vis_off, kept_idx, kept_off, text_ids,

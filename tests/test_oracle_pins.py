@@ -564,3 +564,38 @@ def test_project_gates_fewest_lowest_logit_groups():
             g2[idx // 4, idx % 4] = 1
             assert O.prefill_cost_xG(dims, 56, g2.sum(axis=1)) > limit
     assert hits >= 4
+
+
+# ----------------------------------------------------------------------------
+# gated decode (defined without a cache)
+# ----------------------------------------------------------------------------
+def test_decode_reference_first_step_equals_dense_library_forward():
+    """All gates on, keep all: the first fed token's logits are the dense
+    library transformer's last-row logits over prompt + token."""
+    dims = SMALL_ID
+    w = np_weights(dims)
+    x, ids = _sample(dims)
+    L, G = dims.n_layers, dims.n_groups
+    fed = np.array([7, 3])
+    first, steps = O.decode_reference(dims, w, x, ids, 1.0, np.ones(L, np.uint8), np.ones((L, G), np.uint8), fed,
+                                      mode="fp64")
+    X0 = _packed_rows(dims, w, x, np.arange(x.shape[0]), np.concatenate([ids, fed[:1]]))
+    _, logits = dense_forward(X0, w["layers"], w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(steps[0]["logits"], logits, rtol=1e-10, atol=1e-10)
+    assert steps[0]["k"] == steps[1]["k"] == first["k"] == x.shape[0]
+
+
+def test_decode_reference_is_causal():
+    """Appending tokens leaves the hidden states of earlier rows unchanged
+    (what lets a cache keep them), under gates and a budget-fixed k."""
+    dims = synth.reduced(SMALL, n_prefix=1)
+    w = np_weights(dims, seed=5)
+    x, ids = _sample(dims, seed=6)
+    lg = np.array([1, 1, 0], np.uint8)
+    gg = np.array([[1, 1], [0, 1], [1, 1]], np.uint8)
+    first, steps = O.decode_reference(dims, w, x, ids, 0.6, lg, gg, np.array([1, 2, 3]), mode="fp64")
+    prev = first["hidden"]
+    for st in steps:
+        np.testing.assert_allclose(st["hidden"][:prev.shape[0]], prev, rtol=1e-12, atol=1e-12)
+        assert st["hidden"].shape[0] == prev.shape[0] + 1
+        prev = st["hidden"]
