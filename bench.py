@@ -50,6 +50,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-hbm-sweep", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--hbm-only", type=str, default="",
                     help="comma-separated batch multipliers: run only the token-controller/pack sweep "
                          "(for small profiler captures)")
@@ -400,6 +401,10 @@ def run_ours(args, rank, world, local_rank):
     if not args.no_e2e:
         e2e = run_e2e(args, svl, model, batches, dims, world, dev)
 
+    dec = None
+    if rank == 0 and not args.no_decode:
+        dec = run_decode(svl, model, batches[1], dims, dev, pk)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         nl = 16
@@ -423,10 +428,67 @@ def run_ours(args, rank, world, local_rank):
             "per_budget": per_budget, "roofline": roofline, "kernels": kernels,
             "gpu_launches": int(launches), "gpu_launches_per_step": launches / args.steps,
             "wall_s_timed": t_wall, "clocks": clk.summary(), "e2e": e2e, "cpu_baseline": cpu,
-            "hbm_kernels_sweep": hbm,
+            "hbm_kernels_sweep": hbm, "decode": dec,
         }
         print(json.dumps(line), flush=True)
     model.close()
+
+
+def run_decode(svl, model, bt, dims, dev, pk, steps=16, warm=3):
+    """Gated decode after a KV-cache prefill of the budget-0.5 batch: tokens
+    per second over `steps` teacher-forced steps (CUDA events) and the bytes
+    each step must read -- every weight of the active groups once plus the
+    cached keys and values of the active heads -- against the measured HBM
+    bandwidth (decode is bound by streaming them)."""
+    B = bt["B"]
+    nv, nt = int(bt["vis"].shape[0]), int(bt["text_ids"].shape[0])
+    out = model.run(bt, stages=("select", "pack"))
+    max_len = nv // B + nt // B + steps + warm + 8
+    ws, wsb = model.workspace(B, nv, nt, dev, ("prefill",))
+    kv = torch.empty(svl.svl_kv_cache_size(model.handle, B, max_len), dtype=torch.uint8, device=dev)
+    cache_len = torch.zeros(B, dtype=torch.int32, device=dev)
+    svl.svl_gated_prefill_kv(model.handle, B, nv + nt, out["X"], out["cu_seqlens"], out["pos"], bt["layer_gate"],
+                             bt["group_gate"], svl.SVL_LOGITS_LAST, out["logits"], kv, max_len, cache_len, ws, wsb)
+    dws = torch.empty(svl.svl_decode_workspace_size(model.handle, B), dtype=torch.uint8, device=dev)
+    g = torch.Generator(device=dev).manual_seed(SEED + 99)
+    fed = torch.randint(0, dims.vocab, (warm + steps, B), generator=g, device=dev, dtype=torch.int32)
+    logits = torch.empty(B, dims.vocab, dtype=torch.float32, device=dev)
+    nxt = torch.empty(B, dtype=torch.int32, device=dev)
+    for t in range(warm):
+        svl.svl_decode_step(model.handle, B, fed[t], kv, max_len, cache_len, bt["layer_gate"], bt["group_gate"],
+                            logits, nxt, dws, dws.numel())
+    torch.cuda.synchronize()
+    len0 = cache_len.clone()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for t in range(warm, warm + steps):
+        svl.svl_decode_step(model.handle, B, fed[t], kv, max_len, cache_len, bt["layer_gate"], bt["group_gate"],
+                            logits, nxt, dws, dws.numel())
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    d = dims
+    dh = d.d_model // d.n_heads
+    on = effective_on(bt, d)  # active (layer, group) pairs per sample
+    per_group = d.d_model * (d.n_heads * dh * 2 + 2 * d.n_kv_heads * dh) // d.n_groups + 3 * d.d_model * d.d_ffn // d.n_groups
+    w_bytes = 2 * (int(on.any(dim=0).sum()) * per_group + d.vocab * d.d_model)  # groups active in any sample
+    ctx = float((len0.double() + steps / 2).mean())
+    kv_bytes = 2 * 2 * float(on.sum()) * (d.n_kv_heads // d.n_groups) * dh * ctx
+    nbytes = w_bytes + kv_bytes
+    return {"batch": B, "steps": steps, "ms_per_step": ms, "tokens_per_s": B / (ms / 1000.0),
+            "context_mean": ctx, "bytes_per_step": nbytes, "gb_s": nbytes / (ms / 1000.0) / 1e9,
+            "frac_of_measured_hbm": nbytes / (ms / 1000.0) / 1e9 / pk["hbm_gbs"],
+            "note": "teacher-forced, budget-0.5 batch, prefill gates; bytes = active-group weights once "
+                    "(shared by the batch) + cached K/V of the active heads"}
+
+
+def effective_on(bt, d):
+    """[B, L, G] bool: group j of layer l runs for sample b (prefix layers always)."""
+    lg = bt["layer_gate"].bool()[:, :, None]
+    gg = bt["group_gate"].bool()
+    on = lg & gg
+    on[:, :d.n_prefix, :] = True
+    return on.cpu()
 
 
 def run_hbm_sweep(svl, model, wl, dev, pk, reps=5, mults=(1, 4, 16)):
