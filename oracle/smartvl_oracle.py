@@ -9,7 +9,11 @@ Adaptation for Multimodal LLMs", arXiv 2607.20357).
 Arithmetic is float64 throughout. A storage mode rounds the tensors that the
 GPU stores in memory: ``"fp64"`` (no rounding), ``"fp32"`` or ``"bf16"``
 (round-to-nearest-even emulation of bfloat16 storage). Token logits are never
-rounded.
+rounded. ``"fp8"`` is bf16 storage with the four gated projections of every
+decoder layer (QKV, O, gate/up, down) computed from e4m3 operands: each weight
+row (output channel) and each activation row is scaled so that its largest
+magnitude maps to 448, the largest finite e4m3 value, and rounded to e4m3; the
+product of the codes is scaled back by both scales after the sum.
 
 What each function follows:
 
@@ -41,6 +45,10 @@ What each function follows:
   written without a cache: after feeding tokens t_1..t_n, the logits are
   those of the forward over [kept visual][text][t_1..t_n] under the prompt's
   gates, the kept visual tokens fixed by the prompt's own selection.
+* ``round_e4m3`` / ``quantize_rows_e4m3`` / ``linear_e4m3`` -- FP8 weights
+  for the gated GEMMs, which the paper calls orthogonal to its method
+  (Sec. 5); e4m3 is the OCP 8-bit float with 4 exponent bits (bias 7) and 3
+  mantissa bits, no infinities, largest finite value 448.
 * ``paper_rule_sample`` -- Sec. 3.1 and Sec. 3.3 "Inference", the paper's own
   rule: tokens with sigma(z) > 0.5 survive, gates are the compute
   controller's logits thresholded at 0, and for b < 1 the budget projection
@@ -88,9 +96,75 @@ def make_store(mode: str):
         return lambda a: np.asarray(a, dtype=np.float64)
     if mode == "fp32":
         return lambda a: np.asarray(a, dtype=np.float32).astype(np.float64)
-    if mode == "bf16":
+    if mode in ("bf16", "fp8"):
         return round_bf16
     raise ValueError(mode)
+
+
+# ----------------------------------------------------------------------------
+# e4m3 (FP8) operands of the gated projections
+# ----------------------------------------------------------------------------
+E4M3_MAX = 448.0  # largest finite e4m3 value: exponent field 15, mantissa 110
+
+
+def round_e4m3(a) -> np.ndarray:
+    """Round float32 values to the nearest e4m3 value (ties to the even
+    mantissa), saturating to +-448; returned as float64. NaN stays NaN.
+
+    e4m3 has 3 mantissa bits, so in the binade [2^e, 2^(e+1)) the spacing
+    is 2^(e-3); below the smallest normal 2^-6 the spacing stays 2^-9
+    (subnormals).
+    """
+    f = np.asarray(a, dtype=np.float32).astype(np.float64)
+    m = np.abs(f)
+    _, ex = np.frexp(m)                       # m = fr * 2^ex, fr in [0.5, 1)
+    e = np.maximum(ex.astype(np.int64) - 1, -6)
+    q = np.ldexp(1.0, e - 3)                  # spacing in m's binade
+    r = np.rint(m / q) * q                    # exact quotient; rint rounds half to even
+    r = np.minimum(r, E4M3_MAX)
+    out = np.copysign(r, f)
+    out[np.isnan(f)] = np.nan
+    return out
+
+
+def quantize_rows_e4m3(a):
+    """Per-row e4m3 quantisation of a 2-D array (rows = activation rows or
+    weight output channels). In float32 arithmetic: amax = max |a| of the
+    row, inv = 448 / amax, scale = amax / 448 (0 and 0 for an all-zero row);
+    the codes are round_e4m3(a * inv). Returns (code values, scales), both
+    float64; the row's value is codes * scale."""
+    a32 = np.asarray(a, dtype=np.float32)
+    amax = np.max(np.abs(a32), axis=1)
+    nz = amax > 0
+    safe = np.where(nz, amax, np.float32(1))
+    inv = np.where(nz, np.float32(E4M3_MAX) / safe, np.float32(0)).astype(np.float32)
+    scale = np.where(nz, safe / np.float32(E4M3_MAX), np.float32(0)).astype(np.float32)
+    codes = round_e4m3((a32 * inv[:, None]).astype(np.float32))
+    return codes, scale.astype(np.float64)
+
+
+def linear_e4m3(x, wq):
+    """x W^T with both operands in e4m3: x's rows are quantised here, the
+    weight arrives quantised (codes, per-row scales); the sum of code
+    products is scaled by the activation row's and the output channel's
+    scale afterwards."""
+    xv, xs = quantize_rows_e4m3(x)
+    wv, ws = wq
+    return (xv @ wv.T) * xs[:, None] * ws[None, :]
+
+
+def fp8_layer_weights(lw):
+    """e4m3 weights of one layer's gated projections. The RMSNorm gains are
+    folded into the columns of the projections they feed (W diag(gain), held
+    in bf16 as the folded weights are stored), then every output channel is
+    quantised on its own."""
+    out = {}
+    for name, gain in (("wq", "attn_norm"), ("wk", "attn_norm"), ("wv", "attn_norm"),
+                       ("wg", "ffn_norm"), ("wu", "ffn_norm")):
+        out[name] = quantize_rows_e4m3(round_bf16(lw[name] * lw[gain][None, :]))
+    for name in ("wo", "wd"):
+        out[name] = quantize_rows_e4m3(lw[name])
+    return out
 
 
 # ----------------------------------------------------------------------------
@@ -282,8 +356,9 @@ def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_cou
     X = np.concatenate([X, tok[None, :]], axis=0)
     pos = np.concatenate([pos, [len(pos)]])
     on = np.ones(G, dtype=np.int64)
+    qws = [fp8_layer_weights(lw) if mode == "fp8" else None for lw in weights["layers"]]
     for l in range(P):
-        X = decoder_layer(X, pos, weights["layers"][l], on, dims, store)
+        X = decoder_layer(X, pos, weights["layers"][l], on, dims, store, qws[l])
     gate_logits = controller_gate_logits(dims, weights, X[-1], kappa)
     full_logits = np.zeros((L, G))
     full_logits[P:] = gate_logits
@@ -296,7 +371,7 @@ def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_cou
         gates, flags = project_gates(dims, budget, x.shape[0], len(text_ids), k, gates, full_logits)
     for l in range(P, L):
         if gates[l].any():
-            X = decoder_layer(X, pos, weights["layers"][l], gates[l], dims, store)
+            X = decoder_layer(X, pos, weights["layers"][l], gates[l], dims, store, qws[l])
     y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
     logits = make_store("fp64" if mode == "fp64" else "fp32")(weights["lm_head"] @ y)
     return {"z": z, "kappa": kappa, "k": k, "kept": kept, "gate_logits": gate_logits, "gates": gates,
@@ -343,23 +418,38 @@ def causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
     return p @ v
 
 
-def decoder_layer(X, pos, lw, groups, dims, store):
+def decoder_layer(X, pos, lw, groups, dims, store, qw=None):
     """One gated decoder layer on one sample's rows X [S, D] (Sec. 3.2).
 
     ``groups`` is e_{l,:} (length G). Head h belongs to group h // (A/G);
     FFN channel c to group c // (D_int/G) (reading R3). Off groups give zero
     attention output and zero FFN channels; no rescaling by 1/alpha. With
     every group off the layer is the identity (residual bypass).
+
+    With ``qw`` (``fp8_layer_weights``) the four projections take e4m3
+    operands: the stored residual rows X are quantised as they are and the
+    RMSNorm enters as the row factor 1/rms(X) after the product (the gain is
+    in the folded weights); the attention output and the SwiGLU output are
+    quantised as stored.
     """
     A, Akv, dh, G = dims.n_heads, dims.n_kv_heads, dims.d_head, dims.n_groups
     S = X.shape[0]
     if not np.any(groups):
         return X
     hpg = A // G
-    xn = store(rmsnorm(X, lw["attn_norm"], dims.rms_eps))
-    q = (xn @ lw["wq"].T).reshape(S, A, dh)
-    k = (xn @ lw["wk"].T).reshape(S, Akv, dh)
-    v = (xn @ lw["wv"].T).reshape(S, Akv, dh)
+
+    def inv_rms(Y):
+        return 1.0 / np.sqrt(np.mean(Y * Y, axis=1, keepdims=True) + dims.rms_eps)
+
+    if qw is None:
+        xn = store(rmsnorm(X, lw["attn_norm"], dims.rms_eps))
+        q, k, v = xn @ lw["wq"].T, xn @ lw["wk"].T, xn @ lw["wv"].T
+    else:
+        r = inv_rms(X)
+        q, k, v = (r * linear_e4m3(X, qw[n]) for n in ("wq", "wk", "wv"))
+    q = q.reshape(S, A, dh)
+    k = k.reshape(S, Akv, dh)
+    v = v.reshape(S, Akv, dh)
     q = store(rope(q, pos, dims.rope_theta))
     k = store(rope(k, pos, dims.rope_theta))
     v = store(v)
@@ -369,16 +459,20 @@ def decoder_layer(X, pos, lw, groups, dims, store):
             kv = h // (A // Akv)
             o[:, h, :] = causal_attention(q[:, h, :], k[:, kv, :], v[:, kv, :])
     o = store(o.reshape(S, A * dh))
-    X = store(X + o @ lw["wo"].T)
+    X = store(X + (o @ lw["wo"].T if qw is None else linear_e4m3(o, qw["wo"])))
 
-    xn = store(rmsnorm(X, lw["ffn_norm"], dims.rms_eps))
-    u = silu(xn @ lw["wg"].T) * (xn @ lw["wu"].T)
+    if qw is None:
+        xn = store(rmsnorm(X, lw["ffn_norm"], dims.rms_eps))
+        u = silu(xn @ lw["wg"].T) * (xn @ lw["wu"].T)
+    else:
+        r = inv_rms(X)
+        u = silu(r * linear_e4m3(X, qw["wg"])) * (r * linear_e4m3(X, qw["wu"]))
     cpg = dims.d_ffn // G
     for j in range(G):
         if not groups[j]:
             u[:, j * cpg:(j + 1) * cpg] = 0.0
     u = store(u)
-    return store(X + u @ lw["wd"].T)
+    return store(X + (u @ lw["wd"].T if qw is None else linear_e4m3(u, qw["wd"])))
 
 
 def project_visual(x, weights, dims, store):
@@ -423,7 +517,8 @@ def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
     e = effective_groups(layer_gate, group_gate, dims.n_prefix)
     nl = dims.n_layers if n_layers is None else n_layers
     for l in range(nl):
-        X = decoder_layer(X, pos, weights["layers"][l], e[l], dims, store)
+        qw = fp8_layer_weights(weights["layers"][l]) if mode == "fp8" else None
+        X = decoder_layer(X, pos, weights["layers"][l], e[l], dims, store, qw)
     y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
     logits = make_store("fp64" if mode == "fp64" else "fp32")(weights["lm_head"] @ y)
     return {"z": z, "k": k, "flags": flags, "kept": kept, "hidden": X, "logits": logits}

@@ -599,3 +599,121 @@ def test_decode_reference_is_causal():
         np.testing.assert_allclose(st["hidden"][:prev.shape[0]], prev, rtol=1e-12, atol=1e-12)
         assert st["hidden"].shape[0] == prev.shape[0] + 1
         prev = st["hidden"]
+
+
+# ----------------------------------------------------------------------------- e4m3 (FP8 gated GEMMs)
+def _e4m3_table():
+    """All finite e4m3 values, decoded from the bit fields: sign, 4-bit
+    exponent (bias 7), 3-bit mantissa; exponent field 0 is subnormal
+    (2^-6 * m/8); S.1111.111 is NaN."""
+    vals = []
+    for code in range(256):
+        s, e, m = code >> 7, (code >> 3) & 15, code & 7
+        if e == 15 and m == 7:
+            continue
+        v = (m / 8.0) * 2.0 ** -6 if e == 0 else (1 + m / 8.0) * 2.0 ** (e - 7)
+        vals.append((-v if s else v, code))
+    return vals
+
+
+def test_e4m3_table_brute_force_nearest_ties_even():
+    table = _e4m3_table()
+    vals = np.array([v for v, _ in table])
+    codes = np.array([c for _, c in table])
+    assert vals.max() == O.E4M3_MAX == 448.0 and len(set(vals.tolist())) == 253  # +0 and -0 coincide
+    rng = np.random.default_rng(5)
+    mag = np.exp(rng.uniform(np.log(2.0 ** -12), np.log(500.0), size=20000))
+    x = (mag * rng.choice([-1.0, 1.0], size=mag.size)).astype(np.float32)
+    # every value exactly halfway between two neighbours, as a tie test
+    pos = np.unique(vals[vals >= 0])
+    mids = ((pos[:-1] + pos[1:]) / 2).astype(np.float32)
+    x = np.concatenate([x, mids, -mids, vals.astype(np.float32), [460.0, 464.0, 1e6, -1e6]]).astype(np.float32)
+    got = O.round_e4m3(x)
+    for xi, gi in zip(x.astype(np.float64), got):
+        if abs(xi) > 448.0:
+            assert gi == np.copysign(448.0, xi)
+            continue
+        d = np.abs(vals - xi)
+        best = np.flatnonzero(d == d.min())
+        cand = [(vals[i], codes[i]) for i in best]
+        if len({c[0] for c in cand}) > 1:  # a tie: the even mantissa wins
+            cand = [c for c in cand if (c[1] & 1) == 0]
+        assert gi == cand[0][0], (xi, gi, cand)
+
+
+def test_e4m3_matches_torch_float8_conversion():
+    rng = np.random.default_rng(6)
+    x = (rng.normal(size=50000) * 10.0 ** rng.uniform(-4, 2.4, size=50000)).astype(np.float32)
+    x = np.clip(x, -448, 448)
+    ref = torch.from_numpy(x).to(torch.float8_e4m3fn).to(torch.float64).numpy()
+    np.testing.assert_array_equal(O.round_e4m3(x), ref)
+
+
+def test_quantize_rows_scale_and_error_bound():
+    rng = np.random.default_rng(7)
+    a = rng.normal(size=(64, 300)) * 10.0 ** rng.uniform(-3, 3, size=(64, 1))
+    a[3] = 0.0  # an all-zero row: zero codes, zero scale
+    a = O.round_bf16(a)
+    codes, scale = O.quantize_rows_e4m3(a)
+    assert scale[3] == 0.0 and not codes[3].any()
+    rows = [r for r in range(64) if r != 3]
+    amax = np.abs(a[rows]).max(axis=1)
+    # the largest magnitude lands on +-448 and the scale is amax / 448 in float32
+    np.testing.assert_array_equal(np.abs(codes[rows]).max(axis=1), 448.0)
+    np.testing.assert_array_equal(scale[rows], (amax.astype(np.float32) / np.float32(448)).astype(np.float64))
+    # relative error of the dequantised value: half a spacing, 2^-4, in the normal range
+    deq = codes * scale[:, None]
+    normal = (np.abs(a) >= (2.0 ** -6) * scale[:, None] * 1.01) & (a != 0)
+    err = np.abs(deq - a)[normal] / np.abs(a)[normal]
+    assert err.max() <= 2.0 ** -4 * (1 + 1e-6)
+    # below it the absolute error is half the subnormal spacing 2^-9, times the scale
+    sub = ~normal & (np.arange(64)[:, None] != 3)
+    assert (np.abs(deq - a)[sub] <= 2.0 ** -10 * scale[:, None].repeat(300, 1)[sub] * (1 + 1e-6)).all()
+
+
+def test_linear_e4m3_is_exact_on_the_grid():
+    """Rows whose entries are e4m3 values and whose largest magnitude is 448
+    have scale 1: the product must equal the exact matrix product."""
+    rng = np.random.default_rng(8)
+    grid = np.array([v for v, _ in _e4m3_table()])
+    x = rng.choice(grid, size=(17, 96))
+    w = rng.choice(grid, size=(40, 96))
+    x[:, 5] = 448.0
+    w[:, 7] = -448.0
+    got = O.linear_e4m3(x, O.quantize_rows_e4m3(w))
+    np.testing.assert_array_equal(got, x @ w.T)
+    # scaling a row by a power of two scales its output row and nothing else
+    x2 = x.copy()
+    x2[4] *= 2.0 ** -20
+    got2 = O.linear_e4m3(x2, O.quantize_rows_e4m3(w))
+    np.testing.assert_array_equal(got2[4], got[4] * 2.0 ** -20)
+    np.testing.assert_array_equal(np.delete(got2, 4, 0), np.delete(got, 4, 0))
+
+
+def test_fp8_forward_against_dense_library_forward():
+    """The e4m3 forward stays within e4m3's rounding of the exact dense
+    forward, and is measurably further from it than bf16 storage alone (so
+    the quantisation is really applied). Bound: each e4m3 operand carries a
+    relative rounding error of at most 2^-4, a product of two such operands
+    at most sqrt(2) 2^-4 in the RMS sense, and L layers add L independent
+    errors: sqrt(2 L) 2^-4. A missing scale or norm factor is off by O(1)."""
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 2)
+    L, G = dims.n_layers, dims.n_groups
+    lg, gg = np.ones(L, np.uint8), np.ones((L, G), np.uint8)
+    n = x.shape[0]
+    outs = {m: O.forward_sample(dims, w, x, ids, 1.0, lg, gg, keep_count=n, mode=m) for m in ("bf16", "fp8")}
+    X0 = _packed_rows(dims, w, x, np.arange(n), ids)
+    hid, logits = dense_forward(X0, w["layers"], w["final_norm"], w["lm_head"], dims)
+
+    def rel(a, b):
+        return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+
+    e8, e16 = rel(outs["fp8"]["hidden"], hid.numpy() if hasattr(hid, "numpy") else hid), \
+        rel(outs["bf16"]["hidden"], hid.numpy() if hasattr(hid, "numpy") else hid)
+    bound = math.sqrt(2 * L) * 2.0 ** -4
+    assert e8 < bound, (e8, bound)
+    assert e8 > 2 * e16, (e8, e16)
+    l8 = rel(outs["fp8"]["logits"], logits.numpy() if hasattr(logits, "numpy") else logits)
+    assert l8 < bound, (l8, bound)
