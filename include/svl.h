@@ -65,7 +65,19 @@ typedef enum svl_status {
  * A_kv % G == 0 (each group owns whole KV heads); (D_int / G) % 64 == 0;
  * (A / G) * d_head % 64 == 0; D a multiple of 128; C_v, proj_hidden
  * multiples of 64;
- * H in {16, 32, ..., 128}; proj_hidden == 0 requires C_v == D. */
+ * H in {16, 32, ..., 128}; proj_hidden == 0 requires C_v == D.
+ *
+ * gemm_format selects the operand type of the four gated projections of
+ * every decoder layer (QKV, O, gate/up, down): SVL_GEMM_BF16, or
+ * SVL_GEMM_E4M3 -- FP8 weights, which the paper calls orthogonal to its
+ * method (Sec. 5). With e4m3, svl_model_create quantises each weight output
+ * channel (row of W, norm gains folded in) to e4m3 with the scale
+ * amax / 448; each activation row feeding those GEMMs is quantised the same
+ * way on the fly (svl_quantize_rows_e4m3 is the definition), and the fp32
+ * accumulator of the code products is scaled by both rows' scales. The
+ * projector, token controller and LM head stay bf16. */
+#define SVL_GEMM_BF16 0
+#define SVL_GEMM_E4M3 1
 typedef struct svl_model_desc {
   int32_t n_layers;     /* L */
   int32_t d_model;      /* D */
@@ -81,6 +93,7 @@ typedef struct svl_model_desc {
   float rms_eps;
   float rope_theta;
   int32_t max_seq;      /* longest per-sample sequence the model will see */
+  int32_t gemm_format;  /* SVL_GEMM_BF16 or SVL_GEMM_E4M3 (gated projections) */
 } svl_model_desc;
 
 /* One decoder layer's weights: device bf16, nn.Linear layout [out, in]. */
@@ -257,6 +270,30 @@ svl_status svl_controlled_prefill(svl_model* model, int32_t B, int32_t t_cap, vo
  * svl_kv_cache_size: its bytes (0 on bad arguments). */
 size_t svl_kv_cache_size(const svl_model* model, int32_t B, int32_t max_len);
 
+/* e4m3 quantisation of bf16 rows, as the SVL_GEMM_E4M3 path applies it to
+ * weight output channels and activation rows. For each of the `rows` rows
+ * of `cols` values (device bf16, `ld_src` elements apart): amax = max |x|,
+ * inv = 448 / amax and scale[r] = amax / 448 in float32 with correct
+ * rounding (both 0 when amax is 0), and dst[r * ld_dst + c] =
+ * e4m3(x * inv) rounded to nearest even and saturated to +-448 (OCP e4m3:
+ * 4 exponent bits with bias 7, 3 mantissa bits, no infinities). dst is
+ * device uint8 codes, scale device float32 [rows]; the caller owns both.
+ * Requires cols and ld_src multiples of 8, ld_dst >= cols and a multiple
+ * of 8, src 16-byte and dst 8-byte aligned (else SVL_ERR_INVALID_ARG).
+ * Asynchronous on `stream`. */
+svl_status svl_quantize_rows_e4m3(const void* src, int64_t rows, int32_t cols, int64_t ld_src, void* dst,
+                                  int64_t ld_dst, float* scale, void* stream);
+
+/* The e4m3 GEMM of the gated projections on its own, with an fp32 output:
+ * C[m, n] = a_scale[m] * b_scale[n] * sum_k A[m, k] B[n, k], A [M, K] and
+ * B [N, K] device uint8 e4m3 codes (row-major, K contiguous, 16-byte
+ * aligned), scales float32, C float32 [M, N] row-major; all caller-owned.
+ * Requires K a multiple of 128 and N a multiple of 32 (else
+ * SVL_ERR_INVALID_ARG). The model supplies the device status word and the
+ * SM count only. Asynchronous on `stream`. */
+svl_status svl_gemm_e4m3(svl_model* model, const void* A, const float* a_scale, const void* B, const float* b_scale,
+                         int32_t M, int32_t N, int32_t K, float* C, void* stream);
+
 /* svl_gated_prefill that also stores every layer's keys and values of the
  * prompt into the cache and writes cache_len[B] (device int32) = the prompt
  * length S_b of each sample. Errors: as svl_gated_prefill; prompt rows past
@@ -393,7 +430,8 @@ typedef struct svl_kernel_time {
 #define SVL_TAG_DOWN 11
 #define SVL_TAG_LMHEAD 12
 #define SVL_TAG_COPY 13
-#define SVL_TAG_COUNT 14
+#define SVL_TAG_QUANT 14 /* e4m3 quantisation of the gated GEMMs' activation rows */
+#define SVL_TAG_COUNT 15
 
 svl_status svl_profile_start(svl_model* model, uint32_t tag_mask); /* bit t: record SVL_TAG t */
 svl_status svl_profile_stop(svl_model* model, svl_kernel_time* out, int32_t cap, int32_t* n_out);

@@ -14,6 +14,9 @@ decoder layer (QKV, O, gate/up, down) computed from e4m3 operands: each weight
 row (output channel) and each activation row is scaled so that its largest
 magnitude maps to 448, the largest finite e4m3 value, and rounded to e4m3; the
 product of the codes is scaled back by both scales after the sum.
+``"fp8_s32"`` is the same with fp32 storage: how far it lands from ``"fp8"``
+measures how strongly e4m3's rounding boundaries amplify storage-level
+differences (a value moved across a boundary jumps by a whole e4m3 step).
 
 What each function follows:
 
@@ -98,6 +101,8 @@ def make_store(mode: str):
         return lambda a: np.asarray(a, dtype=np.float32).astype(np.float64)
     if mode in ("bf16", "fp8"):
         return round_bf16
+    if mode == "fp8_s32":
+        return lambda a: np.asarray(a, dtype=np.float32).astype(np.float64)
     raise ValueError(mode)
 
 
@@ -356,7 +361,7 @@ def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_cou
     X = np.concatenate([X, tok[None, :]], axis=0)
     pos = np.concatenate([pos, [len(pos)]])
     on = np.ones(G, dtype=np.int64)
-    qws = [fp8_layer_weights(lw) if mode == "fp8" else None for lw in weights["layers"]]
+    qws = [fp8_layer_weights(lw) if mode in ("fp8", "fp8_s32") else None for lw in weights["layers"]]
     for l in range(P):
         X = decoder_layer(X, pos, weights["layers"][l], on, dims, store, qws[l])
     gate_logits = controller_gate_logits(dims, weights, X[-1], kappa)
@@ -504,11 +509,13 @@ def pack_sample(dims, weights, x, kept, text_ids, store):
 
 
 def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
-                   keep_count=-1, mode="fp32", n_layers=None):
+                   keep_count=-1, mode="fp32", n_layers=None, qws=None):
     """Token controller + pack + gated decoder + final norm + last-row logits.
 
     ``n_layers`` (default: all) runs only the first layers -- used to bound
     the oracle's time; the final norm and LM head then apply after them.
+    ``qws`` passes the per-layer e4m3 weights of the fp8 modes when the
+    caller has them already (they depend on the weights only).
     """
     store = make_store(mode)
     z, k, flags, kept = score_select_sample(dims, weights, x, budget, len(text_ids),
@@ -517,8 +524,11 @@ def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
     e = effective_groups(layer_gate, group_gate, dims.n_prefix)
     nl = dims.n_layers if n_layers is None else n_layers
     for l in range(nl):
-        qw = fp8_layer_weights(weights["layers"][l]) if mode == "fp8" else None
-        X = decoder_layer(X, pos, weights["layers"][l], e[l], dims, store, qw)
+        lw = weights["layers"][l]
+        qw = None
+        if mode in ("fp8", "fp8_s32"):
+            qw = qws[l] if qws is not None else fp8_layer_weights(lw)
+        X = decoder_layer(X, pos, lw, e[l], dims, store, qw)
     y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
     logits = make_store("fp64" if mode == "fp64" else "fp32")(weights["lm_head"] @ y)
     return {"z": z, "k": k, "flags": flags, "kept": kept, "hidden": X, "logits": logits}
@@ -542,13 +552,17 @@ def forward_batch(dims, weights, batch, mode="fp32", n_layers=None, samples=None
     (keys as produced by the input generator, converted to numpy)."""
     out = []
     B = batch["B"]
+    qws = None
+    if mode in ("fp8", "fp8_s32"):
+        nl = dims.n_layers if n_layers is None else n_layers
+        qws = [fp8_layer_weights(weights["layers"][l]) for l in range(nl)]
     for b in (range(B) if samples is None else samples):
         v0, v1 = batch["vis_off"][b], batch["vis_off"][b + 1]
         t0, t1 = batch["text_off"][b], batch["text_off"][b + 1]
         out.append(forward_sample(
             dims, weights, batch["vis"][v0:v1], batch["text_ids"][t0:t1], batch["budget"][b],
             batch["layer_gate"][b], batch["group_gate"][b], int(batch["keep_count"][b]),
-            mode=mode, n_layers=n_layers))
+            mode=mode, n_layers=n_layers, qws=qws))
     return out
 
 

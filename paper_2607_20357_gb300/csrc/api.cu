@@ -27,6 +27,15 @@ struct svl_model {
   // layers whose gains are not all ones): per layer q, k, v, g, u or nullptr
   std::vector<void*> folded;
   CUtensorMap tm_ctrl_w1, tm_proj_w1, tm_proj_w2, tm_lm_head;
+  // e4m3 gated projections (gemm_format SVL_GEMM_E4M3): per layer the codes
+  // of q, k, v, o, g, u, d with their per-row scales, and uint8 tensor maps.
+  // The O and down weights hold each group's K columns padded to a multiple
+  // of 128 (one K block), so that gated-off groups skip whole blocks.
+  bool e4m3 = false;
+  int kgo_p = 0, kgd_p = 0;
+  std::vector<void*> f8_mem;           // one allocation per layer
+  std::vector<const float*> f8_scale;  // per layer q, k, v, o, g, u, d
+  std::vector<CUtensorMap> tm8;        // per layer q, k, v, o, g, u, d
   // kernel timing (svl_profile_start / svl_profile_stop)
   bool prof = false;
   uint32_t prof_mask = 0;
@@ -69,7 +78,23 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uin
   return r == CUDA_SUCCESS;
 }
 
+// The same for uint8 e4m3 codes: boxes of 128 x box_rows (128 bytes per row).
+bool make_map8(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows = 128) {
+  auto fn = encode_fn();
+  if (!fn || !ptr || rows == 0 || cols == 0 || (reinterpret_cast<uintptr_t>(ptr) & 15) || (cols & 15)) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBK8), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int round128(int x) { return (x + 127) & ~127; }
 
 // Each call keeps its scratch at the start of the workspace: no data flows
 // between calls through the workspace, so the three layouts overlap and the
@@ -84,8 +109,9 @@ struct PreLayout {
   int64_t t_cap, t_pad;
   int n_pad, mt_max, qkv_cap, o_cap, gu_cap, dn_cap, attn_cap;
   int ss_slots, ks_units;
+  int64_t aq_cols;  // e4m3: widest quantised activation row (0 for bf16)
   size_t xn, q, k, v, ao, hmid, yl, ss_a, ss_b, ks_part, ks_ticket, ks_info, act, seg, qkv, o, gu, dn, attn, counts,
-      total;
+      aq, as, total;
 };
 
 struct Bump {
@@ -165,6 +191,14 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   L.dn = b.take(sizeof(int4) * nl * L.dn_cap);
   L.attn = b.take(sizeof(int4) * nl * L.attn_cap);
   L.counts = b.take(sizeof(int) * 5 * nl);
+  // e4m3: the quantised rows of the current GEMM input and their scales
+  if (d.gemm_format == SVL_GEMM_E4M3) {
+    const int64_t o_cols = static_cast<int64_t>(G) * round128(static_cast<int>(hq / G));
+    const int64_t d_cols = static_cast<int64_t>(G) * round128(d.d_ffn / G);
+    L.aq_cols = std::max<int64_t>(d.d_model, std::max(o_cols, d_cols));
+    L.aq = b.take(static_cast<size_t>(t_cap) * L.aq_cols);
+    L.as = b.take(sizeof(float) * (t_cap + 64));
+  }
   L.total = b.off;
   return L;
 }
@@ -254,10 +288,11 @@ struct Launch {
   }
 };
 
-svl_status launch(EpiKind kind, svl_model* m, int tag, const GemmParams& p, int64_t tiles, cudaStream_t s) {
+svl_status launch(EpiKind kind, svl_model* m, int tag, const GemmParams& p, int64_t tiles, cudaStream_t s,
+                  bool e4m3 = false) {
   if (tiles <= 0) return SVL_OK;
   Launch L(m, tag, s);
-  return launch_gemm(kind, p, gemm_grid(m, tiles), s) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
+  return launch_gemm(kind, p, gemm_grid(m, tiles), s, e4m3) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
 }
 
 svl_status last_error() { return cudaGetLastError() == cudaSuccess ? SVL_OK : SVL_ERR_CUDA; }
@@ -300,6 +335,7 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   if (d.d_model % 128 || d.c_vis % 64 || d.proj_hidden % 64) return SVL_ERR_UNSUPPORTED;
   if (d.h_ctrl % 16 || d.h_ctrl > 128) return SVL_ERR_UNSUPPORTED;
   if (d.proj_hidden == 0 && d.c_vis != d.d_model) return SVL_ERR_UNSUPPORTED;
+  if (d.gemm_format != SVL_GEMM_BF16 && d.gemm_format != SVL_GEMM_E4M3) return SVL_ERR_INVALID_ARG;
   // Eq. 8 times G must stay exact in double precision at the longest sequence
   {
     const double S = d.max_seq, D = d.d_model, Dkv = static_cast<double>(d.n_kv_heads) * dh;
@@ -371,6 +407,57 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
       return SVL_ERR_CUDA;
     }
   }
+  if (d.gemm_format == SVL_GEMM_E4M3) {
+    // e4m3 copies of the (gain-folded) gated projections, one allocation per
+    // layer: codes then per-row scales of q, k, v, o, g, u, d
+    m->e4m3 = true;
+    const int G = d.n_groups;
+    m->kgo_p = round128(static_cast<int>(hq / G));
+    m->kgd_p = round128(d.d_ffn / G);
+    const int64_t rows[7] = {hq, dkv, dkv, d.d_model, d.d_ffn, d.d_ffn, d.d_model};
+    const int groups[7] = {1, 1, 1, G, 1, 1, G};
+    const int kg[7] = {d.d_model, d.d_model, d.d_model, static_cast<int>(hq / G), d.d_model, d.d_model, d.d_ffn / G};
+    const int kgp[7] = {d.d_model, d.d_model, d.d_model, m->kgo_p, d.d_model, d.d_model, m->kgd_p};
+    size_t code_off[7], scale_off[7], total = 0;
+    for (int i = 0; i < 7; ++i) {
+      code_off[i] = total;
+      total = align256(total + static_cast<size_t>(rows[i]) * groups[i] * kgp[i]);
+      scale_off[i] = total;
+      total = align256(total + sizeof(float) * (rows[i] + 64));
+    }
+    m->f8_mem.assign(d.n_layers, nullptr);
+    m->f8_scale.assign(static_cast<size_t>(d.n_layers) * 7, nullptr);
+    m->tm8.resize(static_cast<size_t>(d.n_layers) * 7);
+    for (int l = 0; l < d.n_layers && ok; ++l) {
+      const svl_layer_weights& lw = m->layers[l];
+      const void* src[7] = {lw.wq, lw.wk, lw.wv, lw.wo, lw.wg, lw.wu, lw.wd};
+      uint8_t* base = nullptr;
+      ok = cudaMalloc(&base, total) == cudaSuccess && cudaMemset(base, 0, total) == cudaSuccess;
+      if (!ok) break;
+      m->f8_mem[l] = base;
+      for (int i = 0; i < 7 && ok; ++i) {
+        QuantArgs qa;
+        std::memset(&qa, 0, sizeof(qa));
+        qa.src = static_cast<const __nv_bfloat16*>(src[i]);
+        qa.ld_src = static_cast<int64_t>(groups[i]) * kg[i];
+        qa.rows = rows[i];
+        qa.G = groups[i];
+        qa.kg = kg[i];
+        qa.kgp = kgp[i];
+        qa.dst = base + code_off[i];
+        qa.ld_dst = static_cast<int64_t>(groups[i]) * kgp[i];
+        qa.scale = reinterpret_cast<float*>(base + scale_off[i]);
+        m->f8_scale[static_cast<size_t>(l) * 7 + i] = qa.scale;
+        ok = launch_quant_rows(qa, 0) == cudaSuccess &&
+             make_map8(&m->tm8[static_cast<size_t>(l) * 7 + i], qa.dst, rows[i], qa.ld_dst);
+        g_launches++;
+      }
+    }
+    if (!ok || cudaDeviceSynchronize() != cudaSuccess) {
+      svl_model_destroy(m);
+      return SVL_ERR_CUDA;
+    }
+  }
   m->tm_layer.resize(static_cast<size_t>(d.n_layers) * 7);
   for (int l = 0; l < d.n_layers && ok; ++l) {
     const svl_layer_weights& lw = m->layers[l];
@@ -411,6 +498,8 @@ void svl_model_destroy(svl_model* m) {
   if (m->d_status) cudaFree(m->d_status);
   if (m->rope_cs) cudaFree(m->rope_cs);
   for (void* f : m->folded)
+    if (f) cudaFree(f);
+  for (void* f : m->f8_mem)
     if (f) cudaFree(f);
   delete m;
 }
@@ -756,6 +845,54 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   if (!make_map(&map_x, X, t_cap, d.d_model) || !make_map(&map_xn, xn, t_cap, d.d_model) ||
       !make_map(&map_ao, ao, t_cap, hq) || !make_map(&map_hm, hm, t_cap, d.d_ffn))
     return SVL_ERR_CUDA;
+  // e4m3: every gated GEMM reads the quantised rows of its input (aq, with
+  // per-row scales as) -- X for QKV and gate/up, the attention output for
+  // O, the SwiGLU output for down (both group-padded to whole K blocks)
+  const bool f8 = m->e4m3;
+  const int G = d.n_groups;
+  uint8_t* aq = f8 ? at<uint8_t>(ws, L.aq) : nullptr;
+  float* as = f8 ? at<float>(ws, L.as) : nullptr;
+  CUtensorMap map_aq_x, map_aq_o, map_aq_h;
+  if (f8 && (!make_map8(&map_aq_x, aq, t_cap, d.d_model) ||
+             !make_map8(&map_aq_o, aq, t_cap, static_cast<uint64_t>(G) * m->kgo_p) ||
+             !make_map8(&map_aq_h, aq, t_cap, static_cast<uint64_t>(G) * m->kgd_p)))
+    return SVL_ERR_CUDA;
+  auto quant = [&](const __nv_bfloat16* src, int64_t ld_src, int groups, int kg, int kgp, int layer) {
+    QuantArgs qa;
+    std::memset(&qa, 0, sizeof(qa));
+    qa.src = src;
+    qa.ld_src = ld_src;
+    qa.rows = t_cap;
+    qa.G = groups;
+    qa.kg = kg;
+    qa.kgp = kgp;
+    qa.dst = aq;
+    qa.ld_dst = static_cast<int64_t>(groups) * kgp;
+    qa.scale = as;
+    qa.cu_seqlens = cu_seqlens;
+    qa.B = B;
+    if (layer >= 0) {
+      qa.layer_gate = layer_gate;
+      qa.group_gate = group_gate;
+      qa.L = nl;
+      qa.l = layer;
+      qa.P = d.n_prefix;
+    }
+    Launch L1(m, SVL_TAG_QUANT, s);
+    return launch_quant_rows(qa, s) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
+  };
+  auto set_f8 = [&](GemmParams& p, const CUtensorMap& mapA, const CUtensorMap* tm8, const float* const* sc,
+                    std::initializer_list<int> mats) {
+    p.mapA = mapA;
+    int i = 0;
+    for (int mat : mats) {
+      p.mapB[i] = tm8[mat];
+      p.b_scale[i] = sc[mat];
+      ++i;
+    }
+    p.a_scale = as;
+  };
+
   // fused RMSNorm: per-row partial sums of squares of X (see GemmParams)
   float* ss_a = at<float>(ws, L.ss_a);
   float* ss_b = at<float>(ws, L.ss_b);
@@ -822,13 +959,18 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
       }
     }
 
+    const CUtensorMap* tm8 = f8 ? &m->tm8[static_cast<size_t>(l) * 7] : nullptr;
+    const float* const* sc8 = f8 ? &m->f8_scale[static_cast<size_t>(l) * 7] : nullptr;
     // attention input norm fused into the QKV GEMM (gain folded into W_qkv)
+    if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), d.d_model, 1, d.d_model, d.d_model, -1)) != SVL_OK)
+      return st;
     GemmParams p = base_params(m);
     set_norm(p, ss_a, nullptr);
     p.mapA = map_x;
     p.mapB[0] = tm[0];
     p.mapB[1] = tm[1];
     p.mapB[2] = tm[2];
+    if (f8) set_f8(p, map_aq_x, tm8, sc8, {0, 1, 2});
     p.tiles = sa.qkv_tiles + static_cast<size_t>(l) * L.qkv_cap;
     p.tile_count = counts + l;
     p.max_tiles = L.qkv_cap;
@@ -844,7 +986,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.rope_cs = m->rope_cs;
     p.rope_rows = d.max_seq;
     p.d_head = dh;
-    if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8)) != SVL_OK) return st;
 
     const size_t layer_kv = static_cast<size_t>(B) * (kvx ? kvx->max_len : 0) * dkv;
     if (kvx && kvx->decode) {
@@ -897,6 +1039,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
       if (launch_attention_tc(aa, gemm_grid(m, L.attn_cap), s) != cudaSuccess) return SVL_ERR_CUDA;
     }
 
+    if (f8 && (st = quant(ao, hq, G, hq / G, m->kgo_p, l)) != SVL_OK) return st;
     p = base_params(m);
     p.mapA = map_ao;
     p.mapB[0] = tm[3];
@@ -905,20 +1048,28 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.max_tiles = L.o_cap;
     p.K = hq;
     p.kgroup = hq / d.n_groups;
+    if (f8) {
+      set_f8(p, map_aq_o, tm8, sc8, {3});
+      p.K = G * m->kgo_p;
+      p.kgroup = m->kgo_p;
+    }
     p.out[0] = X;
     p.ld[0] = d.d_model;
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
     set_norm(p, nullptr, ss_b);  // sums of squares of the updated rows for the MLP norm
-    if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s, f8)) != SVL_OK) return st;
 
     // MLP input norm fused into the gate/up GEMM (gain folded into W_g, W_u)
+    if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), d.d_model, 1, d.d_model, d.d_model, -1)) != SVL_OK)
+      return st;
     p = base_params(m);
     set_norm(p, ss_b, nullptr);
     p.mapA = map_x;
     p.mapB[0] = tm[4];
     p.mapB[1] = tm[5];
+    if (f8) set_f8(p, map_aq_x, tm8, sc8, {4, 5});
     p.b_split = 1;
     p.tiles = sa.gu_tiles + static_cast<size_t>(l) * L.gu_cap;
     p.tile_count = counts + 2 * nl + l;
@@ -927,8 +1078,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.kgroup = d.d_model;
     p.out[0] = hm;
     p.ld[0] = d.d_ffn;
-    if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8)) != SVL_OK) return st;
 
+    if (f8 && (st = quant(hm, d.d_ffn, G, d.d_ffn / G, m->kgd_p, l)) != SVL_OK) return st;
     p = base_params(m);
     p.mapA = map_hm;
     p.mapB[0] = tm[6];
@@ -937,13 +1089,18 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.max_tiles = L.dn_cap;
     p.K = d.d_ffn;
     p.kgroup = d.d_ffn / d.n_groups;
+    if (f8) {
+      set_f8(p, map_aq_h, tm8, sc8, {6});
+      p.K = G * m->kgd_p;
+      p.kgroup = m->kgd_p;
+    }
     p.out[0] = X;
     p.ld[0] = d.d_model;
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8 + 4;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;
     set_norm(p, nullptr, ss_a);  // for the next layer's attention norm
-    if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s)) != SVL_OK) return st;
+    if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s, f8)) != SVL_OK) return st;
   }
 
   // final norm + LM head
@@ -1085,6 +1242,50 @@ svl_status svl_decode_step(svl_model* m, int32_t B, const int32_t* tokens, void*
                       ws_bytes - (xb + cb + pb), stream, nullptr, &kx);
 }
 
+svl_status svl_quantize_rows_e4m3(const void* src, int64_t rows, int32_t cols, int64_t ld_src, void* dst,
+                                  int64_t ld_dst, float* scale, void* stream) {
+  if (!src || !dst || !scale || rows < 0 || cols <= 0 || (cols & 7) || ld_src < cols || (ld_src & 7) ||
+      ld_dst < cols || (ld_dst & 7) || !aligned16(src) || (reinterpret_cast<uintptr_t>(dst) & 7) ||
+      (reinterpret_cast<uintptr_t>(scale) & 3))
+    return SVL_ERR_INVALID_ARG;
+  QuantArgs qa;
+  std::memset(&qa, 0, sizeof(qa));
+  qa.src = static_cast<const __nv_bfloat16*>(src);
+  qa.ld_src = ld_src;
+  qa.rows = rows;
+  qa.G = 1;
+  qa.kg = cols;
+  qa.kgp = cols;
+  qa.dst = static_cast<uint8_t*>(dst);
+  qa.ld_dst = ld_dst;
+  qa.scale = scale;
+  g_launches++;
+  if (launch_quant_rows(qa, static_cast<cudaStream_t>(stream)) != cudaSuccess) return SVL_ERR_CUDA;
+  return last_error();
+}
+
+svl_status svl_gemm_e4m3(svl_model* m, const void* A, const float* a_scale, const void* B, const float* b_scale,
+                         int32_t M, int32_t N, int32_t K, float* C, void* stream) {
+  if (!m || !A || !a_scale || !B || !b_scale || !C || M <= 0 || N <= 0 || K <= 0 || (K % kBK8) || (N & 31))
+    return SVL_ERR_INVALID_ARG;
+  GemmParams p = base_params(m);
+  if (!make_map8(&p.mapA, A, M, K) || !make_map8(&p.mapB[0], B, N, K)) return SVL_ERR_INVALID_ARG;
+  p.grid_m = (M + kBM - 1) / kBM;
+  p.bn = std::min(N, 256);
+  p.grid_n = (N + p.bn - 1) / p.bn;
+  p.m_limit = M;
+  p.n_limit = N;
+  p.K = K;
+  p.kgroup = K;
+  p.out[0] = C;
+  p.ld[0] = N;
+  p.a_scale = a_scale;
+  p.b_scale[0] = b_scale;
+  svl_status st = launch(EPI_F32, m, SVL_TAG_LMHEAD, p, static_cast<int64_t>(p.grid_m) * p.grid_n,
+                         static_cast<cudaStream_t>(stream), true);
+  return st != SVL_OK ? st : last_error();
+}
+
 svl_status svl_flops(const svl_model_desc* d, int32_t s_text, int32_t s_vis, int32_t n_vis, const uint8_t* lg,
                      const uint8_t* gg, double* eq8, double* exec) {
   if (!d || s_text < 0 || s_vis < 0 || n_vis < 0 || d->n_heads <= 0 || d->n_groups <= 0) return SVL_ERR_INVALID_ARG;
@@ -1223,7 +1424,7 @@ svl_status svl_profile_launches(svl_model* m, int32_t* tags, float* ms, int32_t 
 const char* svl_tag_name(int32_t tag) {
   static const char* names[SVL_TAG_COUNT] = {"budget_embed", "score", "select", "pack", "projector",
                                               "schedule", "rmsnorm", "qkv_gemm", "attention", "o_gemm",
-                                              "gateup_gemm", "down_gemm", "lm_head", "host_copy"};
+                                              "gateup_gemm", "down_gemm", "lm_head", "host_copy", "quant"};
   return (tag >= 0 && tag < SVL_TAG_COUNT) ? names[tag] : "unknown";
 }
 

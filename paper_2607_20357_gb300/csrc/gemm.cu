@@ -1,10 +1,12 @@
 // Persistent warp-specialised tcgen05 GEMM with fused epilogues (sm_103a).
 //
-//   warp 0      one thread issues TMA loads of A (128 x 64) and B (up to
-//               2 x 128 x 64) per stage into a 4-stage shared-memory ring;
+//   warp 0      one thread issues TMA loads of A (128 rows x 128 bytes) and B
+//               (up to 2 x 128 rows x 128 bytes) per stage into a 4-stage
+//               shared-memory ring: 64 K of bf16 or 128 K of e4m3;
 //   warp 1      allocates 512 TMEM columns; one thread issues
-//               tcgen05.mma (M = 128, N <= 256, K = 16 per instruction) and
-//               commits stage releases and accumulator-ready signals;
+//               tcgen05.mma (M = 128, N <= 256, K = 16 per bf16 instruction,
+//               32 per e4m3 one) and commits stage releases and
+//               accumulator-ready signals;
 //   warps 2-5   epilogue: tcgen05.ld of their 32-lane quarter of the
 //               accumulator, fused math, global stores. Two accumulators
 //               alternate so the epilogue of tile i overlaps tile i+1.
@@ -121,11 +123,12 @@ struct StageCfg<EPI_SCORE_WIDE> {
 };
 
 // ------------------------------------------------------------------ producer
-template <int NST, int SBYTES>
+template <int NST, int SBYTES, bool F8>
 SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* full,
                               uint64_t* empty, volatile int* abort) {
+  constexpr int BK = F8 ? kBK8 : kBK;
   const int ntiles = num_tiles(p);
-  const int nkb = p.K / kBK, kgb = p.kgroup / kBK;
+  const int nkb = p.K / BK, kgb = p.kgroup / BK;
   int s = 0;
   uint32_t ph = 0;
   for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
@@ -150,9 +153,9 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
       uint8_t* sa = stages + s * SBYTES;
       uint8_t* sb = sa + kABytes;
       mbar_arrive_expect_tx(&full[s], bytes);
-      tma_load_2d(sa, &p.mapA, &full[s], kb * kBK, ti.m0);
-      tma_load_2d(sb, mb0, &full[s], kb * kBK, ti.n0);
-      if (halves == 2) tma_load_2d(sb + kBHalfBytes, mb1, &full[s], kb * kBK, y1);
+      tma_load_2d(sa, &p.mapA, &full[s], kb * BK, ti.m0);
+      tma_load_2d(sb, mb0, &full[s], kb * BK, ti.n0);
+      if (halves == 2) tma_load_2d(sb + kBHalfBytes, mb1, &full[s], kb * BK, y1);
       if (++s == NST) {
         s = 0;
         ph ^= 1;
@@ -162,11 +165,12 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
 }
 
 // ------------------------------------------------------------------ MMA issuer
-template <int NST, int SBYTES>
+template <int NST, int SBYTES, bool F8>
 SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, uint64_t* empty,
                          uint64_t* tfull, uint64_t* tempty, uint32_t tmem, volatile int* abort) {
+  constexpr int BK = F8 ? kBK8 : kBK;
   const int ntiles = num_tiles(p);
-  const int nkb = p.K / kBK, kgb = p.kgroup / kBK;
+  const int nkb = p.K / BK, kgb = p.kgroup / BK;
   int s = 0, it = 0;
   uint32_t ph = 0;
   for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
@@ -180,7 +184,7 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
     }
     tc_fence_after();
     const int n = p.b_split ? 2 * kBHalf : ((ti.ncols + 15) & ~15);
-    const uint32_t idesc = idesc_bf16_f32(kBM, n);
+    const uint32_t idesc = F8 ? idesc_e4m3_f32(kBM, n) : idesc_bf16_f32(kBM, n);
     const uint32_t d = tmem + acc * kAccCols;
     uint32_t accumulate = 0;
     int i0, i1;
@@ -193,10 +197,13 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
       tc_fence_after();
       const uint32_t a0 = smem_u32(stages + s * SBYTES);
       const uint32_t b0 = a0 + kABytes;
+      // four instructions per stage, each over the next 32 bytes of K
 #pragma unroll
-      for (int k = 0; k < kBK / 16; ++k) {
-        tc_mma_bf16(d, smem_desc_sw128(a0 + k * 32), smem_desc_sw128(b0 + k * 32), idesc,
-                    accumulate);
+      for (int k = 0; k < 4; ++k) {
+        if constexpr (F8)
+          tc_mma_e4m3(d, smem_desc_sw128(a0 + k * 32), smem_desc_sw128(b0 + k * 32), idesc, accumulate);
+        else
+          tc_mma_bf16(d, smem_desc_sw128(a0 + k * 32), smem_desc_sw128(b0 + k * 32), idesc, accumulate);
         accumulate = 1;
       }
       tc_commit(&empty[s]);
@@ -261,14 +268,31 @@ SVL_DEVINL float store_bf16_ss(__nv_bfloat16* dst, const float* v, int n /*16 or
   return ss;
 }
 
-template <int KIND>
+// e4m3 dequantisation of 32 accumulator columns: v[j] *= f * cs[j] (cs
+// 16-byte aligned; the same addresses in every lane of the warp)
+SVL_DEVINL void scale_cols(float* v, const float* cs, float f) {
+  const float4* c4 = reinterpret_cast<const float4*>(cs);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 c = __ldg(c4 + i);
+    v[4 * i] *= f * c.x;
+    v[4 * i + 1] *= f * c.y;
+    v[4 * i + 2] *= f * c.z;
+    v[4 * i + 3] *= f * c.w;
+  }
+}
+
+template <int KIND, bool F8>
 SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, bool rv,
                               uint32_t taddr) {
   float v[32];
+  // row factor of e4m3 operands (the activation row's scale)
+  const float af = (F8 && rv) ? p.a_scale[row] : 1.f;
   if constexpr (KIND == EPI_QKV_ROPE) {
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[ti.mat]);
     const size_t ld = static_cast<size_t>(p.ld[ti.mat]);
-    const float rs = (p.ss_in && rv) ? row_rms_scale(p, row) : 1.f;
+    const float rs = ((p.ss_in && rv) ? row_rms_scale(p, row) : 1.f) * af;
+    const float* bsc = F8 ? p.b_scale[ti.mat] + ti.n0 : nullptr;
     if (ti.mat < 2) {
       const int dh = p.d_head, half = dh / 2;
       int prow = rv ? p.pos[row] : 0;
@@ -283,6 +307,10 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
           tmem_ld32(taddr + hb + i0, v);
           tmem_ld32(taddr + hb + half + i0, w);
           if (rv) {
+            if constexpr (F8) {
+              scale_cols(v, bsc + hb + i0, 1.f);
+              scale_cols(w, bsc + hb + half + i0, 1.f);
+            }
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
               const float2 c = cs[i0 + j];
@@ -302,6 +330,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
       for (int c = 0; c < ti.ncols; c += 32) {
         tmem_ld32(taddr + c, v);
         if (rv) {
+          if constexpr (F8) scale_cols(v, bsc + c, 1.f);
 #pragma unroll
           for (int j = 0; j < 32; ++j)
             if (c + j < ti.ncols) out[static_cast<size_t>(ti.n0 + c + j) * ld + row] = __float2bfloat16_rn(v[j] * rs);
@@ -330,6 +359,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
       }
       tmem_ld32(taddr + c, v);
       if (rv) {
+        if constexpr (F8) scale_cols(v, p.b_scale[0] + ti.n0 + c, af);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const uint32_t w[4] = {xa[i].x, xa[i].y, xa[i].z, xa[i].w};
@@ -358,11 +388,15 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
     __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(p.out[0]);
     const size_t ld = static_cast<size_t>(p.ld[0]);
     float u[32];
-    const float rs = (p.ss_in && rv) ? row_rms_scale(p, row) : 1.f;
+    const float rs = ((p.ss_in && rv) ? row_rms_scale(p, row) : 1.f) * af;
     for (int c = 0; c < ti.ncols; c += 32) {
       tmem_ld32(taddr + c, v);
       tmem_ld32(taddr + kBHalf + c, u);
       if (rv) {
+        if constexpr (F8) {
+          scale_cols(v, p.b_scale[0] + ti.n0 + c, 1.f);
+          scale_cols(u, p.b_scale[1] + ti.n0 + c, 1.f);
+        }
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j] * rs) * (u[j] * rs);
         store_bf16(out + static_cast<size_t>(row) * ld + ti.n0 + c, v, min(32, ti.ncols - c));
@@ -399,6 +433,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
     for (int c = 0; c < ti.ncols; c += 32) {
       tmem_ld32(taddr + c, v);
       if (rv) {
+        if constexpr (F8) scale_cols(v, p.b_scale[0] + ti.n0 + c, af);
         float* o = out + static_cast<size_t>(row) * ld + ti.n0 + c;
 #pragma unroll
         for (int j = 0; j < 32; ++j)
@@ -472,6 +507,7 @@ SVL_DEVINL int ld_acquire(const int* p) {
 // this CTA sums all shares in order for its 1/nsplit of the tile's rows, adds
 // them to the residual rows and writes their norm partial sums. Every wait is
 // bounded; returns false on a time-out.
+template <bool F8>
 SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, uint32_t taddr, bool empty, KsSync& ks,
                             volatile int* abort) {
   const size_t unit = static_cast<size_t>(ti.slot) * ti.nsplit;
@@ -540,6 +576,7 @@ SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, u
           v[4 * i + 3] += f[i].w;
         }
       }
+      if constexpr (F8) scale_cols(v, p.b_scale[0] + ti.n0 + c, p.a_scale[row]);
       const uint4* xs = reinterpret_cast<const uint4*>(orow + c);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -562,7 +599,7 @@ SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, u
   return true;
 }
 
-template <int KIND>
+template <int KIND, bool F8>
 SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem,
                               volatile int* abort, KsSync& ks) {
   const int ntiles = num_tiles(p);
@@ -597,16 +634,17 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
     if constexpr (KIND == EPI_RESID) {
       if (ti.nsplit > 1) {
         int i0, i1;
-        k_share(ti, p.K / kBK, p.kgroup / kBK, i0, i1);
-        if (!ksplit_tile(p, ti, q * 32 + lane, taddr, i0 == i1, ks, abort)) {
+        constexpr int BK = F8 ? kBK8 : kBK;
+        k_share(ti, p.K / BK, p.kgroup / BK, i0, i1);
+        if (!ksplit_tile<F8>(p, ti, q * 32 + lane, taddr, i0 == i1, ks, abort)) {
           set_abort(abort, p.status);
           return;
         }
       } else {
-        epilogue_tile<KIND>(p, ti, row, rv, taddr);
+        epilogue_tile<KIND, F8>(p, ti, row, rv, taddr);
       }
     } else {
-      epilogue_tile<KIND>(p, ti, row, rv, taddr);
+      epilogue_tile<KIND, F8>(p, ti, row, rv, taddr);
     }
     tc_fence_before();
     mbar_arrive(&tempty[acc]);
@@ -615,7 +653,7 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
 }
 
 // ------------------------------------------------------------------ kernel
-template <int KIND>
+template <int KIND, bool F8>
 __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
   constexpr int NST = StageCfg<KIND>::stages, SBYTES = StageCfg<KIND>::bytes;
   extern __shared__ uint8_t smem_raw[];
@@ -661,11 +699,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   pdl_wait();
 
   if (warp == 0) {
-    if (lane == 0) producer_loop<NST, SBYTES>(p, stages, full, empty, abort);
+    if (lane == 0) producer_loop<NST, SBYTES, F8>(p, stages, full, empty, abort);
   } else if (warp == 1) {
-    if (lane == 0) mma_loop<NST, SBYTES>(p, stages, full, empty, tfull, tempty, tmem, abort);
+    if (lane == 0) mma_loop<NST, SBYTES, F8>(p, stages, full, empty, tfull, tempty, tmem, abort);
   } else {
-    epilogue_loop<KIND>(p, tfull, tempty, tmem, abort, ks);
+    epilogue_loop<KIND, F8>(p, tfull, tempty, tmem, abort, ks);
   }
 
   __syncwarp();
@@ -684,20 +722,30 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   }
 }
 
-template <int KIND>
+template <int KIND, bool F8 = false>
 static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t stream) {
   constexpr int smem = StageCfg<KIND>::stages * StageCfg<KIND>::bytes + 1024 + 256;
   static_assert(smem <= 232448, "shared memory per CTA");
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<KIND, F8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  return launch_pdl(gemm_kernel<KIND>, grid, kGemmThreads, smem, stream, p);
+  return launch_pdl(gemm_kernel<KIND, F8>, grid, kGemmThreads, smem, stream, p);
 }
 
-cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream) {
+cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3) {
+  if (e4m3) {
+    if (!p.a_scale || !p.b_scale[0]) return cudaErrorInvalidValue;
+    switch (kind) {
+      case EPI_QKV_ROPE: return launch_kind<EPI_QKV_ROPE, true>(p, grid, stream);
+      case EPI_RESID: return launch_kind<EPI_RESID, true>(p, grid, stream);
+      case EPI_SWIGLU: return launch_kind<EPI_SWIGLU, true>(p, grid, stream);
+      case EPI_F32: return launch_kind<EPI_F32, true>(p, grid, stream);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (kind) {
     case EPI_QKV_ROPE: return launch_kind<EPI_QKV_ROPE>(p, grid, stream);
     case EPI_RESID: return launch_kind<EPI_RESID>(p, grid, stream);

@@ -1,6 +1,7 @@
 // Persistent tcgen05/TMEM GEMM for sm_103a: C[M,N] = A[M,K] * B[N,K]^T with
-// bf16 K-major operands staged by TMA (128-byte swizzle) and an fp32
-// accumulator in tensor memory, followed by a fused epilogue.
+// bf16 (or, for the gated projections, e4m3) K-major operands staged by TMA
+// (128-byte swizzle) and an fp32 accumulator in tensor memory, followed by a
+// fused epilogue.
 //
 // Work arrives either as an explicit device tile list (the gated layers: one
 // tile per (row segment, column run) of active groups) or as a dense grid.
@@ -11,7 +12,8 @@
 namespace svl {
 
 constexpr int kBM = 128;           // rows per tile (TMEM lanes)
-constexpr int kBK = 64;            // K per stage: one 128-byte swizzle row
+constexpr int kBK = 64;            // K per stage: one 128-byte swizzle row (bf16)
+constexpr int kBK8 = 128;          // the same 128 bytes of e4m3
 constexpr int kBHalf = 128;        // B rows per TMA box; a stage holds two
 constexpr int kStages = 4;
 constexpr int kABytes = kBM * kBK * 2;
@@ -53,8 +55,8 @@ struct GemmParams {
   const int* m_limit_dev;  // rows bound read on the device (nullptr: use m_limit)
   int m_limit, n_limit;
   // K loop
-  int K;       // multiple of 64
-  int kgroup;  // K elements per gate group (kmask), multiple of 64
+  int K;       // multiple of 64 (e4m3: 128)
+  int kgroup;  // K elements per gate group (kmask), multiple of 64 (e4m3: 128)
   int b_split; // 1: B rows 0-127 from mapB[0], rows 128-255 from mapB[1] (gate | up)
   int b_box_rows;  // rows of one B box when mapB has boxes of fewer than 128 rows (0: 128)
   // epilogue operands
@@ -88,9 +90,15 @@ struct GemmParams {
   const int* ks_info;  // [3] on the device, or nullptr
   float* ks_part;      // [tail tiles * parts][128][256]
   int* ks_ticket;      // [tail tiles]
+  // e4m3 operands (QKV, residual and SwiGLU epilogues): the accumulator is
+  // the sum of code products; the epilogue scales element (r, n) by
+  // a_scale[r] * b_scale[mat][n] before anything else. The b_scale arrays
+  // are readable 32 floats past their last column.
+  const float* a_scale;
+  const float* b_scale[3];
   uint32_t* status;
 };
 
-cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream);
+cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3 = false);
 
 }  // namespace svl

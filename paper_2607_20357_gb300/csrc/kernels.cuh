@@ -77,6 +77,29 @@ SVL_DEVINL int find_sample(const int* cu, int B, int r) {
   return lo;
 }
 
+// ---------------------------------------------------------------- e4m3 operands
+// Per-row e4m3 quantisation of bf16 rows. Row r of src holds G groups of kg
+// columns; dst row r holds G groups of kgp >= kg codes (the tail of each
+// group zero, so that every group starts on a 128-byte K block). Only the
+// groups active for the row's sample are read and quantised (the others are
+// written as zeros): gates of layer l when group_gate is given, else all.
+// Rows at or past cu_seqlens[B] (when given) are left untouched.
+struct QuantArgs {
+  const __nv_bfloat16* src;
+  int64_t ld_src;
+  int64_t rows;
+  int G, kg, kgp;
+  uint8_t* dst;
+  int64_t ld_dst;
+  float* scale;  // [rows]: amax / 448 (0 for a row without a non-zero value)
+  const int* cu_seqlens;
+  int B;
+  const uint8_t* layer_gate;  // [B, L] or nullptr
+  const uint8_t* group_gate;  // [B, L, G] or nullptr
+  int L, l, P;
+};
+cudaError_t launch_quant_rows(const QuantArgs& a, cudaStream_t s);
+
 // ---------------------------------------------------------------- decode
 // Cache of one layer: [B][max_len][dkv] bf16 for K and for V.
 struct KvArgs {

@@ -1,0 +1,79 @@
+// e4m3 operands of the gated projections (FP8 weights, which the paper
+// calls orthogonal to its method, Sec. 5). Every row -- an output channel of
+// a weight matrix, or an activation row feeding one of the four gated GEMMs
+// -- is scaled so that its largest magnitude maps to 448, the largest finite
+// e4m3 value, and rounded to nearest even with saturation:
+//
+//   amax = max |x|, inv = 448 / amax, scale = amax / 448 (float32, correctly
+//   rounded; 0 and 0 when amax = 0), code = e4m3(x * inv).
+//
+// The GEMM multiplies codes and scales its accumulator by both rows' scales.
+#include "kernels.cuh"
+
+namespace svl {
+
+constexpr int kQuantWarps = 8;
+
+__global__ void __launch_bounds__(kQuantWarps * 32) quant_rows_kernel(QuantArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t r = static_cast<int64_t>(blockIdx.x) * kQuantWarps + warp;
+  int64_t rows = a.rows;
+  if (a.cu_seqlens) rows = min(rows, static_cast<int64_t>(a.cu_seqlens[a.B]));
+  if (r >= rows) return;
+  int mask = (1 << a.G) - 1;
+  if (a.group_gate && a.l >= a.P) {
+    const int b = find_sample(a.cu_seqlens, a.B, static_cast<int>(r));
+    const size_t bl = static_cast<size_t>(b) * a.L + a.l;
+    mask = 0;
+    if (a.layer_gate[bl])
+      for (int j = 0; j < a.G; ++j) mask |= a.group_gate[bl * a.G + j] ? (1 << j) : 0;
+  }
+  const __nv_bfloat16* src = a.src + r * a.ld_src;
+  float amax = 0.f;
+  for (int j = 0; j < a.G; ++j) {
+    if (!((mask >> j) & 1)) continue;
+    const uint4* s4 = reinterpret_cast<const uint4*>(src + static_cast<size_t>(j) * a.kg);
+    for (int c = lane; c < a.kg / 8; c += 32) {
+      const uint4 u = s4[c];
+      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = unpack_bf16x2(w[q]);
+        amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+  const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
+  uint8_t* dst = a.dst + r * a.ld_dst;
+  for (int j = 0; j < a.G; ++j) {
+    const bool on = (mask >> j) & 1;
+    const uint4* s4 = reinterpret_cast<const uint4*>(src + static_cast<size_t>(j) * a.kg);
+    uint2* d8 = reinterpret_cast<uint2*>(dst + static_cast<size_t>(j) * a.kgp);
+    for (int c = lane; c < a.kgp / 8; c += 32) {
+      uint2 o = make_uint2(0, 0);
+      if (on && c < a.kg / 8) {
+        const uint4 u = s4[c];
+        const float2 f0 = unpack_bf16x2(u.x), f1 = unpack_bf16x2(u.y), f2 = unpack_bf16x2(u.z),
+                     f3 = unpack_bf16x2(u.w);
+        o.x = static_cast<uint32_t>(e4m3x2(__fmul_rn(f0.x, inv), __fmul_rn(f0.y, inv))) |
+              (static_cast<uint32_t>(e4m3x2(__fmul_rn(f1.x, inv), __fmul_rn(f1.y, inv))) << 16);
+        o.y = static_cast<uint32_t>(e4m3x2(__fmul_rn(f2.x, inv), __fmul_rn(f2.y, inv))) |
+              (static_cast<uint32_t>(e4m3x2(__fmul_rn(f3.x, inv), __fmul_rn(f3.y, inv))) << 16);
+      }
+      d8[c] = o;
+    }
+  }
+  if (lane == 0) a.scale[r] = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
+}
+
+cudaError_t launch_quant_rows(const QuantArgs& a, cudaStream_t s) {
+  if (a.rows <= 0) return cudaSuccess;
+  const int64_t blocks = (a.rows + kQuantWarps - 1) / kQuantWarps;
+  return launch_pdl(quant_rows_kernel, dim3(static_cast<unsigned>(blocks)), kQuantWarps * 32, 0, s, a);
+}
+
+}  // namespace svl

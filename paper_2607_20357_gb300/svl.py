@@ -23,16 +23,18 @@ SVL_LOGITS_ALL = 1
 SVL_FLAG_OVER_BUDGET = 1
 SVL_FLAG_GROUPS_DROPPED = 2
 SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
+SVL_GEMM_BF16, SVL_GEMM_E4M3 = 0, 1
 
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
            "svl_prefill_from_host", "svl_host_workspace_size", "svl_profile_start", "svl_profile_stop",
            "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches", "svl_selftest_wait_timeout",
            "svl_workspace_size_for", "svl_score_select_paper", "svl_pack_controlled", "svl_controlled_prefill",
-           "svl_kv_cache_size", "svl_gated_prefill_kv", "svl_decode_workspace_size", "svl_decode_step"]
+           "svl_kv_cache_size", "svl_gated_prefill_kv", "svl_decode_workspace_size", "svl_decode_step",
+           "svl_quantize_rows_e4m3", "svl_gemm_e4m3"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
-        "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy"]
+        "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy", "quant"]
 
 
 class KernelTime(ctypes.Structure):
@@ -42,7 +44,8 @@ class KernelTime(ctypes.Structure):
 class ModelDesc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in ("n_layers", "d_model", "n_heads", "n_kv_heads", "d_ffn", "vocab",
                                               "n_groups", "n_prefix", "c_vis", "h_ctrl", "proj_hidden")] + \
-               [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float), ("max_seq", ctypes.c_int32)]
+               [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float), ("max_seq", ctypes.c_int32),
+                ("gemm_format", ctypes.c_int32)]
 
 
 class LayerWeights(ctypes.Structure):
@@ -120,6 +123,10 @@ def lib():
         L.svl_selftest_wait_timeout.restype = ctypes.c_int
         L.svl_workspace_size_for.argtypes = [vp, ctypes.c_uint32, i32, i64, i64]
         L.svl_workspace_size_for.restype = sz
+        L.svl_quantize_rows_e4m3.argtypes = [vp, i64, i32, i64, vp, i64, vp, vp]
+        L.svl_quantize_rows_e4m3.restype = ctypes.c_int
+        L.svl_gemm_e4m3.argtypes = [vp] * 5 + [i32, i32, i32, vp, vp]
+        L.svl_gemm_e4m3.restype = ctypes.c_int
         _lib = L
     return _lib
 
@@ -203,6 +210,16 @@ def svl_gated_prefill_kv(model, B, t_cap, X, cu_seqlens, pos, layer_gate, group_
         model, int(B), int(t_cap), _p(X), _p(cu_seqlens), _p(pos), _p(layer_gate), _p(group_gate),
         int(logits_mode), _p(logits), _p(kv_cache), int(max_len), _p(cache_len), _p(workspace),
         int(workspace_bytes), _stream(stream)))
+
+
+def svl_quantize_rows_e4m3(src, rows, cols, ld_src, dst, ld_dst, scale, stream=None):
+    _check("svl_quantize_rows_e4m3", lib().svl_quantize_rows_e4m3(
+        _p(src), int(rows), int(cols), int(ld_src), _p(dst), int(ld_dst), _p(scale), _stream(stream)))
+
+
+def svl_gemm_e4m3(model, A, a_scale, B, b_scale, M, N, K, C, stream=None):
+    _check("svl_gemm_e4m3", lib().svl_gemm_e4m3(model, _p(A), _p(a_scale), _p(B), _p(b_scale), int(M), int(N),
+                                                int(K), _p(C), _stream(stream)))
 
 
 def svl_decode_workspace_size(model, B) -> int:
@@ -324,11 +341,12 @@ def svl_profile_stop(model) -> dict:
 
 
 # --------------------------------------------------------------------------- plumbing
-def model_desc(dims, max_seq: int) -> ModelDesc:
+def model_desc(dims, max_seq: int, gemm_format: int = SVL_GEMM_BF16) -> ModelDesc:
     return ModelDesc(n_layers=dims.n_layers, d_model=dims.d_model, n_heads=dims.n_heads,
                      n_kv_heads=dims.n_kv_heads, d_ffn=dims.d_ffn, vocab=dims.vocab, n_groups=dims.n_groups,
                      n_prefix=dims.n_prefix, c_vis=dims.c_vis, h_ctrl=dims.h_ctrl, proj_hidden=dims.proj_hidden,
-                     rms_eps=dims.rms_eps, rope_theta=dims.rope_theta, max_seq=int(max_seq))
+                     rms_eps=dims.rms_eps, rope_theta=dims.rope_theta, max_seq=int(max_seq),
+                     gemm_format=int(gemm_format))
 
 
 class GatedPrefill:
@@ -337,12 +355,14 @@ class GatedPrefill:
     ``weights`` is a dict as produced by the input generator, tensors on the
     CUDA device (bf16, nn.Linear layout). ``run`` allocates the outputs and
     the workspace with torch and calls the three C entry points in order.
+    ``gemm_format`` = SVL_GEMM_E4M3 runs the gated projections on e4m3
+    operands (the model quantises its weights once, at creation).
     """
 
-    def __init__(self, dims, weights: dict, max_seq: int = 8192):
+    def __init__(self, dims, weights: dict, max_seq: int = 8192, gemm_format: int = SVL_GEMM_BF16):
         self.dims = dims
         self.w = weights
-        self.desc = model_desc(dims, max_seq)
+        self.desc = model_desc(dims, max_seq, gemm_format)
         lw = (LayerWeights * dims.n_layers)()
         for i, l in enumerate(weights["layers"]):
             lw[i] = LayerWeights(*[l[n].data_ptr() for n in ("wq", "wk", "wv", "wo", "wg", "wu", "wd",

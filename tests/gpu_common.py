@@ -89,7 +89,7 @@ def numpy_weights_lazy(w):
 class Case:
     """Seeded model + batch on the GPU and the oracle's view of both."""
 
-    def __init__(self, dims, wl, seed, batch=None, budget=None, max_seq=8192, std=0.02):
+    def __init__(self, dims, wl, seed, batch=None, budget=None, max_seq=8192, std=0.02, gemm_format=svl.SVL_GEMM_BF16):
         self.dims = dims
         w = synth.make_weights(dims, seed, std=std)
         b = synth.make_batch(wl, seed, budget=budget, batch=batch, dims=dims)
@@ -97,7 +97,7 @@ class Case:
         self.b_np = O.to_numpy_batch(b)
         self.w = to_device(w)
         self.b = to_device(b)
-        self.model = svl.GatedPrefill(dims, self.w, max_seq=max_seq)
+        self.model = svl.GatedPrefill(dims, self.w, max_seq=max_seq, gemm_format=gemm_format)
 
     def run(self, logits_mode=svl.SVL_LOGITS_LAST):
         out = self.model.run(self.b, logits_mode=logits_mode)
