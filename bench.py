@@ -51,6 +51,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-hbm-sweep", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-fp8", action="store_true", help="skip the e4m3 (FP8 gated projections) pass")
     ap.add_argument("--hbm-only", type=str, default="",
                     help="comma-separated batch multipliers: run only the token-controller/pack sweep "
                          "(for small profiler captures)")
@@ -405,6 +406,11 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and not args.no_decode:
         dec = run_decode(svl, model, batches[1], dims, dev, pk)
 
+    fp8 = None
+    if rank == 0 and not args.no_fp8:
+        model.close()  # its workspace and outputs go; the e4m3 model holds its own weight codes
+        fp8 = run_fp8(args, svl, wl, weights, batches, dev, pk, max_seq)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         nl = 16
@@ -428,13 +434,90 @@ def run_ours(args, rank, world, local_rank):
             "per_budget": per_budget, "roofline": roofline, "kernels": kernels,
             "gpu_launches": int(launches), "gpu_launches_per_step": launches / args.steps,
             "wall_s_timed": t_wall, "clocks": clk.summary(), "e2e": e2e, "cpu_baseline": cpu,
-            "hbm_kernels_sweep": hbm, "decode": dec,
+            "hbm_kernels_sweep": hbm, "decode": dec, "fp8": fp8,
         }
         print(json.dumps(line), flush=True)
     model.close()
 
 
-def run_decode(svl, model, bt, dims, dev, pk, steps=16, warm=3):
+def run_fp8(args, svl, wl, weights, batches, dev, pk, max_seq):
+    """The same workload with SVL_GEMM_E4M3: the four gated projections on
+    e4m3 operands (per-channel weight and per-row activation scales). Not the
+    headline (reduced precision): its own tokens/s, executed TFLOP/s against
+    the fp8 peak (measured bf16 sustained peak x 2, the nominal fp8/bf16
+    ratio), the per-kernel breakdown including the activation quantisation,
+    and e4m3 decode."""
+    dims = wl.dims
+    model = svl.GatedPrefill(dims, weights, max_seq=max_seq, gemm_format=svl.SVL_GEMM_E4M3)
+    outs = [model.alloc_outputs(bt) for bt in batches]
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        model.run(batches[i % len(batches)], out=outs[i % len(batches)])
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    status = svl.svl_get_device_status(model.handle)
+    if status:
+        raise RuntimeError(f"device status {status:#x} in the e4m3 pass")
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    svl.svl_profile_start(model.handle, tags=["gateup_gemm"])
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        for i in range(args.steps):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+    live = svl.svl_profile_stop(model.handle)
+    svl.svl_profile_start(model.handle)
+    for i in range(args.steps):
+        step(i)
+    kern = svl.svl_profile_stop(model.handle)
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    tokens, fexec, kind = 0, 0.0, {}
+    per_budget = []
+    for j, bt in enumerate(batches):
+        idx = list(range(j, args.steps, len(batches)))
+        if not idx:
+            continue
+        k = outs[j]["k"].cpu().numpy()
+        nv = (bt["vis_off"][1:] - bt["vis_off"][:-1]).cpu().numpy()
+        st = (bt["text_off"][1:] - bt["text_off"][:-1]).cpu().numpy()
+        lg, gg = bt["layer_gate"].cpu(), bt["group_gate"].cpu()
+        toks = int(nv.sum() + st.sum())
+        fex = executed_flops(svl, model.desc, k, st, nv, lg, gg)
+        ms = statistics.mean(step_ms[i] for i in idx)
+        per_budget.append({"budget": float(bt["budget"][0]), "ms_per_step": ms, "tokens_per_s": toks / (ms / 1e3),
+                           "exec_tflops": fex / (ms / 1e3) / 1e12})
+        tokens += toks * len(idx)
+        fexec += fex * len(idx)
+        for kk, v in per_kind_flops(dims, k, st, lg.numpy(), gg.numpy()).items():
+            kind[kk] = kind.get(kk, 0.0) + v * len(idx)
+    total_ms = sum(step_ms)
+    peak8 = 2.0 * pk["bf16_tflops_sustained"]
+    n_l, t_l = live["gateup_gemm"]
+    gu = kind["gateup_gemm"] / (t_l / 1e3) / 1e12
+    tot_k = max(sum(v[1] for v in kern.values()), 1e-9)
+    kernels = {t: {"launches": n, "total_ms": ms, "share": ms / tot_k}
+               for t, (n, ms) in sorted(kern.items(), key=lambda kv: -kv[1][1])}
+    for t in kind:
+        if t in kernels:
+            kernels[t]["tflops"] = kind[t] / (kernels[t]["total_ms"] / 1e3) / 1e12
+    dec = None
+    if not args.no_decode:
+        dec = run_decode(svl, model, batches[1], dims, dev, pk, layer_weight_bytes=1)
+    model.close()
+    return {"gemm_format": "e4m3 (gated projections; projector, token controller, attention, LM head bf16)",
+            "value": tokens / (total_ms / 1e3), "unit": "tokens/s", "ms_per_step": total_ms / args.steps,
+            "exec_tflops": fexec / (total_ms / 1e3) / 1e12,
+            "exec_tflops_frac_of_fp8_peak": fexec / (total_ms / 1e3) / 1e12 / peak8,
+            "fp8_peak_tflops": peak8, "fp8_peak_source": pk["source"] + " bf16 sustained x 2 (nominal fp8/bf16)",
+            "gateup_gemm": {"launches": n_l, "avg_launch_ms": t_l / n_l, "tflops": gu, "frac": gu / peak8},
+            "per_budget": per_budget, "kernels": kernels, "clocks": clk.summary(), "decode": dec}
+
+
+def run_decode(svl, model, bt, dims, dev, pk, steps=16, warm=3, layer_weight_bytes=2):
     """Gated decode after a KV-cache prefill of the budget-0.5 batch: tokens
     per second over `steps` teacher-forced steps (CUDA events) and the bytes
     each step must read -- every weight of the active groups once plus the
@@ -467,17 +550,26 @@ def run_decode(svl, model, bt, dims, dev, pk, steps=16, warm=3):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / steps
+    # device time per kernel kind over a few more steps (events around every launch)
+    svl.svl_profile_start(model.handle)
+    for t in range(warm):
+        svl.svl_decode_step(model.handle, B, fed[t], kv, max_len, cache_len, bt["layer_gate"], bt["group_gate"],
+                            logits, nxt, dws, dws.numel())
+    kern = svl.svl_profile_stop(model.handle)
+    kernel_ms = {k: round(v[1] / warm, 4) for k, v in sorted(kern.items(), key=lambda kv: -kv[1][1])}
     d = dims
     dh = d.d_model // d.n_heads
     on = effective_on(bt, d)  # active (layer, group) pairs per sample
     per_group = d.d_model * (d.n_heads * dh * 2 + 2 * d.n_kv_heads * dh) // d.n_groups + 3 * d.d_model * d.d_ffn // d.n_groups
-    w_bytes = 2 * (int(on.any(dim=0).sum()) * per_group + d.vocab * d.d_model)  # groups active in any sample
+    # groups active in any sample (e4m3 models: one byte per gated-projection weight)
+    w_bytes = layer_weight_bytes * int(on.any(dim=0).sum()) * per_group + 2 * d.vocab * d.d_model
     ctx = float((len0.double() + steps / 2).mean())
     kv_bytes = 2 * 2 * float(on.sum()) * (d.n_kv_heads // d.n_groups) * dh * ctx
     nbytes = w_bytes + kv_bytes
     return {"batch": B, "steps": steps, "ms_per_step": ms, "tokens_per_s": B / (ms / 1000.0),
             "context_mean": ctx, "bytes_per_step": nbytes, "gb_s": nbytes / (ms / 1000.0) / 1e9,
             "frac_of_measured_hbm": nbytes / (ms / 1000.0) / 1e9 / pk["hbm_gbs"],
+            "kernel_ms_per_step_profiled": kernel_ms,
             "note": "teacher-forced, budget-0.5 batch, prefill gates; bytes = active-group weights once "
                     "(shared by the batch) + cached K/V of the active heads"}
 
