@@ -289,10 +289,10 @@ struct Launch {
 };
 
 svl_status launch(EpiKind kind, svl_model* m, int tag, const GemmParams& p, int64_t tiles, cudaStream_t s,
-                  bool e4m3 = false) {
+                  bool e4m3 = false, bool thin = false) {
   if (tiles <= 0) return SVL_OK;
   Launch L(m, tag, s);
-  return launch_gemm(kind, p, gemm_grid(m, tiles), s, e4m3) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
+  return launch_gemm(kind, p, gemm_grid(m, tiles), s, e4m3, thin) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
 }
 
 svl_status last_error() { return cudaGetLastError() == cudaSuccess ? SVL_OK : SVL_ERR_CUDA; }
@@ -841,9 +841,13 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   __nv_bfloat16* vb = at<__nv_bfloat16>(ws, L.v);
   __nv_bfloat16* ao = at<__nv_bfloat16>(ws, L.ao);
   __nv_bfloat16* hm = at<__nv_bfloat16>(ws, L.hmid);
+  // decode-sized batches (one row per sample) stream the weights through the
+  // gated GEMMs with A boxes of kThinRows rows and deeper stages
+  const bool thin = t_cap <= kThinRows;
+  const uint32_t a_rows = thin ? kThinRows : 128;
   CUtensorMap map_x, map_xn, map_ao, map_hm;
-  if (!make_map(&map_x, X, t_cap, d.d_model) || !make_map(&map_xn, xn, t_cap, d.d_model) ||
-      !make_map(&map_ao, ao, t_cap, hq) || !make_map(&map_hm, hm, t_cap, d.d_ffn))
+  if (!make_map(&map_x, X, t_cap, d.d_model, a_rows) || !make_map(&map_xn, xn, t_cap, d.d_model) ||
+      !make_map(&map_ao, ao, t_cap, hq, a_rows) || !make_map(&map_hm, hm, t_cap, d.d_ffn, a_rows))
     return SVL_ERR_CUDA;
   // e4m3: every gated GEMM reads the quantised rows of its input (aq, with
   // per-row scales as) -- X for QKV and gate/up, the attention output for
@@ -853,9 +857,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   uint8_t* aq = f8 ? at<uint8_t>(ws, L.aq) : nullptr;
   float* as = f8 ? at<float>(ws, L.as) : nullptr;
   CUtensorMap map_aq_x, map_aq_o, map_aq_h;
-  if (f8 && (!make_map8(&map_aq_x, aq, t_cap, d.d_model) ||
-             !make_map8(&map_aq_o, aq, t_cap, static_cast<uint64_t>(G) * m->kgo_p) ||
-             !make_map8(&map_aq_h, aq, t_cap, static_cast<uint64_t>(G) * m->kgd_p)))
+  if (f8 && (!make_map8(&map_aq_x, aq, t_cap, d.d_model, a_rows) ||
+             !make_map8(&map_aq_o, aq, t_cap, static_cast<uint64_t>(G) * m->kgo_p, a_rows) ||
+             !make_map8(&map_aq_h, aq, t_cap, static_cast<uint64_t>(G) * m->kgd_p, a_rows)))
     return SVL_ERR_CUDA;
   auto quant = [&](const __nv_bfloat16* src, int64_t ld_src, int groups, int kg, int kgp, int layer) {
     QuantArgs qa;
@@ -986,7 +990,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.rope_cs = m->rope_cs;
     p.rope_rows = d.max_seq;
     p.d_head = dh;
-    if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8)) != SVL_OK) return st;
+    if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8, thin)) != SVL_OK) return st;
 
     const size_t layer_kv = static_cast<size_t>(B) * (kvx ? kvx->max_len : 0) * dkv;
     if (kvx && kvx->decode) {
@@ -1059,7 +1063,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
     set_norm(p, nullptr, ss_b);  // sums of squares of the updated rows for the MLP norm
-    if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s, f8)) != SVL_OK) return st;
+    if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s, f8, thin)) != SVL_OK) return st;
 
     // MLP input norm fused into the gate/up GEMM (gain folded into W_g, W_u)
     if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), d.d_model, 1, d.d_model, d.d_model, -1)) != SVL_OK)
@@ -1078,7 +1082,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.kgroup = d.d_model;
     p.out[0] = hm;
     p.ld[0] = d.d_ffn;
-    if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8)) != SVL_OK) return st;
+    if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8, thin)) != SVL_OK) return st;
 
     if (f8 && (st = quant(hm, d.d_ffn, G, d.d_ffn / G, m->kgd_p, l)) != SVL_OK) return st;
     p = base_params(m);
@@ -1100,7 +1104,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;
     set_norm(p, nullptr, ss_a);  // for the next layer's attention norm
-    if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s, f8)) != SVL_OK) return st;
+    if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s, f8, thin)) != SVL_OK) return st;
   }
 
   // final norm + LM head

@@ -88,10 +88,29 @@ void launch_decode_prep(int B, int D, int V, const int* tokens, const int* cache
 // query against the cached keys 0..len-1 and its own key (position len),
 // softmax in float32, output row of O. The block of the first query head of
 // each KV head also appends the new key and value to the cache. Each warp
-// takes every 8th position with an online softmax; the warps are merged at
-// the end. Memory-bound on the cache (2 * (len + 1) * d_head * 2 bytes).
+// takes runs of kDecRun consecutive positions (every kDecWarps-th run),
+// loading all their K and V rows before using any (lane i holds d_head / 32
+// consecutive dimensions, one 4- or 8-byte load per row), and folds the run
+// into its online softmax at once; the warps are merged at the end. Four
+// blocks fit per SM, so a batch of 16 samples x 32 heads runs in one wave.
+// Memory-bound on the cache (2 * (len + 1) * d_head * 2 bytes per head).
 constexpr int kDecWarps = 8;
-__global__ void __launch_bounds__(kDecWarps * 32) decode_attn_kernel(DecAttnArgs a) {
+constexpr int kDecRun = 4;
+
+template <int PER>  // d_head / 32: 2 or 4
+SVL_DEVINL void load_row(const __nv_bfloat16* src, float* out) {
+  if constexpr (PER == 4) {
+    const uint2 u = *reinterpret_cast<const uint2*>(src);
+    const float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+    out[0] = a.x; out[1] = a.y; out[2] = b.x; out[3] = b.y;
+  } else {
+    const float2 a = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(src));
+    out[0] = a.x; out[1] = a.y;
+  }
+}
+
+template <int PER>
+__global__ void __launch_bounds__(kDecWarps * 32, 4) decode_attn_kernel(DecAttnArgs a) {
   __shared__ float sm_m[kDecWarps], sm_l[kDecWarps];
   __shared__ float sm_o[kDecWarps][128];
   pdl_trigger();
@@ -104,111 +123,142 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_attn_kernel(DecAttnArgs
   const int dh = a.dh, kvh = h / (a.A / a.Akv);
   const int len = a.cache_len[b];
   if (len < 0 || len >= a.max_len) return;  // reported by decode_prep
-  const size_t cbase = static_cast<size_t>(b) * a.max_len * a.dkv + static_cast<size_t>(kvh) * dh;
-  const int per = dh / 32;  // d_head / 32 dims per lane (2 or 4)
-  float q[4], kn[4], vn[4];
+  const size_t cbase = static_cast<size_t>(b) * a.max_len * a.dkv + static_cast<size_t>(kvh) * dh + lane * PER;
+  float q[PER], kn[PER], vn[PER];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int d = lane * per + i;
-    q[i] = i < per ? __bfloat162float(a.q[static_cast<size_t>(b) * a.ldq + h * dh + d]) : 0.f;
-    kn[i] = i < per ? __bfloat162float(a.k[static_cast<size_t>(b) * a.dkv + kvh * dh + d]) : 0.f;
-    vn[i] = i < per ? __bfloat162float(a.vt[static_cast<size_t>(kvh * dh + d) * a.t_pad + b]) : 0.f;
+  for (int i = 0; i < PER; ++i) {
+    const int d = lane * PER + i;
+    q[i] = __bfloat162float(a.q[static_cast<size_t>(b) * a.ldq + h * dh + d]) * a.scale;
+    kn[i] = __bfloat162float(a.k[static_cast<size_t>(b) * a.dkv + kvh * dh + d]);
+    vn[i] = __bfloat162float(a.vt[static_cast<size_t>(kvh * dh + d) * a.t_pad + b]);
   }
   if (h % (a.A / a.Akv) == 0 && warp == 0) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (i < per) {
-        const int d = lane * per + i;
-        a.k_cache[cbase + static_cast<size_t>(len) * a.dkv + d] = __float2bfloat16_rn(kn[i]);
-        a.v_cache[cbase + static_cast<size_t>(len) * a.dkv + d] = __float2bfloat16_rn(vn[i]);
-      }
+    for (int i = 0; i < PER; ++i) {
+      a.k_cache[cbase + static_cast<size_t>(len) * a.dkv + i] = __float2bfloat16_rn(kn[i]);
+      a.v_cache[cbase + static_cast<size_t>(len) * a.dkv + i] = __float2bfloat16_rn(vn[i]);
+    }
   }
-  float m = -INFINITY, l = 0.f, o[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int p = warp; p <= len; p += kDecWarps) {
-    float kk[4], vv[4];
-    if (p == len) {
+  float m = -INFINITY, l = 0.f, o[PER];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        kk[i] = kn[i];
-        vv[i] = vn[i];
-      }
-    } else {
-      const __nv_bfloat16* kr = a.k_cache + cbase + static_cast<size_t>(p) * a.dkv + lane * per;
-      const __nv_bfloat16* vr = a.v_cache + cbase + static_cast<size_t>(p) * a.dkv + lane * per;
+  for (int i = 0; i < PER; ++i) o[i] = 0.f;
+  for (int p0 = warp * kDecRun; p0 <= len; p0 += kDecWarps * kDecRun) {
+    float kk[kDecRun][PER], vv[kDecRun][PER], sc[kDecRun];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        kk[i] = i < per ? __bfloat162float(kr[i]) : 0.f;
-        vv[i] = i < per ? __bfloat162float(vr[i]) : 0.f;
+    for (int u = 0; u < kDecRun; ++u) {
+      const int p = p0 + u;
+      if (p < len) {
+        load_row<PER>(a.k_cache + cbase + static_cast<size_t>(p) * a.dkv, kk[u]);
+        load_row<PER>(a.v_cache + cbase + static_cast<size_t>(p) * a.dkv, vv[u]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < PER; ++i) {
+          kk[u][i] = p == len ? kn[i] : 0.f;
+          vv[u][i] = p == len ? vn[i] : 0.f;
+        }
       }
     }
-    float sdot = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) sdot = fmaf(q[i], kk[i], sdot);
+    for (int u = 0; u < kDecRun; ++u) {
+      float d = 0.f;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) sdot += __shfl_xor_sync(0xffffffffu, sdot, off);
-    const float sc = sdot * a.scale;
-    const float mn = fmaxf(m, sc);
-    const float corr = __expf(m - mn), e = __expf(sc - mn);
-    l = l * corr + e;
+      for (int i = 0; i < PER; ++i) d = fmaf(q[i], kk[u][i], d);
+      sc[u] = d;
+    }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) o[i] = fmaf(o[i], corr, e * vv[i]);
-    m = mn;
+    for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+      for (int u = 0; u < kDecRun; ++u) sc[u] += __shfl_xor_sync(0xffffffffu, sc[u], off);
+    float mr = m;
+#pragma unroll
+    for (int u = 0; u < kDecRun; ++u)
+      if (p0 + u <= len) mr = fmaxf(mr, sc[u]);
+    const float corr = __expf(m - mr);
+    l *= corr;
+#pragma unroll
+    for (int i = 0; i < PER; ++i) o[i] *= corr;
+#pragma unroll
+    for (int u = 0; u < kDecRun; ++u) {
+      const float e = p0 + u <= len ? __expf(sc[u] - mr) : 0.f;
+      l += e;
+#pragma unroll
+      for (int i = 0; i < PER; ++i) o[i] = fmaf(e, vv[u][i], o[i]);
+    }
+    m = mr;
   }
   if (lane == 0) {
     sm_m[warp] = m;
     sm_l[warp] = l;
   }
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
-    if (i < per) sm_o[warp][lane * per + i] = o[i];
+  for (int i = 0; i < PER; ++i) sm_o[warp][lane * PER + i] = o[i];
   __syncthreads();
   if (warp == 0) {
     float M = -INFINITY;
     for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, sm_m[w]);
-    float L = 0.f, acc[4] = {0.f, 0.f, 0.f, 0.f};
+    float L = 0.f, acc[PER];
+#pragma unroll
+    for (int i = 0; i < PER; ++i) acc[i] = 0.f;
     for (int w = 0; w < kDecWarps; ++w) {
       const float f = sm_m[w] == -INFINITY ? 0.f : __expf(sm_m[w] - M);
       L += sm_l[w] * f;
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (i < per) acc[i] += sm_o[w][lane * per + i] * f;
+      for (int i = 0; i < PER; ++i) acc[i] += sm_o[w][lane * PER + i] * f;
     }
     const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (i < per) a.out[static_cast<size_t>(b) * a.ldo + h * dh + lane * per + i] = __float2bfloat16_rn(acc[i] * inv);
+    for (int i = 0; i < PER; ++i)
+      a.out[static_cast<size_t>(b) * a.ldo + h * dh + lane * PER + i] = __float2bfloat16_rn(acc[i] * inv);
   }
 }
 
 void launch_decode_attn(const DecAttnArgs& a, cudaStream_t s) {
-  launch_pdl(decode_attn_kernel, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
+  if (a.dh == 128)
+    launch_pdl(decode_attn_kernel<4>, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
+  else
+    launch_pdl(decode_attn_kernel<2>, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
 }
 
 // Greedy next token per sample (largest logit; equal logits: lower id) and
-// the cache length advanced by the fed token.
-__global__ void decode_finish_kernel(int B, int V, const float* logits, int* next_token, int* cache_len) {
-  __shared__ float bv[32];
-  __shared__ int bi[32];
+// the cache length advanced by the fed token. One 1024-thread block per
+// sample; with V a multiple of 4 each thread reads float4s (4 consecutive ids,
+// kept in id order, so the tie rule holds).
+constexpr int kFinThreads = 1024;
+
+SVL_DEVINL void arg_better(float x, int v, float& best, int& idx) {
+  if (x > best || (x == best && v < idx)) {
+    best = x;
+    idx = v;
+  }
+}
+
+__global__ void __launch_bounds__(kFinThreads) decode_finish_kernel(int B, int V, const float* logits, int* next_token,
+                                                                    int* cache_len) {
+  __shared__ float bv[kFinThreads / 32];
+  __shared__ int bi[kFinThreads / 32];
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const float* row = logits + static_cast<size_t>(b) * V;
   float best = -INFINITY;
   int idx = 0x7fffffff;
-  for (int v = tid; v < V; v += blockDim.x) {
-    const float x = logits[static_cast<size_t>(b) * V + v];
-    if (x > best || (x == best && v < idx)) {
-      best = x;
-      idx = v;
+  if ((V & 3) == 0) {
+    const float4* r4 = reinterpret_cast<const float4*>(row);
+    for (int c = tid; c < V / 4; c += kFinThreads) {
+      const float4 x = r4[c];
+      arg_better(x.x, 4 * c, best, idx);
+      arg_better(x.y, 4 * c + 1, best, idx);
+      arg_better(x.z, 4 * c + 2, best, idx);
+      arg_better(x.w, 4 * c + 3, best, idx);
     }
+  } else {
+    for (int v = tid; v < V; v += kFinThreads) arg_better(row[v], v, best, idx);
   }
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     const float ob = __shfl_xor_sync(0xffffffffu, best, off);
     const int oi = __shfl_xor_sync(0xffffffffu, idx, off);
-    if (ob > best || (ob == best && oi < idx)) {
-      best = ob;
-      idx = oi;
-    }
+    arg_better(ob, oi, best, idx);
   }
   if (lane == 0) {
     bv[warp] = best;
@@ -216,18 +266,14 @@ __global__ void decode_finish_kernel(int B, int V, const float* logits, int* nex
   }
   __syncthreads();
   if (tid == 0) {
-    for (int w = 1; w < static_cast<int>(blockDim.x >> 5); ++w)
-      if (bv[w] > best || (bv[w] == best && bi[w] < idx)) {
-        best = bv[w];
-        idx = bi[w];
-      }
+    for (int w = 1; w < kFinThreads / 32; ++w) arg_better(bv[w], bi[w], best, idx);
     if (next_token) next_token[b] = idx == 0x7fffffff ? 0 : idx;
     cache_len[b] += 1;
   }
 }
 
 void launch_decode_finish(int B, int V, const float* logits, int* next_token, int* cache_len, cudaStream_t s) {
-  launch_pdl(decode_finish_kernel, B, 256, 0, s, B, V, logits, next_token, cache_len);
+  launch_pdl(decode_finish_kernel, B, kFinThreads, 0, s, B, V, logits, next_token, cache_len);
 }
 
 }  // namespace svl

@@ -106,24 +106,38 @@ SVL_DEVINL void set_abort(volatile int* abort, uint32_t* status) {
 // Stage geometry per epilogue: the token-score GEMM streams the features
 // once and reads a B box of only H rows per stage (H <= 64: 24 KB stages,
 // nine deep; H <= 128: 32 KB, six deep), keeping more feature bytes in flight.
-template <int KIND>
+// THIN launches (at most kThinRows rows of A, e.g. one row per sample in
+// decode) are weight-streaming: their A box is kThinRows rows, so a stage is
+// 36 KB and six of them keep 192 KB of weights in flight per SM. The MMA
+// still reads 128 rows of A; rows past kThinRows come from the B tile that
+// follows in the stage and only reach accumulator rows that are never stored.
+template <int KIND, bool THIN = false>
 struct StageCfg {
   static constexpr int stages = kStages;
+  static constexpr int abytes = kABytes;
   static constexpr int bytes = kStageBytes;
 };
+template <int KIND>
+struct StageCfg<KIND, true> {
+  static constexpr int stages = 6;
+  static constexpr int abytes = kThinRows * 128;
+  static constexpr int bytes = abytes + 2 * kBHalfBytes;
+};
 template <>
-struct StageCfg<EPI_SCORE> {
+struct StageCfg<EPI_SCORE, false> {
   static constexpr int stages = 9;
+  static constexpr int abytes = kABytes;
   static constexpr int bytes = kABytes + kBHalfBytes / 2;
 };
 template <>
-struct StageCfg<EPI_SCORE_WIDE> {
+struct StageCfg<EPI_SCORE_WIDE, false> {
   static constexpr int stages = 6;
+  static constexpr int abytes = kABytes;
   static constexpr int bytes = kABytes + kBHalfBytes;
 };
 
 // ------------------------------------------------------------------ producer
-template <int NST, int SBYTES, bool F8>
+template <int NST, int SBYTES, int ABYTES, bool F8>
 SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* full,
                               uint64_t* empty, volatile int* abort) {
   constexpr int BK = F8 ? kBK8 : kBK;
@@ -138,7 +152,7 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
     const CUtensorMap* mb0 = p.b_split ? &p.mapB[0] : &p.mapB[ti.mat];
     const CUtensorMap* mb1 = p.b_split ? &p.mapB[1] : &p.mapB[ti.mat];
     const int y1 = p.b_split ? ti.n0 : ti.n0 + kBHalf;
-    const uint32_t bytes = kABytes + halves * (p.b_box_rows ? p.b_box_rows * 128 : kBHalfBytes);
+    const uint32_t bytes = ABYTES + halves * (p.b_box_rows ? p.b_box_rows * 128 : kBHalfBytes);
     KWalk w(nkb, kgb, ti.kmask);
     int i0, i1;
     k_share(ti, nkb, kgb, i0, i1);
@@ -151,7 +165,7 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
         return;
       }
       uint8_t* sa = stages + s * SBYTES;
-      uint8_t* sb = sa + kABytes;
+      uint8_t* sb = sa + ABYTES;
       mbar_arrive_expect_tx(&full[s], bytes);
       tma_load_2d(sa, &p.mapA, &full[s], kb * BK, ti.m0);
       tma_load_2d(sb, mb0, &full[s], kb * BK, ti.n0);
@@ -165,7 +179,7 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
 }
 
 // ------------------------------------------------------------------ MMA issuer
-template <int NST, int SBYTES, bool F8>
+template <int NST, int SBYTES, int ABYTES, bool F8>
 SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, uint64_t* empty,
                          uint64_t* tfull, uint64_t* tempty, uint32_t tmem, volatile int* abort) {
   constexpr int BK = F8 ? kBK8 : kBK;
@@ -196,7 +210,7 @@ SVL_DEVINL void mma_loop(const GemmParams& p, uint8_t* stages, uint64_t* full, u
       }
       tc_fence_after();
       const uint32_t a0 = smem_u32(stages + s * SBYTES);
-      const uint32_t b0 = a0 + kABytes;
+      const uint32_t b0 = a0 + ABYTES;
       // four instructions per stage, each over the next 32 bytes of K
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
@@ -512,17 +526,21 @@ SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, u
                             volatile int* abort) {
   const size_t unit = static_cast<size_t>(ti.slot) * ti.nsplit;
   float* mine = p.ks_part + ((unit + ti.part) * kBM + lrow) * kAccCols;
+  // rows past the tile's end are never reduced: no partial for them
+  const bool stored = ti.m0 + lrow < ti.m_end;
   float v[32];
   for (int c = 0; c < ti.ncols; c += 32) {
     if (!empty) {
-      tmem_ld32(taddr + c, v);
+      tmem_ld32(taddr + c, v);  // warp-collective: every lane loads
     } else {
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = 0.f;
     }
-    float4* d = reinterpret_cast<float4*>(mine + c);
+    if (stored) {
+      float4* d = reinterpret_cast<float4*>(mine + c);
 #pragma unroll
-    for (int i = 0; i < 8; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      for (int i = 0; i < 8; ++i) d[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
   }
   __threadfence();
   mbar_arrive(ks.gather);
@@ -547,19 +565,27 @@ SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, u
   ks.phase ^= 1;
   __syncwarp();
   if (!__all_sync(0xffffffffu, got) || !*ks.flag) return false;
-  // this share's rows [r0, r1) of the tile; one work item = (row, 128 columns)
-  const int r0 = (kBM * ti.part) / ti.nsplit, r1 = (kBM * (ti.part + 1)) / ti.nsplit;
+  // The tile's valid rows x 128-column slots form the groups of the
+  // reduction; the shares take every nsplit-th group, so the work is spread
+  // over all of them even when only a few rows are valid (one row per
+  // sample in decode). Four adjacent lanes take the four 32-column chunks of
+  // a group and combine their sums of squares for the norm slot.
+  const int nr = ti.m_end - ti.m0;
   const int nsl = (ti.ncols + 127) / 128;
-  const int items = (r1 - r0) * nsl;
+  const int ngroups = nr * nsl;
+  const int n_mine = ti.part < ngroups ? (ngroups - ti.part + ti.nsplit - 1) / ti.nsplit : 0;
   const int et = threadIdx.x - 2 * 32;  // 0..127
+  const int chunk = et & 3;
   const float* base = p.ks_part + unit * kBM * kAccCols;
-  for (int w = et; w < items; w += 4 * 32) {
-    const int lr = r0 + w / nsl, sl = w % nsl;
+  for (int k0 = 0; k0 < n_mine; k0 += 32) {  // uniform over the CTA
+    const int i = k0 + (et >> 2);
+    const bool act = i < n_mine;
+    const int g = ti.part + i * ti.nsplit;
+    const int lr = act ? g / nsl : 0, sl = act ? g - lr * nsl : 0;
     const int row = ti.m0 + lr;
-    if (row >= ti.m_end) continue;
-    __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out[0]) + static_cast<size_t>(row) * p.ld[0] + ti.n0;
+    const int c = sl * 128 + chunk * 32;
     float hss = 0.f;
-    for (int c = sl * 128; c < min(ti.ncols, sl * 128 + 128); c += 32) {
+    if (act && c < ti.ncols) {
       const int n = min(32, ti.ncols - c);
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = 0.f;
@@ -567,34 +593,40 @@ SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, u
         const float4* src = reinterpret_cast<const float4*>(base + (static_cast<size_t>(q) * kBM + lr) * kAccCols + c);
         float4 f[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) f[i] = __ldcg(src + i);
+        for (int i4 = 0; i4 < 8; ++i4) f[i4] = __ldcg(src + i4);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          v[4 * i] += f[i].x;
-          v[4 * i + 1] += f[i].y;
-          v[4 * i + 2] += f[i].z;
-          v[4 * i + 3] += f[i].w;
+        for (int i4 = 0; i4 < 8; ++i4) {
+          v[4 * i4] += f[i4].x;
+          v[4 * i4 + 1] += f[i4].y;
+          v[4 * i4 + 2] += f[i4].z;
+          v[4 * i4 + 3] += f[i4].w;
         }
       }
       if constexpr (F8) scale_cols(v, p.b_scale[0] + ti.n0 + c, p.a_scale[row]);
+      __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out[0]) + static_cast<size_t>(row) * p.ld[0] + ti.n0;
       const uint4* xs = reinterpret_cast<const uint4*>(orow + c);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        if (i * 8 < n) {
-          const uint4 x = xs[i];
+      for (int i4 = 0; i4 < 4; ++i4) {
+        if (i4 * 8 < n) {
+          const uint4 x = xs[i4];
           const uint32_t wd[4] = {x.x, x.y, x.z, x.w};
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             const float2 f = unpack_bf16x2(wd[k]);
-            v[8 * i + 2 * k] += f.x;
-            v[8 * i + 2 * k + 1] += f.y;
+            v[8 * i4 + 2 * k] += f.x;
+            v[8 * i4 + 2 * k + 1] += f.y;
           }
         }
       }
-      if (p.ss_out) hss += store_bf16_ss(orow + c, v, n);
+      if (p.ss_out) hss = store_bf16_ss(orow + c, v, n);
       else store_bf16(orow + c, v, n);
     }
-    if (p.ss_out) p.ss_out[static_cast<size_t>((ti.n0 >> 7) + sl) * p.ss_ld + row] = hss;
+    if (p.ss_out) {
+      // the group's four chunks sit in four adjacent lanes: chunk order kept
+      hss += __shfl_xor_sync(0xffffffffu, hss, 1);
+      hss += __shfl_xor_sync(0xffffffffu, hss, 2);
+      if (act && chunk == 0) p.ss_out[static_cast<size_t>((ti.n0 >> 7) + sl) * p.ss_ld + row] = hss;
+    }
   }
   return true;
 }
@@ -653,9 +685,10 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
 }
 
 // ------------------------------------------------------------------ kernel
-template <int KIND, bool F8>
+template <int KIND, bool F8, bool THIN>
 __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_constant__ GemmParams p) {
-  constexpr int NST = StageCfg<KIND>::stages, SBYTES = StageCfg<KIND>::bytes;
+  constexpr int NST = StageCfg<KIND, THIN>::stages, SBYTES = StageCfg<KIND, THIN>::bytes;
+  constexpr int ABYTES = StageCfg<KIND, THIN>::abytes;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* stages = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(stages + NST * SBYTES);
@@ -699,9 +732,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   pdl_wait();
 
   if (warp == 0) {
-    if (lane == 0) producer_loop<NST, SBYTES, F8>(p, stages, full, empty, abort);
+    if (lane == 0) producer_loop<NST, SBYTES, ABYTES, F8>(p, stages, full, empty, abort);
   } else if (warp == 1) {
-    if (lane == 0) mma_loop<NST, SBYTES, F8>(p, stages, full, empty, tfull, tempty, tmem, abort);
+    if (lane == 0) mma_loop<NST, SBYTES, ABYTES, F8>(p, stages, full, empty, tfull, tempty, tmem, abort);
   } else {
     epilogue_loop<KIND, F8>(p, tfull, tempty, tmem, abort, ks);
   }
@@ -722,22 +755,37 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   }
 }
 
-template <int KIND, bool F8 = false>
+template <int KIND, bool F8 = false, bool THIN = false>
 static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t stream) {
-  constexpr int smem = StageCfg<KIND>::stages * StageCfg<KIND>::bytes + 1024 + 256;
+  constexpr int smem = StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256;
   static_assert(smem <= 232448, "shared memory per CTA");
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<KIND, F8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(gemm_kernel<KIND, F8, THIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  return launch_pdl(gemm_kernel<KIND, F8>, grid, kGemmThreads, smem, stream, p);
+  return launch_pdl(gemm_kernel<KIND, F8, THIN>, grid, kGemmThreads, smem, stream, p);
 }
 
-cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3) {
+cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3, bool thin) {
+  if (e4m3 && (!p.a_scale || !p.b_scale[0])) return cudaErrorInvalidValue;
+  if (thin) {
+    switch (kind) {
+      case EPI_QKV_ROPE:
+        return e4m3 ? launch_kind<EPI_QKV_ROPE, true, true>(p, grid, stream)
+                    : launch_kind<EPI_QKV_ROPE, false, true>(p, grid, stream);
+      case EPI_RESID:
+        return e4m3 ? launch_kind<EPI_RESID, true, true>(p, grid, stream)
+                    : launch_kind<EPI_RESID, false, true>(p, grid, stream);
+      case EPI_SWIGLU:
+        return e4m3 ? launch_kind<EPI_SWIGLU, true, true>(p, grid, stream)
+                    : launch_kind<EPI_SWIGLU, false, true>(p, grid, stream);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   if (e4m3) {
-    if (!p.a_scale || !p.b_scale[0]) return cudaErrorInvalidValue;
     switch (kind) {
       case EPI_QKV_ROPE: return launch_kind<EPI_QKV_ROPE, true>(p, grid, stream);
       case EPI_RESID: return launch_kind<EPI_RESID, true>(p, grid, stream);

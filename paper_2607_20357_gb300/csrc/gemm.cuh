@@ -16,6 +16,7 @@ constexpr int kBK = 64;            // K per stage: one 128-byte swizzle row (bf1
 constexpr int kBK8 = 128;          // the same 128 bytes of e4m3
 constexpr int kBHalf = 128;        // B rows per TMA box; a stage holds two
 constexpr int kStages = 4;
+constexpr int kThinRows = 32;      // A rows of a THIN launch (see launch_gemm)
 constexpr int kABytes = kBM * kBK * 2;
 constexpr int kBHalfBytes = kBHalf * kBK * 2;
 constexpr int kStageBytes = kABytes + 2 * kBHalfBytes;
@@ -99,6 +100,10 @@ struct GemmParams {
   uint32_t* status;
 };
 
-cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3 = false);
+// `thin`: every tile has at most kThinRows rows and mapA has boxes of
+// kThinRows rows (QKV, residual and SwiGLU epilogues): deeper weight
+// pipeline for decode-sized batches.
+cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3 = false,
+                        bool thin = false);
 
 }  // namespace svl

@@ -8,6 +8,8 @@
 //   rounded; 0 and 0 when amax = 0), code = e4m3(x * inv).
 //
 // The GEMM multiplies codes and scales its accumulator by both rows' scales.
+#include <algorithm>
+
 #include "kernels.cuh"
 
 namespace svl {
@@ -71,87 +73,96 @@ __global__ void __launch_bounds__(kQuantWarps * 32) quant_rows_kernel(QuantArgs 
   if (lane == 0) a.scale[r] = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
 }
 
-// One CTA of 128 threads per row: thread t holds the row's 16-byte chunks
-// t, t + 128, ... (NCH of them) in registers between the amax and the code
-// pass, so each bf16 value is read from memory once.
+// 128-thread CTAs walking the rows (row = blockIdx.x + i * gridDim.x, so a
+// grid sized for the SMs serves any row count without idle CTAs): thread t
+// holds the row's 16-byte chunks t, t + 128, ... (NCH of them) in registers
+// between the amax and the code pass, so each bf16 value is read once.
 constexpr int kQuantThreads = 128;
 
 template <int NCH>
 __global__ void __launch_bounds__(kQuantThreads) quant_row_cta_kernel(QuantArgs a) {
-  __shared__ float red[kQuantThreads / 32];
-  __shared__ int s_mask;
+  __shared__ float red[2][kQuantThreads / 32];
+  __shared__ int s_mask[2];
   pdl_trigger();
   pdl_wait();
-  const int64_t r = blockIdx.x;
   int64_t rows = a.rows;
   if (a.cu_seqlens) rows = min(rows, static_cast<int64_t>(a.cu_seqlens[a.B]));
-  if (r >= rows) return;  // uniform across the block
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) {
-    int mask = (1 << a.G) - 1;
-    if (a.group_gate && a.l >= a.P) {
-      const int b = find_sample(a.cu_seqlens, a.B, static_cast<int>(r));
-      const size_t bl = static_cast<size_t>(b) * a.L + a.l;
-      mask = 0;
-      if (a.layer_gate[bl])
-        for (int j = 0; j < a.G; ++j) mask |= a.group_gate[bl * a.G + j] ? (1 << j) : 0;
+  int par = 0;  // the shared slots alternate between consecutive rows
+  for (int64_t r = blockIdx.x; r < rows; r += gridDim.x, par ^= 1) {
+    if (tid == 0) {
+      int mask = (1 << a.G) - 1;
+      if (a.group_gate && a.l >= a.P) {
+        const int b = find_sample(a.cu_seqlens, a.B, static_cast<int>(r));
+        const size_t bl = static_cast<size_t>(b) * a.L + a.l;
+        mask = 0;
+        if (a.layer_gate[bl])
+          for (int j = 0; j < a.G; ++j) mask |= a.group_gate[bl * a.G + j] ? (1 << j) : 0;
+      }
+      s_mask[par] = mask;
     }
-    s_mask = mask;
-  }
-  __syncthreads();
-  const int mask = s_mask;
-  const int per_g = a.kgp / 8, src_per_g = a.kg / 8, nchunk = a.G * per_g;
-  const __nv_bfloat16* src = a.src + r * a.ld_src;
-  uint4 v[NCH];
-  float amax = 0.f;
+    __syncthreads();
+    const int mask = s_mask[par];
+    const int per_g = a.kgp / 8, src_per_g = a.kg / 8, nchunk = a.G * per_g;
+    const __nv_bfloat16* src = a.src + r * a.ld_src;
+    uint4 v[NCH];
+    float amax = 0.f;
 #pragma unroll
-  for (int i = 0; i < NCH; ++i) {
-    const int c = tid + i * kQuantThreads;
-    v[i] = make_uint4(0, 0, 0, 0);
-    if (c < nchunk) {
-      const int j = c / per_g, cc = c - j * per_g;
-      if (((mask >> j) & 1) && cc < src_per_g)
-        v[i] = *reinterpret_cast<const uint4*>(src + static_cast<size_t>(j) * a.kg + static_cast<size_t>(cc) * 8);
+    for (int i = 0; i < NCH; ++i) {
+      const int c = tid + i * kQuantThreads;
+      v[i] = make_uint4(0, 0, 0, 0);
+      if (c < nchunk) {
+        const int j = c / per_g, cc = c - j * per_g;
+        if (((mask >> j) & 1) && cc < src_per_g)
+          v[i] = *reinterpret_cast<const uint4*>(src + static_cast<size_t>(j) * a.kg + static_cast<size_t>(cc) * 8);
+      }
     }
-  }
 #pragma unroll
-  for (int i = 0; i < NCH; ++i) {
-    const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
+    for (int i = 0; i < NCH; ++i) {
+      const uint32_t w[4] = {v[i].x, v[i].y, v[i].z, v[i].w};
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float2 f = unpack_bf16x2(w[q]);
-      amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = unpack_bf16x2(w[q]);
+        amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
     }
-  }
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
-  if (lane == 0) red[warp] = amax;
-  __syncthreads();
-  amax = fmaxf(fmaxf(red[0], red[1]), fmaxf(red[2], red[3]));
-  const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
-  uint8_t* dst = a.dst + r * a.ld_dst;
+    for (int off = 16; off > 0; off >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+    if (lane == 0) red[par][warp] = amax;
+    __syncthreads();
+    amax = fmaxf(fmaxf(red[par][0], red[par][1]), fmaxf(red[par][2], red[par][3]));
+    const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
+    uint8_t* dst = a.dst + r * a.ld_dst;
 #pragma unroll
-  for (int i = 0; i < NCH; ++i) {
-    const int c = tid + i * kQuantThreads;
-    if (c < nchunk) {
-      const float2 f0 = unpack_bf16x2(v[i].x), f1 = unpack_bf16x2(v[i].y), f2 = unpack_bf16x2(v[i].z),
-                   f3 = unpack_bf16x2(v[i].w);
-      uint2 o;
-      o.x = static_cast<uint32_t>(e4m3x2(__fmul_rn(f0.x, inv), __fmul_rn(f0.y, inv))) |
-            (static_cast<uint32_t>(e4m3x2(__fmul_rn(f1.x, inv), __fmul_rn(f1.y, inv))) << 16);
-      o.y = static_cast<uint32_t>(e4m3x2(__fmul_rn(f2.x, inv), __fmul_rn(f2.y, inv))) |
-            (static_cast<uint32_t>(e4m3x2(__fmul_rn(f3.x, inv), __fmul_rn(f3.y, inv))) << 16);
-      // chunk c of the padded row sits at byte 8 c (groups are kgp apart)
-      *reinterpret_cast<uint2*>(dst + static_cast<size_t>(c) * 8) = o;
+    for (int i = 0; i < NCH; ++i) {
+      const int c = tid + i * kQuantThreads;
+      if (c < nchunk) {
+        const float2 f0 = unpack_bf16x2(v[i].x), f1 = unpack_bf16x2(v[i].y), f2 = unpack_bf16x2(v[i].z),
+                     f3 = unpack_bf16x2(v[i].w);
+        uint2 o;
+        o.x = static_cast<uint32_t>(e4m3x2(__fmul_rn(f0.x, inv), __fmul_rn(f0.y, inv))) |
+              (static_cast<uint32_t>(e4m3x2(__fmul_rn(f1.x, inv), __fmul_rn(f1.y, inv))) << 16);
+        o.y = static_cast<uint32_t>(e4m3x2(__fmul_rn(f2.x, inv), __fmul_rn(f2.y, inv))) |
+              (static_cast<uint32_t>(e4m3x2(__fmul_rn(f3.x, inv), __fmul_rn(f3.y, inv))) << 16);
+        // chunk c of the padded row sits at byte 8 c (groups are kgp apart)
+        *reinterpret_cast<uint2*>(dst + static_cast<size_t>(c) * 8) = o;
+      }
     }
+    if (tid == 0) a.scale[r] = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
   }
-  if (tid == 0) a.scale[r] = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
 }
 
 cudaError_t launch_quant_rows(const QuantArgs& a, cudaStream_t s) {
   if (a.rows <= 0) return cudaSuccess;
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 1;
+  }
   const int64_t chunks = static_cast<int64_t>(a.G) * (a.kgp / 8);
-  const dim3 grid(static_cast<unsigned>(a.rows));
+  const dim3 grid(static_cast<unsigned>(std::min<int64_t>(a.rows, static_cast<int64_t>(sms) * 8)));
   if (chunks <= 4 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<4>, grid, kQuantThreads, 0, s, a);
   if (chunks <= 8 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<8>, grid, kQuantThreads, 0, s, a);
   if (chunks <= 12 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<12>, grid, kQuantThreads, 0, s, a);
