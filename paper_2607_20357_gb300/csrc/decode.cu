@@ -87,104 +87,117 @@ void launch_decode_prep(int B, int D, int V, const int* tokens, const int* cache
 // One block per (sample, query head) of an active group: the new token's
 // query against the cached keys 0..len-1 and its own key (position len),
 // softmax in float32, output row of O. The block of the first query head of
-// each KV head also appends the new key and value to the cache. Each warp
-// takes runs of kDecRun consecutive positions (every kDecWarps-th run),
-// loading all their K and V rows before using any (lane i holds d_head / 32
-// consecutive dimensions, one 4- or 8-byte load per row), and folds the run
-// into its online softmax at once; the warps are merged at the end. Four
-// blocks fit per SM, so a batch of 16 samples x 32 heads runs in one wave.
+// each KV head also appends the new key and value to the cache. Each of the
+// 8 warps takes a contiguous run of positions, 32 at a time: lane j scores
+// key j on its own (its whole K row as 16-byte loads against q in shared
+// memory, no shuffles per key), the warp folds the 32 scores into its online
+// softmax, then every lane accumulates its d_head / 32 output dimensions over
+// the 32 V rows (independent loads). The warps are merged at the end.
 // Memory-bound on the cache (2 * (len + 1) * d_head * 2 bytes per head).
 constexpr int kDecWarps = 8;
-constexpr int kDecRun = 4;
 
-template <int PER>  // d_head / 32: 2 or 4
-SVL_DEVINL void load_row(const __nv_bfloat16* src, float* out) {
-  if constexpr (PER == 4) {
-    const uint2 u = *reinterpret_cast<const uint2*>(src);
-    const float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
-    out[0] = a.x; out[1] = a.y; out[2] = b.x; out[3] = b.y;
-  } else {
-    const float2 a = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(src));
-    out[0] = a.x; out[1] = a.y;
-  }
-}
-
-template <int PER>
+template <int DH>  // d_head: 64 or 128
 __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_attn_kernel(DecAttnArgs a) {
+  constexpr int PER = DH / 32;
+  __shared__ __align__(16) float sq[DH];  // q * scale
+  __shared__ __align__(16) float snv[DH];  // the new value row
   __shared__ float sm_m[kDecWarps], sm_l[kDecWarps];
-  __shared__ float sm_o[kDecWarps][128];
+  __shared__ float sm_o[kDecWarps][DH];
+  __shared__ float sp[kDecWarps][32];
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x, h = blockIdx.y;
   const int G = a.G, hpg = a.A / G, g = h / hpg;
   if (!(a.layer_gate[b * a.L + a.l] && a.group_gate[(static_cast<size_t>(b) * a.L + a.l) * G + g]) && a.l >= a.P)
     return;  // gated off: no keys, no values, no output
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int dh = a.dh, kvh = h / (a.A / a.Akv);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
+  const int kvh = h / (a.A / a.Akv);
   const int len = a.cache_len[b];
   if (len < 0 || len >= a.max_len) return;  // reported by decode_prep
-  const size_t cbase = static_cast<size_t>(b) * a.max_len * a.dkv + static_cast<size_t>(kvh) * dh + lane * PER;
-  float q[PER], kn[PER], vn[PER];
-#pragma unroll
-  for (int i = 0; i < PER; ++i) {
-    const int d = lane * PER + i;
-    q[i] = __bfloat162float(a.q[static_cast<size_t>(b) * a.ldq + h * dh + d]) * a.scale;
-    kn[i] = __bfloat162float(a.k[static_cast<size_t>(b) * a.dkv + kvh * dh + d]);
-    vn[i] = __bfloat162float(a.vt[static_cast<size_t>(kvh * dh + d) * a.t_pad + b]);
-  }
-  if (h % (a.A / a.Akv) == 0 && warp == 0) {
-#pragma unroll
-    for (int i = 0; i < PER; ++i) {
-      a.k_cache[cbase + static_cast<size_t>(len) * a.dkv + i] = __float2bfloat16_rn(kn[i]);
-      a.v_cache[cbase + static_cast<size_t>(len) * a.dkv + i] = __float2bfloat16_rn(vn[i]);
+  const __nv_bfloat16* knew = a.k + static_cast<size_t>(b) * a.dkv + kvh * DH;
+  if (tid < DH) {
+    sq[tid] = __bfloat162float(a.q[static_cast<size_t>(b) * a.ldq + h * DH + tid]) * a.scale;
+    const __nv_bfloat16 vnew = a.vt[static_cast<size_t>(kvh * DH + tid) * a.t_pad + b];
+    snv[tid] = __bfloat162float(vnew);
+    if (h % (a.A / a.Akv) == 0) {  // append the new key and value to the cache
+      const size_t at = (static_cast<size_t>(b) * a.max_len + len) * a.dkv + kvh * DH + tid;
+      a.k_cache[at] = knew[tid];
+      a.v_cache[at] = vnew;
     }
   }
+  __syncthreads();
+  const size_t cbase = static_cast<size_t>(b) * a.max_len * a.dkv + static_cast<size_t>(kvh) * DH;
+  const int n = len + 1, per_warp = (n + kDecWarps - 1) / kDecWarps;
+  const int p_begin = warp * per_warp, p_end = min(n, p_begin + per_warp);
   float m = -INFINITY, l = 0.f, o[PER];
 #pragma unroll
   for (int i = 0; i < PER; ++i) o[i] = 0.f;
-  for (int p0 = warp * kDecRun; p0 <= len; p0 += kDecWarps * kDecRun) {
-    float kk[kDecRun][PER], vv[kDecRun][PER], sc[kDecRun];
+  for (int p0 = p_begin; p0 < p_end; p0 += 32) {
+    const int p = p0 + lane;
+    float sc = -INFINITY;
+    if (p < p_end) {
+      const uint4* kr = reinterpret_cast<const uint4*>(p < len ? a.k_cache + cbase + static_cast<size_t>(p) * a.dkv
+                                                               : knew);
+      uint4 u[DH / 8];
 #pragma unroll
-    for (int u = 0; u < kDecRun; ++u) {
-      const int p = p0 + u;
-      if (p < len) {
-        load_row<PER>(a.k_cache + cbase + static_cast<size_t>(p) * a.dkv, kk[u]);
-        load_row<PER>(a.v_cache + cbase + static_cast<size_t>(p) * a.dkv, vv[u]);
-      } else {
+      for (int c = 0; c < DH / 8; ++c) u[c] = kr[c];
+      float acc = 0.f;
 #pragma unroll
-        for (int i = 0; i < PER; ++i) {
-          kk[u][i] = p == len ? kn[i] : 0.f;
-          vv[u][i] = p == len ? vn[i] : 0.f;
-        }
+      for (int c = 0; c < DH / 8; ++c) {
+        const float4 q0 = *reinterpret_cast<const float4*>(sq + 8 * c);
+        const float4 q1 = *reinterpret_cast<const float4*>(sq + 8 * c + 4);
+        const float2 k0 = unpack_bf16x2(u[c].x), k1 = unpack_bf16x2(u[c].y), k2 = unpack_bf16x2(u[c].z),
+                     k3 = unpack_bf16x2(u[c].w);
+        acc = fmaf(q0.x, k0.x, acc);
+        acc = fmaf(q0.y, k0.y, acc);
+        acc = fmaf(q0.z, k1.x, acc);
+        acc = fmaf(q0.w, k1.y, acc);
+        acc = fmaf(q1.x, k2.x, acc);
+        acc = fmaf(q1.y, k2.y, acc);
+        acc = fmaf(q1.z, k3.x, acc);
+        acc = fmaf(q1.w, k3.y, acc);
       }
+      sc = acc;
     }
+    float mx = sc;
 #pragma unroll
-    for (int u = 0; u < kDecRun; ++u) {
-      float d = 0.f;
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    const float mn = fmaxf(m, mx);
+    const float e = p < p_end ? __expf(sc - mn) : 0.f;
+    float es = e;
 #pragma unroll
-      for (int i = 0; i < PER; ++i) d = fmaf(q[i], kk[u][i], d);
-      sc[u] = d;
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1)
-#pragma unroll
-      for (int u = 0; u < kDecRun; ++u) sc[u] += __shfl_xor_sync(0xffffffffu, sc[u], off);
-    float mr = m;
-#pragma unroll
-    for (int u = 0; u < kDecRun; ++u)
-      if (p0 + u <= len) mr = fmaxf(mr, sc[u]);
-    const float corr = __expf(m - mr);
-    l *= corr;
+    for (int off = 16; off > 0; off >>= 1) es += __shfl_xor_sync(0xffffffffu, es, off);
+    const float corr = __expf(m - mn);  // 0 while m is -inf
+    l = l * corr + es;
 #pragma unroll
     for (int i = 0; i < PER; ++i) o[i] *= corr;
+    m = mn;
+    sp[warp][lane] = e;
+    __syncwarp();
+    const int nk = min(32, p_end - p0);
+#pragma unroll 8
+    for (int j = 0; j < nk; ++j) {
+      const int pj = p0 + j;
+      const float ej = sp[warp][j];
+      float vv[PER];
+      if (pj < len) {
+        const __nv_bfloat16* vr = a.v_cache + cbase + static_cast<size_t>(pj) * a.dkv + lane * PER;
+        if constexpr (PER == 4) {
+          const uint2 w = *reinterpret_cast<const uint2*>(vr);
+          const float2 v0 = unpack_bf16x2(w.x), v1 = unpack_bf16x2(w.y);
+          vv[0] = v0.x; vv[1] = v0.y; vv[2] = v1.x; vv[3] = v1.y;
+        } else {
+          const float2 v0 = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(vr));
+          vv[0] = v0.x; vv[1] = v0.y;
+        }
+      } else {
 #pragma unroll
-    for (int u = 0; u < kDecRun; ++u) {
-      const float e = p0 + u <= len ? __expf(sc[u] - mr) : 0.f;
-      l += e;
+        for (int i = 0; i < PER; ++i) vv[i] = snv[lane * PER + i];
+      }
 #pragma unroll
-      for (int i = 0; i < PER; ++i) o[i] = fmaf(e, vv[u][i], o[i]);
+      for (int i = 0; i < PER; ++i) o[i] = fmaf(ej, vv[i], o[i]);
     }
-    m = mr;
+    __syncwarp();
   }
   if (lane == 0) {
     sm_m[warp] = m;
@@ -208,15 +221,15 @@ __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_attn_kernel(DecAttnA
     const float inv = L > 0.f ? 1.f / L : 0.f;
 #pragma unroll
     for (int i = 0; i < PER; ++i)
-      a.out[static_cast<size_t>(b) * a.ldo + h * dh + lane * PER + i] = __float2bfloat16_rn(acc[i] * inv);
+      a.out[static_cast<size_t>(b) * a.ldo + h * DH + lane * PER + i] = __float2bfloat16_rn(acc[i] * inv);
   }
 }
 
 void launch_decode_attn(const DecAttnArgs& a, cudaStream_t s) {
   if (a.dh == 128)
-    launch_pdl(decode_attn_kernel<4>, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
+    launch_pdl(decode_attn_kernel<128>, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
   else
-    launch_pdl(decode_attn_kernel<2>, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
+    launch_pdl(decode_attn_kernel<64>, dim3(a.B, a.A), kDecWarps * 32, 0, s, a);
 }
 
 // Greedy next token per sample (largest logit; equal logits: lower id) and
