@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--no-hbm-sweep", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-fp8", action="store_true", help="skip the e4m3 (FP8 gated projections) pass")
+    ap.add_argument("--decode-only", action="store_true",
+                    help="profiling aid: only the decode measurement (bf16, and e4m3 unless --no-fp8)")
     ap.add_argument("--hbm-only", type=str, default="",
                     help="comma-separated batch multipliers: run only the token-controller/pack sweep "
                          "(for small profiler captures)")
@@ -275,6 +277,16 @@ def run_ours(args, rank, world, local_rank):
         return
     seed = SEED + 17 * rank
     batches = [synth.make_batch(wl, seed, budget=b, device=dev) for b in wl.budgets]
+    if args.decode_only:
+        out = {"decode": run_decode(svl, model, batches[1], dims, dev, pk)}
+        model.close()
+        if not args.no_fp8:
+            m8 = svl.GatedPrefill(dims, weights, max_seq=max_seq, gemm_format=svl.SVL_GEMM_E4M3)
+            out["fp8_decode"] = run_decode(svl, m8, batches[1], dims, dev, pk, layer_weight_bytes=1)
+            m8.close()
+        if rank == 0:
+            print(json.dumps(out), flush=True)
+        return
     outs = [model.alloc_outputs(bt) for bt in batches]
     stream = torch.cuda.current_stream()
 
