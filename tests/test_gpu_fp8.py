@@ -209,3 +209,20 @@ def test_fp8_decode_matches_extended_prefill():
         compared += 1
     assert compared >= 1
     case.close()
+
+
+def test_fp8_prefill_qwen_gqa_two_layers():
+    """Qwen2-VL-7B widths with e4m3 projections: GQA 28/4 (one KV head per
+    group), d 3584, FFN 18,944 (4,736 channels per group, no padding), no
+    projector, 2 layers, one group gated off in one sample's second layer."""
+    wl = synth.WORKLOADS["qwen"]
+    dims = synth.reduced(wl.dims, n_layers=2)
+    case = Case(dims, wl, seed=7, batch=2, gemm_format=E4M3)
+    b = synth.make_batch(wl, 7, n_vis_list=[256, 300], s_text_list=[128, 128], keep_list=[-1, -1],
+                         budget_list=[0.6, 0.9], dims=dims)
+    b["group_gate"][1, 1, 2] = 0
+    case.b_np = O.to_numpy_batch(b)
+    case.b = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in b.items()}
+    out = case.run()
+    _compare(case, out, 2, 1)
+    case.close()
