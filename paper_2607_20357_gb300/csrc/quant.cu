@@ -162,8 +162,14 @@ cudaError_t launch_quant_rows(const QuantArgs& a, cudaStream_t s) {
     if (sms <= 0) sms = 1;
   }
   const int64_t chunks = static_cast<int64_t>(a.G) * (a.kgp / 8);
-  const dim3 grid(static_cast<unsigned>(std::min<int64_t>(a.rows, static_cast<int64_t>(sms) * 8)));
-  if (chunks <= 4 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<4>, grid, kQuantThreads, 0, s, a);
+  // enough CTAs to fill every SM (16 resident for the 4-chunk rows, fewer
+  // for the wider ones, which are limited by registers)
+  auto grid_for = [&](int per_sm) {
+    return dim3(static_cast<unsigned>(std::min<int64_t>(a.rows, static_cast<int64_t>(sms) * per_sm)));
+  };
+  const dim3 grid = grid_for(8);
+  if (chunks <= 4 * kQuantThreads)
+    return launch_pdl(quant_row_cta_kernel<4>, grid_for(16), kQuantThreads, 0, s, a);
   if (chunks <= 8 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<8>, grid, kQuantThreads, 0, s, a);
   if (chunks <= 12 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<12>, grid, kQuantThreads, 0, s, a);
   if (chunks <= 16 * kQuantThreads) return launch_pdl(quant_row_cta_kernel<16>, grid, kQuantThreads, 0, s, a);
