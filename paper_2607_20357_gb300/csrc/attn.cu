@@ -463,6 +463,385 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
   }
 }
 
+// ------------------------------------------------------------------------
+// Pipelined variant: two independent query-block pipelines ("slots") per
+// CTA. A unit of work is one block of up to 128 queries of one (sample,
+// active head); every item of the device schedule gives two units (its two
+// 128-query halves), and slot s of CTA c takes units 2c + s, 2c + s + 2G, ...
+// of the list [all first halves][all second halves], so neither slot waits
+// for the other's chain. Keys come in tiles of 64. Per slot:
+//   S = Q K^T   into one of two S buffers in TMEM (64 columns each), so S of
+//               tile j+1 is computed while the softmax works on tile j;
+//   P           bf16 into the slot's shared-memory P buffer;
+//   O += P V    in TMEM (d_head columns), rescaled lazily as in the kernel
+//               above; K and V^T tiles through the slot's own 4-stage ring
+//               (K of tile j+1 can load while tiles j-1 and j are in use).
+// A full block's output goes through the P buffer and TMA tensor stores (one
+// 64-column atom at a time); a partial block's rows are stored by their
+// threads.
+// Warps: 0 / 6 TMA producers of slot 0 / 1; 1 / 7 MMA issuers (warp 1 also
+// owns the TMEM allocation); 2-5 / 8-11 softmax and output of slot 0 / 1.
+constexpr int kPipeThreads = 384;
+constexpr int kPipeKeys = 64;
+constexpr int kPipeRing = 4;
+
+template <int DH>
+struct PipeSmem {
+  static constexpr int kQAtom = 128 * 128;            // 128 rows x 128 B
+  static constexpr int kQ = 128 * DH * 2;             // DH/64 atoms
+  static constexpr int kKAtom = kPipeKeys * 128;      // 64 keys x 128 B
+  static constexpr int kKV = kPipeKeys * DH * 2;      // K tile (DH/64 atoms) or V^T tile (DH rows x 128 B)
+  static constexpr int kP = 128 * kPipeKeys * 2;      // 128 rows x 64 keys
+  static constexpr int q0 = 0;
+  static constexpr int p0 = q0 + kQ;
+  static constexpr int r0 = p0 + kP;
+  static constexpr int slot = r0 + kPipeRing * kKV;   // bytes per slot (multiple of 1024)
+  static constexpr int bars = 2 * slot;
+  static constexpr int total = bars + 512 + 1024;
+};
+static_assert(PipeSmem<128>::total <= 232448, "pipelined attention shared memory");
+
+struct PipeBars {
+  uint64_t q_full, q_empty, r_full[kPipeRing], r_empty[kPipeRing], s_full[2], p_full[2], pv_done[2];
+  uint64_t epi;  // the slot's 128 softmax threads meeting around the output stores
+};
+
+// Unit u of the list [first halves][second halves] of n_items items.
+SVL_DEVINL bool pipe_unit(const AttnTcArgs& a, int n_items, int u, int4& it, int& qb0, int& qend, int& ntiles) {
+  const int item = u < n_items ? u : u - n_items;
+  const int half = u < n_items ? 0 : 1;
+  it = a.items[item];
+  qb0 = it.x + 128 * half;
+  qend = min(qb0 + 128, it.y);
+  if (qend <= qb0) return false;
+  const int key_base = it.z & ~7;
+  ntiles = (qend - key_base + kPipeKeys - 1) / kPipeKeys;
+  return true;
+}
+
+template <int DH>
+__global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid_constant__ AttnTcArgs a) {
+  using L = PipeSmem<DH>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  PipeBars* bars = reinterpret_cast<PipeBars*>(sm + L::bars);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int sl = 0; sl < 2; ++sl) {
+      PipeBars* b = bars + sl;
+      mbar_init(&b->q_full, 1);
+      mbar_init(&b->q_empty, 1);
+      for (int i = 0; i < kPipeRing; ++i) {
+        mbar_init(&b->r_full[i], 1);
+        mbar_init(&b->r_empty[i], 1);
+      }
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(&b->s_full[i], 1);
+        mbar_init(&b->p_full[i], 128);
+        mbar_init(&b->pv_done[i], 1);
+      }
+      mbar_init(&b->epi, 128);
+    }
+    *abort = 0;
+    fence_barrier_init();
+    fence_proxy_async();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
+  const int n_items = min(*a.count, a.cap);
+  const int n_units = 2 * n_items;
+  const int group = a.A / a.Akv;
+  const int slot = warp < 6 ? 0 : 1;
+  const int role = warp < 6 ? warp : warp - 6;  // 0 producer, 1 MMA, 2-5 softmax
+  PipeBars* bar = bars + slot;
+  uint8_t* ss = sm + slot * L::slot;
+  const uint32_t tbase = tmem + 256 * slot;      // S0, S1 at +0, +64; O at +128
+  const int worker = 2 * blockIdx.x + slot, stride = 2 * gridDim.x;
+
+  if (role == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int g = 0, nq = 0;
+      bool ok = true;
+      for (int u = worker; u < n_units && ok; u += stride) {
+        int4 it;
+        int qb0, qend, n;
+        if (!pipe_unit(a, n_items, u, it, qb0, qend, n)) continue;
+        const int kvh = it.w / group, key_base = it.z & ~7;
+        if (!mbar_wait(&bar->q_empty, (nq & 1) ^ 1, abort)) { ok = false; break; }
+        ++nq;
+        mbar_arrive_expect_tx(&bar->q_full, L::kQ);
+        for (int at = 0; at < DH / 64; ++at)
+          tma_load_2d(ss + L::q0 + at * L::kQAtom, &a.mapQ, &bar->q_full, it.w * DH + at * 64, qb0);
+        for (int p = 0; p < 2 * n && ok; ++p, ++g) {
+          const bool is_k = p == 0 || (p & 1 && p < 2 * n - 1);
+          const int tile = is_k ? (p + 1) >> 1 : (p == 2 * n - 1 ? n - 1 : (p >> 1) - 1);
+          const int st = g % kPipeRing;
+          if (!mbar_wait(&bar->r_empty[st], ((g / kPipeRing) & 1) ^ 1, abort)) { ok = false; break; }
+          mbar_arrive_expect_tx(&bar->r_full[st], L::kKV);
+          uint8_t* dst = ss + L::r0 + st * L::kKV;
+          const int key0 = key_base + tile * kPipeKeys;
+          if (is_k) {
+            for (int at = 0; at < DH / 64; ++at)
+              tma_load_2d(dst + at * L::kKAtom, &a.mapK64, &bar->r_full[st], kvh * DH + at * 64, key0);
+          } else {
+            tma_load_2d(dst, &a.mapVt, &bar->r_full[st], key0, kvh * DH);
+          }
+        }
+      }
+      if (!ok) attn_abort(abort, a.status);
+    }
+  } else if (role == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      const uint32_t id_s = idesc_bf16_f32(128, kPipeKeys), id_o = idesc_bf16_f32(128, DH);
+      int g = 0, nq = 0, t = 0;  // ring position, units, tiles so far
+      bool ok = true;
+      auto ring_wait = [&](int pos) -> bool {
+        if (!mbar_wait(&bar->r_full[pos % kPipeRing], (pos / kPipeRing) & 1, abort)) return false;
+        tc_fence_after();
+        return true;
+      };
+      auto mma_s = [&](int b, int pos) {
+        const uint64_t dq = smem_desc_sw128(smem_u32(ss + L::q0));
+        const uint64_t dk = smem_desc_sw128(smem_u32(ss + L::r0 + (pos % kPipeRing) * L::kKV));
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const uint32_t offq = ((kk >> 2) * L::kQAtom + (kk & 3) * 32) >> 4;
+          const uint32_t offk = ((kk >> 2) * L::kKAtom + (kk & 3) * 32) >> 4;
+          tc_mma_bf16(tbase + 64 * b, dq + offq, dk + offk, id_s, kk > 0);
+        }
+        tc_commit(&bar->s_full[b]);
+      };
+      auto mma_pv = [&](int b, int pos, bool acc) {
+        const uint64_t dp = smem_desc_sw128(smem_u32(ss + L::p0));
+        const uint64_t dv = smem_desc_sw128(smem_u32(ss + L::r0 + (pos % kPipeRing) * L::kKV));
+#pragma unroll
+        for (int kk = 0; kk < kPipeKeys / 16; ++kk)
+          tc_mma_bf16(tbase + 128, dp + ((kk * 32) >> 4), dv + ((kk * 32) >> 4), id_o, (acc || kk > 0) ? 1u : 0u);
+        tc_commit(&bar->pv_done[b]);
+      };
+      for (int u = worker; u < n_units && ok; u += stride) {
+        int4 it;
+        int qb0, qend, n;
+        if (!pipe_unit(a, n_items, u, it, qb0, qend, n)) continue;
+        ok = mbar_wait(&bar->q_full, nq & 1, abort);
+        ++nq;
+        if (!ok) break;
+        tc_fence_after();
+        // S of tile 0
+        ok = ring_wait(g + pos_k(0));
+        if (!ok) break;
+        mma_s(t & 1, g + pos_k(0));
+        if (n == 1) tc_commit(&bar->q_empty);
+        tc_commit(&bar->r_empty[(g + pos_k(0)) % kPipeRing]);
+        for (int j = 0; j < n && ok; ++j) {
+          if (j + 1 < n) {
+            // its S buffer was last read by the softmax of tile t+j-1,
+            // whose P V was issued (after p_full) in the previous round
+            const int gk = g + pos_k(j + 1);
+            ok = ring_wait(gk);
+            if (!ok) break;
+            mma_s((t + j + 1) & 1, gk);
+            if (j + 1 == n - 1) tc_commit(&bar->q_empty);
+            tc_commit(&bar->r_empty[gk % kPipeRing]);
+          }
+          const int tj = t + j;
+          ok = mbar_wait(&bar->p_full[tj & 1], (tj >> 1) & 1, abort);
+          if (!ok) break;
+          tc_fence_after();
+          const int gv = g + pos_v(j, n);
+          ok = ring_wait(gv);
+          if (!ok) break;
+          mma_pv(tj & 1, gv, j > 0);
+          tc_commit(&bar->r_empty[gv % kPipeRing]);
+        }
+        t += n;
+        g += 2 * n;
+      }
+      if (!ok) attn_abort(abort, a.status);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax + output
+    const int q = warp & 3;         // TMEM lane quarter this warp may access
+    const int row = q * 32 + lane;  // query row within the block = TMEM lane
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const uint32_t t_o = tbase + 128 + lane_off;
+    const float sc = a.scale_log2;
+    const uint64_t sc2 = f2(sc, sc);
+    int t = 0;
+    uint32_t epi_phase = 0;
+    bool ok = true;
+    auto wait_all = [&](uint64_t* b, uint32_t parity) -> bool {
+      const bool got = mbar_wait(b, parity, abort);
+      __syncwarp();
+      return __all_sync(0xffffffffu, got);
+    };
+    // bounded meeting of the slot's softmax threads
+    auto slot_sync = [&]() -> bool {
+      mbar_arrive(&bar->epi);
+      const bool got = wait_all(&bar->epi, epi_phase & 1);
+      ++epi_phase;
+      return got;
+    };
+    for (int u = worker; u < n_units && ok; u += stride) {
+      int4 it;
+      int qb0, qend, n;
+      if (!pipe_unit(a, n_items, u, it, qb0, qend, n)) continue;
+      const int qg = qb0 + row;
+      const int key_base = it.z & ~7;
+      float m_run = -INFINITY, l_run = 0.f;
+      for (int j = 0; j < n; ++j, ++t) {
+        const int b = t & 1;
+        if (!wait_all(&bar->s_full[b], (t >> 1) & 1)) { ok = false; break; }
+        tc_fence_after();
+        const int kbase = key_base + j * kPipeKeys;
+        const bool full = kbase >= it.z && kbase + kPipeKeys - 1 <= qb0;
+        const int lo = full ? 0 : max(it.z - kbase, 0);
+        const int hi = full ? kPipeKeys : max(min(min(qg + 1, qend) - kbase, kPipeKeys), lo);
+        const unsigned span = static_cast<unsigned>(hi - lo);
+        uint32_t sv[64];
+        tmem_ld32_async(tbase + 64 * b + lane_off, sv);
+        tmem_ld32_async(tbase + 64 * b + 32 + lane_off, sv + 32);
+        tmem_ld_wait32(sv);
+        tmem_ld_wait32(sv + 32);
+        const float m_tile = row_max64(sv, 0, full, lo, span, -INFINITY) * sc;
+        if (j == 0) {
+          m_run = m_tile;
+        } else {
+          const bool need = m_tile > m_run + kRescaleLog2;
+          if (__any_sync(0xffffffffu, need)) {
+            // O must hold P V of every earlier tile before it is rescaled
+            if (!wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
+            tc_fence_after();
+            const float corr = need ? ex2(m_run - m_tile) : 1.f;
+            if (need) {
+              l_run *= corr;
+              m_run = m_tile;
+            }
+#pragma unroll 1
+            for (int cc = 0; cc < DH; cc += 32) {
+              uint32_t ov[32];
+              tmem_ld32_async(t_o + cc, ov);
+              tmem_ld_wait32(ov);
+#pragma unroll
+              for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
+              tmem_st32(t_o + cc, ov);
+            }
+            tmem_st_wait();
+          }
+        }
+        // the P buffer was read by P V of tile t-1
+        if (t >= 1 && !wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
+        const float mref = (m_run == -INFINITY) ? 0.f : m_run;
+        const uint64_t nm2 = f2(-mref, -mref);
+        l_run += exp_store64(sv, 0, full, lo, span, sc2, nm2, ss + L::p0 + row * 128, row);
+        fence_proxy_async();  // P written by threads, read by the tensor core
+        tc_fence_before();
+        mbar_arrive(&bar->p_full[b]);
+      }
+      if (!ok) break;
+      // block done: O of the last P V, divided by the row sum
+      if (!wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
+      tc_fence_after();
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+      if (qend - qb0 == 128) {
+        // full block: 64 columns at a time into the P buffer (swizzled like a
+        // TMA box), then one TMA store per atom, issued by row 0's thread
+        uint8_t* prow = ss + L::p0 + row * 128;
+#pragma unroll 1
+        for (int h = 0; h < DH / 64; ++h) {
+          if (h > 0) {
+            if (row == 0) bulk_wait_read0();  // the previous atom has left shared memory
+            if (!(ok = slot_sync())) break;
+          }
+#pragma unroll 1
+          for (int c2 = 0; c2 < 2; ++c2) {
+            uint32_t ov[32];
+            tmem_ld32_async(t_o + 64 * h + 32 * c2, ov);
+            tmem_ld_wait32(ov);
+#pragma unroll
+            for (int d = 0; d < 32; d += 8) {
+              const int chunk = (32 * c2 + d) / 8;  // 16-byte chunk of the 128-byte row
+              *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) = make_uint4(
+                  pack_bf16x2(__uint_as_float(ov[d]) * inv, __uint_as_float(ov[d + 1]) * inv),
+                  pack_bf16x2(__uint_as_float(ov[d + 2]) * inv, __uint_as_float(ov[d + 3]) * inv),
+                  pack_bf16x2(__uint_as_float(ov[d + 4]) * inv, __uint_as_float(ov[d + 5]) * inv),
+                  pack_bf16x2(__uint_as_float(ov[d + 6]) * inv, __uint_as_float(ov[d + 7]) * inv));
+            }
+          }
+          fence_proxy_async();  // generic-proxy writes, read by the TMA unit
+          if (!(ok = slot_sync())) break;
+          if (row == 0) {
+            tma_store_2d(&a.mapO, ss + L::p0, it.w * DH + 64 * h, qb0);
+            bulk_commit();
+          }
+        }
+        // the next unit writes P only after the last atom has been read
+        if (row == 0) bulk_wait_read0();
+        if (ok) ok = slot_sync();
+        if (!ok) break;
+      } else {
+        uint4* dst = reinterpret_cast<uint4*>(a.O + static_cast<size_t>(qg) * a.ldo + static_cast<size_t>(it.w) * DH);
+#pragma unroll 1
+        for (int cc = 0; cc < DH; cc += 32) {
+          uint32_t ov[32];
+          tmem_ld32_async(t_o + cc, ov);
+          tmem_ld_wait32(ov);
+          if (qg < qend) {
+#pragma unroll
+            for (int d = 0; d < 32; d += 8)
+              dst[(cc + d) / 8] = make_uint4(
+                  pack_bf16x2(__uint_as_float(ov[d]) * inv, __uint_as_float(ov[d + 1]) * inv),
+                  pack_bf16x2(__uint_as_float(ov[d + 2]) * inv, __uint_as_float(ov[d + 3]) * inv),
+                  pack_bf16x2(__uint_as_float(ov[d + 4]) * inv, __uint_as_float(ov[d + 5]) * inv),
+                  pack_bf16x2(__uint_as_float(ov[d + 6]) * inv, __uint_as_float(ov[d + 7]) * inv));
+          }
+        }
+      }
+      tc_fence_before();  // O read before the next unit's first P V overwrites it
+    }
+    if (row == 0) bulk_wait0();  // this thread's output stores are complete
+    if (!ok) attn_abort(abort, a.status);
+  }
+
+  __syncwarp();
+  if (*abort) {
+    long long t0 = clock64();
+    while (clock64() - t0 < 20000000LL) {
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+template <int DH>
+static cudaError_t launch_pipe(const AttnTcArgs& a, int grid, cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(attn_pipe_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         PipeSmem<DH>::total);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  return launch_pdl(attn_pipe_kernel<DH>, grid, kPipeThreads, PipeSmem<DH>::total, s, a);
+}
+
 template <int DH>
 static cudaError_t launch_dh(const AttnTcArgs& a, int grid, cudaStream_t s) {
   static bool configured = false;
@@ -477,6 +856,7 @@ static cudaError_t launch_dh(const AttnTcArgs& a, int grid, cudaStream_t s) {
 
 cudaError_t launch_attention_tc(const AttnTcArgs& a, int grid, cudaStream_t s) {
   if (a.cap <= 0) return cudaSuccess;
+  if (a.pipe) return a.dh == 128 ? launch_pipe<128>(a, grid, s) : launch_pipe<64>(a, grid, s);
   return a.dh == 128 ? launch_dh<128>(a, grid, s) : launch_dh<64>(a, grid, s);
 }
 
