@@ -476,9 +476,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_c
 //   O += P V    in TMEM (d_head columns), rescaled lazily as in the kernel
 //               above; K and V^T tiles through the slot's own 4-stage ring
 //               (K of tile j+1 can load while tiles j-1 and j are in use).
-// A full block's output goes through the P buffer and TMA tensor stores (one
-// 64-column atom at a time); a partial block's rows are stored by their
-// threads.
+// Each softmax warp writes its own 32 output rows: through its part of the P
+// buffer and a TMA tensor store per 64 columns when all 32 rows exist, with
+// per-thread stores otherwise; no meeting of the four warps is needed.
 // Warps: 0 / 6 TMA producers of slot 0 / 1; 1 / 7 MMA issuers (warp 1 also
 // owns the TMEM allocation); 2-5 / 8-11 softmax and output of slot 0 / 1.
 constexpr int kPipeThreads = 384;
@@ -503,7 +503,6 @@ static_assert(PipeSmem<128>::total <= 232448, "pipelined attention shared memory
 
 struct PipeBars {
   uint64_t q_full, q_empty, r_full[kPipeRing], r_empty[kPipeRing], s_full[2], p_full[2], pv_done[2];
-  uint64_t epi;  // the slot's 128 softmax threads meeting around the output stores
 };
 
 // Unit u of the list [first halves][second halves] of n_items items.
@@ -543,7 +542,6 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid
         mbar_init(&b->p_full[i], 128);
         mbar_init(&b->pv_done[i], 1);
       }
-      mbar_init(&b->epi, 128);
     }
     *abort = 0;
     fence_barrier_init();
@@ -681,19 +679,11 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid
     const float sc = a.scale_log2;
     const uint64_t sc2 = f2(sc, sc);
     int t = 0;
-    uint32_t epi_phase = 0;
     bool ok = true;
     auto wait_all = [&](uint64_t* b, uint32_t parity) -> bool {
       const bool got = mbar_wait(b, parity, abort);
       __syncwarp();
       return __all_sync(0xffffffffu, got);
-    };
-    // bounded meeting of the slot's softmax threads
-    auto slot_sync = [&]() -> bool {
-      mbar_arrive(&bar->epi);
-      const bool got = wait_all(&bar->epi, epi_phase & 1);
-      ++epi_phase;
-      return got;
     };
     for (int u = worker; u < n_units && ok; u += stride) {
       int4 it;
@@ -746,6 +736,10 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid
         if (t >= 1 && !wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
         const float mref = (m_run == -INFINITY) ? 0.f : m_run;
         const uint64_t nm2 = f2(-mref, -mref);
+        // this warp's rows of the P buffer may still be the source of its
+        // last output store
+        if (lane == 0) bulk_wait_read0();
+        __syncwarp();
         l_run += exp_store64(sv, 0, full, lo, span, sc2, nm2, ss + L::p0 + row * 128, row);
         fence_proxy_async();  // P written by threads, read by the tensor core
         tc_fence_before();
@@ -756,15 +750,16 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid
       if (!wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      if (qend - qb0 == 128) {
-        // full block: 64 columns at a time into the P buffer (swizzled like a
-        // TMA box), then one TMA store per atom, issued by row 0's thread
+      const int wrow0 = q * 32;  // this warp's first row in the block
+      if (qb0 + wrow0 + 32 <= qend) {
+        // all 32 rows exist: 64 columns at a time into this warp's rows of the
+        // P buffer (swizzled like a TMA box), one TMA store each by lane 0
         uint8_t* prow = ss + L::p0 + row * 128;
 #pragma unroll 1
         for (int h = 0; h < DH / 64; ++h) {
           if (h > 0) {
-            if (row == 0) bulk_wait_read0();  // the previous atom has left shared memory
-            if (!(ok = slot_sync())) break;
+            if (lane == 0) bulk_wait_read0();  // the previous 64 columns have left shared memory
+            __syncwarp();
           }
 #pragma unroll 1
           for (int c2 = 0; c2 < 2; ++c2) {
@@ -782,16 +777,12 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid
             }
           }
           fence_proxy_async();  // generic-proxy writes, read by the TMA unit
-          if (!(ok = slot_sync())) break;
-          if (row == 0) {
-            tma_store_2d(&a.mapO, ss + L::p0, it.w * DH + 64 * h, qb0);
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_2d(&a.mapO, ss + L::p0 + wrow0 * 128, it.w * DH + 64 * h, qb0 + wrow0);
             bulk_commit();
           }
         }
-        // the next unit writes P only after the last atom has been read
-        if (row == 0) bulk_wait_read0();
-        if (ok) ok = slot_sync();
-        if (!ok) break;
       } else {
         uint4* dst = reinterpret_cast<uint4*>(a.O + static_cast<size_t>(qg) * a.ldo + static_cast<size_t>(it.w) * DH);
 #pragma unroll 1
@@ -812,7 +803,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid
       }
       tc_fence_before();  // O read before the next unit's first P V overwrites it
     }
-    if (row == 0) bulk_wait0();  // this thread's output stores are complete
+    if (lane == 0) bulk_wait0();  // this warp's output stores are complete
     if (!ok) attn_abort(abort, a.status);
   }
 
