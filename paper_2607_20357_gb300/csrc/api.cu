@@ -925,11 +925,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     return SVL_ERR_CUDA;
   AttnTcArgs aa;
   std::memset(&aa, 0, sizeof(aa));
-  if (!make_map(&aa.mapQ, qb, t_cap, hq) || !make_map(&aa.mapK, kb, t_cap, dkv) ||
-      !make_map(&aa.mapVt, vb, dkv, L.t_pad, static_cast<uint32_t>(dh)) || !make_map(&aa.mapK64, kb, t_cap, dkv, 64) ||
-      !make_map(&aa.mapO, ao, t_cap, hq, 32))
+  if (!make_map(&aa.mapQ, qb, t_cap, hq) || !make_map(&aa.mapVt, vb, dkv, L.t_pad, static_cast<uint32_t>(dh)) ||
+      !make_map(&aa.mapK64, kb, t_cap, dkv, 64) || !make_map(&aa.mapO, ao, t_cap, hq, 32))
     return SVL_ERR_CUDA;
-  aa.pipe = 1;
   aa.cap = L.attn_cap;
   aa.A = d.n_heads;
   aa.Akv = d.n_kv_heads;

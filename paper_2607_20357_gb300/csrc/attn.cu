@@ -1,64 +1,46 @@
 // Variable-length causal attention over active heads only (Sec. 3.2: the
 // heads of a gated-off group are never computed), on tcgen05 tensor cores.
 //
-// Persistent kernel, one CTA per SM. A work item from the device schedule is
-// (sample, active head, up to 256 consecutive queries); its first 128 queries
-// are block A, the rest block B. Each block owns a Q buffer, an S and an O
-// accumulator in TMEM, a P buffer in shared memory and four softmax warps.
-// Both blocks walk the same key tiles, so every K and V^T tile is loaded once
-// for 256 queries. Per tile of 128 keys and block:
-//   S = Q K^T      tcgen05.mma M=128 N=128 K=d_head into the block's S columns
+// Persistent kernel, one CTA per SM, two independent query-block pipelines
+// ("slots") per CTA. A unit of work is one block of up to 128 queries of one
+// (sample, active head); every item of the device schedule (up to 256
+// queries) gives two units, its two 128-query halves, and slot s of CTA c
+// takes units 2c + s, 2c + s + 2G, ... of the list [all first halves][all
+// second halves], so neither slot ever waits for the other's chain. Keys come
+// in tiles of 64. Per slot and tile:
+//   S = Q K^T      tcgen05.mma M=128 N=64 K=d_head into one of two S buffers
+//                  in TMEM, so S of tile j+1 is computed while the softmax
+//                  works on tile j;
 //   softmax        one query row per thread: row max, P = exp2(S*scale - m)
-//                  rounded to bf16 and written to shared memory in the
-//                  128-byte-swizzled K-major layout, row sum
-//   O += P V       tcgen05.mma M=128 N=d_head K=128 into the block's O columns
+//                  rounded to bf16 and written to the slot's shared-memory P
+//                  buffer in the 128-byte-swizzled K-major layout, row sum;
+//   O += P V       tcgen05.mma M=128 N=d_head K=64 into the slot's O columns.
 // The running max m is only moved when a tile's max exceeds it by more than
 // 2^8 (then O and the row sum are rescaled in place); otherwise P is formed
 // against the stale max, its entries stay below 256 and O needs no per-tile
-// correction. O / rowsum is written out once per item.
+// correction. O / rowsum is written out once per unit.
 //
-// The MMA thread works in rounds: in round j, for each block whose softmax of
-// tile j-1 is done, it issues S of tile j and P V of tile j-1, so one block's
-// softmax overlaps the other block's products. V arrives transposed (V^T,
-// keys contiguous) so that both operands are K-major; K and V^T tiles share a
-// ring of shared-memory stages that the producer fills in the order the MMA
-// thread consumes them. Key tiles start at the sample's first row rounded down
-// to a multiple of 8 (TMA needs a 16-byte aligned innermost coordinate); keys
-// of the neighbouring sample that this pulls in are masked, like every key
-// after the query (causal) or past the sample's end.
+// V arrives transposed (V^T, keys contiguous) so that both operands are
+// K-major. K and V^T tiles go through the slot's own 4-stage ring, which the
+// producer fills in the order the MMA thread consumes them (K of tile j+1
+// can load while tiles j-1 and j are in use). Key tiles start at the sample's
+// first row rounded down to a multiple of 8 (TMA needs a 16-byte aligned
+// innermost coordinate); keys of the neighbouring sample that this pulls in
+// are masked, like every key after the query (causal) or past the sample's
+// end. Each softmax warp writes its own 32 output rows: through its part of
+// the P buffer and a TMA tensor store per 64 columns when all 32 rows exist,
+// with per-thread stores otherwise.
 //
-// Warp 0: TMA producer. Warp 1: TMEM allocation and the MMA-issuing thread.
-// Warps 2-5: block A softmax and output; warps 6-9: block B.
-// Every barrier completes at most once ahead of its waiter; every wait is
-// bounded.
+// Warps: 0 / 6 TMA producers of slot 0 / 1; 1 / 7 MMA issuers (warp 1 also
+// owns the TMEM allocation: slot s uses columns 256 s .. 256 s + 255 for S0,
+// S1 and O); 2-5 / 8-11 softmax and output of slot 0 / 1. Every barrier
+// completes at most once ahead of its waiter; every wait is bounded.
 #include "kernels.cuh"
 
 namespace svl {
 
-constexpr int kAttnThreads = 320;
-constexpr int kKeyTile = 128;
-constexpr int kRing = 3;
 constexpr float kRescaleLog2 = 8.f;  // move the running max when it grows by more than 2^8
 static_assert(kAttnQ == 256, "an attention item is two blocks of 128 queries");
-
-template <int DH>
-struct AttnSmem {
-  static constexpr int kAtom = 128 * 128;     // 128 rows x 128 B
-  static constexpr int kQ = 128 * DH * 2;     // Q tile: DH/64 atoms
-  static constexpr int kStage = 128 * DH * 2; // K tile (DH/64 atoms of 128 keys) or V^T tile (2 x DH rows x 128 B)
-  static constexpr int kVAtom = DH * 128;     // V^T: DH rows x 64 keys
-  static constexpr int kP = 128 * kKeyTile * 2;
-  static constexpr int q0 = 0;
-  static constexpr int p0 = q0 + 2 * kQ;
-  static constexpr int r0 = p0 + 2 * kP;
-  static constexpr int bars = r0 + kRing * kStage;
-  static constexpr int total = bars + 256 + 1024;  // + barriers + alignment slack
-};
-static_assert(AttnSmem<128>::total <= 232448, "attention shared memory");
-
-struct AttnBars {
-  uint64_t q_full[2], q_empty[2], r_full[kRing], r_empty[kRing], s_full[2], p_full[2], pv_done[2];
-};
 
 SVL_DEVINL void attn_abort(volatile int* abort, uint32_t* status) {
   *abort = 1;
@@ -93,22 +75,6 @@ SVL_DEVINL uint64_t add2(uint64_t a, uint64_t b) {
 }
 SVL_DEVINL float lo2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v)); }
 SVL_DEVINL float hi2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
-
-// Tile counts of an item {q0, q_end, r0, head}: block A is queries
-// [q0, min(q0 + 128, q_end)), block B the rest (possibly empty). Key tiles
-// start at r0 rounded down to 8; a block needs the tiles up to its last query.
-struct ItemTiles {
-  int na, nb, n;
-};
-SVL_DEVINL ItemTiles item_tiles(const int4& it) {
-  const int key_base = it.z & ~7;
-  const int a_end = min(it.x + 128, it.y);
-  ItemTiles t;
-  t.na = (a_end - key_base + kKeyTile - 1) / kKeyTile;
-  t.nb = it.y > a_end ? (it.y - key_base + kKeyTile - 1) / kKeyTile : 0;
-  t.n = max(t.na, t.nb);
-  return t;
-}
 
 // Ring positions of an item's 2n tiles relative to its first: K(0), then per
 // round j = 1..n: K(j) (while j < n) and V(j-1).
@@ -163,324 +129,6 @@ SVL_DEVINL float exp_store64(const uint32_t* sv, int base, bool full, int lo, un
   return lo2(acc) + hi2(acc);
 }
 
-// TMEM columns: block x holds S at 256*x and O at 256*x + 128.
-template <int DH>
-__global__ void __launch_bounds__(kAttnThreads, 1) attn_tc_kernel(const __grid_constant__ AttnTcArgs a) {
-  using L = AttnSmem<DH>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  AttnBars* bar = reinterpret_cast<AttnBars*>(sm + L::bars);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 1);
-  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&bar->q_full[i], 1);
-      mbar_init(&bar->q_empty[i], 1);
-      mbar_init(&bar->s_full[i], 1);
-      mbar_init(&bar->p_full[i], 128);
-      mbar_init(&bar->pv_done[i], 1);
-    }
-    for (int i = 0; i < kRing; ++i) {
-      mbar_init(&bar->r_full[i], 1);
-      mbar_init(&bar->r_empty[i], 1);
-    }
-    *abort = 0;
-    fence_barrier_init();
-    fence_proxy_async();
-  }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
-  }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  pdl_trigger();
-  pdl_wait();
-  const int n_items = min(*a.count, a.cap);
-  const int group = a.A / a.Akv;
-
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      int base = 0, nq[2] = {0, 0};
-      bool ok = true;
-      int4 it = blockIdx.x < n_items ? a.items[blockIdx.x] : make_int4(0, 0, 0, 0);
-      auto load_q = [&](int x, const int4& cur) -> bool {
-        if (!mbar_wait(&bar->q_empty[x], (nq[x] & 1) ^ 1, abort)) return false;
-        ++nq[x];
-        mbar_arrive_expect_tx(&bar->q_full[x], L::kQ);
-        for (int at = 0; at < DH / 64; ++at)
-          tma_load_2d(sm + L::q0 + x * L::kQ + at * L::kAtom, &a.mapQ, &bar->q_full[x], cur.w * DH + at * 64,
-                      cur.x + 128 * x);
-        return true;
-      };
-      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
-        const int4 cur = it;
-        if (i + gridDim.x < n_items) it = a.items[i + gridDim.x];  // next item, loaded early
-        const ItemTiles nt = item_tiles(cur);
-        const int kvh = cur.w / group, key_base = cur.z & ~7;
-        ok = load_q(0, cur);
-        // block B's Q after the first two key tiles: its buffer frees only
-        // when the previous item's last S of block B is done
-        const int p_qb = min(1, 2 * nt.n - 1);
-        for (int p = 0; p < 2 * nt.n && ok; ++p) {
-          // position p of this item: K(j) or V(m), see pos_k / pos_v
-          const bool is_k = p == 0 || (p & 1 && p < 2 * nt.n - 1);
-          const int tile = is_k ? (p + 1) >> 1 : (p == 2 * nt.n - 1 ? nt.n - 1 : (p >> 1) - 1);
-          const int g = base + p, st = g % kRing;
-          if (!mbar_wait(&bar->r_empty[st], ((g / kRing) & 1) ^ 1, abort)) { ok = false; break; }
-          mbar_arrive_expect_tx(&bar->r_full[st], L::kStage);
-          uint8_t* dst = sm + L::r0 + st * L::kStage;
-          const int key0 = key_base + tile * kKeyTile;
-          if (is_k) {
-            for (int at = 0; at < DH / 64; ++at)
-              tma_load_2d(dst + at * L::kAtom, &a.mapK, &bar->r_full[st], kvh * DH + at * 64, key0);
-          } else {
-            for (int h2 = 0; h2 < 2; ++h2)
-              tma_load_2d(dst + h2 * L::kVAtom, &a.mapVt, &bar->r_full[st], key0 + 64 * h2, kvh * DH);
-          }
-          if (p == p_qb && nt.nb > 0) ok = load_q(1, cur);
-        }
-        base += 2 * nt.n;
-      }
-      if (!ok) attn_abort(abort, a.status);
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t id_s = idesc_bf16_f32(128, kKeyTile), id_o = idesc_bf16_f32(128, DH);
-      int base = 0, nq[2] = {0, 0}, np[2] = {0, 0};
-      bool ok = true;
-      auto ring_wait = [&](int g) -> bool {
-        if (!mbar_wait(&bar->r_full[g % kRing], (g / kRing) & 1, abort)) return false;
-        tc_fence_after();
-        return true;
-      };
-      auto mma_s = [&](int x, int g) {
-        // descriptors advance by (byte offset >> 4) in their start-address field
-        const uint64_t dq = smem_desc_sw128(smem_u32(sm + L::q0 + x * L::kQ));
-        const uint64_t dk = smem_desc_sw128(smem_u32(sm + L::r0 + (g % kRing) * L::kStage));
-#pragma unroll
-        for (int kk = 0; kk < DH / 16; ++kk) {
-          const uint32_t off = ((kk >> 2) * L::kAtom + (kk & 3) * 32) >> 4;
-          tc_mma_bf16(tmem + 256 * x, dq + off, dk + off, id_s, kk > 0);
-        }
-        tc_commit(&bar->s_full[x]);
-      };
-      auto mma_pv = [&](int x, int g, bool acc) {
-        const uint64_t dp = smem_desc_sw128(smem_u32(sm + L::p0 + x * L::kP));
-        const uint64_t dv = smem_desc_sw128(smem_u32(sm + L::r0 + (g % kRing) * L::kStage));
-#pragma unroll
-        for (int kk = 0; kk < kKeyTile / 16; ++kk) {
-          const uint32_t offp = ((kk >> 2) * L::kAtom + (kk & 3) * 32) >> 4;
-          const uint32_t offv = ((kk >> 2) * L::kVAtom + (kk & 3) * 32) >> 4;
-          tc_mma_bf16(tmem + 256 * x + 128, dp + offp, dv + offv, id_o, (acc || kk > 0) ? 1u : 0u);
-        }
-        tc_commit(&bar->pv_done[x]);
-      };
-      int4 it = blockIdx.x < n_items ? a.items[blockIdx.x] : make_int4(0, 0, 0, 0);
-      for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
-        const ItemTiles nt = item_tiles(it);
-        if (i + gridDim.x < n_items) it = a.items[i + gridDim.x];  // next item, loaded early
-        const int ntx[2] = {nt.na, nt.nb};
-        // round 0: S of tile 0 for both blocks
-        ok = ring_wait(base + pos_k(0));
-#pragma unroll
-        for (int x = 0; x < 2; ++x) {
-          if (ok && ntx[x] > 0) {
-            ok = mbar_wait(&bar->q_full[x], nq[x] & 1, abort);
-            if (ok) {
-              tc_fence_after();
-              mma_s(x, base + pos_k(0));
-              if (ntx[x] == 1) tc_commit(&bar->q_empty[x]);
-              ++nq[x];
-            }
-          }
-        }
-        if (!ok) break;
-        tc_commit(&bar->r_empty[(base + pos_k(0)) % kRing]);
-        // rounds 1..n: S of tile j and P V of tile j-1
-        for (int j = 1; j <= nt.n && ok; ++j) {
-          const int gk = base + pos_k(j), gv = base + pos_v(j - 1, nt.n);
-          bool k_ready = false, v_ready = false;
-#pragma unroll
-          for (int x = 0; x < 2; ++x) {
-            if (ok && j - 1 < ntx[x]) {
-              ok = mbar_wait(&bar->p_full[x], np[x] & 1, abort);
-              ++np[x];
-              if (ok) tc_fence_after();
-              if (ok && j < ntx[x]) {
-                if (!k_ready) ok = k_ready = ring_wait(gk);
-                if (ok) {
-                  mma_s(x, gk);
-                  if (j == ntx[x] - 1) tc_commit(&bar->q_empty[x]);
-                }
-              }
-              if (ok && !v_ready) ok = v_ready = ring_wait(gv);
-              if (ok) mma_pv(x, gv, j > 1);
-            }
-          }
-          if (!ok) break;
-          if (j < nt.n) tc_commit(&bar->r_empty[gk % kRing]);
-          tc_commit(&bar->r_empty[gv % kRing]);
-        }
-        base += 2 * nt.n;
-      }
-      if (!ok) attn_abort(abort, a.status);
-    }
-  } else {
-    // ------------------------------------------------------------ softmax + output
-    const int x = (warp - 2) >> 2;  // block: 0 = A, 1 = B
-    const int q = warp & 3;         // TMEM lane quarter this warp may access
-    const int row = q * 32 + lane;  // query row within the block = TMEM lane
-    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
-    const uint32_t t_s = tmem + 256 * x + lane_off, t_o = tmem + 256 * x + 128 + lane_off;
-    uint8_t* prow = sm + L::p0 + x * L::kP + row * 128;
-    const float sc = a.scale_log2;
-    const uint64_t sc2 = f2(sc, sc);
-    int t = 0;  // tiles of this block so far (barrier phases)
-    bool ok = true;
-    auto wait_all = [&](uint64_t* b, uint32_t parity) -> bool {
-      const bool got = mbar_wait(b, parity, abort);
-      __syncwarp();
-      return __all_sync(0xffffffffu, got);
-    };
-    for (int i = blockIdx.x; i < n_items && ok; i += gridDim.x) {
-      const int4 cur = a.items[i];
-      const ItemTiles ntt = item_tiles(cur);
-      const int nt = x == 0 ? ntt.na : ntt.nb;
-      if (nt == 0) continue;
-      const int qb0 = cur.x + 128 * x;  // first query of this block
-      const int qg = qb0 + row;         // global query row
-      const int key_base = cur.z & ~7;
-      float m_run = -INFINITY, l_run = 0.f;
-      for (int j = 0; j < nt; ++j, ++t) {
-        if (!wait_all(&bar->s_full[x], t & 1)) { ok = false; break; }
-        tc_fence_after();
-        // keys kbase + [lo, hi) are valid for this row; a tile wholly inside
-        // the sample and before the block's first query needs no mask
-        const int kbase = key_base + j * kKeyTile;
-        const bool full = kbase >= cur.z && kbase + kKeyTile - 1 <= qb0;
-        const int lo = full ? 0 : max(cur.z - kbase, 0);
-        // (a row that precedes the whole tile has no valid key: empty range)
-        const int hi = full ? kKeyTile : max(min(min(qg + 1, cur.y) - kbase, kKeyTile), lo);
-        const unsigned span = static_cast<unsigned>(hi - lo);
-        // row max over both halves of the tile; the second half stays in
-        // registers, the first is read again for the exponentials
-        uint32_t sv[64];
-        tmem_ld32_async(t_s, sv);
-        tmem_ld32_async(t_s + 32, sv + 32);
-        tmem_ld_wait32(sv);
-        tmem_ld_wait32(sv + 32);
-        float mx = row_max64(sv, 0, full, lo, span, -INFINITY);
-        tmem_ld32_async(t_s + 64, sv);
-        tmem_ld32_async(t_s + 96, sv + 32);
-        tmem_ld_wait32(sv);
-        tmem_ld_wait32(sv + 32);
-        mx = row_max64(sv, 64, full, lo, span, mx);
-        const float m_tile = mx * sc;
-        if (j == 0) {
-          m_run = m_tile;
-        } else {
-          // P V of the previous tile must be done: it reads the P buffer and
-          // accumulates into O
-          if (!wait_all(&bar->pv_done[x], (t - 1) & 1)) { ok = false; break; }
-          tc_fence_after();
-          const bool need = m_tile > m_run + kRescaleLog2;
-          if (__any_sync(0xffffffffu, need)) {
-            const float corr = need ? ex2(m_run - m_tile) : 1.f;
-            if (need) {
-              l_run *= corr;
-              m_run = m_tile;
-            }
-#pragma unroll 1
-            for (int cc = 0; cc < DH; cc += 32) {
-              uint32_t ov[32];
-              tmem_ld32_async(t_o + cc, ov);
-              tmem_ld_wait32(ov);
-#pragma unroll
-              for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * corr);
-              tmem_st32(t_o + cc, ov);
-            }
-            tmem_st_wait();
-          }
-        }
-        const float mref = (m_run == -INFINITY) ? 0.f : m_run;
-        const uint64_t nm2 = f2(-mref, -mref);
-        float rs = exp_store64(sv, 64, full, lo, span, sc2, nm2, prow + L::kAtom, row);
-        tmem_ld32_async(t_s, sv);
-        tmem_ld32_async(t_s + 32, sv + 32);
-        tmem_ld_wait32(sv);
-        tmem_ld_wait32(sv + 32);
-        rs += exp_store64(sv, 0, full, lo, span, sc2, nm2, prow, row);
-        l_run += rs;
-        fence_proxy_async();  // P written by threads, read by the tensor core
-        tc_fence_before();
-        mbar_arrive(&bar->p_full[x]);
-      }
-      if (!ok) break;
-      // block done: O of the last P V, divided by the row sum
-      if (!wait_all(&bar->pv_done[x], (t - 1) & 1)) { ok = false; break; }
-      tc_fence_after();
-      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      uint4* dst = reinterpret_cast<uint4*>(a.O + static_cast<size_t>(qg) * a.ldo + static_cast<size_t>(cur.w) * DH);
-#pragma unroll 1
-      for (int cc = 0; cc < DH; cc += 32) {
-        uint32_t ov[32];
-        tmem_ld32_async(t_o + cc, ov);
-        tmem_ld_wait32(ov);
-        if (qg < cur.y) {
-#pragma unroll
-          for (int d = 0; d < 32; d += 8)
-            dst[(cc + d) / 8] = make_uint4(
-                pack_bf16x2(__uint_as_float(ov[d]) * inv, __uint_as_float(ov[d + 1]) * inv),
-                pack_bf16x2(__uint_as_float(ov[d + 2]) * inv, __uint_as_float(ov[d + 3]) * inv),
-                pack_bf16x2(__uint_as_float(ov[d + 4]) * inv, __uint_as_float(ov[d + 5]) * inv),
-                pack_bf16x2(__uint_as_float(ov[d + 6]) * inv, __uint_as_float(ov[d + 7]) * inv));
-        }
-      }
-      tc_fence_before();  // O read before the next item's first P V overwrites it
-    }
-    if (!ok) attn_abort(abort, a.status);
-  }
-
-  __syncwarp();
-  if (*abort) {
-    long long t0 = clock64();
-    while (clock64() - t0 < 20000000LL) {
-    }
-  }
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, 512);
-  }
-}
-
-// ------------------------------------------------------------------------
-// Pipelined variant: two independent query-block pipelines ("slots") per
-// CTA. A unit of work is one block of up to 128 queries of one (sample,
-// active head); every item of the device schedule gives two units (its two
-// 128-query halves), and slot s of CTA c takes units 2c + s, 2c + s + 2G, ...
-// of the list [all first halves][all second halves], so neither slot waits
-// for the other's chain. Keys come in tiles of 64. Per slot:
-//   S = Q K^T   into one of two S buffers in TMEM (64 columns each), so S of
-//               tile j+1 is computed while the softmax works on tile j;
-//   P           bf16 into the slot's shared-memory P buffer;
-//   O += P V    in TMEM (d_head columns), rescaled lazily as in the kernel
-//               above; K and V^T tiles through the slot's own 4-stage ring
-//               (K of tile j+1 can load while tiles j-1 and j are in use).
-// Each softmax warp writes its own 32 output rows: through its part of the P
-// buffer and a TMA tensor store per 64 columns when all 32 rows exist, with
-// per-thread stores otherwise; no meeting of the four warps is needed.
-// Warps: 0 / 6 TMA producers of slot 0 / 1; 1 / 7 MMA issuers (warp 1 also
-// owns the TMEM allocation); 2-5 / 8-11 softmax and output of slot 0 / 1.
 constexpr int kPipeThreads = 384;
 constexpr int kPipeKeys = 64;
 constexpr int kPipeRing = 4;
@@ -519,7 +167,7 @@ SVL_DEVINL bool pipe_unit(const AttnTcArgs& a, int n_items, int u, int4& it, int
 }
 
 template <int DH>
-__global__ void __launch_bounds__(kPipeThreads, 1) attn_pipe_kernel(const __grid_constant__ AttnTcArgs a) {
+__global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_constant__ AttnTcArgs a) {
   using L = PipeSmem<DH>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -825,30 +473,17 @@ template <int DH>
 static cudaError_t launch_pipe(const AttnTcArgs& a, int grid, cudaStream_t s) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_pipe_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          PipeSmem<DH>::total);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  return launch_pdl(attn_pipe_kernel<DH>, grid, kPipeThreads, PipeSmem<DH>::total, s, a);
-}
-
-template <int DH>
-static cudaError_t launch_dh(const AttnTcArgs& a, int grid, cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         AttnSmem<DH>::total);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
-  return launch_pdl(attn_tc_kernel<DH>, grid, kAttnThreads, AttnSmem<DH>::total, s, a);
+  return launch_pdl(attn_tc_kernel<DH>, grid, kPipeThreads, PipeSmem<DH>::total, s, a);
 }
 
 cudaError_t launch_attention_tc(const AttnTcArgs& a, int grid, cudaStream_t s) {
   if (a.cap <= 0) return cudaSuccess;
-  if (a.pipe) return a.dh == 128 ? launch_pipe<128>(a, grid, s) : launch_pipe<64>(a, grid, s);
-  return a.dh == 128 ? launch_dh<128>(a, grid, s) : launch_dh<64>(a, grid, s);
+  return a.dh == 128 ? launch_pipe<128>(a, grid, s) : launch_pipe<64>(a, grid, s);
 }
 
 }  // namespace svl

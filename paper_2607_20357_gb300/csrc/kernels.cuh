@@ -203,11 +203,9 @@ void launch_final_last_rows(const NormArgs& a, int n_pad, cudaStream_t s);
 
 struct AttnTcArgs {
   CUtensorMap mapQ;         // Q   [T_cap, A*dh]      boxes 64 x 128
-  CUtensorMap mapK;         // K   [T_cap, A_kv*dh]   boxes 64 x 128
   CUtensorMap mapVt;        // V^T [A_kv*dh, T_pad]   boxes 64 x dh
-  CUtensorMap mapK64;       // K   [T_cap, A_kv*dh]   boxes 64 x 64 (pipelined kernel)
-  CUtensorMap mapO;         // O   [T_cap, A*dh]      boxes 64 x 32 (pipelined kernel's output stores)
-  int pipe;                 // 1: the pipelined kernel (two independent query-block slots per CTA)
+  CUtensorMap mapK64;       // K   [T_cap, A_kv*dh]   boxes 64 x 64
+  CUtensorMap mapO;         // O   [T_cap, A*dh]      boxes 64 x 32 (output stores)
   const int4* items;        // {q0, q_end, r0, head}
   const int* count;
   int cap;
