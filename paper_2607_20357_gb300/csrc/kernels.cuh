@@ -6,7 +6,7 @@
 namespace svl {
 
 constexpr int kSelectThreads = 512;
-constexpr int kAttnQ = 256;       // query rows per attention work item: two 128-row blocks sharing K/V
+constexpr int kAttnQ = 256;       // query rows per attention work item (the kernel runs its two 128-row halves as units)
 constexpr int kNBand = 8;         // n-tiles per raster band in the tile lists
 constexpr int kBM_SCHED = 128;    // tile rows (the GEMM's M)
 

@@ -76,3 +76,24 @@ def test_binding_argument_counts_match_header(svl_lib):
     for name in svl.SYMBOLS:
         fn = getattr(svl_lib, name)
         assert len(fn.argtypes) == counts[name], (name, len(fn.argtypes), counts[name])
+
+
+def test_e4m3_entry_points_reject_bad_args_without_gpu(svl_lib):
+    """Host-side checks return SVL_ERR_INVALID_ARG (1) before anything is
+    launched: the pointers below are never dereferenced."""
+    buf = ctypes.create_string_buffer(4096 + 16)
+    base = (ctypes.addressof(buf) + 15) & ~15
+    src, dst, sc = ctypes.c_void_p(base), ctypes.c_void_p(base + 1024), ctypes.c_void_p(base + 2048)
+    q = svl_lib.svl_quantize_rows_e4m3
+    assert q(None, 4, 16, 16, dst, 16, sc, None) == 1        # null source
+    assert q(src, 4, 12, 16, dst, 16, sc, None) == 1         # cols not a multiple of 8
+    assert q(src, 4, 16, 12, dst, 16, sc, None) == 1         # ld_src < cols
+    assert q(src, 4, 16, 16, dst, 8, sc, None) == 1          # ld_dst < cols
+    assert q(src, -1, 16, 16, dst, 16, sc, None) == 1        # negative rows
+    assert q(ctypes.c_void_p(base + 2), 4, 16, 16, dst, 16, sc, None) == 1  # misaligned source
+    g = svl_lib.svl_gemm_e4m3
+    assert g(None, src, sc, dst, sc, 128, 32, 128, sc, None) == 1  # no model
+    d = svl.model_desc(synth.WORKLOADS["tiny"].dims, 256, gemm_format=7)  # unknown operand format
+    w = svl.Weights()
+    h = ctypes.c_void_p()
+    assert svl_lib.svl_model_create(ctypes.byref(d), ctypes.byref(w), ctypes.byref(h)) == 1
