@@ -41,6 +41,26 @@ WORKLOAD = "llava"
 SEED = 1000
 
 
+def rank_seed(rank: int) -> int:
+    """Each rank runs its own batch (replicas over independent samples)."""
+    return SEED + 17 * rank
+
+
+def job_aggregate(max_part, sum_part, device="cpu"):
+    """Whole-job figures over the ranks of the default process group: the
+    maximum of each entry of `max_part` (times) and the sum of each entry of
+    `sum_part` (tokens, FLOPs). Without a group of more than one rank the
+    values come back as given. This is the only collective of the bench."""
+    dist = torch.distributed
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return [float(v) for v in max_part], [float(v) for v in sum_part]
+    mx = torch.tensor([float(v) for v in max_part], dtype=torch.float64, device=device)
+    sm = torch.tensor([float(v) for v in sum_part], dtype=torch.float64, device=device)
+    dist.all_reduce(mx, op=dist.ReduceOp.MAX)
+    dist.all_reduce(sm, op=dist.ReduceOp.SUM)
+    return mx.tolist(), sm.tolist()
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -275,7 +295,7 @@ def run_ours(args, rank, world, local_rank):
         print(json.dumps({"hbm_kernels_sweep": run_hbm_sweep(svl, model, wl, dev, pk, mults=mults)}), flush=True)
         model.close()
         return
-    seed = SEED + 17 * rank
+    seed = rank_seed(rank)
     batches = [synth.make_batch(wl, seed, budget=b, device=dev) for b in wl.budgets]
     if args.decode_only:
         out = {"decode": run_decode(svl, model, batches[1], dims, dev, pk)}
@@ -397,12 +417,7 @@ def run_ours(args, rank, world, local_rank):
             kernels[t]["tflops"] = kind_flops[t] / (kernels[t]["total_ms"] / 1000.0) / 1e12
 
     # whole-job aggregate over ranks: max time, summed tokens
-    if world > 1:
-        tt = torch.tensor([total_ms, float(tokens_total), fexec_total], dtype=torch.float64, device=dev)
-        mx = tt.clone()
-        torch.distributed.all_reduce(mx[:1], op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.all_reduce(tt[1:], op=torch.distributed.ReduceOp.SUM)
-        total_ms, tokens_total, fexec_total = float(mx[0]), float(tt[1]), float(tt[2])
+    (total_ms,), (tokens_total, fexec_total) = job_aggregate([total_ms], [tokens_total, fexec_total], dev)
     value = tokens_total / (total_ms / 1000.0)
 
     hbm = None
@@ -676,11 +691,7 @@ def run_e2e(args, svl, model, batches, dims, world, dev):
     h2d = sum(int(h0[k].numel() * h0[k].element_size()) for k in
               ("vis", "vis_off", "text_ids", "text_off", "budget", "keep_count", "layer_gate", "group_gate"))
     d2h = int(h0["logits"].numel() * 4 + h0["k"].numel() * 4)
-    if world > 1:
-        t = torch.tensor([ms, float(tokens)], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t[:1], op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.all_reduce(t[1:], op=torch.distributed.ReduceOp.SUM)
-        ms, tokens = float(t[0]), float(t[1])
+    (ms,), (tokens,) = job_aggregate([ms], [tokens], dev)
     return {"value": tokens / (ms / 1000.0), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "entry_point": "svl_prefill_from_host (pinned host buffers)"}
 
