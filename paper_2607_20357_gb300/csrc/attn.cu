@@ -76,8 +76,9 @@ SVL_DEVINL uint64_t add2(uint64_t a, uint64_t b) {
 SVL_DEVINL float lo2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v)); }
 SVL_DEVINL float hi2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
 
-// Ring positions of an item's 2n tiles relative to its first: K(0), then per
-// round j = 1..n: K(j) (while j < n) and V(j-1).
+// Ring positions of a unit's 2n tiles relative to its first, in the order the
+// MMA thread consumes them: K(0), then per round j = 1..n: K(j) (while j < n)
+// and V(j-1).
 SVL_DEVINL int pos_k(int j) { return j == 0 ? 0 : 2 * j - 1; }
 SVL_DEVINL int pos_v(int m, int n) { return m + 1 < n ? 2 * m + 2 : 2 * m + 1; }
 
