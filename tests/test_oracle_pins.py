@@ -717,3 +717,37 @@ def test_fp8_forward_against_dense_library_forward():
     assert e8 > 2 * e16, (e8, e16)
     l8 = rel(outs["fp8"]["logits"], logits.numpy() if hasattr(logits, "numpy") else logits)
     assert l8 < bound, (l8, bound)
+
+
+def test_fp8_group_off_equals_zeroed_projection_rows():
+    """In the e4m3 forward too, a gated-off group equals the same group with
+    its Q, K, V rows and its gate/up channels zeroed: zero rows quantise to
+    zero codes on their own (per-channel scales), the group's attention output
+    and SwiGLU channels are then exactly zero, and nothing else changes -- the
+    activation rows' and the other channels' scales are untouched."""
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 3)
+    L, G, A, Akv, dh = dims.n_layers, dims.n_groups, dims.n_heads, dims.n_kv_heads, dims.d_head
+    gg = np.ones((L, G), np.uint8)
+    gg[0, 1] = 0
+    gg[2, 0] = 0
+    lg = np.ones(L, np.uint8)
+    gated = O.forward_sample(dims, w, x, ids, 1.0, lg, gg, keep_count=12, mode="fp8")
+    wz = dict(w)
+    layers = []
+    hpg, kpg, cpg = A // G, Akv // G, dims.d_ffn // G
+    for l, lw in enumerate(w["layers"]):
+        lw = {k: v.copy() for k, v in lw.items()}
+        for j in range(G):
+            if not gg[l, j]:
+                lw["wq"][j * hpg * dh:(j + 1) * hpg * dh] = 0.0
+                lw["wk"][j * kpg * dh:(j + 1) * kpg * dh] = 0.0
+                lw["wv"][j * kpg * dh:(j + 1) * kpg * dh] = 0.0
+                lw["wg"][j * cpg:(j + 1) * cpg] = 0.0
+                lw["wu"][j * cpg:(j + 1) * cpg] = 0.0
+        layers.append(lw)
+    wz["layers"] = layers
+    dense = O.forward_sample(dims, wz, x, ids, 1.0, lg, np.ones((L, G), np.uint8), keep_count=12, mode="fp8")
+    np.testing.assert_array_equal(gated["hidden"], dense["hidden"])
+    np.testing.assert_array_equal(gated["logits"], dense["logits"])
