@@ -27,6 +27,21 @@
  *    workspace must be ordered on one stream.
  *  - Gates are bytes, 0 = off, anything else = on. For layers l < n_prefix
  *    the gates are ignored and every group runs (Sec. 3.2 prefix layers).
+ *  - The GEMM and attention kernels are persistent (one CTA per SM) and the
+ *    shares of a GEMM's K-split tail wait for each other inside one launch.
+ *    Run the calls of one GPU on one stream (or ordered streams): two of them
+ *    running concurrently can keep each other's CTAs off the SMs until a
+ *    bounded wait gives up (SVL_DEV_TIMEOUT in the status word).
+ *
+ * Beyond the three calls of the path: svl_score_select_paper (the paper's own
+ * inference rule, Sec. 3.1 and Sec. 3.3), svl_pack_controlled and
+ * svl_controlled_prefill (the LLM-side compute controller, Sec. 3.2, Eq. 7),
+ * svl_gated_prefill_kv and svl_decode_step (gated decode with a KV cache,
+ * which the paper leaves open, Sec. 5), gemm_format = SVL_GEMM_E4M3 with
+ * svl_quantize_rows_e4m3 and svl_gemm_e4m3 (FP8 gated projections; Sec. 5
+ * calls quantisation orthogonal to the method), svl_prefill_from_host (the
+ * path from host buffers), svl_flops (Eq. 8 on the host) and the profiling and
+ * self-test calls.
  */
 #ifndef SVL_H
 #define SVL_H
