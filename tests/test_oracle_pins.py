@@ -751,3 +751,20 @@ def test_fp8_group_off_equals_zeroed_projection_rows():
     dense = O.forward_sample(dims, wz, x, ids, 1.0, lg, np.ones((L, G), np.uint8), keep_count=12, mode="fp8")
     np.testing.assert_array_equal(gated["hidden"], dense["hidden"])
     np.testing.assert_array_equal(gated["logits"], dense["logits"])
+
+
+def test_fp8_decode_reference_is_causal():
+    """The e4m3 forward keeps causality exactly: weight scales are fixed and
+    every activation row is quantised on its own, so appending tokens leaves
+    the earlier rows bit for bit unchanged (what lets an e4m3 decode cache
+    them)."""
+    dims = synth.reduced(SMALL, n_prefix=1)
+    w = np_weights(dims, seed=5)
+    x, ids = _sample(dims, seed=6)
+    lg = np.array([1, 1, 0], np.uint8)
+    gg = np.array([[1, 1], [0, 1], [1, 1]], np.uint8)
+    first, steps = O.decode_reference(dims, w, x, ids, 0.6, lg, gg, np.array([1, 2, 3]), mode="fp8")
+    prev = first["hidden"]
+    for st in steps:
+        np.testing.assert_array_equal(st["hidden"][:prev.shape[0]], prev)
+        prev = st["hidden"]
