@@ -9,14 +9,20 @@ Adaptation for Multimodal LLMs", arXiv 2607.20357).
 Arithmetic is float64 throughout. A storage mode rounds the tensors that the
 GPU stores in memory: ``"fp64"`` (no rounding), ``"fp32"`` or ``"bf16"``
 (round-to-nearest-even emulation of bfloat16 storage). Token logits are never
-rounded. ``"fp8"`` is bf16 storage with the four gated projections of every
-decoder layer (QKV, O, gate/up, down) computed from e4m3 operands: each weight
-row (output channel) and each activation row is scaled so that its largest
-magnitude maps to 448, the largest finite e4m3 value, and rounded to e4m3; the
-product of the codes is scaled back by both scales after the sum.
-``"fp8_s32"`` is the same with fp32 storage: how far it lands from ``"fp8"``
-measures how strongly e4m3's rounding boundaries amplify storage-level
-differences (a value moved across a boundary jumps by a whole e4m3 step).
+rounded, and neither are the RMS-normalised rows that feed a projection: they
+are an intermediate of the projection, not a stored tensor. ``"fp8"`` is bf16
+storage with the four gated projections of every decoder layer (QKV, O,
+gate/up, down) computed from e4m3 operands, stated plainly: the projection's
+input -- RMSNorm(X) * gain for QKV and gate/up, the attention output for O, the
+SwiGLU output for down -- and the weight W as given (no gain folded in) are
+quantised row by row: each activation row and each weight row (output
+channel) is scaled so that its largest magnitude maps to 448, the largest
+finite e4m3 value, and rounded to e4m3; the product of the codes is scaled
+back by both scales after the sum. ``"fp8_s32"`` is the same with fp32
+storage: how far it lands from ``"fp8"`` measures how strongly e4m3's
+rounding boundaries amplify storage-level differences (a value moved across
+a boundary jumps by a whole e4m3 step). ``"fp8_s64"`` stores nothing rounded
+(the e4m3 definition on its own, for pinning it against library routines).
 
 What each function follows:
 
@@ -37,7 +43,11 @@ What each function follows:
 * ``decoder_layer`` -- Sec. 3.2 gating: group j of layer l switches its
   attention heads and its slice of FFN channels together; alpha_l = 0 skips
   the layer through its residual connection. Gated-off parts contribute zero
-  (masked-dense definition).
+  (masked-dense definition). Its stages, each usable on its own:
+  ``attention_projections`` (RMSNorm, Q/K/V, RoPE), ``attention_heads``
+  (causal attention of the active heads), ``attention_residual`` (O
+  projection + residual), ``mlp_hidden`` (RMSNorm, gate/up, SwiGLU on the
+  active channels), ``mlp_residual`` (down projection + residual).
 * ``forward_sample`` / ``forward_batch`` -- the whole path, sample by sample.
 * ``survival_rate`` / ``controller_gate_logits`` / ``forward_controlled`` --
   Sec. 3.2 LLM-side compute controller: the budget token (Eq. 5 encoding,
@@ -103,6 +113,8 @@ def make_store(mode: str):
         return round_bf16
     if mode == "fp8_s32":
         return lambda a: np.asarray(a, dtype=np.float32).astype(np.float64)
+    if mode == "fp8_s64":
+        return lambda a: np.asarray(a, dtype=np.float64)
     raise ValueError(mode)
 
 
@@ -159,17 +171,11 @@ def linear_e4m3(x, wq):
 
 
 def fp8_layer_weights(lw):
-    """e4m3 weights of one layer's gated projections. The RMSNorm gains are
-    folded into the columns of the projections they feed (W diag(gain), held
-    in bf16 as the folded weights are stored), then every output channel is
-    quantised on its own."""
-    out = {}
-    for name, gain in (("wq", "attn_norm"), ("wk", "attn_norm"), ("wv", "attn_norm"),
-                       ("wg", "ffn_norm"), ("wu", "ffn_norm")):
-        out[name] = quantize_rows_e4m3(round_bf16(lw[name] * lw[gain][None, :]))
-    for name in ("wo", "wd"):
-        out[name] = quantize_rows_e4m3(lw[name])
-    return out
+    """e4m3 weights of one layer's gated projections: every output channel
+    (row of W, as given) quantised on its own. The RMSNorm gains stay on the
+    activation side (they scale the normalised rows before those are
+    quantised)."""
+    return {name: quantize_rows_e4m3(lw[name]) for name in ("wq", "wk", "wv", "wo", "wg", "wu", "wd")}
 
 
 # ----------------------------------------------------------------------------
@@ -361,7 +367,7 @@ def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_cou
     X = np.concatenate([X, tok[None, :]], axis=0)
     pos = np.concatenate([pos, [len(pos)]])
     on = np.ones(G, dtype=np.int64)
-    qws = [fp8_layer_weights(lw) if mode in ("fp8", "fp8_s32") else None for lw in weights["layers"]]
+    qws = [fp8_layer_weights(lw) if mode in ("fp8", "fp8_s32", "fp8_s64") else None for lw in weights["layers"]]
     for l in range(P):
         X = decoder_layer(X, pos, weights["layers"][l], on, dims, store, qws[l])
     gate_logits = controller_gate_logits(dims, weights, X[-1], kappa)
@@ -412,15 +418,86 @@ def rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
     return np.concatenate([x1 * cos - x2 * sin, x2 * cos + x1 * sin], axis=-1)
 
 
-def causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray) -> np.ndarray:
-    """softmax(q k^T / sqrt(d) + causal mask) v for one head; q,k,v are [S, d]."""
+def causal_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, p_bf16: bool = False) -> np.ndarray:
+    """softmax(q k^T / sqrt(d) + causal mask) v for one head; q,k,v are [S, d].
+
+    ``p_bf16`` is a variant, not the definition: the unnormalised
+    probabilities exp(s - rowmax) are rounded to bfloat16 before the product
+    with v and the row sum is taken of the unrounded values -- the precision
+    at which a kernel that feeds the probabilities to a bf16 tensor-core
+    product computes this.
+    """
     S, d = q.shape
     s = (q @ k.T) / np.sqrt(d)
     s = np.where(np.tril(np.ones((S, S), dtype=bool)), s, -np.inf)
     s = s - s.max(axis=1, keepdims=True)
     p = np.exp(s)
+    if p_bf16:
+        return (round_bf16(p) @ v) / p.sum(axis=1, keepdims=True)
     p = p / p.sum(axis=1, keepdims=True)
     return p @ v
+
+
+def attention_projections(X, pos, lw, dims, store, qw=None):
+    """Q, K, V of one sample's rows (Sec. 3.2, attention block): the
+    RMS-normalised rows times the norm gain, times W_q, W_k, W_v; RoPE on Q
+    and K at positions ``pos``. Every head is computed (the gated-off ones
+    are ignored downstream). With ``qw`` the three products take e4m3
+    operands: the normalised, gain-scaled rows and the weights, each
+    quantised per row. Returns q [S, A, d_h], k and v [S, A_kv, d_h]."""
+    A, Akv, dh = dims.n_heads, dims.n_kv_heads, dims.d_head
+    S = X.shape[0]
+    xn = rmsnorm(X, lw["attn_norm"], dims.rms_eps)
+    if qw is None:
+        q, k, v = xn @ lw["wq"].T, xn @ lw["wk"].T, xn @ lw["wv"].T
+    else:
+        q, k, v = (linear_e4m3(xn, qw[n]) for n in ("wq", "wk", "wv"))
+    q = store(rope(q.reshape(S, A, dh), pos, dims.rope_theta))
+    k = store(rope(k.reshape(S, Akv, dh), pos, dims.rope_theta))
+    return q, k, store(v.reshape(S, Akv, dh))
+
+
+def attention_heads(q, k, v, groups, dims, store, p_bf16=False):
+    """Causal attention of the heads whose group is on; gated-off heads give
+    zero (Sec. 3.2). GQA: query head h reads KV head h // (A / A_kv).
+    Returns the attention output [S, A * d_h]."""
+    A, Akv, dh, G = dims.n_heads, dims.n_kv_heads, dims.d_head, dims.n_groups
+    S = q.shape[0]
+    hpg = A // G
+    o = np.zeros((S, A, dh))
+    for h in range(A):
+        if groups[h // hpg]:
+            kv = h // (A // Akv)
+            o[:, h, :] = causal_attention(q[:, h, :], k[:, kv, :], v[:, kv, :], p_bf16)
+    return store(o.reshape(S, A * dh))
+
+
+def attention_residual(X, o, lw, store, qw=None):
+    """X + o W_O^T (e4m3 operands with ``qw``: o quantised per row)."""
+    return store(X + (o @ lw["wo"].T if qw is None else linear_e4m3(o, qw["wo"])))
+
+
+def mlp_hidden(X, lw, groups, dims, store, qw=None):
+    """SwiGLU of the RMS-normalised, gain-scaled rows: SiLU(xn W_g^T) * (xn
+    W_u^T), with the FFN channels of gated-off groups set to zero (channel c
+    belongs to group c // (D_int / G), reading R3). With ``qw`` both products
+    take e4m3 operands (xn and the weights quantised per row)."""
+    G = dims.n_groups
+    xn = rmsnorm(X, lw["ffn_norm"], dims.rms_eps)
+    if qw is None:
+        u = silu(xn @ lw["wg"].T) * (xn @ lw["wu"].T)
+    else:
+        u = silu(linear_e4m3(xn, qw["wg"])) * linear_e4m3(xn, qw["wu"])
+    cpg = dims.d_ffn // G
+    for j in range(G):
+        if not groups[j]:
+            u[:, j * cpg:(j + 1) * cpg] = 0.0
+    return store(u)
+
+
+def mlp_residual(X, u, lw, store, qw=None):
+    """X + u W_down^T (e4m3 operands with ``qw``: u quantised per row)."""
+    return store(X + (u @ lw["wd"].T if qw is None else linear_e4m3(u, qw["wd"])))
 
 
 def decoder_layer(X, pos, lw, groups, dims, store, qw=None):
@@ -429,55 +506,14 @@ def decoder_layer(X, pos, lw, groups, dims, store, qw=None):
     ``groups`` is e_{l,:} (length G). Head h belongs to group h // (A/G);
     FFN channel c to group c // (D_int/G) (reading R3). Off groups give zero
     attention output and zero FFN channels; no rescaling by 1/alpha. With
-    every group off the layer is the identity (residual bypass).
-
-    With ``qw`` (``fp8_layer_weights``) the four projections take e4m3
-    operands: the stored residual rows X are quantised as they are and the
-    RMSNorm enters as the row factor 1/rms(X) after the product (the gain is
-    in the folded weights); the attention output and the SwiGLU output are
-    quantised as stored.
+    every group off the layer is the identity (residual bypass). With ``qw``
+    (``fp8_layer_weights``) the four projections take e4m3 operands.
     """
-    A, Akv, dh, G = dims.n_heads, dims.n_kv_heads, dims.d_head, dims.n_groups
-    S = X.shape[0]
     if not np.any(groups):
         return X
-    hpg = A // G
-
-    def inv_rms(Y):
-        return 1.0 / np.sqrt(np.mean(Y * Y, axis=1, keepdims=True) + dims.rms_eps)
-
-    if qw is None:
-        xn = store(rmsnorm(X, lw["attn_norm"], dims.rms_eps))
-        q, k, v = xn @ lw["wq"].T, xn @ lw["wk"].T, xn @ lw["wv"].T
-    else:
-        r = inv_rms(X)
-        q, k, v = (r * linear_e4m3(X, qw[n]) for n in ("wq", "wk", "wv"))
-    q = q.reshape(S, A, dh)
-    k = k.reshape(S, Akv, dh)
-    v = v.reshape(S, Akv, dh)
-    q = store(rope(q, pos, dims.rope_theta))
-    k = store(rope(k, pos, dims.rope_theta))
-    v = store(v)
-    o = np.zeros((S, A, dh))
-    for h in range(A):
-        if groups[h // hpg]:
-            kv = h // (A // Akv)
-            o[:, h, :] = causal_attention(q[:, h, :], k[:, kv, :], v[:, kv, :])
-    o = store(o.reshape(S, A * dh))
-    X = store(X + (o @ lw["wo"].T if qw is None else linear_e4m3(o, qw["wo"])))
-
-    if qw is None:
-        xn = store(rmsnorm(X, lw["ffn_norm"], dims.rms_eps))
-        u = silu(xn @ lw["wg"].T) * (xn @ lw["wu"].T)
-    else:
-        r = inv_rms(X)
-        u = silu(r * linear_e4m3(X, qw["wg"])) * (r * linear_e4m3(X, qw["wu"]))
-    cpg = dims.d_ffn // G
-    for j in range(G):
-        if not groups[j]:
-            u[:, j * cpg:(j + 1) * cpg] = 0.0
-    u = store(u)
-    return store(X + (u @ lw["wd"].T if qw is None else linear_e4m3(u, qw["wd"])))
+    q, k, v = attention_projections(X, pos, lw, dims, store, qw)
+    X = attention_residual(X, attention_heads(q, k, v, groups, dims, store), lw, store, qw)
+    return mlp_residual(X, mlp_hidden(X, lw, groups, dims, store, qw), lw, store, qw)
 
 
 def project_visual(x, weights, dims, store):
@@ -526,7 +562,7 @@ def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
     for l in range(nl):
         lw = weights["layers"][l]
         qw = None
-        if mode in ("fp8", "fp8_s32"):
+        if mode in ("fp8", "fp8_s32", "fp8_s64"):
             qw = qws[l] if qws is not None else fp8_layer_weights(lw)
         X = decoder_layer(X, pos, lw, e[l], dims, store, qw)
     y = store(rmsnorm(X[-1], weights["final_norm"], dims.rms_eps))
@@ -553,7 +589,7 @@ def forward_batch(dims, weights, batch, mode="fp32", n_layers=None, samples=None
     out = []
     B = batch["B"]
     qws = None
-    if mode in ("fp8", "fp8_s32"):
+    if mode in ("fp8", "fp8_s32", "fp8_s64"):
         nl = dims.n_layers if n_layers is None else n_layers
         qws = [fp8_layer_weights(weights["layers"][l]) for l in range(nl)]
     for b in (range(B) if samples is None else samples):

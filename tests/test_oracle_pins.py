@@ -15,7 +15,7 @@ import torch
 
 from oracle import smartvl_oracle as O
 from paper_2607_20357_gb300 import synth
-from tests.dense_reference import dense_forward, rope_complex
+from tests.dense_reference import dense_forward, dense_forward_fp8, project_visual, rope_complex
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
@@ -267,10 +267,29 @@ def _sample(dims, seed=0, n_vis=24, s_text=7):
 
 
 def _packed_rows(dims, w, x, kept, ids):
+    """The packed rows built from library layers (projector: Linear, erf
+    GELU, Linear from torch.nn.functional)."""
     vis = x[kept]
     if dims.proj_hidden:
-        vis = O.gelu(vis @ w["proj_w1"].T) @ w["proj_w2"].T
+        vis = project_visual(vis, w["proj_w1"], w["proj_w2"])
     return np.concatenate([vis, w["embed"][ids]], 0)
+
+
+def test_project_visual_matches_library_layers():
+    """The LLaVA projector W2 GELU(W1 x) (no biases, exact GELU) against
+    torch.nn.functional.linear and gelu(approximate='none'); with bf16
+    storage the hidden and output rows are those values rounded."""
+    dims = SMALL
+    w = np_weights(dims, seed=11)
+    x, _ = _sample(dims, seed=12, n_vis=40)
+    got = O.project_visual(x, w, dims, O.make_store("fp64"))
+    ref = project_visual(x, w["proj_w1"], w["proj_w2"])
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-14)
+    # an identity projector when C_v = D and no hidden width
+    np.testing.assert_array_equal(O.project_visual(x, w, SMALL_ID, O.make_store("fp64")), x)
+    # bf16 storage: the stored output is the bf16 rounding of W2 bf16(GELU(W1 x))
+    h = O.round_bf16(torch.nn.functional.gelu(torch.as_tensor(x @ w["proj_w1"].T), approximate="none").numpy())
+    np.testing.assert_array_equal(O.project_visual(x, w, dims, O.round_bf16), O.round_bf16(h @ w["proj_w2"].T))
 
 
 @pytest.mark.parametrize("dims", [SMALL, SMALL_ID])
@@ -768,3 +787,118 @@ def test_fp8_decode_reference_is_causal():
     for st in steps:
         np.testing.assert_array_equal(st["hidden"][:prev.shape[0]], prev)
         prev = st["hidden"]
+
+
+def _random_gains(w, seed):
+    """A copy of the weights whose RMSNorm gains are drawn from U[0.5, 1.5]
+    (bf16 values) instead of 1."""
+    rng = np.random.default_rng(seed)
+    w = dict(w)
+    layers = []
+    for lw in w["layers"]:
+        lw = dict(lw)
+        for g in ("attn_norm", "ffn_norm"):
+            lw[g] = O.round_bf16(rng.uniform(0.5, 1.5, size=lw[g].shape))
+        layers.append(lw)
+    w["layers"] = layers
+    return w
+
+
+def test_fp8_plain_definition_with_random_gains_matches_library_fp8():
+    """The oracle's e4m3 forward is the plain definition: e4m3(RMSNorm(X) *
+    gain) against e4m3(W) per output channel, no gain folded into W. With
+    non-unit gains it must equal a forward built from PyTorch's float8_e4m3fn
+    conversion, F.rms_norm and F.linear (nothing stored rounded on either
+    side). The same forward with the gains folded into the weights before
+    their quantisation -- algebraically identical, quantised differently --
+    must fail that comparison by orders of magnitude: the pin sees the
+    folding."""
+    dims = SMALL
+    w = _random_gains(np_weights(dims, seed=21), seed=22)
+    x, ids = _sample(dims, seed=23)
+    L, G = dims.n_layers, dims.n_groups
+    lg, gg = np.ones(L, np.uint8), np.ones((L, G), np.uint8)
+    n = x.shape[0]
+    got = O.forward_sample(dims, w, x, ids, 1.0, lg, gg, keep_count=n, mode="fp8_s64")
+    X0 = _packed_rows(dims, w, x, np.arange(n), ids)
+    hid, logits = dense_forward_fp8(X0, w["layers"], w["final_norm"], w["lm_head"], dims)
+
+    def rel(a, b):
+        return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+
+    tol = 1e-9
+    assert rel(got["hidden"], hid) < tol
+    assert rel(got["logits"], logits) < 2.0 ** -23  # logits are returned as float32
+    # planted mistake: the gains folded into W before quantising, the rows
+    # normalised without them (the arrangement of an earlier kernel)
+    w_mis = dict(w)
+    w_mis["layers"] = [dict(lw, attn_norm=np.ones_like(lw["attn_norm"]), ffn_norm=np.ones_like(lw["ffn_norm"]))
+                       for lw in w["layers"]]
+    qws = []
+    for lw in w["layers"]:
+        q = O.fp8_layer_weights(lw)
+        for name, g in (("wq", "attn_norm"), ("wk", "attn_norm"), ("wv", "attn_norm"),
+                        ("wg", "ffn_norm"), ("wu", "ffn_norm")):
+            q[name] = O.quantize_rows_e4m3(O.round_bf16(lw[name] * lw[g][None, :]))
+        qws.append(q)
+    mis = O.forward_sample(dims, w_mis, x, ids, 1.0, lg, gg, keep_count=n, mode="fp8_s64", qws=qws)
+    assert rel(mis["hidden"], hid) > 1e4 * tol
+    # and a gain applied twice (folded into W while the rows keep it)
+    mis2 = O.forward_sample(dims, w, x, ids, 1.0, lg, gg, keep_count=n, mode="fp8_s64", qws=qws)
+    assert rel(mis2["hidden"], hid) > 1e4 * tol
+
+
+def _e4m3_midpoint_distance(q):
+    """Relative distance of each |q| to the nearest midpoint between two
+    adjacent e4m3 values (spacing 2^(e-3) in [2^e, 2^(e+1)), 2^-9 below
+    2^-6)."""
+    m = np.abs(np.asarray(q, dtype=np.float64))
+    _, ex = np.frexp(m)
+    sp = np.ldexp(1.0, np.maximum(ex.astype(np.int64) - 1, -6) - 3)
+    f = m / sp - np.floor(m / sp)
+    return np.abs(f - 0.5) * sp / np.maximum(m, 1e-300)
+
+
+@pytest.mark.parametrize("unit_gain", [True, False])
+def test_fp8_prescaled_rows_equal_plain_definition(unit_gain):
+    """The kernels' arrangement of the e4m3 QKV and gate/up products: they
+    quantise the rows X * gain (exact float32 products of bf16 values) and
+    multiply by 1/rms(X) after the product. Per-row scales make this the plain
+    definition: 1/rms scales a whole row, so the codes of X * gain equal those
+    of RMSNorm(X) * gain and the scales differ by the factor rms -- up to
+    float32 rounding of the two quotients, which can only split a value that
+    lies within a few float32 ulps of a midpoint between two e4m3 values
+    (bf16 inputs put about 0.1 % of the values exactly on one). Checked at
+    LLaVA-7B width for unit and random gains: every differing code is such a
+    near-tie, one e4m3 step apart, and the products agree to float rounding
+    plus those steps."""
+    rng = np.random.default_rng(31 + unit_gain)
+    D, R, N, eps = 4096, 48, 256, 1e-5
+    X = O.round_bf16(rng.normal(size=(R, D)) * 10.0 ** rng.uniform(-2, 2, size=(R, 1)))
+    X[0, 7] = 40.0  # an outlier row
+    gain = np.ones(D) if unit_gain else O.round_bf16(rng.uniform(0.5, 1.5, size=D))
+    W = O.round_bf16(rng.normal(size=(N, D)) * 0.02)
+    wq = O.quantize_rows_e4m3(W)
+    y = O.rmsnorm(X, gain, eps)
+    pc, ps = O.quantize_rows_e4m3(y)
+    fc, fs = O.quantize_rows_e4m3((X.astype(np.float32) * gain.astype(np.float32)).astype(np.float64))
+    inv_rms = 1.0 / np.sqrt(np.mean(X * X, axis=1) + eps)
+    # scales: amax(X * gain) / 448 times 1/rms is amax(y) / 448
+    np.testing.assert_allclose(fs * inv_rms, ps, rtol=2.0 ** -21)
+    diff = pc != fc
+    # bf16 rows make exact e4m3 ties common (x / amax is a ratio of 8-bit
+    # significands): float32 rounding of either quotient splits those
+    assert diff.mean() < 5e-3, diff.mean()
+    if diff.any():
+        y32 = y.astype(np.float32)
+        inv = (np.float32(448) / np.abs(y32).max(axis=1)).astype(np.float32)
+        quot = (y32 * inv[:, None]).astype(np.float64)
+        assert (_e4m3_midpoint_distance(quot[diff]) < 2.0 ** -19).all()
+        assert (np.abs(pc[diff] - fc[diff]) <= np.maximum(np.abs(pc[diff]), np.abs(fc[diff])) * 2.0 ** -3 + 2.0 ** -9).all()
+    plain = O.linear_e4m3(y, wq)
+    fused = (fc @ wq[0].T) * fs[:, None] * wq[1][None, :] * inv_rms[:, None]
+    err = np.abs(fused - plain)
+    # float rounding of the scales, plus one e4m3 step per differing code
+    step = np.abs(pc - fc) @ np.abs(wq[0]).T * ps[:, None] * wq[1][None, :]
+    bound = 2.0 ** -20 * (np.abs(pc) @ np.abs(wq[0]).T) * ps[:, None] * wq[1][None, :] + step
+    assert (err <= bound + 1e-300).all()
