@@ -86,11 +86,13 @@ typedef enum svl_status {
  * every decoder layer (QKV, O, gate/up, down): SVL_GEMM_BF16, or
  * SVL_GEMM_E4M3 -- FP8 weights, which the paper calls orthogonal to its
  * method (Sec. 5). With e4m3, svl_model_create quantises each weight output
- * channel (row of W, norm gains folded in) to e4m3 with the scale
- * amax / 448; each activation row feeding those GEMMs is quantised the same
- * way on the fly (svl_quantize_rows_e4m3 is the definition), and the fp32
- * accumulator of the code products is scaled by both rows' scales. The
- * projector, token controller and LM head stay bf16. */
+ * channel (row of W as given) to e4m3 with the scale amax / 448; each
+ * activation row feeding those GEMMs -- RMSNorm(X) * gain for QKV and
+ * gate/up, the attention output for O, the SwiGLU output for down -- is
+ * quantised the same way on the fly (svl_quantize_rows_e4m3 is the
+ * definition), and the fp32 accumulator of the code products is scaled by
+ * both rows' scales. The projector, token controller and LM head stay
+ * bf16. */
 #define SVL_GEMM_BF16 0
 #define SVL_GEMM_E4M3 1
 typedef struct svl_model_desc {
@@ -287,17 +289,20 @@ size_t svl_kv_cache_size(const svl_model* model, int32_t B, int32_t max_len);
 
 /* e4m3 quantisation of bf16 rows, as the SVL_GEMM_E4M3 path applies it to
  * weight output channels and activation rows. For each of the `rows` rows
- * of `cols` values (device bf16, `ld_src` elements apart): amax = max |x|,
- * inv = 448 / amax and scale[r] = amax / 448 in float32 with correct
- * rounding (both 0 when amax is 0), and dst[r * ld_dst + c] =
- * e4m3(x * inv) rounded to nearest even and saturated to +-448 (OCP e4m3:
- * 4 exponent bits with bias 7, 3 mantissa bits, no infinities). dst is
- * device uint8 codes, scale device float32 [rows]; the caller owns both.
- * Requires cols and ld_src multiples of 8, ld_dst >= cols and a multiple
- * of 8, src 16-byte and dst 8-byte aligned (else SVL_ERR_INVALID_ARG).
- * Asynchronous on `stream`. */
-svl_status svl_quantize_rows_e4m3(const void* src, int64_t rows, int32_t cols, int64_t ld_src, void* dst,
-                                  int64_t ld_dst, float* scale, void* stream);
+ * of `cols` values (device bf16, `ld_src` elements apart), with
+ * x = src[r, c] * gain[c] (float32, exact; gain is a device bf16 [cols]
+ * vector, or NULL for x = src[r, c]): amax = max |x|, inv = 448 / amax and
+ * scale[r] = amax / 448 in float32 with correct rounding (both 0 when amax
+ * is 0), and dst[r * ld_dst + c] = e4m3(x * inv) rounded to nearest even and
+ * saturated to +-448 (OCP e4m3: 4 exponent bits with bias 7, 3 mantissa
+ * bits, no infinities). The prefill quantises the QKV and gate/up inputs
+ * with their RMSNorm gain this way (the norm's 1/rms is a factor of the row,
+ * applied after the product). dst is device uint8 codes, scale device
+ * float32 [rows]; the caller owns both. Requires cols and ld_src multiples
+ * of 8, ld_dst >= cols and a multiple of 8, src (and gain) 16-byte and dst
+ * 8-byte aligned (else SVL_ERR_INVALID_ARG). Asynchronous on `stream`. */
+svl_status svl_quantize_rows_e4m3(const void* src, const void* gain, int64_t rows, int32_t cols, int64_t ld_src,
+                                  void* dst, int64_t ld_dst, float* scale, void* stream);
 
 /* The e4m3 GEMM of the gated projections on its own, with an fp32 output:
  * C[m, n] = a_scale[m] * b_scale[n] * sum_k A[m, k] B[n, k], A [M, K] and
@@ -326,7 +331,10 @@ svl_status svl_gated_prefill_kv(svl_model* model, int32_t B, int32_t t_cap, void
  * NULL) the largest logit (equal logits: lower id), and cache_len[b] is
  * advanced by one. Workspace: svl_decode_workspace_size(model, B) bytes.
  * A fed id outside [0, V) or a full cache sets SVL_DEV_BAD_INDEX (the id is
- * read as 0; a full cache skips the sample's attention). */
+ * read as 0). A sample whose cache is full (cache_len[b] >= max_len) takes
+ * no step: nothing is appended, its attention output is zero, cache_len[b]
+ * stays at max_len and next_token[b] is -1. Check the status word after the
+ * steps of a batch. */
 size_t svl_decode_workspace_size(const svl_model* model, int32_t B);
 svl_status svl_decode_step(svl_model* model, int32_t B, const int32_t* tokens, void* kv_cache, int32_t max_len,
                            int32_t* cache_len, const uint8_t* layer_gate, const uint8_t* group_gate, float* logits,
@@ -389,6 +397,37 @@ svl_status svl_gated_prefill(svl_model* model, int32_t B, int32_t t_cap, void* X
                              const uint8_t* layer_gate, const uint8_t* group_gate,
                              int32_t logits_mode, float* logits,
                              void* workspace, size_t workspace_bytes, void* stream);
+
+/* One stage of decoder layer `layer` of (3) on caller buffers: the layer
+ * piecewise, with exactly the kernels and launch configuration the prefill
+ * uses (the stage inside svl_gated_prefill is the same code path). Serves
+ * per-stage checks of a layer and callers that interleave their own work
+ * between the stages. Gates, cu_seqlens, pos, t_cap and the workspace are as
+ * for svl_gated_prefill (a workspace sized for the prefill suffices); the
+ * RMSNorm sums of squares that the prefill carries from the previous stage
+ * are recomputed from X. d_h = D / A, t_pad = t_cap rounded up to 8.
+ *  SVL_LAYER_QKV:    X -> q [t_cap, A*d_h], k [t_cap, A_kv*d_h] (RoPE at pos)
+ *                    and vt [A_kv*d_h, t_pad] (V transposed), for the heads of
+ *                    active groups (other columns untouched)
+ *  SVL_LAYER_ATTN:   q, k, vt -> ao [t_cap, A*d_h]: causal attention of the
+ *                    active heads (key columns of vt past the packed rows
+ *                    must hold finite values)
+ *  SVL_LAYER_OPROJ:  X += ao W_O^T over the active heads' rows of W_O
+ *  SVL_LAYER_GATEUP: X -> h [t_cap, D_int] = SiLU(xn W_g^T) * (xn W_u^T),
+ *                    xn = RMSNorm(X) * gain, active groups' channels only
+ *  SVL_LAYER_DOWN:   X += h W_down^T over the active channels
+ * Buffers a stage does not use may be NULL. All bf16, device, caller-owned,
+ * 16-byte aligned. Errors: as svl_gated_prefill; a bad stage or layer, or a
+ * missing buffer the stage needs: SVL_ERR_INVALID_ARG. */
+#define SVL_LAYER_QKV 0
+#define SVL_LAYER_ATTN 1
+#define SVL_LAYER_OPROJ 2
+#define SVL_LAYER_GATEUP 3
+#define SVL_LAYER_DOWN 4
+svl_status svl_layer_stage(svl_model* model, int32_t stage, int32_t layer, int32_t B, int32_t t_cap, void* X,
+                           const int32_t* cu_seqlens, const int32_t* pos, const uint8_t* layer_gate,
+                           const uint8_t* group_gate, void* q, void* k, void* vt, void* ao, void* h,
+                           void* workspace, size_t workspace_bytes, void* stream);
 
 /* Eq. 8 for one sample, host only, no GPU: writes G * C(S) (exact integer
  * arithmetic, 8 D^2 generalised to 4 D^2 + 4 D D_kv) for S = s_text + s_vis
@@ -472,6 +511,20 @@ const char* svl_status_string(svl_status s);
 /* Number of kernels launched by this library since the process started
  * (host-side counter, used to report launches per step). */
 uint64_t svl_launch_count(void);
+
+/* The launch rule of the residual GEMMs' K-split tail, host only (no GPU):
+ * the number of K shares (1 = no split) the last wave of a residual GEMM
+ * list of `tiles` tiles (list capacity `cap`) is cut into, on a persistent
+ * grid of num_sms CTAs of which blocks_per_sm fit on one SM, with `units`
+ * partial tiles of workspace. The shares wait for each other inside one
+ * launch, so the tail is split only when the whole grid is resident at once
+ * (blocks_per_sm >= 1); svl_model_create queries the occupancy of the
+ * residual GEMM and the prefill disables the split when it is 0. Beyond
+ * that: a last wave of r = tiles % num_sms tiles is split only when
+ * 0 < r <= num_sms / 2, into min(num_sms / r, 8, units / r,
+ * 1 + (cap - tiles) / r) shares, if that is at least 2. The paper has no
+ * counterpart; this is the library's load balancing of partial waves. */
+int32_t svl_ksplit_plan(int32_t tiles, int32_t cap, int32_t num_sms, int32_t blocks_per_sm, int32_t units);
 
 #ifdef __cplusplus
 }

@@ -19,6 +19,9 @@ struct svl_model {
   std::vector<svl_layer_weights> layers;
   int device = 0;
   int num_sms = 0;
+  // every CTA of the persistent residual GEMM fits on the GPU at once, so
+  // the shares of a K-split tail can wait for each other (else no split)
+  bool ks_resident = false;
   uint32_t* d_status = nullptr;
   float2* rope_cs = nullptr;
   // B-operand tensor maps of the weights: per layer q, k, v, o, g, u, d
@@ -317,6 +320,12 @@ const char* svl_status_string(svl_status s) {
 
 uint64_t svl_launch_count(void) { return g_launches.load(); }
 
+int32_t svl_ksplit_plan(int32_t tiles, int32_t cap, int32_t num_sms, int32_t blocks_per_sm, int32_t units) {
+  // one CTA per SM: the grid is resident at once iff an SM holds a CTA
+  if (blocks_per_sm < 1) return 1;
+  return ksplit_shares(tiles, cap, num_sms, units);
+}
+
 svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, svl_model** out) {
   if (!desc || !w || !out) return SVL_ERR_INVALID_ARG;
   *out = nullptr;
@@ -357,6 +366,9 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   m->w.layers = m->layers.data();
   cudaGetDevice(&m->device);
   cudaDeviceGetAttribute(&m->num_sms, cudaDevAttrMultiProcessorCount, m->device);
+  // the persistent residual GEMM runs one CTA per SM: resident at once iff
+  // one CTA fits on an SM (the rule svl_ksplit_plan applies)
+  m->ks_resident = gemm_resid_blocks_per_sm(d.gemm_format == SVL_GEMM_E4M3) >= 1;
   const int64_t dkv = static_cast<int64_t>(d.n_kv_heads) * dh, hq = static_cast<int64_t>(d.n_heads) * dh;
   bool ok = true;
   for (int l = 0; l < d.n_layers && ok; ++l) {
@@ -370,8 +382,12 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   // RMSNorm runs fused into the GEMMs after it (x / rms(x) scales the
   // accumulator rows), so each norm gain is folded into the columns of the
   // projections it feeds: W' = W diag(gain). Layers whose gains are exactly 1
-  // keep the caller's weights.
-  {
+  // keep the caller's weights. e4m3 models fold nothing: their activation
+  // quantiser multiplies the rows by the gain (the e4m3 definition quantises
+  // RMSNorm(X) * gain and W as given), so their codes come from the caller's
+  // weights.
+  m->folded.assign(static_cast<size_t>(d.n_layers) * 5, nullptr);
+  if (d.gemm_format != SVL_GEMM_E4M3) {
     int* flags = nullptr;
     std::vector<int> host(2 * static_cast<size_t>(d.n_layers), 1);
     ok = cudaMalloc(&flags, sizeof(int) * host.size()) == cudaSuccess &&
@@ -384,7 +400,6 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
     }
     ok = ok && cudaMemcpy(host.data(), flags, sizeof(int) * host.size(), cudaMemcpyDeviceToHost) == cudaSuccess;
     if (flags) cudaFree(flags);
-    m->folded.assign(static_cast<size_t>(d.n_layers) * 5, nullptr);
     for (int l = 0; l < d.n_layers && ok; ++l) {
       svl_layer_weights& lw = m->layers[l];
       const void** src[5] = {&lw.wq, &lw.wk, &lw.wv, &lw.wg, &lw.wu};
@@ -408,8 +423,8 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
     }
   }
   if (d.gemm_format == SVL_GEMM_E4M3) {
-    // e4m3 copies of the (gain-folded) gated projections, one allocation per
-    // layer: codes then per-row scales of q, k, v, o, g, u, d
+    // e4m3 copies of the gated projections, one allocation per layer: codes
+    // then per-row scales of q, k, v, o, g, u, d
     m->e4m3 = true;
     const int G = d.n_groups;
     m->kgo_p = round128(static_cast<int>(hq / G));
@@ -745,6 +760,14 @@ svl_status svl_pack_controlled(svl_model* m, int32_t B, int32_t n_vis_total, int
 }
 
 namespace {
+// One stage of one layer on caller buffers (svl_layer_stage): the stage's
+// inputs and outputs replace the workspace copies of Q, K, V^T, the
+// attention output and the SwiGLU output.
+struct StageSel {
+  int stage, layer;
+  __nv_bfloat16 *q, *k, *vt, *ao, *h;
+};
+
 // KV cache of a prefill (store each layer's K, V) or a decode step (one new
 // row per sample: embedding of the fed token, attention against the cache,
 // greedy next token).
@@ -765,8 +788,8 @@ struct StepCtx {
 svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
                         const int32_t* pos, const uint8_t* layer_gate, const uint8_t* group_gate,
                         int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream,
-                        const CtlArgs* ctl, const StepCtx* kvx = nullptr) {
-  if (!m || B <= 0 || t_cap <= 0 || !X || !cu_seqlens || !pos || !layer_gate || !group_gate || !logits)
+                        const CtlArgs* ctl, const StepCtx* kvx = nullptr, const StageSel* only = nullptr) {
+  if (!m || B <= 0 || t_cap <= 0 || !X || !cu_seqlens || !pos || !layer_gate || !group_gate || (!logits && !only))
     return SVL_ERR_INVALID_ARG;
   if (logits_mode != SVL_LOGITS_LAST && logits_mode != SVL_LOGITS_ALL) return SVL_ERR_INVALID_ARG;
   if (!aligned16(X)) return SVL_ERR_INVALID_ARG;
@@ -819,7 +842,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   sa.attn_cap = L.attn_cap;
   sa.attn_count = counts + 4 * nl;
   sa.ks_info = at<int>(ws, L.ks_info);
-  sa.ks_units = L.ks_units;
+  sa.ks_units = m->ks_resident ? L.ks_units : 0;
   sa.status = m->d_status;
   if (ctl) {
     // controller path: every group on until the controller has decided
@@ -836,11 +859,11 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   }
 
   __nv_bfloat16* xn = at<__nv_bfloat16>(ws, L.xn);
-  __nv_bfloat16* qb = at<__nv_bfloat16>(ws, L.q);
-  __nv_bfloat16* kb = at<__nv_bfloat16>(ws, L.k);
-  __nv_bfloat16* vb = at<__nv_bfloat16>(ws, L.v);
-  __nv_bfloat16* ao = at<__nv_bfloat16>(ws, L.ao);
-  __nv_bfloat16* hm = at<__nv_bfloat16>(ws, L.hmid);
+  __nv_bfloat16* qb = only ? only->q : at<__nv_bfloat16>(ws, L.q);
+  __nv_bfloat16* kb = only ? only->k : at<__nv_bfloat16>(ws, L.k);
+  __nv_bfloat16* vb = only ? only->vt : at<__nv_bfloat16>(ws, L.v);
+  __nv_bfloat16* ao = only ? only->ao : at<__nv_bfloat16>(ws, L.ao);
+  __nv_bfloat16* hm = only ? only->h : at<__nv_bfloat16>(ws, L.hmid);
   // decode-sized batches (one row per sample) stream the weights through the
   // gated GEMMs with A boxes of kThinRows rows and deeper stages
   const bool thin = t_cap <= kThinRows;
@@ -861,10 +884,12 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
              !make_map8(&map_aq_o, aq, t_cap, static_cast<uint64_t>(G) * m->kgo_p, a_rows) ||
              !make_map8(&map_aq_h, aq, t_cap, static_cast<uint64_t>(G) * m->kgd_p, a_rows)))
     return SVL_ERR_CUDA;
-  auto quant = [&](const __nv_bfloat16* src, int64_t ld_src, int groups, int kg, int kgp, int layer) {
+  auto quant = [&](const __nv_bfloat16* src, const void* gain, int64_t ld_src, int groups, int kg, int kgp,
+                   int layer) {
     QuantArgs qa;
     std::memset(&qa, 0, sizeof(qa));
     qa.src = src;
+    qa.gain = static_cast<const __nv_bfloat16*>(gain);
     qa.ld_src = ld_src;
     qa.rows = t_cap;
     qa.G = groups;
@@ -920,8 +945,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   na.cu_seqlens = cu_seqlens;
 
   // V^T is read in 128-key tiles that may run past the rows written in this
-  // call; zero it once so those (masked) keys hold finite values
-  if (cudaMemsetAsync(vb, 0, sizeof(__nv_bfloat16) * static_cast<size_t>(L.t_pad) * dkv, s) != cudaSuccess)
+  // call; zero it once so those (masked) keys hold finite values (a single
+  // stage reads or writes the caller's V^T as it is)
+  if (!only && cudaMemsetAsync(vb, 0, sizeof(__nv_bfloat16) * static_cast<size_t>(L.t_pad) * dkv, s) != cudaSuccess)
     return SVL_ERR_CUDA;
   AttnTcArgs aa;
   std::memset(&aa, 0, sizeof(aa));
@@ -938,12 +964,17 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   aa.status = m->d_status;
 
   {
+    // sums of squares of the input rows: for the first layer's attention
+    // norm, or for the MLP norm when a single gate/up stage runs
     Launch L1(m, SVL_TAG_RMSNORM, s);
-    launch_norm_init(static_cast<const __nv_bfloat16*>(X), cu_seqlens, B, static_cast<int>(t_cap), d.d_model, ss_a,
-                     ss_ld, L.ss_slots, s);
+    launch_norm_init(static_cast<const __nv_bfloat16*>(X), cu_seqlens, B, static_cast<int>(t_cap), d.d_model,
+                     only && only->stage == SVL_LAYER_GATEUP ? ss_b : ss_a, ss_ld, L.ss_slots, s);
   }
+  // a stage of the layer runs unless a single other stage was asked for
+  auto want = [&](int l, int stage) { return !only || (only->layer == l && only->stage == stage); };
 
   for (int l = 0; l < nl; ++l) {
+    if (only && l != only->layer) continue;
     const CUtensorMap* tm = &m->tm_layer[static_cast<size_t>(l) * 7];
     if (ctl && l == std::min(d.n_prefix, nl)) {
       // the budget token's state after the prefix layers decides the gates
@@ -965,10 +996,14 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
 
     const CUtensorMap* tm8 = f8 ? &m->tm8[static_cast<size_t>(l) * 7] : nullptr;
     const float* const* sc8 = f8 ? &m->f8_scale[static_cast<size_t>(l) * 7] : nullptr;
-    // attention input norm fused into the QKV GEMM (gain folded into W_qkv)
-    if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), d.d_model, 1, d.d_model, d.d_model, -1)) != SVL_OK)
+    GemmParams p;
+    if (want(l, SVL_LAYER_QKV)) {
+    // attention input norm fused into the QKV GEMM (bf16: gain folded into
+    // W_qkv; e4m3: the quantiser multiplies the rows by the gain)
+    if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), m->layers[l].attn_norm, d.d_model, 1, d.d_model,
+                          d.d_model, -1)) != SVL_OK)
       return st;
-    GemmParams p = base_params(m);
+    p = base_params(m);
     set_norm(p, ss_a, nullptr);
     p.mapA = map_x;
     p.mapB[0] = tm[0];
@@ -991,7 +1026,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.rope_rows = d.max_seq;
     p.d_head = dh;
     if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8, thin)) != SVL_OK) return st;
+    }
 
+    if (want(l, SVL_LAYER_ATTN)) {
     const size_t layer_kv = static_cast<size_t>(B) * (kvx ? kvx->max_len : 0) * dkv;
     if (kvx && kvx->decode) {
       DecAttnArgs da;
@@ -1042,8 +1079,10 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
       Launch L1(m, SVL_TAG_ATTENTION, s);
       if (launch_attention_tc(aa, gemm_grid(m, L.attn_cap), s) != cudaSuccess) return SVL_ERR_CUDA;
     }
+    }
 
-    if (f8 && (st = quant(ao, hq, G, hq / G, m->kgo_p, l)) != SVL_OK) return st;
+    if (want(l, SVL_LAYER_OPROJ)) {
+    if (f8 && (st = quant(ao, nullptr, hq, G, hq / G, m->kgo_p, l)) != SVL_OK) return st;
     p = base_params(m);
     p.mapA = map_ao;
     p.mapB[0] = tm[3];
@@ -1064,9 +1103,13 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
     set_norm(p, nullptr, ss_b);  // sums of squares of the updated rows for the MLP norm
     if ((st = launch(EPI_RESID, m, SVL_TAG_OPROJ, p, L.o_cap, s, f8, thin)) != SVL_OK) return st;
+    }
 
-    // MLP input norm fused into the gate/up GEMM (gain folded into W_g, W_u)
-    if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), d.d_model, 1, d.d_model, d.d_model, -1)) != SVL_OK)
+    if (want(l, SVL_LAYER_GATEUP)) {
+    // MLP input norm fused into the gate/up GEMM (bf16: gain folded into W_g,
+    // W_u; e4m3: applied by the quantiser)
+    if (f8 && (st = quant(static_cast<const __nv_bfloat16*>(X), m->layers[l].ffn_norm, d.d_model, 1, d.d_model,
+                          d.d_model, -1)) != SVL_OK)
       return st;
     p = base_params(m);
     set_norm(p, ss_b, nullptr);
@@ -1083,8 +1126,10 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.out[0] = hm;
     p.ld[0] = d.d_ffn;
     if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8, thin)) != SVL_OK) return st;
+    }
 
-    if (f8 && (st = quant(hm, d.d_ffn, G, d.d_ffn / G, m->kgd_p, l)) != SVL_OK) return st;
+    if (want(l, SVL_LAYER_DOWN)) {
+    if (f8 && (st = quant(hm, nullptr, d.d_ffn, G, d.d_ffn / G, m->kgd_p, l)) != SVL_OK) return st;
     p = base_params(m);
     p.mapA = map_hm;
     p.mapB[0] = tm[6];
@@ -1105,7 +1150,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;
     set_norm(p, nullptr, ss_a);  // for the next layer's attention norm
     if ((st = launch(EPI_RESID, m, SVL_TAG_DOWN, p, L.dn_cap, s, f8, thin)) != SVL_OK) return st;
+    }
   }
+  if (only) return last_error();
 
   // final norm + LM head
   na.gain = static_cast<const __nv_bfloat16*>(m->w.final_norm);
@@ -1151,7 +1198,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   }
   if (kvx && kvx->decode) {
     Launch L1(m, SVL_TAG_LMHEAD, s);
-    launch_decode_finish(B, d.vocab, logits, kvx->next_token, kvx->cache_len, s);
+    launch_decode_finish(B, d.vocab, logits, kvx->next_token, kvx->cache_len, kvx->max_len, s);
   } else if (kvx && kvx->cache_len) {
     launch_offsets_diff(cu_seqlens, kvx->cache_len, B, s);  // cache length = prompt length
     g_launches++;
@@ -1165,6 +1212,26 @@ svl_status svl_gated_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, co
                              int32_t logits_mode, float* logits, void* ws, size_t ws_bytes, void* stream) {
   return prefill_impl(m, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, logits_mode, logits, ws, ws_bytes,
                       stream, nullptr);
+}
+
+svl_status svl_layer_stage(svl_model* m, int32_t stage, int32_t layer, int32_t B, int32_t t_cap, void* X,
+                           const int32_t* cu_seqlens, const int32_t* pos, const uint8_t* layer_gate,
+                           const uint8_t* group_gate, void* q, void* k, void* vt, void* ao, void* h, void* ws,
+                           size_t ws_bytes, void* stream) {
+  if (!m || stage < SVL_LAYER_QKV || stage > SVL_LAYER_DOWN || layer < 0 || layer >= m->d.n_layers)
+    return SVL_ERR_INVALID_ARG;
+  const bool need_qkv = stage == SVL_LAYER_QKV || stage == SVL_LAYER_ATTN;
+  if ((need_qkv && (!q || !k || !vt)) || ((stage == SVL_LAYER_ATTN || stage == SVL_LAYER_OPROJ) && !ao) ||
+      ((stage == SVL_LAYER_GATEUP || stage == SVL_LAYER_DOWN) && !h))
+    return SVL_ERR_INVALID_ARG;
+  for (const void* p : {q, k, vt, ao, h})
+    if (p && !aligned16(p)) return SVL_ERR_INVALID_ARG;
+  // buffers the stage does not use still need a valid address for the
+  // tensor maps made up front: X stands in for them (never read or written)
+  auto or_x = [&](void* p) { return static_cast<__nv_bfloat16*>(p ? p : X); };
+  StageSel sel{stage, layer, or_x(q), or_x(k), or_x(vt), or_x(ao), or_x(h)};
+  return prefill_impl(m, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, SVL_LOGITS_LAST, nullptr, ws,
+                      ws_bytes, stream, nullptr, nullptr, &sel);
 }
 
 svl_status svl_controlled_prefill(svl_model* m, int32_t B, int32_t t_cap, void* X, const int32_t* cu_seqlens,
@@ -1246,15 +1313,16 @@ svl_status svl_decode_step(svl_model* m, int32_t B, const int32_t* tokens, void*
                       ws_bytes - (xb + cb + pb), stream, nullptr, &kx);
 }
 
-svl_status svl_quantize_rows_e4m3(const void* src, int64_t rows, int32_t cols, int64_t ld_src, void* dst,
-                                  int64_t ld_dst, float* scale, void* stream) {
+svl_status svl_quantize_rows_e4m3(const void* src, const void* gain, int64_t rows, int32_t cols, int64_t ld_src,
+                                  void* dst, int64_t ld_dst, float* scale, void* stream) {
   if (!src || !dst || !scale || rows < 0 || cols <= 0 || (cols & 7) || ld_src < cols || (ld_src & 7) ||
       ld_dst < cols || (ld_dst & 7) || !aligned16(src) || (reinterpret_cast<uintptr_t>(dst) & 7) ||
-      (reinterpret_cast<uintptr_t>(scale) & 3))
+      (reinterpret_cast<uintptr_t>(scale) & 3) || (gain && !aligned16(gain)))
     return SVL_ERR_INVALID_ARG;
   QuantArgs qa;
   std::memset(&qa, 0, sizeof(qa));
   qa.src = static_cast<const __nv_bfloat16*>(src);
+  qa.gain = static_cast<const __nv_bfloat16*>(gain);
   qa.ld_src = ld_src;
   qa.rows = rows;
   qa.G = 1;
@@ -1524,9 +1592,11 @@ extern "C" svl_status svl_score_select_noalloc(svl_model* m, int32_t B, int32_t 
   // Every scratch element read below is written earlier in the same call
   // (e_b by the budget MLP, kept_local[vis_off[b] ..] by the select kernel
   // before compaction reads it), so nothing has to be cleared first.
-  g_launches++;
-  launch_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.bud_w1),
-                      static_cast<const __nv_bfloat16*>(m->w.bud_w2), d.h_ctrl, B, e_b, s);
+  {
+    Launch L(m, SVL_TAG_BUDGET_EMBED, s);
+    launch_budget_embed(budget, static_cast<const __nv_bfloat16*>(m->w.bud_w1),
+                        static_cast<const __nv_bfloat16*>(m->w.bud_w2), d.h_ctrl, B, e_b, s);
+  }
   if (n_vis_total > 0) {
     GemmParams p = base_params(m);
     if (!make_map(&p.mapA, vis_feats, n_vis_total, d.c_vis)) return SVL_ERR_INVALID_ARG;
@@ -1545,9 +1615,8 @@ extern "C" svl_status svl_score_select_noalloc(svl_model* m, int32_t B, int32_t 
     p.w2 = static_cast<const __nv_bfloat16*>(m->w.ctrl_w2);
     p.c2 = m->w.ctrl_c2;
     p.b_box_rows = d.h_ctrl;
-    g_launches++;
-    if (launch_gemm(d.h_ctrl <= 64 ? EPI_SCORE : EPI_SCORE_WIDE, p, gemm_grid(m, p.grid_m), s) != cudaSuccess)
-      return SVL_ERR_CUDA;
+    st = launch(d.h_ctrl <= 64 ? EPI_SCORE : EPI_SCORE_WIDE, m, SVL_TAG_SCORE, p, p.grid_m, s);
+    if (st != SVL_OK) return st;
   }
   SelectArgs a;
   std::memset(&a, 0, sizeof(a));
@@ -1568,9 +1637,13 @@ extern "C" svl_status svl_score_select_noalloc(svl_model* m, int32_t B, int32_t 
   a.k_out = k;
   a.flags = sample_flags;
   a.kept_local = kept_local;
-  g_launches++;
-  launch_select(a, B, s);
-  g_launches++;
-  launch_compact(B, vis_off, k, kept_local, kept_idx, kept_off, nullptr, s);
+  {
+    Launch L1(m, SVL_TAG_SELECT, s);
+    launch_select(a, B, s);
+  }
+  {
+    Launch L2(m, SVL_TAG_SELECT, s);
+    launch_compact(B, vis_off, k, kept_local, kept_idx, kept_off, nullptr, s);
+  }
   return last_error();
 }

@@ -113,7 +113,13 @@ __global__ void __launch_bounds__(kDecWarps * 32, 4) decode_attn_kernel(DecAttnA
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, tid = threadIdx.x;
   const int kvh = h / (a.A / a.Akv);
   const int len = a.cache_len[b];
-  if (len < 0 || len >= a.max_len) return;  // reported by decode_prep
+  if (len < 0 || len >= a.max_len) {
+    // full (or corrupt) cache, reported by decode_prep: the head's output is
+    // zero, so the step's logits for this sample are defined, and nothing is
+    // appended
+    if (tid < DH) a.out[static_cast<size_t>(b) * a.ldo + h * DH + tid] = __float2bfloat16(0.f);
+    return;
+  }
   const __nv_bfloat16* knew = a.k + static_cast<size_t>(b) * a.dkv + kvh * DH;
   if (tid < DH) {
     sq[tid] = __bfloat162float(a.q[static_cast<size_t>(b) * a.ldq + h * DH + tid]) * a.scale;
@@ -246,7 +252,7 @@ SVL_DEVINL void arg_better(float x, int v, float& best, int& idx) {
 }
 
 __global__ void __launch_bounds__(kFinThreads) decode_finish_kernel(int B, int V, const float* logits, int* next_token,
-                                                                    int* cache_len) {
+                                                                    int* cache_len, int max_len) {
   __shared__ float bv[kFinThreads / 32];
   __shared__ int bi[kFinThreads / 32];
   pdl_trigger();
@@ -280,13 +286,18 @@ __global__ void __launch_bounds__(kFinThreads) decode_finish_kernel(int B, int V
   __syncthreads();
   if (tid == 0) {
     for (int w = 1; w < kFinThreads / 32; ++w) arg_better(bv[w], bi[w], best, idx);
-    if (next_token) next_token[b] = idx == 0x7fffffff ? 0 : idx;
-    cache_len[b] += 1;
+    // a sample whose cache was already full took no step: its length stays
+    // and it has no next token
+    const int len = cache_len[b];
+    const bool stepped = len >= 0 && len < max_len;
+    if (next_token) next_token[b] = !stepped ? -1 : (idx == 0x7fffffff ? 0 : idx);
+    if (stepped) cache_len[b] = len + 1;
   }
 }
 
-void launch_decode_finish(int B, int V, const float* logits, int* next_token, int* cache_len, cudaStream_t s) {
-  launch_pdl(decode_finish_kernel, B, kFinThreads, 0, s, B, V, logits, next_token, cache_len);
+void launch_decode_finish(int B, int V, const float* logits, int* next_token, int* cache_len, int max_len,
+                          cudaStream_t s) {
+  launch_pdl(decode_finish_kernel, B, kFinThreads, 0, s, B, V, logits, next_token, cache_len, max_len);
 }
 
 }  // namespace svl

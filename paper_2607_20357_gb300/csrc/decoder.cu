@@ -90,11 +90,9 @@ __device__ int split_k_tail(int4* tiles, int count, int cap, int num_sms, int un
   info[0] = count;
   info[1] = 0;
   info[2] = 1;
-  const int r = count % num_sms;
-  if (r == 0 || 2 * r > num_sms) return count;
-  int sp = min(min(num_sms / r, 8), units / r);
-  sp = min(sp, 1 + (cap - count) / r);
+  const int sp = ksplit_shares(count, cap, num_sms, units);
   if (sp < 2) return count;
+  const int r = count % num_sms;
   const int first = count - r;
   for (int part = 1; part < sp; ++part)
     for (int i = 0; i < r; ++i) tiles[count + (part - 1) * r + i] = tiles[first + i];

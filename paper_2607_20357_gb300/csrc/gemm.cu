@@ -769,6 +769,24 @@ static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t strea
   return launch_pdl(gemm_kernel<KIND, F8, THIN>, grid, kGemmThreads, smem, stream, p);
 }
 
+template <int KIND, bool F8, bool THIN>
+static int blocks_per_sm_kind() {
+  constexpr int smem = StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256;
+  int n = 0;
+  if (cudaFuncSetAttribute(gemm_kernel<KIND, F8, THIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+          cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemm_kernel<KIND, F8, THIN>, kGemmThreads, smem) !=
+          cudaSuccess)
+    return 0;
+  return n;
+}
+
+int gemm_resid_blocks_per_sm(bool e4m3) {
+  const int a = e4m3 ? blocks_per_sm_kind<EPI_RESID, true, false>() : blocks_per_sm_kind<EPI_RESID, false, false>();
+  const int b = e4m3 ? blocks_per_sm_kind<EPI_RESID, true, true>() : blocks_per_sm_kind<EPI_RESID, false, true>();
+  return a < b ? a : b;
+}
+
 cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3, bool thin) {
   if (e4m3 && (!p.a_scale || !p.b_scale[0])) return cudaErrorInvalidValue;
   if (thin) {

@@ -106,4 +106,8 @@ struct GemmParams {
 cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3 = false,
                         bool thin = false);
 
+// CTAs of the residual (EPI_RESID) GEMM that fit on one SM at once, the
+// smaller of the wide and THIN instantiations (0 if the query fails).
+int gemm_resid_blocks_per_sm(bool e4m3);
+
 }  // namespace svl

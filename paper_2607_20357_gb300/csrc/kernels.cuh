@@ -78,7 +78,8 @@ SVL_DEVINL int find_sample(const int* cu, int B, int r) {
 }
 
 // ---------------------------------------------------------------- e4m3 operands
-// Per-row e4m3 quantisation of bf16 rows. Row r of src holds G groups of kg
+// Per-row e4m3 quantisation of bf16 rows (times a gain vector when given:
+// the input norm's gain of the QKV and gate/up projections). Row r of src holds G groups of kg
 // columns; dst row r holds G groups of kgp >= kg codes (the tail of each
 // group zero, so that every group starts on a 128-byte K block). Only the
 // groups active for the row's sample are read and quantised (the others are
@@ -86,6 +87,7 @@ SVL_DEVINL int find_sample(const int* cu, int B, int r) {
 // Rows at or past cu_seqlens[B] (when given) are left untouched.
 struct QuantArgs {
   const __nv_bfloat16* src;
+  const __nv_bfloat16* gain;  // [G * kg] multiplies each row before quantising, or nullptr
   int64_t ld_src;
   int64_t rows;
   int G, kg, kgp;
@@ -129,7 +131,8 @@ struct DecAttnArgs {
   __nv_bfloat16* out;       // [B, A*dh]
 };
 void launch_decode_attn(const DecAttnArgs& a, cudaStream_t s);
-void launch_decode_finish(int B, int V, const float* logits, int* next_token, int* cache_len, cudaStream_t s);
+void launch_decode_finish(int B, int V, const float* logits, int* next_token, int* cache_len, int max_len,
+                          cudaStream_t s);
 
 // ---------------------------------------------------------------- decoder
 struct ScheduleArgs {
@@ -152,6 +155,25 @@ struct ScheduleArgs {
   uint32_t* status;
 };
 void launch_schedule(const ScheduleArgs& a, cudaStream_t s);
+
+// Number of K shares the last wave of a residual GEMM's `count` tiles is cut
+// into (1: no split). The persistent grid has num_sms CTAs, so the last wave
+// holds r = count % num_sms tiles; it is split only when at most half full,
+// into at most 8 and at most num_sms / r shares, within the `units` partial
+// tiles of the workspace and the list capacity `cap`. The shares meet inside
+// one launch, so the caller passes units = 0 unless every CTA of the grid is
+// resident at once. Shared by the device schedule and svl_ksplit_plan.
+__host__ __device__ inline int ksplit_shares(int count, int cap, int num_sms, int units) {
+  if (num_sms <= 0 || count <= 0) return 1;
+  const int r = count % num_sms;
+  if (r == 0 || 2 * r > num_sms) return 1;
+  int sp = num_sms / r;
+  sp = sp < 8 ? sp : 8;
+  sp = sp < units / r ? sp : units / r;
+  const int room = 1 + (cap - count) / r;
+  sp = sp < room ? sp : room;
+  return sp < 2 ? 1 : sp;
+}
 
 // LLM-side compute controller (Sec. 3.2, Eq. 7), one block per sample: the
 // budget token's state after the prefix layers plus MLP_kappa(PE(kappa)),

@@ -24,6 +24,7 @@ SVL_FLAG_OVER_BUDGET = 1
 SVL_FLAG_GROUPS_DROPPED = 2
 SVL_DEV_NONFINITE, SVL_DEV_TIMEOUT, SVL_DEV_BAD_INDEX = 1, 2, 4
 SVL_GEMM_BF16, SVL_GEMM_E4M3 = 0, 1
+SVL_LAYER_QKV, SVL_LAYER_ATTN, SVL_LAYER_OPROJ, SVL_LAYER_GATEUP, SVL_LAYER_DOWN = 0, 1, 2, 3, 4
 
 SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_score_select", "svl_pack",
            "svl_gated_prefill", "svl_flops", "svl_get_device_status", "svl_status_string", "svl_launch_count",
@@ -31,7 +32,7 @@ SYMBOLS = ["svl_model_create", "svl_model_destroy", "svl_workspace_size", "svl_s
            "svl_tag_name", "svl_score_select_noalloc", "svl_profile_launches", "svl_selftest_wait_timeout",
            "svl_workspace_size_for", "svl_score_select_paper", "svl_pack_controlled", "svl_controlled_prefill",
            "svl_kv_cache_size", "svl_gated_prefill_kv", "svl_decode_workspace_size", "svl_decode_step",
-           "svl_quantize_rows_e4m3", "svl_gemm_e4m3"]
+           "svl_quantize_rows_e4m3", "svl_gemm_e4m3", "svl_layer_stage", "svl_ksplit_plan"]
 
 TAGS = ["budget_embed", "score", "select", "pack", "projector", "schedule", "rmsnorm", "qkv_gemm", "attention",
         "o_gemm", "gateup_gemm", "down_gemm", "lm_head", "host_copy", "quant"]
@@ -123,10 +124,14 @@ def lib():
         L.svl_selftest_wait_timeout.restype = ctypes.c_int
         L.svl_workspace_size_for.argtypes = [vp, ctypes.c_uint32, i32, i64, i64]
         L.svl_workspace_size_for.restype = sz
-        L.svl_quantize_rows_e4m3.argtypes = [vp, i64, i32, i64, vp, i64, vp, vp]
+        L.svl_quantize_rows_e4m3.argtypes = [vp, vp, i64, i32, i64, vp, i64, vp, vp]
         L.svl_quantize_rows_e4m3.restype = ctypes.c_int
         L.svl_gemm_e4m3.argtypes = [vp] * 5 + [i32, i32, i32, vp, vp]
         L.svl_gemm_e4m3.restype = ctypes.c_int
+        L.svl_layer_stage.argtypes = [vp, i32, i32, i32, i32] + [vp] * 10 + [vp, sz, vp]
+        L.svl_layer_stage.restype = ctypes.c_int
+        L.svl_ksplit_plan.argtypes = [i32] * 5
+        L.svl_ksplit_plan.restype = i32
         _lib = L
     return _lib
 
@@ -212,14 +217,28 @@ def svl_gated_prefill_kv(model, B, t_cap, X, cu_seqlens, pos, layer_gate, group_
         int(workspace_bytes), _stream(stream)))
 
 
-def svl_quantize_rows_e4m3(src, rows, cols, ld_src, dst, ld_dst, scale, stream=None):
+def svl_quantize_rows_e4m3(src, rows, cols, ld_src, dst, ld_dst, scale, stream=None, gain=None):
     _check("svl_quantize_rows_e4m3", lib().svl_quantize_rows_e4m3(
-        _p(src), int(rows), int(cols), int(ld_src), _p(dst), int(ld_dst), _p(scale), _stream(stream)))
+        _p(src), _p(gain), int(rows), int(cols), int(ld_src), _p(dst), int(ld_dst), _p(scale), _stream(stream)))
 
 
 def svl_gemm_e4m3(model, A, a_scale, B, b_scale, M, N, K, C, stream=None):
     _check("svl_gemm_e4m3", lib().svl_gemm_e4m3(model, _p(A), _p(a_scale), _p(B), _p(b_scale), int(M), int(N),
                                                 int(K), _p(C), _stream(stream)))
+
+
+def svl_layer_stage(model, stage, layer, B, t_cap, X, cu_seqlens, pos, layer_gate, group_gate, q=None, k=None,
+                    vt=None, ao=None, h=None, workspace=None, workspace_bytes=0, stream=None):
+    """One stage of one decoder layer on caller buffers (see svl.h)."""
+    _check("svl_layer_stage", lib().svl_layer_stage(
+        model, int(stage), int(layer), int(B), int(t_cap), _p(X), _p(cu_seqlens), _p(pos), _p(layer_gate),
+        _p(group_gate), _p(q), _p(k), _p(vt), _p(ao), _p(h), _p(workspace), int(workspace_bytes),
+        _stream(stream)))
+
+
+def svl_ksplit_plan(tiles, cap, num_sms, blocks_per_sm, units) -> int:
+    """K shares of a residual GEMM's last wave (1 = no split); host only."""
+    return int(lib().svl_ksplit_plan(int(tiles), int(cap), int(num_sms), int(blocks_per_sm), int(units)))
 
 
 def svl_decode_workspace_size(model, B) -> int:

@@ -7,10 +7,14 @@ import os
 import sys
 
 sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__)))))
-from oracle import smartvl_oracle as O  # noqa: E402
-from paper_2607_20357_gb300.synth import WORKLOADS  # noqa: E402
+from collections import namedtuple  # noqa: E402
 
-dims = WORKLOADS["llava"].dims
+from oracle import smartvl_oracle as O  # noqa: E402
+
+# LLaVA-1.5-7B decoder widths (32 layers, d 4096, MHA, SwiGLU 11008, vocab
+# 32000, 4 head groups), written out here so that only the oracle computes
+Dims = namedtuple("Dims", "n_layers d_model d_kv d_ffn vocab n_groups")
+dims = Dims(n_layers=32, d_model=4096, d_kv=4096, d_ffn=11008, vocab=32000, n_groups=4)
 ks = {}
 for b in ("0.1", "0.25", "0.5", "0.75", "1.0"):
     ks[b] = O.budget_keep_count(dims, float(b), 576, 64, [dims.n_groups] * dims.n_layers)[0]

@@ -89,9 +89,17 @@ def numpy_weights_lazy(w):
 class Case:
     """Seeded model + batch on the GPU and the oracle's view of both."""
 
-    def __init__(self, dims, wl, seed, batch=None, budget=None, max_seq=8192, std=0.02, gemm_format=svl.SVL_GEMM_BF16):
+    def __init__(self, dims, wl, seed, batch=None, budget=None, max_seq=8192, std=0.02, gemm_format=svl.SVL_GEMM_BF16,
+                 random_gains=False):
         self.dims = dims
         w = synth.make_weights(dims, seed, std=std)
+        if random_gains:
+            # RMSNorm gains drawn from U[0.5, 1.5] instead of 1
+            g = torch.Generator().manual_seed(seed + 7919)
+            for lw in w["layers"]:
+                for key in ("attn_norm", "ffn_norm"):
+                    lw[key] = (0.5 + torch.rand(dims.d_model, generator=g)).to(torch.bfloat16)
+            w["final_norm"] = (0.5 + torch.rand(dims.d_model, generator=g)).to(torch.bfloat16)
         b = synth.make_batch(wl, seed, budget=budget, batch=batch, dims=dims)
         self.w_np = O.to_numpy_weights(w)
         self.b_np = O.to_numpy_batch(b)

@@ -85,15 +85,48 @@ def test_e4m3_entry_points_reject_bad_args_without_gpu(svl_lib):
     base = (ctypes.addressof(buf) + 15) & ~15
     src, dst, sc = ctypes.c_void_p(base), ctypes.c_void_p(base + 1024), ctypes.c_void_p(base + 2048)
     q = svl_lib.svl_quantize_rows_e4m3
-    assert q(None, 4, 16, 16, dst, 16, sc, None) == 1        # null source
-    assert q(src, 4, 12, 16, dst, 16, sc, None) == 1         # cols not a multiple of 8
-    assert q(src, 4, 16, 12, dst, 16, sc, None) == 1         # ld_src < cols
-    assert q(src, 4, 16, 16, dst, 8, sc, None) == 1          # ld_dst < cols
-    assert q(src, -1, 16, 16, dst, 16, sc, None) == 1        # negative rows
-    assert q(ctypes.c_void_p(base + 2), 4, 16, 16, dst, 16, sc, None) == 1  # misaligned source
+    assert q(None, None, 4, 16, 16, dst, 16, sc, None) == 1        # null source
+    assert q(src, None, 4, 12, 16, dst, 16, sc, None) == 1         # cols not a multiple of 8
+    assert q(src, None, 4, 16, 12, dst, 16, sc, None) == 1         # ld_src < cols
+    assert q(src, None, 4, 16, 16, dst, 8, sc, None) == 1          # ld_dst < cols
+    assert q(src, None, -1, 16, 16, dst, 16, sc, None) == 1        # negative rows
+    assert q(ctypes.c_void_p(base + 2), None, 4, 16, 16, dst, 16, sc, None) == 1  # misaligned source
+    assert q(src, ctypes.c_void_p(base + 3074), 4, 16, 16, dst, 16, sc, None) == 1  # misaligned gain
     g = svl_lib.svl_gemm_e4m3
     assert g(None, src, sc, dst, sc, 128, 32, 128, sc, None) == 1  # no model
     d = svl.model_desc(synth.WORKLOADS["tiny"].dims, 256, gemm_format=7)  # unknown operand format
     w = svl.Weights()
     h = ctypes.c_void_p()
     assert svl_lib.svl_model_create(ctypes.byref(d), ctypes.byref(w), ctypes.byref(h)) == 1
+
+
+def test_ksplit_plan_launch_rule(svl_lib):
+    """The K-split launch rule on the host: no split unless the persistent
+    grid is resident at once, and otherwise the documented share count."""
+    plan = svl.svl_ksplit_plan
+    sms = 152
+    # LLaVA-7B O projection at b = 0.5: 41 row tiles x 16 column tiles = 656
+    # tiles, last wave 656 - 4 * 152 = 48 tiles -> 152 // 48 = 3 shares
+    assert plan(656, 1024, sms, 1, 256) == 3
+    assert plan(656, 1024, sms, 0, 256) == 1          # grid not resident at once: never split
+    assert plan(656, 1024, sms, 1, 0) == 1            # no partial-tile workspace
+    assert plan(4 * sms, 1024, sms, 1, 256) == 1      # full last wave
+    assert plan(3 * sms + 77, 1024, sms, 1, 256) == 1  # last wave more than half full
+    assert plan(3 * sms + 76, 1024, sms, 1, 256) == 2  # exactly half full
+    assert plan(16, 1024, sms, 1, 256) == 8            # decode-sized: at most 8 shares
+    assert plan(16, 1024, sms, 1, 64) == 4             # limited by the partial tiles (64 // 16)
+    assert plan(16, 40, sms, 1, 256) == 2              # limited by the list capacity (1 + 24 // 16)
+    assert plan(1, 1024, sms, 1, 256) == 8
+    assert plan(0, 1024, sms, 1, 256) == 1
+    # brute force over small grids against the stated rule
+    for n in (4, 7, 16):
+        for tiles in range(0, 5 * n):
+            for units in (0, 3, 8, 40):
+                for cap in (tiles, tiles + 5, tiles + 100):
+                    r = tiles % n if tiles else 0
+                    want = 1
+                    if r and 2 * r <= n:
+                        sp = min(n // r, 8, units // r, 1 + (cap - tiles) // r)
+                        want = sp if sp >= 2 else 1
+                    assert plan(tiles, cap, n, 1, units) == want, (n, tiles, units, cap)
+                    assert plan(tiles, cap, n, 0, units) == 1

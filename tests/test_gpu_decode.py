@@ -111,3 +111,63 @@ def test_decode_llava_width_two_layers():
             got = r["logits"][t][i].double().numpy()
             assert rel_err(got, s32[t]["logits"]) < bar_for(s32[t], s16[t], "logits"), (i, t)
     case.close()
+
+
+def test_decode_past_full_cache_saturates():
+    """Stepping a batch past max_len: a sample whose cache is full takes no
+    step -- its length stays at max_len, its next token is -1 -- and the
+    status word reports SVL_DEV_BAD_INDEX, while the other samples keep
+    decoding as before (their logits equal those of a run that never hit
+    the limit)."""
+    dims = synth.reduced(TINY.dims, n_layers=2)
+    n_vis, s_text = [40, 20], [10, 6]
+    wl = TINY
+    case = Case(dims, wl, seed=75, batch=None, max_seq=256)
+    b = synth.make_batch(wl, 75, n_vis_list=n_vis, s_text_list=s_text, keep_list=[-1, -1], budget_list=[1.0, 1.0],
+                         dims=dims)
+    B = 2
+    b["group_gate"] = torch.ones(B, dims.n_layers, dims.n_groups, dtype=torch.uint8)
+    b["layer_gate"] = torch.ones(B, dims.n_layers, dtype=torch.uint8)
+    bd = {k: (v.cuda() if isinstance(v, torch.Tensor) else v) for k, v in b.items()}
+    m = case.model
+    fed = torch.randint(0, dims.vocab, (5, B), generator=torch.Generator().manual_seed(76), dtype=torch.int32)
+
+    def run(max_len):
+        out = m.run(bd, stages=("select", "pack"))
+        nv, nt = int(bd["vis"].shape[0]), int(bd["text_ids"].shape[0])
+        ws, wsb = m.workspace(B, nv, nt, "cuda", ("prefill",))
+        kv = torch.zeros(svl.svl_kv_cache_size(m.handle, B, max_len), dtype=torch.uint8, device="cuda")
+        cache_len = torch.zeros(B, dtype=torch.int32, device="cuda")
+        svl.svl_gated_prefill_kv(m.handle, B, nv + nt, out["X"], out["cu_seqlens"], out["pos"], bd["layer_gate"],
+                                 bd["group_gate"], svl.SVL_LOGITS_LAST, out["logits"], kv, max_len, cache_len, ws, wsb)
+        dws = torch.empty(svl.svl_decode_workspace_size(m.handle, B), dtype=torch.uint8, device="cuda")
+        logits = torch.empty(B, dims.vocab, dtype=torch.float32, device="cuda")
+        nxt = torch.empty(B, dtype=torch.int32, device="cuda")
+        lens, nexts, lg = [], [], []
+        for t in range(fed.shape[0]):
+            svl.svl_decode_step(m.handle, B, fed[t].cuda(), kv, max_len, cache_len, bd["layer_gate"],
+                                bd["group_gate"], logits, nxt, dws, dws.numel())
+            lens.append(cache_len.cpu().clone())
+            nexts.append(nxt.cpu().clone())
+            lg.append(logits.cpu().clone())
+        torch.cuda.synchronize()
+        return np.diff(out["cu_seqlens"].cpu().numpy()), lens, nexts, lg
+
+    prompt, lens_ok, _, lg_ok = run(128)  # never full
+    assert svl.svl_get_device_status(m.handle) == 0
+    full = int(prompt.max())
+    assert prompt[0] == full > prompt[1]
+    max_len = full + 2  # sample 0 fills after two steps
+    _, lens, nexts, lg = run(max_len)
+    status = svl.svl_get_device_status(m.handle)
+    assert status & svl.SVL_DEV_BAD_INDEX, status
+    for t in range(fed.shape[0]):
+        assert int(lens[t][0]) == min(full + t + 1, max_len)
+        assert int(lens[t][1]) == prompt[1] + t + 1
+        if full + t >= max_len:
+            assert int(nexts[t][0]) == -1
+        else:
+            assert int(nexts[t][0]) >= 0
+        # the sample that still has room decodes exactly as without the limit
+        np.testing.assert_array_equal(lg[t][1].numpy(), lg_ok[t][1].numpy())
+    case.close()

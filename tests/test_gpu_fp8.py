@@ -7,16 +7,21 @@ float32 on both sides from the same bf16 inputs, so they must agree exactly.
 The e4m3 GEMM on its own (svl_gemm_e4m3) must equal the exact product of
 the decoded codes times both scales to float32 accumulation error.
 
-The forward compares with the oracle's fp8 definition. An activation is
+The forward compares with the oracle's plain fp8 definition: e4m3 of
+RMSNorm(X) * gain (QKV, gate/up), of the attention output (O) and of the
+SwiGLU output (down) against e4m3 of W as given, per row. An activation is
 quantised from values the GPU computes in float32 with bf16 storage and
 the oracle in float64: where the two differ by a bf16 step, a value can sit
 on opposite sides of an e4m3 rounding boundary and jump by a whole e4m3 step
-(6-12 %). The bar is therefore 1.5x the distance between the oracle's fp8
-forward with bf16 storage and with fp32 storage (the same definition under
-storage-level perturbation), at least 2e-2. The layers' update of the
-residual stream (final hidden minus the packed input rows) must also sit
-closer to the fp8 definition's than to the bf16 one's, which shows the e4m3
-arithmetic is what ran."""
+(6-12 %). The end-to-end bar is therefore 1.5x the distance between the
+oracle's fp8 forward with bf16 storage and with fp32 storage (the same
+definition under storage-level perturbation), at least 2e-2; at widths up to
+512, where that sensitivity is small, the layers' update of the residual
+stream (final hidden minus the packed input rows) must in addition lie
+within 2e-2 (L2) of the definition's. The update must also sit closer to the
+fp8 definition's than to the bf16 one's, which shows the e4m3 arithmetic is
+what ran. Per-stage checks at LLaVA-7B width (tests/test_gpu_stages.py)
+carry the element-wise claim."""
 import numpy as np
 import pytest
 import torch
@@ -125,17 +130,19 @@ def _compare(case, out, n_samples, min_compared):
         e8 = l2_err(d_got, refs["fp8"][i]["hidden"] - x0)
         e16 = l2_err(d_got, refs["bf16"][i]["hidden"] - x0)
         assert e8 < e16, (i, e8, e16)
+        if case.dims.d_model <= 512:
+            assert e8 < 2e-2, (i, e8)
         compared += 1
     assert compared >= min_compared
     return refs
 
 
-@pytest.mark.parametrize("prefix", [0, 1])
-def test_fp8_prefill_tiny_gated(prefix):
+@pytest.mark.parametrize("prefix,random_gains", [(0, False), (1, False), (0, True)])
+def test_fp8_prefill_tiny_gated(prefix, random_gains):
     dims = synth.reduced(TINY.dims, n_layers=4, n_prefix=prefix)
     wl = synth.Workload("fp8", dims, batch=6, n_vis=(40, 64), s_text=(5, 40), budgets=(1.0,),
                         gates="bern_heads", features="normal", keep_count=24)
-    case = Case(dims, wl, seed=81 + prefix, batch=6, max_seq=512, gemm_format=E4M3)
+    case = Case(dims, wl, seed=81 + prefix, batch=6, max_seq=512, gemm_format=E4M3, random_gains=random_gains)
     out = case.run()
     _compare(case, out, 6, 4)
     case.close()
