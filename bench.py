@@ -72,6 +72,8 @@ def parse():
     ap.add_argument("--no-hbm-sweep", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-fp8", action="store_true", help="skip the e4m3 (FP8 gated projections) pass")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the mixed / gating-sweep / video / Qwen passes")
     ap.add_argument("--decode-only", action="store_true",
                     help="profiling aid: only the decode measurement (bf16, and e4m3 unless --no-fp8)")
     ap.add_argument("--hbm-only", type=str, default="",
@@ -237,8 +239,14 @@ def cpu_oracle_baseline(dims, weights_cpu_layers, weights_rest, batch_cpu, budge
 
 # --------------------------------------------------------------------------- reference arm
 def run_reference(args, rank, world):
-    """The CPU oracle as the reference arm: one sample per step, layers
-    0-1 of 32 timed and scaled to the full depth."""
+    """The CPU oracle as the reference arm. One step is a bounded sample of
+    the benchmark batch: one of its samples (they cycle through the batch
+    and the budgets), its token controller, pack, final norm and LM head
+    whole and decoder layers 0-1 of 32. ``ms_per_step`` is the time of that
+    sample as measured; ``value`` is the sample's input tokens over the time
+    the whole 32-layer path would take at the measured per-layer rate
+    (front + 16 x two layers). Samples are independent, so the oracle's
+    throughput on the batch is its per-sample throughput."""
     if rank != 0:
         return
     wl = synth.WORKLOADS[args.workload]
@@ -247,28 +255,35 @@ def run_reference(args, rank, world):
     w = synth.make_weights(dims, SEED, device="cpu", layers=range(nl))
     from oracle import smartvl_oracle as O
     w_np = O.to_numpy_weights(w)
-    batches = [synth.make_batch(wl, SEED, budget=b, batch=1) for b in wl.budgets]
-    times, tokens = [], []
+    bt = synth.make_batch(wl, SEED)  # the budgets below only change k; features are the same for each
+    budgets = list(wl.budgets)
+    measured, extrapolated, tokens = [], [], []
     for i in range(args.warmup + args.steps):
-        bt = batches[i % len(batches)]
-        x = bt["vis"].double().numpy()
-        ids = bt["text_ids"].numpy()
-        t0 = time.perf_counter()
-        front, per_layer, _ = oracle_sample_seconds(dims, w_np, x, ids, float(bt["budget"][0]),
-                                                    bt["layer_gate"][0].numpy(), bt["group_gate"][0].numpy(), nl)
-        t_full = front + per_layer * dims.n_layers
+        budget = budgets[i % len(budgets)]
+        b = (i // len(budgets)) % bt["B"]
+        v0, v1 = int(bt["vis_off"][b]), int(bt["vis_off"][b + 1])
+        t0, t1 = int(bt["text_off"][b]), int(bt["text_off"][b + 1])
+        x = bt["vis"][v0:v1].double().numpy()
+        ids = bt["text_ids"][t0:t1].numpy()
+        front, per_layer, wall = oracle_sample_seconds(dims, w_np, x, ids, budget,
+                                                       bt["layer_gate"][b].numpy(), bt["group_gate"][b].numpy(), nl)
         if i >= args.warmup:
-            times.append(t_full)
+            measured.append(wall + front)  # both forward_sample calls of the step
+            extrapolated.append(front + per_layer * dims.n_layers)
             tokens.append(x.shape[0] + ids.shape[0])
-    value = sum(tokens) / sum(times)
+    value = sum(tokens) / sum(extrapolated)
     cores = os.cpu_count()
-    sample = (f"1 sample per step (budget cycling {list(wl.budgets)}); token controller, pack, final norm and "
-              f"LM head timed whole; decoder layers 0-{nl - 1} timed and scaled x{dims.n_layers // nl} to 32 layers")
+    sample = (f"per step one sample of the B={wl.batch} batch (samples and budgets {list(wl.budgets)} cycle): "
+              f"token controller, pack, final norm and LM head whole, decoder layers 0-{nl - 1} of "
+              f"{dims.n_layers}; value = sample tokens / (front + {dims.n_layers // nl} x the two layers' time)")
+    cfg = workload_config(wl, wl.batch)
+    cfg["reference_step"] = f"one sample, front + {nl} of {dims.n_layers} layers (measured); throughput per sample"
     line = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(times), "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": 1000.0 * statistics.mean(measured), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": workload_config(wl, 1), "impl": "reference",
+        "config": cfg, "impl": "reference",
+        "ms_per_full_sample_extrapolated": 1000.0 * statistics.mean(extrapolated),
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -289,6 +304,9 @@ def run_ours(args, rank, world, local_rank):
 
     weights = synth.make_weights(dims, SEED, device=dev)
     max_seq = wl.n_vis[1] + wl.s_text[1] + 64
+    if args.workload == "llava" and not args.no_workloads and not args.layers:
+        # the mixed (576 + 256) and video (4608 + 64) batches run on this model too
+        max_seq = max(max_seq, synth.WORKLOADS["video"].n_vis[1] + synth.WORKLOADS["video"].s_text[1] + 64)
     model = svl.GatedPrefill(dims, weights, max_seq=max_seq)
     if args.hbm_only:
         mults = tuple(int(x) for x in args.hbm_only.split(","))
@@ -433,6 +451,12 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and not args.no_decode:
         dec = run_decode(svl, model, batches[1], dims, dev, pk)
 
+    gated = None
+    if not args.no_workloads and not args.layers and args.workload == "llava":
+        del outs
+        torch.cuda.empty_cache()
+        gated = run_gated_workloads(args, svl, model, dev, pk)
+
     fp8 = None
     if rank == 0 and not args.no_fp8:
         model.close()  # its workspace and outputs go; the e4m3 model holds its own weight codes
@@ -461,10 +485,233 @@ def run_ours(args, rank, world, local_rank):
             "per_budget": per_budget, "roofline": roofline, "kernels": kernels,
             "gpu_launches": int(launches), "gpu_launches_per_step": launches / args.steps,
             "wall_s_timed": t_wall, "clocks": clk.summary(), "e2e": e2e, "cpu_baseline": cpu,
-            "hbm_kernels_sweep": hbm, "decode": dec, "fp8": fp8,
+            "hbm_kernels_sweep": hbm, "decode": dec, "fp8": fp8, "gated_workloads": gated,
         }
-        print(json.dumps(line), flush=True)
+        # the full record first (no "metric" key), then the bench line:
+        # required keys, roofline, clocks, e2e, CPU baseline and a compact
+        # summary, short enough to survive a log tail
+        print(json.dumps({"bench_details": line}), flush=True)
+        keep = ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+                "vs_baseline", "dtype", "data", "gpu_launches", "roofline", "clocks", "e2e", "cpu_baseline")
+        main_line = {k: line[k] for k in keep}
+        main_line["summary"] = compact_summary(line, gated)
+        main_line["exec_tflops"] = round(line["exec_tflops"], 1)
+        main_line["config"] = {"workload": line["config"]["workload"], "batch": B,
+                               "gates": line["config"]["gates"], "l2": line["config"]["l2"],
+                               "parallelism": line["config"]["parallelism"]}
+        main_line["roofline"] = {k: v for k, v in roofline.items() if k not in ("traffic_note", "timing")}
+        main_line["cpu_baseline"] = dict(cpu, sample=cpu["sample"][:160]) if cpu else None
+        print(json.dumps(main_line), flush=True)
     model.close()
+
+
+def timed_steps(svl, model, batches, outs, steps, warmup, live_tags=("gateup_gemm",)):
+    """`warmup` untimed steps, then `steps` steps cycling over `batches`,
+    CUDA events around each step on the launching stream and around every
+    launch of the kernels named in `live_tags` only. Fails on a non-zero
+    device status word. Returns per-step ms, the live kernel times, the
+    clock summary and the launch count of the timed steps."""
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        model.run(batches[i % len(batches)], out=outs[i % len(batches)])
+
+    for i in range(warmup):
+        step(i)
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    launches0 = svl.svl_launch_count()
+    svl.svl_profile_start(model.handle, tags=list(live_tags))
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        for i in range(steps):
+            ev[i][0].record(stream)
+            step(i)
+            ev[i][1].record(stream)
+        torch.cuda.synchronize()
+    live = svl.svl_profile_stop(model.handle)
+    launches = svl.svl_launch_count() - launches0
+    status = svl.svl_get_device_status(model.handle)
+    if status:
+        raise RuntimeError(f"device status {status:#x} in a timed pass")
+    return [a.elapsed_time(b) for a, b in ev], live, clk.summary(), launches
+
+
+def batch_accounting(svl, model, dims, bt, out):
+    """Input tokens, executed FLOPs (svl_flops: post-gating, causal
+    attention, last-row LM head), per-kind FLOPs, mean k and the executed
+    fraction alpha of the decoder's (layer, group) pairs of one batch."""
+    k = out["k"].cpu().numpy()
+    nv = (bt["vis_off"][1:] - bt["vis_off"][:-1]).cpu().numpy()
+    st = (bt["text_off"][1:] - bt["text_off"][:-1]).cpu().numpy()
+    lg, gg = bt["layer_gate"].cpu(), bt["group_gate"].cpu()
+    on = effective_on(bt, dims)
+    return {"tokens": int(nv.sum() + st.sum()), "fexec": executed_flops(svl, model.desc, k, st, nv, lg, gg),
+            "kind": per_kind_flops(dims, k, st, lg.numpy(), gg.numpy()), "k_mean": float(k.mean()),
+            "alpha": float(on.float().mean())}
+
+
+def pass_summary(svl, model, dims, batches, outs, step_ms, live, pk, label_key=None, labels=None):
+    """Per-batch rows (ms per step, tokens/s, executed TFLOP/s) and the
+    whole pass: tokens/s, executed TFLOP/s and the gate/up GEMM's rate from
+    the live events against the measured sustained bf16 peak."""
+    peak = pk["bf16_tflops_sustained"]
+    rows, tokens, fexec, kind = [], 0, 0.0, {}
+    for j, bt in enumerate(batches):
+        idx = list(range(j, len(step_ms), len(batches)))
+        if not idx:
+            continue
+        acc = batch_accounting(svl, model, dims, bt, outs[j])
+        ms = statistics.mean(step_ms[i] for i in idx)
+        row = {"ms_per_step": round(ms, 3), "tokens_per_s": round(acc["tokens"] / (ms / 1e3), 1),
+               "exec_tflops": round(acc["fexec"] / (ms / 1e3) / 1e12, 1),
+               "exec_tflop_per_step": acc["fexec"] / 1e12, "k_mean": round(acc["k_mean"], 1),
+               "alpha": round(acc["alpha"], 4)}
+        if labels is not None:
+            row[label_key] = labels[j]
+        rows.append(row)
+        tokens += acc["tokens"] * len(idx)
+        fexec += acc["fexec"] * len(idx)
+        for t, f in acc["kind"].items():
+            kind[t] = kind.get(t, 0.0) + f * len(idx)
+    total_s = sum(step_ms) / 1e3
+    out = {"tokens_per_s": round(tokens / total_s, 1), "exec_tflops": round(fexec / total_s / 1e12, 1),
+           "exec_frac_of_peak": round(fexec / total_s / 1e12 / peak, 4), "ms_per_step": sum(step_ms) / len(step_ms),
+           "rows": rows}
+    for tag in ("gateup_gemm", "attention"):
+        if tag in live and kind.get(tag):
+            n_l, t_l = live[tag]
+            ach = kind[tag] / (t_l / 1e3) / 1e12
+            out["roofline" if tag == "gateup_gemm" else "attention_roofline"] = {
+                "kernel": tag, "bound": "tensor", "achieved": round(ach, 1), "peak": peak, "unit": "TFLOP/s",
+                "frac": round(ach / peak, 4), "launches": n_l}
+    return out
+
+
+def scaling_vs(rows, key, ref_value):
+    """t(x)/t(ref) / (F(x)/F(ref)) - 1 for each row, against the row whose
+    `key` equals ref_value (linear scaling in executed FLOPs gives 0)."""
+    ref = [r for r in rows if abs(r[key] - ref_value) < 1e-9]
+    if not ref:
+        return
+    for r in rows:
+        r["time_vs_flops_ratio_minus_1"] = round((r["ms_per_step"] / ref[0]["ms_per_step"]) /
+                                                 (r["exec_tflop_per_step"] / ref[0]["exec_tflop_per_step"]) - 1.0, 4)
+
+
+def gated_batch(wl, seed, dev, alpha=1.0, layer_skip=0.0, keep=288):
+    """The mixed-serving batch shape (576 visual tokens, text U[16, 256]) at a
+    fixed kept count, with exactly round(alpha * G) head groups on in every
+    (sample, layer) -- which ones drawn at random -- and a fraction
+    `layer_skip` of each sample's layers skipped (drawn at random)."""
+    bt = synth.make_batch(wl, seed, budget=1.0, device="cpu")
+    B, L, G = bt["B"], wl.dims.n_layers, wl.dims.n_groups
+    g = torch.Generator().manual_seed(seed + 5)
+    n_on = max(1, round(alpha * G))
+    order = torch.rand(B, L, G, generator=g).argsort(dim=2)
+    gg = (order < n_on).to(torch.uint8)
+    lg = torch.ones(B, L, dtype=torch.uint8)
+    n_skip = round(layer_skip * L)
+    if n_skip:
+        skip = torch.rand(B, L, generator=g).argsort(dim=1) < n_skip
+        lg[skip] = 0
+    bt["group_gate"], bt["layer_gate"] = gg, lg
+    bt["keep_count"] = torch.full((B,), keep, dtype=torch.int32)
+    return {k: (v.to(dev) if isinstance(v, torch.Tensor) else v) for k, v in bt.items()}
+
+
+def run_gated_workloads(args, svl, llava_model, dev, pk):
+    """The other configurations of the benchmark suite, each with its own
+    warm-up and timed steps (CUDA events, clocks sampled):
+
+    * mixed serving (B = 64, text U[16, 256], per-sample budgets U[0.1, 1],
+      head gates Bern(sqrt(b)) and layer skips, LLaVA-7B decoder);
+    * a gating sweep on the mixed shape at a fixed kept count (288 of 576):
+      head-group density alpha = 1, 0.75, 0.5, 0.25, and half the layers
+      skipped -- wall time against executed FLOPs, which shows that gated-off
+      heads, channels and layers are never issued;
+    * video (B = 2, 8 x 576 visual tokens, budgets 0.1 / 0.25 / 0.5);
+    * Qwen2-VL-7B shapes (B = 8, 256..2048 visual tokens, GQA 28/4, vocab
+      152,064, per-sample budgets U[0.2, 1]), its own weights.
+    """
+    res = {}
+    w_steps, t_steps = max(3, min(args.warmup, 3)), max(4, min(args.steps, 6))
+    dims = llava_model.dims
+    wl_m = synth.WORKLOADS["mixed"]
+    bts = [synth.make_batch(wl_m, SEED + 301 + i, device=dev) for i in range(2)]
+    outs = [llava_model.alloc_outputs(bt) for bt in bts]
+    ms, live, clk, _ = timed_steps(svl, llava_model, bts, outs, t_steps, w_steps)
+    res["mixed"] = dict(pass_summary(svl, llava_model, dims, bts, outs, ms, live, pk), clocks=clk)
+    del outs
+    # gating sweep at fixed k
+    points = [("alpha", 1.0, 0.0), ("alpha", 0.75, 0.0), ("alpha", 0.5, 0.0), ("alpha", 0.25, 0.0),
+              ("layer_skip", 1.0, 0.5)]
+    rows = []
+    for kind, alpha, skip in points:
+        bt = gated_batch(wl_m, SEED + 401, dev, alpha=alpha, layer_skip=skip)
+        out = [llava_model.alloc_outputs(bt)]
+        ms, live, clk, _ = timed_steps(svl, llava_model, [bt], out, max(3, t_steps // 2), 2)
+        r = pass_summary(svl, llava_model, dims, [bt], out, ms, live, pk)["rows"][0]
+        r.update({"point": f"{kind} {alpha if kind == 'alpha' else skip}", "sm_mhz": clk.get("sm_mhz")})
+        rows.append(r)
+    ref = rows[0]
+    for r in rows:
+        r["t_over_t1"] = round(r["ms_per_step"] / ref["ms_per_step"], 4)
+        r["f_over_f1"] = round(r["exec_tflop_per_step"] / ref["exec_tflop_per_step"], 4)
+        r["time_vs_flops_ratio_minus_1"] = round(r["t_over_t1"] / r["f_over_f1"] - 1.0, 4)
+    res["gating_sweep"] = {"batch": "mixed shape, B=64, keep 288 of 576, layer gates on unless skipped",
+                           "rows": rows}
+    # video
+    wl_v = synth.WORKLOADS["video"]
+    bts = [synth.make_batch(wl_v, SEED + 501, budget=b, device=dev) for b in wl_v.budgets]
+    outs = [llava_model.alloc_outputs(bt) for bt in bts]
+    ms, live, clk, _ = timed_steps(svl, llava_model, bts, outs, 2 * len(bts), w_steps,
+                                   live_tags=("gateup_gemm", "attention"))
+    v = pass_summary(svl, llava_model, dims, bts, outs, ms, live, pk, "budget", list(wl_v.budgets))
+    scaling_vs(v["rows"], "budget", 0.5)
+    v["clocks"] = clk
+    res["video"] = v
+    del outs
+    # Qwen2-VL-7B shapes
+    wl_q = synth.WORKLOADS["qwen"]
+    wq = synth.make_weights(wl_q.dims, SEED + 7, device=dev)
+    mq = svl.GatedPrefill(wl_q.dims, wq, max_seq=wl_q.n_vis[1] + wl_q.s_text[1] + 64)
+    bts = [synth.make_batch(wl_q, SEED + 601 + i, device=dev) for i in range(2)]
+    outs = [mq.alloc_outputs(bt) for bt in bts]
+    ms, live, clk, _ = timed_steps(svl, mq, bts, outs, t_steps, w_steps)
+    res["qwen"] = dict(pass_summary(svl, mq, wl_q.dims, bts, outs, ms, live, pk), clocks=clk)
+    mq.close()
+    del wq, outs, mq
+    torch.cuda.empty_cache()
+    return res
+
+
+def compact_summary(line, gated):
+    """The figures a reader needs first, small enough for a log tail."""
+    s = {"per_budget": [[p["budget"], round(p["ms_per_step"], 2), round(p.get("time_vs_flops_ratio_minus_1", 0), 4)]
+                        for p in line["per_budget"]],
+         "per_budget_cols": ["budget", "ms_per_step", "t_vs_F_minus_1"]}
+    kern = line.get("kernels", {})
+    s["tflops"] = {t: round(kern[t]["tflops"]) for t in ("qkv_gemm", "o_gemm", "gateup_gemm", "down_gemm", "attention")
+                   if t in kern and "tflops" in kern[t]}
+    if line.get("hbm_kernels_sweep"):
+        s["hbm_frac"] = {f"B{r['batch']}": {n: r[n]["frac_of_measured_hbm"] for n in ("score", "select", "pack")
+                                            if n in r} for r in line["hbm_kernels_sweep"]}
+    if gated:
+        m = gated["mixed"]
+        s["mixed"] = [m["tokens_per_s"], m["exec_tflops"], m.get("roofline", {}).get("frac")]
+        s["gating_sweep"] = [[r["point"], r["t_over_t1"], r["f_over_f1"], r["time_vs_flops_ratio_minus_1"]]
+                             for r in gated["gating_sweep"]["rows"]]
+        v = gated["video"]
+        s["video"] = [[r["budget"], r["ms_per_step"], r.get("time_vs_flops_ratio_minus_1")] for r in v["rows"]]
+        s["video_attention_tflops"] = v.get("attention_roofline", {}).get("achieved")
+        q = gated["qwen"]
+        s["qwen"] = [q["tokens_per_s"], q["exec_tflops"], q.get("roofline", {}).get("frac")]
+    if line.get("fp8"):
+        f = line["fp8"]
+        s["fp8"] = [round(f["value"]), round(f["exec_tflops"]), round(f["gateup_gemm"]["frac"], 3)]
+    if line.get("decode"):
+        s["decode"] = [round(line["decode"]["tokens_per_s"]), round(line["decode"]["frac_of_measured_hbm"], 3)]
+    return s
 
 
 def run_fp8(args, svl, wl, weights, batches, dev, pk, max_seq):

@@ -15,13 +15,13 @@ the oracle in float64: where the two differ by a bf16 step, a value can sit
 on opposite sides of an e4m3 rounding boundary and jump by a whole e4m3 step
 (6-12 %). The end-to-end bar is therefore 1.5x the distance between the
 oracle's fp8 forward with bf16 storage and with fp32 storage (the same
-definition under storage-level perturbation), at least 2e-2; at widths up to
-512, where that sensitivity is small, the layers' update of the residual
-stream (final hidden minus the packed input rows) must in addition lie
-within 2e-2 (L2) of the definition's. The update must also sit closer to the
-fp8 definition's than to the bf16 one's, which shows the e4m3 arithmetic is
-what ran. Per-stage checks at LLaVA-7B width (tests/test_gpu_stages.py)
-carry the element-wise claim."""
+definition under storage-level perturbation), at least 2e-2. The layers'
+update of the residual stream (final hidden minus the packed input rows)
+must lie within 1.5x that storage sensitivity measured on the update itself
+(at these small widths bf16 storage alone moves the update by 5-7 %), and
+closer to the fp8 definition's update than to the bf16 one's, which shows the
+e4m3 arithmetic is what ran. Per-stage checks at LLaVA-7B width
+(tests/test_gpu_stages.py) carry the element-wise claim."""
 import numpy as np
 import pytest
 import torch
@@ -130,8 +130,9 @@ def _compare(case, out, n_samples, min_compared):
         e8 = l2_err(d_got, refs["fp8"][i]["hidden"] - x0)
         e16 = l2_err(d_got, refs["bf16"][i]["hidden"] - x0)
         assert e8 < e16, (i, e8, e16)
-        if case.dims.d_model <= 512:
-            assert e8 < 2e-2, (i, e8)
+        # and within 1.5x the definition's own storage sensitivity on the update
+        sens = l2_err(refs["fp8_s32"][i]["hidden"] - x0, refs["fp8"][i]["hidden"] - x0)
+        assert e8 < 1.5 * sens, (i, e8, sens)
         compared += 1
     assert compared >= min_compared
     return refs

@@ -7,10 +7,15 @@ recomputes the stage in float64 from those same bf16 values and rounds its
 output to bf16. The bar:
 
 * QKV + RoPE, O projection + residual, gate/up + SwiGLU, down projection +
-  residual: every element within one bf16 ulp of the oracle (the GPU's
-  float32 accumulation error is far below half an ulp, so two roundings of
-  nearly the same value differ by at most one ulp); the number of 1-ulp flips
-  is reported, and the L2 relative error must be within 1e-3.
+  residual: every element within one bf16 ulp of the oracle, plus the
+  float32 accumulation error of the GPU's sum, bounded by
+  2^-15 * sum_k |x_k w_k| (twice the recursive-summation bound of the
+  K/16 + 16 fp32 additions a K-deep tensor-core product makes). For a typical
+  element that term is under half an ulp, so two roundings of nearly the same
+  value differ by one ulp at most; it matters only for outputs near zero,
+  where the products cancel. The number of differing elements is reported,
+  and with unit gains and bf16 operands the L2 relative error must be within
+  1e-3.
 * Attention: the kernel rounds the unnormalised probabilities to bf16 before
   the P.V product (relative error at most 2^-8 each) and divides by the
   float32 sum of the unrounded ones, so per element
@@ -139,6 +144,14 @@ def _codes(x):
     return O.quantize_rows_e4m3(x)
 
 
+ACC = 2.0 ** -15  # float32 accumulation, relative to sum |x_k w_k|
+
+
+def _acc_floor(a, w):
+    """Accumulation error bound of a @ w^T on the GPU: ACC * |a| @ |w|^T."""
+    return ACC * (np.abs(a) @ np.abs(w).T)
+
+
 def _norm_step_bound(L, Xb, gain, w_codes):
     """Per-element effect of the one-step code differences between the plain
     codes of RMSNorm(X) * gain and the kernel's codes of X * gain, on
@@ -182,23 +195,23 @@ def run_layer_checks(L):
         qr, kr, vr = O.attention_projections(X_np[r], pos, L.lw, d, store, qw)
         qr, kr, vr = qr.reshape(-1, hq), kr.reshape(-1, dkv), vr.reshape(-1, dkv)
         cq, ck = L.head_cols(b, A), L.head_cols(b, Akv)
-        extra = {"q": 0.0, "k": 0.0, "v": 0.0}
-        if qw is not None:
-            for key, wn, heads, cols, rope in (("q", "wq", A, cq, True), ("k", "wk", Akv, ck, True),
-                                               ("v", "wv", Akv, ck, False)):
-                e, frac = _norm_step_bound(L, X_np[r], L.lw["attn_norm"], qw[wn])
+        extra = {}
+        xn = O.rmsnorm(X_np[r], L.lw["attn_norm"], d.rms_eps)
+        for key, wn, heads, cols, rope in (("q", "wq", A, cq, True), ("k", "wk", Akv, ck, True),
+                                           ("v", "wv", Akv, ck, False)):
+            e = _acc_floor(xn, L.lw[wn]) * (1.15 if qw is not None else 1.0)
+            if qw is not None:
+                step, frac = _norm_step_bound(L, X_np[r], L.lw["attn_norm"], qw[wn])
                 print(f"qkv s{b} {key}: {100 * frac:.3f} % of the activation codes differ (e4m3 ties)")
-                extra[key] = (_rope_pair_sum(e, heads, dh) if rope else e)[:, cols]
-        elif fold:
-            # bf16(W * gain): relative error 2^-8 per weight
-            xn = O.rmsnorm(X_np[r], L.lw["attn_norm"], d.rms_eps)
-            for key, wn, heads, cols, rope in (("q", "wq", A, cq, True), ("k", "wk", Akv, ck, True),
-                                               ("v", "wv", Akv, ck, False)):
-                e = 2.0 ** -8 * (np.abs(xn) @ np.abs(L.lw[wn]).T)
-                extra[key] = (_rope_pair_sum(e, heads, dh) if rope else e)[:, cols]
-        check_close(f"qkv s{b} q", qg[r][:, cq], qr[:, cq], extra["q"])
-        check_close(f"qkv s{b} k", kg[r][:, ck], kr[:, ck], extra["k"])
-        check_close(f"qkv s{b} v", vg[r][:, ck], vr[:, ck], extra["v"])
+                e = e + step
+            elif fold:
+                # bf16(W * gain): relative error 2^-8 per weight
+                e = e + 2.0 ** -8 * (np.abs(xn) @ np.abs(L.lw[wn]).T)
+            extra[key] = (_rope_pair_sum(e, heads, dh) if rope else e)[:, cols]
+        l2_bar = 1e-3 if (qw is None and not fold) else None
+        check_close(f"qkv s{b} q", qg[r][:, cq], qr[:, cq], extra["q"], l2_bar)
+        check_close(f"qkv s{b} k", kg[r][:, ck], kr[:, ck], extra["k"], l2_bar)
+        check_close(f"qkv s{b} v", vg[r][:, ck], vr[:, ck], extra["v"], l2_bar)
         # gated-off heads: never written
         assert np.isnan(qg[r][:, ~cq]).all() and np.isnan(kg[r][:, ~ck]).all()
         assert (vg[r][:, ~ck] == 0).all()
@@ -219,10 +232,10 @@ def run_layer_checks(L):
         W = O.attention_heads(qb, kb, np.abs(vb), groups, d, lambda a: a)
         cq = L.head_cols(b, A)
         got = aog[r][:, cq]
-        check_close(f"attn s{b} vs exact", got, store(exact)[:, cq], 2.0 ** -8 * W[:, cq] * (1 + 1e-3) +
-                    1e-5 * W[:, cq], l2_bar=4e-3)
-        check_close(f"attn s{b} vs bf16-P variant", got, store(var)[:, cq], 2.0 ** -7 * W[:, cq] * (1 + 1e-3) +
-                    1e-5 * W[:, cq], l2_bar=4e-3)
+        check_close(f"attn s{b} vs exact", got, store(exact)[:, cq], (2.0 ** -8 * (1 + 1e-3) + ACC) * W[:, cq],
+                    l2_bar=4e-3)
+        check_close(f"attn s{b} vs bf16-P variant", got, store(var)[:, cq], (2.0 ** -7 * (1 + 1e-3) + ACC) * W[:, cq],
+                    l2_bar=4e-3)
         assert np.isnan(aog[r][:, ~cq]).all()
 
     # ---- O projection + residual (gated-off heads of ao hold NaN: never read)
@@ -233,7 +246,8 @@ def run_layer_checks(L):
         r = L.rows(b)
         o = np.where(L.head_cols(b, A)[None, :], aog[r], 0.0)
         ref = O.attention_residual(X_np[r], o, L.lw, store, qw)
-        check_close(f"oproj s{b}", Xo_np[r], ref)
+        check_close(f"oproj s{b}", Xo_np[r], ref, _acc_floor(o, L.lw["wo"]) * (1.15 if qw is not None else 1.0),
+                    1e-3 if qw is None else None)
     assert (Xo_np[L.T:] == X_np[L.T:]).all()
 
     # ---- gate/up + SwiGLU (on the GPU's residual rows)
@@ -244,20 +258,21 @@ def run_layer_checks(L):
         r = L.rows(b)
         ref = O.mlp_hidden(Xo_np[r], L.lw, L.gg[b, 0], d, store, qw)
         cc = L.chan_cols(b)
-        extra = 0.0
-        if qw is not None or fold:
-            xn = O.rmsnorm(Xo_np[r], L.lw["ffn_norm"], d.rms_eps)
-            if qw is not None:
-                eg, _ = _norm_step_bound(L, Xo_np[r], L.lw["ffn_norm"], qw["wg"])
-                eu, _ = _norm_step_bound(L, Xo_np[r], L.lw["ffn_norm"], qw["wu"])
-                gv, uv = O.linear_e4m3(xn, qw["wg"]), O.linear_e4m3(xn, qw["wu"])
-            else:
-                eg = 2.0 ** -8 * (np.abs(xn) @ np.abs(L.lw["wg"]).T)
-                eu = 2.0 ** -8 * (np.abs(xn) @ np.abs(L.lw["wu"]).T)
-                gv, uv = xn @ L.lw["wg"].T, xn @ L.lw["wu"].T
-            # d(SiLU(g) u) <= 1.1 |u| dg + |SiLU(g)| du + 1.1 dg du  (|SiLU'| <= 1.1)
-            extra = (1.1 * np.abs(uv) * eg + np.abs(O.silu(gv)) * eu + 1.1 * eg * eu)[:, cc]
-        check_close(f"gateup s{b}", hg[r][:, cc], ref[:, cc], extra)
+        xn = O.rmsnorm(Xo_np[r], L.lw["ffn_norm"], d.rms_eps)
+        f8 = 1.15 if qw is not None else 1.0
+        eg, eu = _acc_floor(xn, L.lw["wg"]) * f8, _acc_floor(xn, L.lw["wu"]) * f8
+        if qw is not None:
+            eg = eg + _norm_step_bound(L, Xo_np[r], L.lw["ffn_norm"], qw["wg"])[0]
+            eu = eu + _norm_step_bound(L, Xo_np[r], L.lw["ffn_norm"], qw["wu"])[0]
+            gv, uv = O.linear_e4m3(xn, qw["wg"]), O.linear_e4m3(xn, qw["wu"])
+        else:
+            if fold:
+                eg = eg + 2.0 ** -8 * (np.abs(xn) @ np.abs(L.lw["wg"]).T)
+                eu = eu + 2.0 ** -8 * (np.abs(xn) @ np.abs(L.lw["wu"]).T)
+            gv, uv = xn @ L.lw["wg"].T, xn @ L.lw["wu"].T
+        # d(SiLU(g) u) <= 1.1 |u| dg + |SiLU(g)| du + 1.1 dg du  (|SiLU'| <= 1.1)
+        extra = (1.1 * np.abs(uv) * eg + np.abs(O.silu(gv)) * eu + 1.1 * eg * eu)[:, cc]
+        check_close(f"gateup s{b}", hg[r][:, cc], ref[:, cc], extra, 1e-3 if (qw is None and not fold) else None)
         assert np.isnan(hg[r][:, ~cc]).all()
 
     # ---- down projection + residual (gated-off channels of h hold NaN: never read)
@@ -268,7 +283,8 @@ def run_layer_checks(L):
         r = L.rows(b)
         u = np.where(L.chan_cols(b)[None, :], hg[r], 0.0)
         ref = O.mlp_residual(Xo_np[r], u, L.lw, store, qw)
-        check_close(f"down s{b}", Xd_np[r], ref)
+        check_close(f"down s{b}", Xd_np[r], ref, _acc_floor(u, L.lw["wd"]) * (1.15 if qw is not None else 1.0),
+                    1e-3 if qw is None else None)
     assert (Xd_np[L.T:] == X_np[L.T:]).all()
 
 
