@@ -12,9 +12,13 @@
 //                  in TMEM, so S of tile j+1 is computed while the softmax
 //                  works on tile j;
 //   softmax        one query row per thread: row max, P = exp2(S*scale - m)
-//                  rounded to bf16 and written to the slot's shared-memory P
-//                  buffer in the 128-byte-swizzled K-major layout, row sum;
-//   O += P V       tcgen05.mma M=128 N=d_head K=64 into the slot's O columns.
+//                  rounded to bf16 and written back over the tile's own S
+//                  columns in TMEM (tcgen05.st, two keys per column), row sum;
+//   O += P V       tcgen05.mma M=128 N=d_head K=64 into the slot's O columns,
+//                  A = P read from tensor memory, B = the V^T tile.
+// P never touches shared memory, and the softmax of tile j+1 does not wait
+// for the P V of tile j: the next S MMA into the same buffer is issued after
+// that P V, and the tensor core executes one thread's MMAs in order.
 // The running max m is only moved when a tile's max exceeds it by more than
 // 2^8 (then O and the row sum are rescaled in place); otherwise P is formed
 // against the stale max, its entries stay below 256 and O needs no per-tile
@@ -28,8 +32,8 @@
 // innermost coordinate); keys of the neighbouring sample that this pulls in
 // are masked, like every key after the query (causal) or past the sample's
 // end. Each softmax warp writes its own 32 output rows: through its part of
-// the P buffer and a TMA tensor store per 64 columns when all 32 rows exist,
-// with per-thread stores otherwise.
+// the slot's output staging buffer and a TMA tensor store per 64 columns when
+// all 32 rows exist, with per-thread stores otherwise.
 //
 // Warps: 0 / 6 TMA producers of slot 0 / 1; 1 / 7 MMA issuers (warp 1 also
 // owns the TMEM allocation: slot s uses columns 256 s .. 256 s + 255 for S0,
@@ -102,29 +106,24 @@ SVL_DEVINL float row_max64(const uint32_t* sv, int base, bool full, int lo, unsi
   return fmaxf(m0, m1);
 }
 
-// P = exp2(S*scale - m) for 64 keys, rounded to bf16 into this row of the
-// swizzled P atom; returns the row sum of the unrounded values.
-SVL_DEVINL float exp_store64(const uint32_t* sv, int base, bool full, int lo, unsigned span, uint64_t sc2,
-                             uint64_t nm2, uint8_t* patom_row, int row) {
+// P = exp2(S*scale - m) for 64 keys, rounded to bf16 and packed two keys per
+// 32-bit word (lower key in the low half) into pk[32], the layout of the A
+// operand in tensor memory; returns the row sum of the unrounded values.
+SVL_DEVINL float exp_pack64(const uint32_t* sv, int base, bool full, int lo, unsigned span, uint64_t sc2,
+                            uint64_t nm2, uint32_t* pk) {
   uint64_t acc0 = 0, acc1 = 0;
 #pragma unroll
-  for (int c8 = 0; c8 < 8; ++c8) {
-    uint32_t pk[4];
-#pragma unroll
-    for (int e2 = 0; e2 < 4; ++e2) {
-      const int e = 8 * c8 + 2 * e2;
-      const uint64_t xv = fma2(f2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), sc2, nm2);
-      float x0 = lo2(xv), x1 = hi2(xv);
-      if (!full) {
-        if (static_cast<unsigned>(base + e - lo) >= span) x0 = -INFINITY;
-        if (static_cast<unsigned>(base + e + 1 - lo) >= span) x1 = -INFINITY;
-      }
-      const float p0 = ex2(x0), p1 = ex2(x1);
-      if (e2 & 1) acc1 = add2(acc1, f2(p0, p1)); else acc0 = add2(acc0, f2(p0, p1));
-      pk[e2] = pack_bf16x2(p0, p1);
+  for (int e2 = 0; e2 < 32; ++e2) {
+    const int e = 2 * e2;
+    const uint64_t xv = fma2(f2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), sc2, nm2);
+    float x0 = lo2(xv), x1 = hi2(xv);
+    if (!full) {
+      if (static_cast<unsigned>(base + e - lo) >= span) x0 = -INFINITY;
+      if (static_cast<unsigned>(base + e + 1 - lo) >= span) x1 = -INFINITY;
     }
-    // keys base + 8*c8 .. +7: 16-byte chunk c8 of the row, 128-byte swizzle
-    *reinterpret_cast<uint4*>(patom_row + ((c8 ^ (row & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+    const float p0 = ex2(x0), p1 = ex2(x1);
+    if (e2 & 1) acc1 = add2(acc1, f2(p0, p1)); else acc0 = add2(acc0, f2(p0, p1));
+    pk[e2] = pack_bf16x2(p0, p1);
   }
   const uint64_t acc = add2(acc0, acc1);
   return lo2(acc) + hi2(acc);
@@ -140,7 +139,7 @@ struct PipeSmem {
   static constexpr int kQ = 128 * DH * 2;             // DH/64 atoms
   static constexpr int kKAtom = kPipeKeys * 128;      // 64 keys x 128 B
   static constexpr int kKV = kPipeKeys * DH * 2;      // K tile (DH/64 atoms) or V^T tile (DH rows x 128 B)
-  static constexpr int kP = 128 * kPipeKeys * 2;      // 128 rows x 64 keys
+  static constexpr int kP = 128 * kPipeKeys * 2;      // output staging: 128 rows x 64 columns
   static constexpr int q0 = 0;
   static constexpr int p0 = q0 + kQ;
   static constexpr int r0 = p0 + kP;
@@ -272,11 +271,11 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
         tc_commit(&bar->s_full[b]);
       };
       auto mma_pv = [&](int b, int pos, bool acc) {
-        const uint64_t dp = smem_desc_sw128(smem_u32(ss + L::p0));
+        // P of this tile: 32 columns of packed bf16 over its S buffer
         const uint64_t dv = smem_desc_sw128(smem_u32(ss + L::r0 + (pos % kPipeRing) * L::kKV));
 #pragma unroll
         for (int kk = 0; kk < kPipeKeys / 16; ++kk)
-          tc_mma_bf16(tbase + 128, dp + ((kk * 32) >> 4), dv + ((kk * 32) >> 4), id_o, (acc || kk > 0) ? 1u : 0u);
+          tc_mma_bf16_ts(tbase + 128, tbase + 64 * b + 8 * kk, dv + ((kk * 32) >> 4), id_o, (acc || kk > 0) ? 1u : 0u);
         tc_commit(&bar->pv_done[b]);
       };
       for (int u = worker; u < n_units && ok; u += stride) {
@@ -295,8 +294,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
         tc_commit(&bar->r_empty[(g + pos_k(0)) % kPipeRing]);
         for (int j = 0; j < n && ok; ++j) {
           if (j + 1 < n) {
-            // its S buffer was last read by the softmax of tile t+j-1,
-            // whose P V was issued (after p_full) in the previous round
+            // its S buffer held P of tile t+j-1, read by the P V issued
+            // (after p_full) in the previous round: in-order MMAs
             const int gk = g + pos_k(j + 1);
             ok = ring_wait(gk);
             if (!ok) break;
@@ -381,16 +380,14 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
             tmem_st_wait();
           }
         }
-        // the P buffer was read by P V of tile t-1
-        if (t >= 1 && !wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
         const float mref = (m_run == -INFINITY) ? 0.f : m_run;
         const uint64_t nm2 = f2(-mref, -mref);
-        // this warp's rows of the P buffer may still be the source of its
-        // last output store
-        if (lane == 0) bulk_wait_read0();
-        __syncwarp();
-        l_run += exp_store64(sv, 0, full, lo, span, sc2, nm2, ss + L::p0 + row * 128, row);
-        fence_proxy_async();  // P written by threads, read by the tensor core
+        uint32_t pk[32];
+        l_run += exp_pack64(sv, 0, full, lo, span, sc2, nm2, pk);
+        // P over the first 32 columns of this tile's S buffer (its S values
+        // are in registers already)
+        tmem_st32(tbase + 64 * b + lane_off, pk);
+        tmem_st_wait();
         tc_fence_before();
         mbar_arrive(&bar->p_full[b]);
       }
@@ -402,14 +399,14 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
       const int wrow0 = q * 32;  // this warp's first row in the block
       if (qb0 + wrow0 + 32 <= qend) {
         // all 32 rows exist: 64 columns at a time into this warp's rows of the
-        // P buffer (swizzled like a TMA box), one TMA store each by lane 0
+        // staging buffer (swizzled like a TMA box), one TMA store each by lane 0
         uint8_t* prow = ss + L::p0 + row * 128;
 #pragma unroll 1
         for (int h = 0; h < DH / 64; ++h) {
-          if (h > 0) {
-            if (lane == 0) bulk_wait_read0();  // the previous 64 columns have left shared memory
-            __syncwarp();
-          }
+          // the previous store from these rows (this unit's or the last one's)
+          // has left shared memory
+          if (lane == 0) bulk_wait_read0();
+          __syncwarp();
 #pragma unroll 1
           for (int c2 = 0; c2 < 2; ++c2) {
             uint32_t ov[32];

@@ -171,6 +171,20 @@ SVL_DEVINL void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, u
       : "memory");
 }
 
+// D[tmem] (+)= A[tmem] * B[smem]^T, bf16, fp32 accumulate: A (M = 128 rows,
+// one per TMEM lane) is read from tensor memory, two bf16 values of a row per
+// 32-bit column (lower K index in the low half), K = 16 per instruction, i.e.
+// 8 columns starting at a_tmem.
+SVL_DEVINL void tc_mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                               uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // The same with e4m3 operands (kind::f8f6f4, K = 32 per instruction: the
 // same 32 bytes of each swizzled row as 16 bf16 values).
 SVL_DEVINL void tc_mma_e4m3(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,

@@ -6,10 +6,14 @@
 //  * e_{b,l,j} = (l < P) or (layer_gate[b,l] and group_gate[b,l,j]);
 //  * consecutive samples with the same non-zero group mask form one row
 //    segment (samples with mask 0 skip the layer: residual bypass);
-//  * QKV tiles cover only the Q/K/V columns of active groups (column runs of
-//    consecutive active groups), gate/up tiles only active FFN channels;
-//    O and down tiles carry the mask so their K loop visits only active
-//    groups' rows of W_O / W_down;
+//  * QKV tiles cover only the Q/K/V columns of active groups, gate/up tiles
+//    only active FFN channels. These N-sparse lists are built per group, over
+//    maximal runs of consecutive samples in which that group runs (other
+//    groups' bits do not cut a run), and adjacent groups whose on/off pattern
+//    over the samples is the same share one column block; so mixed masks do
+//    not fragment the row tiles, and all-on batches get the segment tiles;
+//  * O and down tiles carry the segment mask so their K loop visits only
+//    active groups' rows of W_O / W_down;
 //  * attention items are (sample, active head, block of kAttnQ queries).
 #include "kernels.cuh"
 
@@ -102,10 +106,74 @@ __device__ int split_k_tail(int4* tiles, int count, int cap, int num_sms, int un
   return count + r * (sp - 1);
 }
 
+// Group j of layer l runs for sample b.
+SVL_DEVINL bool group_on(const ScheduleArgs& a, int b, int l, int j) {
+  return (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * a.G + j]);
+}
+
+// Emits the tiles of an N-sparse GEMM list of layer l: for each block of
+// adjacent groups with the same on/off pattern over the non-empty samples,
+// the maximal row runs of samples where the block runs, times the block's
+// columns (`cols(j0, j1, nt)` fills the n-tiles). Returns the tile count.
+// Called by the whole block; thread 0 walks groups and samples.
+template <class Cols>
+__device__ int emit_group_runs(const ScheduleArgs& a, int l, int4* tiles, int cap, NTile* nt, int* s_nnt,
+                               int* s_run, Cols cols) {
+  const int tid = threadIdx.x, B = a.B, G = a.G;
+  int off = 0;
+  int j0 = 0;
+  while (j0 < G) {
+    // the block [j0, j1]: following groups with the same pattern
+    if (tid == 0) {
+      int j1 = j0;
+      for (; j1 + 1 < G; ++j1) {
+        bool same = true;
+        for (int b = 0; b < B && same; ++b)
+          if (a.cu_seqlens[b + 1] > a.cu_seqlens[b]) same = group_on(a, b, l, j1 + 1) == group_on(a, b, l, j0);
+        if (!same) break;
+      }
+      s_run[2] = j1;
+      *s_nnt = cols(j0, j1, nt);
+      s_run[3] = 0;  // next sample to look at
+    }
+    __syncthreads();
+    const int j1 = s_run[2];
+    while (true) {
+      if (tid == 0) {
+        // next maximal run of non-empty samples (empty ones are transparent) where the block runs
+        int b = s_run[3], r0 = -1, r1 = -1;
+        for (; b < B; ++b) {
+          const int q0 = a.cu_seqlens[b], q1 = a.cu_seqlens[b + 1];
+          if (q1 <= q0) continue;
+          if (group_on(a, b, l, j0)) {
+            if (r0 < 0) r0 = q0;
+            r1 = q1;
+          } else if (r0 >= 0) {
+            break;
+          }
+        }
+        s_run[0] = r0;
+        s_run[1] = r1;
+        s_run[3] = b;
+      }
+      __syncthreads();
+      const int r0 = s_run[0], r1 = s_run[1];
+      if (r0 < 0) break;
+      emit_tiles(tiles, off, cap, r0, r1, nt, *s_nnt, 0, a.status);
+      off += ((r1 - r0 + kBM_SCHED - 1) / kBM_SCHED) * *s_nnt;
+      __syncthreads();
+    }
+    j0 = j1 + 1;
+    __syncthreads();
+  }
+  return min(off, cap);
+}
+
 __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __shared__ NTile nt[kMaxNT];
   __shared__ int s_nseg, s_nnt;
   __shared__ int s_heads[256];
+  __shared__ int s_run[4];
   pdl_trigger();
   pdl_wait();
   const int l = blockIdx.x, tid = threadIdx.x;
@@ -137,25 +205,18 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   const int nseg = s_nseg;
   const int hq = (a.A / G) * a.dh, hk = (a.Akv / G) * a.dh;
 
-  // ---- QKV (N-sparse over active groups' Q, K, V columns)
-  int off = 0;
-  for (int s = 0; s < nseg; ++s) {
-    const int4 sg = seg[s];
-    if (tid == 0) {
-      int c = build_runs(nt, 0, sg.z, G, hq, 256, 0);
-      c = build_runs(nt, c, sg.z, G, hk, 256, 1);
-      c = build_runs(nt, c, sg.z, G, hk, 256, 2);
-      s_nnt = c;
-    }
-    __syncthreads();
-    emit_tiles(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, sg.x, sg.y, nt, s_nnt, 0, a.status);
-    off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
-    __syncthreads();
-  }
+  // ---- QKV (N-sparse over active groups' Q, K, V columns, per group block)
+  auto qkv_cols = [&](int j0, int j1, NTile* out) {
+    const int mask = ((1 << (j1 + 1)) - 1) & ~((1 << j0) - 1);
+    int c = build_runs(out, 0, mask, G, hq, 256, 0);
+    c = build_runs(out, c, mask, G, hk, 256, 1);
+    return build_runs(out, c, mask, G, hk, 256, 2);
+  };
+  int off = emit_group_runs(a, l, a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, a.qkv_cap, nt, &s_nnt, s_run,
+                            qkv_cols);
   __syncthreads();
   if (tid == 0)
-    a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, min(off, a.qkv_cap), a.qkv_cap,
-                                a.num_sms, a.dh);
+    a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, a.num_sms, a.dh);
 
   // ---- O projection (K-sparse: kmask = segment mask), all D columns
   off = 0;
@@ -183,17 +244,14 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
                                  a.num_sms, a.ks_units, a.ks_info + static_cast<size_t>(l) * 8 + 4);
   __syncthreads();
 
-  // ---- gate/up (N-sparse over active FFN channels, 128 per tile)
-  off = 0;
-  for (int s = 0; s < nseg; ++s) {
-    const int4 sg = seg[s];
-    if (tid == 0) s_nnt = build_runs(nt, 0, sg.z, G, a.Di / G, 128, 0);
-    __syncthreads();
-    emit_tiles(a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, off, a.gu_cap, sg.x, sg.y, nt, s_nnt, 0, a.status);
-    off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
-    __syncthreads();
-  }
-  if (tid == 0) a.gu_count[l] = min(off, a.gu_cap);
+  // ---- gate/up (N-sparse over active FFN channels, 128 per tile, per group block)
+  auto gu_cols = [&](int j0, int j1, NTile* out) {
+    const int mask = ((1 << (j1 + 1)) - 1) & ~((1 << j0) - 1);
+    return build_runs(out, 0, mask, G, a.Di / G, 128, 0);
+  };
+  off = emit_group_runs(a, l, a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, a.gu_cap, nt, &s_nnt, s_run, gu_cols);
+  __syncthreads();
+  if (tid == 0) a.gu_count[l] = off;
 
   // ---- attention items: per active sample, blocks of kAttnQ queries (latest first), active heads
   off = 0;
