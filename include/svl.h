@@ -391,7 +391,8 @@ svl_status svl_pack(svl_model* model, int32_t B, int32_t n_vis_total, int32_t n_
  *  (on return it holds the final hidden state before the final norm).
  *   X [T_cap, D] bf16 in/out; cu_seqlens [B+1]; pos [T_cap] (from svl_pack)
  *   logits float32 [B, V] (LAST) or [T_cap, V] (ALL)
- *   t_cap: rows of X (n_vis_total + n_text_total of the pack call) */
+ *   t_cap: rows of X (n_vis_total + n_text_total of the pack call)
+ *  B <= 4096 samples per call (else SVL_ERR_UNSUPPORTED). */
 svl_status svl_gated_prefill(svl_model* model, int32_t B, int32_t t_cap, void* X,
                              const int32_t* cu_seqlens, const int32_t* pos,
                              const uint8_t* layer_gate, const uint8_t* group_gate,

@@ -99,6 +99,8 @@ size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 int round128(int x) { return (x + 127) & ~127; }
 
+constexpr int kMaxPrefillBatch = 4096;  // samples per prefill call
+
 // Each call keeps its scratch at the start of the workspace: no data flows
 // between calls through the workspace, so the three layouts overlap and the
 // workspace size is the largest of them.
@@ -793,6 +795,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     return SVL_ERR_INVALID_ARG;
   if (logits_mode != SVL_LOGITS_LAST && logits_mode != SVL_LOGITS_ALL) return SVL_ERR_INVALID_ARG;
   if (!aligned16(X)) return SVL_ERR_INVALID_ARG;
+  if (B > kMaxPrefillBatch) return SVL_ERR_UNSUPPORTED;  // the schedule stages per-sample data in shared memory
   const PreLayout L = pre_layout(m->d, B, t_cap);
   svl_status st = check_ws(ws, ws_bytes, L.total);
   if (st != SVL_OK) return st;

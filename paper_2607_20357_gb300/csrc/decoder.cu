@@ -106,10 +106,16 @@ __device__ int split_k_tail(int4* tiles, int count, int cap, int num_sms, int un
   return count + r * (sp - 1);
 }
 
-// Group j of layer l runs for sample b.
-SVL_DEVINL bool group_on(const ScheduleArgs& a, int b, int l, int j) {
-  return (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * a.G + j]);
-}
+// Shared-memory copies of the layer's per-sample inputs: row offsets
+// cu[0..B] and the effective group mask of every sample (bit j: group j
+// runs). Filled by the whole block, so the serial walks below read shared
+// memory only.
+struct SchedShared {
+  int* cu;
+  uint8_t* mask;
+};
+
+SVL_DEVINL bool group_on(const SchedShared& sh, int b, int j) { return (sh.mask[b] >> j) & 1; }
 
 // Emits the tiles of an N-sparse GEMM list of layer l: for each block of
 // adjacent groups with the same on/off pattern over the non-empty samples,
@@ -117,8 +123,8 @@ SVL_DEVINL bool group_on(const ScheduleArgs& a, int b, int l, int j) {
 // columns (`cols(j0, j1, nt)` fills the n-tiles). Returns the tile count.
 // Called by the whole block; thread 0 walks groups and samples.
 template <class Cols>
-__device__ int emit_group_runs(const ScheduleArgs& a, int l, int4* tiles, int cap, NTile* nt, int* s_nnt,
-                               int* s_run, Cols cols) {
+__device__ int emit_group_runs(const ScheduleArgs& a, const SchedShared& sh, int4* tiles, int cap, NTile* nt,
+                               int* s_nnt, int* s_run, Cols cols) {
   const int tid = threadIdx.x, B = a.B, G = a.G;
   int off = 0;
   int j0 = 0;
@@ -129,7 +135,7 @@ __device__ int emit_group_runs(const ScheduleArgs& a, int l, int4* tiles, int ca
       for (; j1 + 1 < G; ++j1) {
         bool same = true;
         for (int b = 0; b < B && same; ++b)
-          if (a.cu_seqlens[b + 1] > a.cu_seqlens[b]) same = group_on(a, b, l, j1 + 1) == group_on(a, b, l, j0);
+          if (sh.cu[b + 1] > sh.cu[b]) same = group_on(sh, b, j1 + 1) == group_on(sh, b, j0);
         if (!same) break;
       }
       s_run[2] = j1;
@@ -143,9 +149,9 @@ __device__ int emit_group_runs(const ScheduleArgs& a, int l, int4* tiles, int ca
         // next maximal run of non-empty samples (empty ones are transparent) where the block runs
         int b = s_run[3], r0 = -1, r1 = -1;
         for (; b < B; ++b) {
-          const int q0 = a.cu_seqlens[b], q1 = a.cu_seqlens[b + 1];
+          const int q0 = sh.cu[b], q1 = sh.cu[b + 1];
           if (q1 <= q0) continue;
-          if (group_on(a, b, l, j0)) {
+          if (group_on(sh, b, j0)) {
             if (r0 < 0) r0 = q0;
             r1 = q1;
           } else if (r0 >= 0) {
@@ -176,20 +182,28 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __shared__ int s_run[4];
   pdl_trigger();
   pdl_wait();
+  extern __shared__ int sched_dyn[];
   const int l = blockIdx.x, tid = threadIdx.x;
   const int B = a.B, G = a.G;
   int4* seg = a.seg + static_cast<size_t>(l) * B;
   uint8_t* act = a.act + static_cast<size_t>(l) * B;
+  const SchedShared sh{sched_dyn, reinterpret_cast<uint8_t*>(sched_dyn + B + 1)};
+  for (int b = tid; b <= B; b += blockDim.x) sh.cu[b] = a.cu_seqlens[b];
+  for (int b = tid; b < B; b += blockDim.x) {
+    int mask = 0;
+    for (int j = 0; j < G; ++j) {
+      const bool e = (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * G + j]);
+      mask |= e ? (1 << j) : 0;
+    }
+    sh.mask[b] = static_cast<uint8_t>(mask);
+  }
+  __syncthreads();
 
   if (tid == 0) {
     int ns = 0;
     for (int b = 0; b < B; ++b) {
-      int mask = 0;
-      for (int j = 0; j < G; ++j) {
-        const bool e = (l < a.P) || (a.layer_gate[b * a.L + l] && a.group_gate[(b * a.L + l) * G + j]);
-        mask |= e ? (1 << j) : 0;
-      }
-      const int r0 = a.cu_seqlens[b], r1 = a.cu_seqlens[b + 1];
+      const int mask = sh.mask[b];
+      const int r0 = sh.cu[b], r1 = sh.cu[b + 1];
       act[b] = (mask != 0 && r1 > r0) ? 1 : 0;
       if (mask == 0 || r1 <= r0) continue;
       if (ns > 0 && seg[ns - 1].z == mask && seg[ns - 1].y == r0) {
@@ -212,7 +226,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     c = build_runs(out, c, mask, G, hk, 256, 1);
     return build_runs(out, c, mask, G, hk, 256, 2);
   };
-  int off = emit_group_runs(a, l, a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, a.qkv_cap, nt, &s_nnt, s_run,
+  int off = emit_group_runs(a, sh, a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, a.qkv_cap, nt, &s_nnt, s_run,
                             qkv_cols);
   __syncthreads();
   if (tid == 0)
@@ -249,7 +263,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     const int mask = ((1 << (j1 + 1)) - 1) & ~((1 << j0) - 1);
     return build_runs(out, 0, mask, G, a.Di / G, 128, 0);
   };
-  off = emit_group_runs(a, l, a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, a.gu_cap, nt, &s_nnt, s_run, gu_cols);
+  off = emit_group_runs(a, sh, a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, a.gu_cap, nt, &s_nnt, s_run, gu_cols);
   __syncthreads();
   if (tid == 0) a.gu_count[l] = off;
 
@@ -272,10 +286,10 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     int lo = 0, hi = B;
     while (hi - lo > 1) {  // first sample of the segment
       const int mid = (lo + hi) >> 1;
-      if (a.cu_seqlens[mid] <= sg.x) lo = mid; else hi = mid;
+      if (sh.cu[mid] <= sg.x) lo = mid; else hi = mid;
     }
-    for (int b = lo; b < B && a.cu_seqlens[b] < sg.y; ++b) {
-      const int r0 = a.cu_seqlens[b], r1 = a.cu_seqlens[b + 1];
+    for (int b = lo; b < B && sh.cu[b] < sg.y; ++b) {
+      const int r0 = sh.cu[b], r1 = sh.cu[b + 1];
       if (r1 <= r0) continue;
       const int nq = (r1 - r0 + kAttnQ - 1) / kAttnQ;
       const int total = nq * nh;
@@ -294,7 +308,9 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   if (tid == 0) a.attn_count[l] = min(off, a.attn_cap);
 }
 
-void launch_schedule(const ScheduleArgs& a, cudaStream_t s) { launch_pdl(schedule_kernel, a.L, 256, 0, s, a); }
+void launch_schedule(const ScheduleArgs& a, cudaStream_t s) {
+  launch_pdl(schedule_kernel, a.L, 256, static_cast<size_t>(a.B + 1) * sizeof(int) + a.B, s, a);
+}
 
 // LLM-side compute controller (Sec. 3.2), one block per sample:
 //   h~ = h_b^(P) + W_k2 SiLU(W_k1 PE(kappa))          (Eq. 7; h_b^(P) = the budget
