@@ -340,9 +340,17 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
       const int qg = qb0 + row;
       const int key_base = it.z & ~7;
       float m_run = -INFINITY, l_run = 0.f;
+      // a warp whose 32 rows all lie past the block's end (the short last
+      // block of a sample) only keeps the tile barriers in step: its rows of
+      // S, P and O are never stored, and the MMA rows are independent
+      const bool idle = qb0 + q * 32 >= qend;
       for (int j = 0; j < n; ++j, ++t) {
         const int b = t & 1;
         if (!wait_all(&bar->s_full[b], (t >> 1) & 1)) { ok = false; break; }
+        if (idle) {
+          mbar_arrive(&bar->p_full[b]);
+          continue;
+        }
         tc_fence_after();
         const int kbase = key_base + j * kPipeKeys;
         const bool full = kbase >= it.z && kbase + kPipeKeys - 1 <= qb0;
@@ -392,6 +400,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
         mbar_arrive(&bar->p_full[b]);
       }
       if (!ok) break;
+      if (idle) continue;  // no rows of this warp to write
       // block done: O of the last P V, divided by the row sum
       if (!wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
       tc_fence_after();
