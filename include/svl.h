@@ -159,7 +159,11 @@ typedef struct svl_model svl_model;
 /* Creates a model on the current CUDA device: validates dims, records the
  * weight pointers, allocates the device status word and the RoPE cos/sin
  * table (max_seq x d_head/2 float2, computed in double precision).
- * Returns SVL_ERR_UNSUPPORTED for dims outside the list above. */
+ * Returns SVL_ERR_UNSUPPORTED for dims outside the list above.
+ * With SVL_PAIR_GEMM=1 in the environment, a bf16 model runs its QKV and
+ * gate/up GEMMs on clusters of two CTAs (256-row tiles, tcgen05
+ * cta_group::2); the results meet the same bars, and the default
+ * single-CTA kernel is as fast on GB300. */
 svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* weights, svl_model** out);
 void svl_model_destroy(svl_model* model);
 

@@ -3,6 +3,7 @@
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <cstdlib>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -22,6 +23,11 @@ struct svl_model {
   // every CTA of the persistent residual GEMM fits on the GPU at once, so
   // the shares of a K-split tail can wait for each other (else no split)
   bool ks_resident = false;
+  // QKV and gate/up on CTA pairs (256-row tiles, tcgen05 cta_group::2):
+  // clusters of two resident at once (0: single-CTA kernel); per layer the
+  // q, k, v, g, u weights as tensor maps with 64-row boxes
+  int pair_clusters = 0;
+  std::vector<CUtensorMap> tm_pair;
   uint32_t* d_status = nullptr;
   float2* rope_cs = nullptr;
   // B-operand tensor maps of the weights: per layer q, k, v, o, g, u, d
@@ -300,6 +306,15 @@ svl_status launch(EpiKind kind, svl_model* m, int tag, const GemmParams& p, int6
   return launch_gemm(kind, p, gemm_grid(m, tiles), s, e4m3, thin) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
 }
 
+// The same for the CTA-pair kernel (QKV, gate/up): up to pair_clusters
+// clusters of two, no more than the list's tiles.
+svl_status launch_pair(EpiKind kind, svl_model* m, int tag, const GemmParams& p, int64_t tiles, cudaStream_t s) {
+  if (tiles <= 0) return SVL_OK;
+  Launch L(m, tag, s);
+  const int pairs = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(m->pair_clusters, tiles)));
+  return launch_gemm_pair(kind, p, pairs, s) == cudaSuccess ? SVL_OK : SVL_ERR_CUDA;
+}
+
 svl_status last_error() { return cudaGetLastError() == cudaSuccess ? SVL_OK : SVL_ERR_CUDA; }
 
 }  // namespace
@@ -492,6 +507,33 @@ svl_status svl_model_create(const svl_model_desc* desc, const svl_weights* w, sv
   if (!ok) {
     svl_model_destroy(m);
     return SVL_ERR_INVALID_ARG;
+  }
+  // CTA-pair QKV and gate/up GEMMs for bf16 models, chosen with
+  // SVL_PAIR_GEMM=1 in the environment at model creation. They move a third
+  // less data through shared memory and L2 per FLOP but run at the same speed
+  // as the single-CTA kernel on GB300, whose GEMMs are held by the power cap,
+  // so the single-CTA kernel stays the default.
+  if (ok && !m->e4m3) {
+    const char* env = std::getenv("SVL_PAIR_GEMM");
+    if (env && env[0] == '1') {
+      const int c = std::min(gemm_pair_max_clusters(EPI_QKV_ROPE), gemm_pair_max_clusters(EPI_SWIGLU));
+      m->pair_clusters = std::min(c, m->num_sms / 2);
+    }
+    cudaGetLastError();  // a failed occupancy query only disables the pair kernel
+    if (m->pair_clusters > 0) {
+      m->tm_pair.resize(static_cast<size_t>(d.n_layers) * 5);
+      for (int l = 0; l < d.n_layers && ok; ++l) {
+        const svl_layer_weights& lw = m->layers[l];
+        CUtensorMap* t = &m->tm_pair[static_cast<size_t>(l) * 5];
+        ok = make_map(t + 0, lw.wq, hq, d.d_model, 64) && make_map(t + 1, lw.wk, dkv, d.d_model, 64) &&
+             make_map(t + 2, lw.wv, dkv, d.d_model, 64) && make_map(t + 3, lw.wg, d.d_ffn, d.d_model, 64) &&
+             make_map(t + 4, lw.wu, d.d_ffn, d.d_model, 64);
+      }
+      if (!ok) {
+        svl_model_destroy(m);
+        return SVL_ERR_INVALID_ARG;
+      }
+    }
   }
   if (cudaMalloc(&m->d_status, sizeof(uint32_t)) != cudaSuccess ||
       cudaMalloc(&m->rope_cs, sizeof(float2) * static_cast<size_t>(d.max_seq) * (dh / 2)) != cudaSuccess) {
@@ -819,6 +861,10 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   sa.G = d.n_groups;
   sa.P = d.n_prefix;
   sa.num_sms = m->num_sms;
+  const bool thin_launch = t_cap <= kThinRows;
+  const bool pair = m->pair_clusters > 0 && !m->e4m3 && !thin_launch;
+  sa.nsparse_rows = pair ? 2 * kBM : kBM;
+  sa.nsparse_wave = pair ? m->pair_clusters : m->num_sms;
   sa.A = d.n_heads;
   sa.Akv = d.n_kv_heads;
   sa.dh = dh;
@@ -1013,6 +1059,12 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.mapB[1] = tm[1];
     p.mapB[2] = tm[2];
     if (f8) set_f8(p, map_aq_x, tm8, sc8, {0, 1, 2});
+    if (pair) {
+      const CUtensorMap* tp = &m->tm_pair[static_cast<size_t>(l) * 5];
+      p.mapB[0] = tp[0];
+      p.mapB[1] = tp[1];
+      p.mapB[2] = tp[2];
+    }
     p.tiles = sa.qkv_tiles + static_cast<size_t>(l) * L.qkv_cap;
     p.tile_count = counts + l;
     p.max_tiles = L.qkv_cap;
@@ -1028,7 +1080,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.rope_cs = m->rope_cs;
     p.rope_rows = d.max_seq;
     p.d_head = dh;
-    if ((st = launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8, thin)) != SVL_OK) return st;
+    if ((st = pair ? launch_pair(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s)
+                   : launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8, thin)) != SVL_OK)
+      return st;
     }
 
     if (want(l, SVL_LAYER_ATTN)) {
@@ -1120,6 +1174,10 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.mapB[0] = tm[4];
     p.mapB[1] = tm[5];
     if (f8) set_f8(p, map_aq_x, tm8, sc8, {4, 5});
+    if (pair) {
+      p.mapB[0] = m->tm_pair[static_cast<size_t>(l) * 5 + 3];
+      p.mapB[1] = m->tm_pair[static_cast<size_t>(l) * 5 + 4];
+    }
     p.b_split = 1;
     p.tiles = sa.gu_tiles + static_cast<size_t>(l) * L.gu_cap;
     p.tile_count = counts + 2 * nl + l;
@@ -1128,7 +1186,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.kgroup = d.d_model;
     p.out[0] = hm;
     p.ld[0] = d.d_ffn;
-    if ((st = launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8, thin)) != SVL_OK) return st;
+    if ((st = pair ? launch_pair(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s)
+                   : launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8, thin)) != SVL_OK)
+      return st;
     }
 
     if (want(l, SVL_LAYER_DOWN)) {

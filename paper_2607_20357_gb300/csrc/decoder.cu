@@ -43,8 +43,8 @@ SVL_DEVINL int build_runs(NTile* out, int cnt, int mask, int G, int width, int s
 // sweeps all m-tiles before the next band starts, so concurrent CTAs share
 // the same weight columns in L2).
 __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const NTile* nt, int n_nt, int kmask,
-                           uint32_t* status) {
-  const int mt = (r1 - r0 + kBM_SCHED - 1) / kBM_SCHED;
+                           uint32_t* status, int bm = kBM_SCHED) {
+  const int mt = (r1 - r0 + bm - 1) / bm;
   const int total = mt * n_nt;
   for (int t = threadIdx.x; t < total; t += blockDim.x) {
     const int band = t / (mt * kNBand);
@@ -52,14 +52,14 @@ __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const
     const int bw = min(kNBand, n_nt - band * kNBand);
     const int mi = rem / bw;
     const int ni = band * kNBand + rem % bw;
-    const int m0 = r0 + mi * kBM_SCHED;
+    const int m0 = r0 + mi * bm;
     const int idx = base + t;
     if (idx >= cap) {
       report(status, SVL_DEV_BAD_INDEX);
       continue;
     }
     const NTile n = nt[ni];
-    tiles[idx] = make_int4(m0, min(m0 + kBM_SCHED, r1), n.n0, n.ncols | (n.mat << 16) | (kmask << 24));
+    tiles[idx] = make_int4(m0, min(m0 + bm, r1), n.n0, n.ncols | (n.mat << 16) | (kmask << 24));
   }
 }
 
@@ -165,8 +165,8 @@ __device__ int emit_group_runs(const ScheduleArgs& a, const SchedShared& sh, int
       __syncthreads();
       const int r0 = s_run[0], r1 = s_run[1];
       if (r0 < 0) break;
-      emit_tiles(tiles, off, cap, r0, r1, nt, *s_nnt, 0, a.status);
-      off += ((r1 - r0 + kBM_SCHED - 1) / kBM_SCHED) * *s_nnt;
+      emit_tiles(tiles, off, cap, r0, r1, nt, *s_nnt, 0, a.status, a.nsparse_rows);
+      off += ((r1 - r0 + a.nsparse_rows - 1) / a.nsparse_rows) * *s_nnt;
       __syncthreads();
     }
     j0 = j1 + 1;
@@ -230,7 +230,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
                             qkv_cols);
   __syncthreads();
   if (tid == 0)
-    a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, a.num_sms, a.dh);
+    a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, a.nsparse_wave, a.dh);
 
   // ---- O projection (K-sparse: kmask = segment mask), all D columns
   off = 0;

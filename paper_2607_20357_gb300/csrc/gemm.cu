@@ -755,6 +755,286 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   }
 }
 
+// ------------------------------------------------------------------ CTA-pair kernel
+// The same GEMM on 256-row tiles computed by a cluster of two CTAs on two SMs
+// (tcgen05 cta_group::2). Each CTA loads its 128 rows of A and half of B (the
+// first or the second N/2 rows of the tile's B, or the gate or the up rows of
+// a gate/up tile) into its own shared memory; the leader (cluster rank 0)
+// issues the MMAs, which read both CTAs' halves and write D rows 0-127 into
+// the leader's tensor memory and rows 128-255 into the peer's. Per SM and K
+// block this moves 32 KB through shared memory for a 128 x N product where the
+// single-CTA kernel moves 48 KB, which is what caps that kernel's tensor pipe.
+//
+//   full[s]    leader only: both CTAs' TMA loads of stage s (the leader posts
+//              the byte count of both, the peer's loads complete on it);
+//   empty[s]   each CTA: stage s consumed (the leader's MMA commit, multicast);
+//   tfull[a]   each CTA: accumulator a ready (commit, multicast);
+//   tempty[a]  leader only: both CTAs' epilogues have read accumulator a.
+// Waits are bounded as in the single-CTA kernel. The two cluster barriers (after
+// set-up and before the tensor memory is released) are reached by every thread
+// of both CTAs on every path; each producer first waits for the release of its
+// last stages, so no MMA completion can arrive after its CTA has exited.
+#ifndef SVL_PAIR_STAGES
+#define SVL_PAIR_STAGES 6
+#endif
+constexpr int kPairStages = SVL_PAIR_STAGES;
+constexpr int kPairBox = 64;                         // B rows per TMA box (64-row tensor maps)
+constexpr int kPairBBytes = kBHalf * kBK * 2;        // up to 128 B rows per CTA
+constexpr int kPairStageBytes = kABytes + kPairBBytes;
+constexpr int kPairSmem = kPairStages * kPairStageBytes + 1024 + 256;
+static_assert(kPairSmem <= 232448, "shared memory per CTA");
+
+// MMA N of a pair tile: gate/up tiles are 128 gate + 128 up rows; others
+// round their columns up to 128 or 256 (each CTA holds N / 2 rows of B).
+SVL_DEVINL int pair_n(const GemmParams& p, const TileInfo& ti) {
+  if (p.b_split) return 2 * kBHalf;
+  return ti.ncols > kBHalf ? 2 * kBHalf : kBHalf;
+}
+
+SVL_DEVINL void pair_producer(const GemmParams& p, uint8_t* stages, uint64_t* full, uint64_t* empty, uint32_t rank,
+                              volatile int* abort) {
+  const int ntiles = num_tiles(p);
+  const int npairs = gridDim.x >> 1, pair = blockIdx.x >> 1;
+  const int nkb = p.K / kBK, kgb = p.kgroup / kBK;
+  int s = 0;
+  uint32_t ph = 0;
+  auto next = [&]() {
+    if (++s == kPairStages) {
+      s = 0;
+      ph ^= 1;
+    }
+  };
+  for (int t = pair; t < ntiles; t += npairs) {
+    const TileInfo ti = get_tile(p, t);
+    if (!ti.valid) continue;
+    const int brows = pair_n(p, ti) / 2;
+    const CUtensorMap* mb = p.b_split ? &p.mapB[rank] : &p.mapB[ti.mat];
+    const int by = p.b_split ? ti.n0 : ti.n0 + static_cast<int>(rank) * brows;
+    const uint32_t bytes = 2u * static_cast<uint32_t>(kABytes + brows * 128);
+    KWalk w(nkb, kgb, ti.kmask);
+    while (w.next()) {
+      if (!mbar_wait(&empty[s], ph ^ 1, abort)) {
+        set_abort(abort, p.status);
+        return;
+      }
+      uint8_t* sa = stages + s * kPairStageBytes;
+      uint8_t* sb = sa + kABytes;
+      if (rank == 0) mbar_arrive_expect_tx(&full[s], bytes);
+      const uint32_t fb = mapa_shared(&full[s], 0);
+      tma_load_2d_pair(sa, &p.mapA, fb, w.kb * kBK, ti.m0 + static_cast<int>(rank) * kBM);
+      for (int r = 0; r < brows; r += kPairBox) tma_load_2d_pair(sb + r * 128, mb, fb, w.kb * kBK, by + r);
+      next();
+    }
+  }
+  // the releases of the last stages (the leader's MMA commits) have arrived here
+  for (int i = 0; i < kPairStages; ++i) {
+    if (!mbar_wait(&empty[s], ph ^ 1, abort)) {
+      set_abort(abort, p.status);
+      return;
+    }
+    next();
+  }
+}
+
+SVL_DEVINL void pair_mma(const GemmParams& p, uint8_t* stages, uint64_t* full, uint64_t* empty, uint64_t* tfull,
+                         uint64_t* tempty, uint32_t tmem, volatile int* abort) {
+  const int ntiles = num_tiles(p);
+  const int npairs = gridDim.x >> 1, pair = blockIdx.x >> 1;
+  const int nkb = p.K / kBK, kgb = p.kgroup / kBK;
+  int s = 0, it = 0;
+  uint32_t ph = 0;
+  for (int t = pair; t < ntiles; t += npairs) {
+    const TileInfo ti = get_tile(p, t);
+    if (!ti.valid) continue;
+    const int acc = it & 1;
+    const uint32_t aph = (it >> 1) & 1;
+    if (!mbar_wait(&tempty[acc], aph ^ 1, abort)) {
+      set_abort(abort, p.status);
+      return;
+    }
+    tc_fence_after();
+    const uint32_t idesc = idesc_bf16_f32(2 * kBM, pair_n(p, ti));
+    const uint32_t d = tmem + acc * kAccCols;
+    uint32_t accumulate = 0;
+    KWalk w(nkb, kgb, ti.kmask);
+    while (w.next()) {
+      if (!mbar_wait(&full[s], ph, abort)) {
+        set_abort(abort, p.status);
+        return;
+      }
+      tc_fence_after();
+      const uint32_t a0 = smem_u32(stages + s * kPairStageBytes);
+      const uint32_t b0 = a0 + kABytes;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        tc_mma_bf16_pair(d, smem_desc_sw128(a0 + k * 32), smem_desc_sw128(b0 + k * 32), idesc, accumulate);
+        accumulate = 1;
+      }
+      tc_commit_pair(&empty[s]);
+      if (++s == kPairStages) {
+        s = 0;
+        ph ^= 1;
+      }
+    }
+    tc_commit_pair(&tfull[acc]);
+    ++it;
+  }
+}
+
+template <int KIND>
+SVL_DEVINL void pair_epilogue(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem, uint32_t rank,
+                              volatile int* abort) {
+  const int ntiles = num_tiles(p);
+  const int npairs = gridDim.x >> 1, pair = blockIdx.x >> 1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int q = warp & 3;  // TMEM lane quarter this warp may access
+  int it = 0;
+  for (int t = pair; t < ntiles; t += npairs) {
+    const TileInfo ti = get_tile(p, t);
+    if (!ti.valid) continue;
+    const int acc = it & 1;
+    const uint32_t aph = (it >> 1) & 1;
+    const bool ok = mbar_wait(&tfull[acc], aph, abort);
+    __syncwarp();
+    if (!__all_sync(0xffffffffu, ok)) {
+      set_abort(abort, p.status);
+      return;
+    }
+    tc_fence_after();
+    const int row = ti.m0 + static_cast<int>(rank) * kBM + q * 32 + lane;
+    const uint32_t taddr = tmem + acc * kAccCols + (static_cast<uint32_t>(q * 32) << 16);
+    epilogue_tile<KIND, false>(p, ti, row, row < ti.m_end, taddr);
+    tc_fence_before();
+    if (rank == 0)
+      mbar_arrive(&tempty[acc]);
+    else
+      mbar_arrive_cluster(mapa_shared(&tempty[acc], 0));
+    ++it;
+  }
+}
+
+template <int KIND>
+__global__ void __launch_bounds__(kGemmThreads, 1) gemm_pair_kernel(const __grid_constant__ GemmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* stages = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(stages + kPairStages * kPairStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + kPairStages;
+  uint64_t* tfull = bars + 2 * kPairStages;
+  uint64_t* tempty = bars + 2 * kPairStages + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kPairStages + 4);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t rank = cluster_rank();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kPairStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&tfull[i], 1);
+      mbar_init(&tempty[i], 2 * 4 * 32);  // the epilogue threads of both CTAs
+    }
+    *abort = 0;
+    fence_barrier_init();
+    fence_proxy_async();
+    prefetch_tmap(&p.mapA);
+    prefetch_tmap(&p.mapB[0]);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  cluster_sync();  // both CTAs' barriers exist before any TMA or arrive reaches them
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
+
+  if (warp == 0) {
+    if (lane == 0) pair_producer(p, stages, full, empty, rank, abort);
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) pair_mma(p, stages, full, empty, tfull, tempty, tmem, abort);
+  } else {
+    pair_epilogue<KIND>(p, tfull, tempty, tmem, rank, abort);
+  }
+
+  __syncwarp();
+  if (*abort) {
+    // let copies and MMAs already issued land before shared and tensor memory go
+    long long t0 = clock64();
+    while (clock64() - t0 < 20000000LL) {
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the peer is done with this CTA's barriers and tensor memory
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, kTmemCols);
+  }
+}
+
+template <int KIND>
+static cudaError_t launch_pair_kind(const GemmParams& p, int pairs, cudaStream_t stream) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_pair_kernel<KIND>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(2 * pairs));
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = kPairSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 2;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, gemm_pair_kernel<KIND>, p);
+}
+
+cudaError_t launch_gemm_pair(EpiKind kind, const GemmParams& p, int pairs, cudaStream_t stream) {
+  if (pairs <= 0) return cudaSuccess;
+  switch (kind) {
+    case EPI_QKV_ROPE: return launch_pair_kind<EPI_QKV_ROPE>(p, pairs, stream);
+    case EPI_SWIGLU: return launch_pair_kind<EPI_SWIGLU>(p, pairs, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+int gemm_pair_max_clusters(EpiKind kind) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2);
+  cfg.blockDim = dim3(kGemmThreads);
+  cfg.dynamicSmemBytes = kPairSmem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  cudaError_t e;
+  if (kind == EPI_QKV_ROPE) {
+    e = cudaFuncSetAttribute(gemm_pair_kernel<EPI_QKV_ROPE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, gemm_pair_kernel<EPI_QKV_ROPE>, &cfg);
+  } else {
+    e = cudaFuncSetAttribute(gemm_pair_kernel<EPI_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPairSmem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveClusters(&n, gemm_pair_kernel<EPI_SWIGLU>, &cfg);
+  }
+  return e == cudaSuccess ? n : 0;
+}
+
 template <int KIND, bool F8 = false, bool THIN = false>
 static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t stream) {
   constexpr int smem = StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256;

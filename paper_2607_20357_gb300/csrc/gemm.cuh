@@ -106,6 +106,14 @@ struct GemmParams {
 cudaError_t launch_gemm(EpiKind kind, const GemmParams& p, int grid, cudaStream_t stream, bool e4m3 = false,
                         bool thin = false);
 
+// The gated QKV / gate-up GEMM on 256-row tiles by clusters of two CTAs
+// (tcgen05 cta_group::2): `pairs` clusters walk the tile list (tiles of up to
+// 256 rows), mapA has 128-row boxes, mapB 64-row boxes. bf16 only.
+cudaError_t launch_gemm_pair(EpiKind kind, const GemmParams& p, int pairs, cudaStream_t stream);
+// Clusters of two of the pair kernel that can be resident at once (0 if the
+// query fails).
+int gemm_pair_max_clusters(EpiKind kind);
+
 // CTAs of the residual (EPI_RESID) GEMM that fit on one SM at once, the
 // smaller of the wide and THIN instantiations (0 if the query fails).
 int gemm_resid_blocks_per_sm(bool e4m3);

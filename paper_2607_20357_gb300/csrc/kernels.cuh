@@ -138,6 +138,8 @@ void launch_decode_finish(int B, int V, const float* logits, int* next_token, in
 struct ScheduleArgs {
   int B, L, G, P;
   int num_sms;              // CTAs of the persistent GEMM (one wave of tiles)
+  int nsparse_rows;         // rows per tile of the QKV and gate/up lists (128, or 256 for CTA pairs)
+  int nsparse_wave;         // tiles of those lists that run at once (CTAs, or CTA pairs)
   int A, Akv, dh, D, Di;
   const int* cu_seqlens;
   const uint8_t* layer_gate;

@@ -294,6 +294,16 @@ def test_stages_bf16_llava_width():
     L.close()
 
 
+def test_stages_bf16_llava_width_cta_pairs(monkeypatch):
+    """The QKV and gate/up stages on CTA pairs (256-row tiles, tcgen05
+    cta_group::2; chosen with SVL_PAIR_GEMM=1 at model creation) against the
+    same bars."""
+    monkeypatch.setenv("SVL_PAIR_GEMM", "1")
+    L = Layer(seed=307)
+    run_layer_checks(L)
+    L.close()
+
+
 def test_stages_bf16_llava_width_random_gains():
     """Non-unit RMSNorm gains: the bf16 path folds them into bf16 copies of
     W_qkv and W_g,u (relative error 2^-8 per weight), which the bar of the
