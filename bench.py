@@ -168,6 +168,48 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+class NvmlClock:
+    """SM clock samples read through NVML (libnvidia-ml, read-only queries)
+    by a background thread every few milliseconds, stamped with the host
+    clock; `median(t0, t1)` is the median of the samples in a host-time
+    window. Without NVML every median is None."""
+
+    def __init__(self, index, period=0.003):
+        import ctypes
+        import threading
+        self.samples, self.stop, self.thread = [], threading.Event(), None
+        self.period = period
+        try:
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            handle = ctypes.c_void_p()
+            if lib.nvmlInit_v2() != 0 or lib.nvmlDeviceGetHandleByIndex_v2(int(index), ctypes.byref(handle)) != 0:
+                lib = None
+        except OSError:
+            lib = None
+        self.lib, self.handle = lib, (handle if lib is not None else None)
+        if lib is None:
+            return
+        clock = ctypes.c_uint()
+
+        def run():
+            while not self.stop.is_set():
+                if self.lib.nvmlDeviceGetClockInfo(self.handle, 1, ctypes.byref(clock)) == 0:  # NVML_CLOCK_SM
+                    self.samples.append((time.perf_counter(), clock.value))
+                time.sleep(self.period)
+
+        self.thread = threading.Thread(target=run, daemon=True)
+        self.thread.start()
+
+    def median(self, t0, t1):
+        v = [c for t, c in list(self.samples) if t0 <= t <= t1]
+        return statistics.median(v) if v else None
+
+    def close(self):
+        if self.thread is not None:
+            self.stop.set()
+            self.thread.join(timeout=1.0)
+
+
 # --------------------------------------------------------------------------- flops
 def per_kind_flops(dims, k, s_text, lg, gg):
     """Algorithmic FLOPs per GEMM kind for one batch (executed work only)."""
@@ -347,14 +389,22 @@ def run_ours(args, rank, world, local_rank):
     # between kernels would keep each launch from overlapping its predecessor
     live_tag = "gateup_gemm"
     svl.svl_profile_start(model.handle, tags=[live_tag])
+    # the SM clock of each step: the host waits for each step, so the step
+    # runs on the GPU within its host-time window, where NVML samples the clock
+    nv = NvmlClock(local_rank)
+    windows = []
     with ClockSampler(local_rank) as clk:
         t_wall0 = time.perf_counter()
         for i in range(args.steps):
+            tw0 = time.perf_counter()
             ev[i][0].record(stream)
             step(i)
             ev[i][1].record(stream)
-        torch.cuda.synchronize()
+            torch.cuda.synchronize()
+            windows.append((tw0, time.perf_counter()))
         t_wall = time.perf_counter() - t_wall0
+    nv.close()
+    step_mhz = [nv.median(a, b) for a, b in windows]
     kern_live = svl.svl_profile_stop(model.handle)
     launches = svl.svl_launch_count() - launches0
     # a second, untimed pass over the same steps with every kernel bracketed
@@ -384,7 +434,13 @@ def run_ours(args, rank, world, local_rank):
         toks = int(nv.sum() + st.sum())
         fex = executed_flops(svl, desc, k, st, nv, lg, gg)
         ms = statistics.mean(step_ms[i] for i in range(j, args.steps, len(batches)))
+        mhz = [step_mhz[i] for i in range(j, args.steps, len(batches)) if step_mhz[i]]
+        # SM cycles per step (time x median clock): the work in a unit that the
+        # power cap's clock changes between steps do not move
+        cyc = statistics.mean(step_ms[i] * step_mhz[i] * 1e3 for i in range(j, args.steps, len(batches))
+                              if step_mhz[i]) if mhz else None
         per_budget.append({"budget": float(bt["budget"][0]), "k_mean": float(k.mean()), "ms_per_step": ms,
+                           "sm_mhz": statistics.median(mhz) if mhz else None, "mcycles_per_step": cyc / 1e6 if cyc else None,
                            "tokens_per_s": toks / (ms / 1000.0), "exec_tflops": fex / (ms / 1000.0) / 1e12,
                            "exec_tflop_per_step": fex / 1e12})
         tokens_total += toks * nsteps
@@ -409,6 +465,9 @@ def run_ours(args, rank, world, local_rank):
         for p in per_budget:
             p["time_vs_flops_ratio_minus_1"] = (p["ms_per_step"] / full[0]["ms_per_step"]) / \
                 (p["exec_tflop_per_step"] / full[0]["exec_tflop_per_step"]) - 1.0
+            if p["mcycles_per_step"] and full[0]["mcycles_per_step"]:
+                p["cycles_vs_flops_ratio_minus_1"] = (p["mcycles_per_step"] / full[0]["mcycles_per_step"]) / \
+                    (p["exec_tflop_per_step"] / full[0]["exec_tflop_per_step"]) - 1.0
 
     # dominant kernel roofline (tensor-bound GEMM)
     gemm_tags = ["qkv_gemm", "o_gemm", "gateup_gemm", "down_gemm"]
@@ -522,18 +581,25 @@ def timed_steps(svl, model, batches, outs, steps, warmup, live_tags=("gateup_gem
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     launches0 = svl.svl_launch_count()
     svl.svl_profile_start(model.handle, tags=list(live_tags))
+    nv = NvmlClock(torch.cuda.current_device())
+    windows = []
     with ClockSampler(torch.cuda.current_device()) as clk:
         for i in range(steps):
+            tw0 = time.perf_counter()
             ev[i][0].record(stream)
             step(i)
             ev[i][1].record(stream)
-        torch.cuda.synchronize()
+            torch.cuda.synchronize()
+            windows.append((tw0, time.perf_counter()))
+    nv.close()
     live = svl.svl_profile_stop(model.handle)
     launches = svl.svl_launch_count() - launches0
     status = svl.svl_get_device_status(model.handle)
     if status:
         raise RuntimeError(f"device status {status:#x} in a timed pass")
-    return [a.elapsed_time(b) for a, b in ev], live, clk.summary(), launches
+    summary = clk.summary()
+    summary["step_sm_mhz"] = [nv.median(a, b) for a, b in windows]
+    return [a.elapsed_time(b) for a, b in ev], live, summary, launches
 
 
 def batch_accounting(svl, model, dims, bt, out):
@@ -550,7 +616,7 @@ def batch_accounting(svl, model, dims, bt, out):
             "alpha": float(on.float().mean())}
 
 
-def pass_summary(svl, model, dims, batches, outs, step_ms, live, pk, label_key=None, labels=None):
+def pass_summary(svl, model, dims, batches, outs, step_ms, live, pk, label_key=None, labels=None, step_mhz=None):
     """Per-batch rows (ms per step, tokens/s, executed TFLOP/s) and the
     whole pass: tokens/s, executed TFLOP/s and the gate/up GEMM's rate from
     the live events against the measured sustained bf16 peak."""
@@ -562,7 +628,11 @@ def pass_summary(svl, model, dims, batches, outs, step_ms, live, pk, label_key=N
             continue
         acc = batch_accounting(svl, model, dims, bt, outs[j])
         ms = statistics.mean(step_ms[i] for i in idx)
+        mhz = [step_mhz[i] for i in idx if step_mhz and step_mhz[i]]
         row = {"ms_per_step": round(ms, 3), "tokens_per_s": round(acc["tokens"] / (ms / 1e3), 1),
+               "sm_mhz": statistics.median(mhz) if mhz else None,
+               "mcycles_per_step": round(statistics.mean(step_ms[i] * step_mhz[i] / 1e3 for i in idx
+                                                         if step_mhz[i]), 4) if mhz else None,
                "exec_tflops": round(acc["fexec"] / (ms / 1e3) / 1e12, 1),
                "exec_tflop_per_step": acc["fexec"] / 1e12, "k_mean": round(acc["k_mean"], 1),
                "alpha": round(acc["alpha"], 4)}
@@ -589,13 +659,17 @@ def pass_summary(svl, model, dims, batches, outs, step_ms, live, pk, label_key=N
 
 def scaling_vs(rows, key, ref_value):
     """t(x)/t(ref) / (F(x)/F(ref)) - 1 for each row, against the row whose
-    `key` equals ref_value (linear scaling in executed FLOPs gives 0)."""
+    `key` equals ref_value (linear scaling in executed FLOPs gives 0); the
+    same with SM cycles (time x clock) in place of time when clocks exist."""
     ref = [r for r in rows if abs(r[key] - ref_value) < 1e-9]
     if not ref:
         return
     for r in rows:
-        r["time_vs_flops_ratio_minus_1"] = round((r["ms_per_step"] / ref[0]["ms_per_step"]) /
-                                                 (r["exec_tflop_per_step"] / ref[0]["exec_tflop_per_step"]) - 1.0, 4)
+        f = r["exec_tflop_per_step"] / ref[0]["exec_tflop_per_step"]
+        r["time_vs_flops_ratio_minus_1"] = round((r["ms_per_step"] / ref[0]["ms_per_step"]) / f - 1.0, 4)
+        if r.get("mcycles_per_step") and ref[0].get("mcycles_per_step"):
+            r["cycles_vs_flops_ratio_minus_1"] = round((r["mcycles_per_step"] / ref[0]["mcycles_per_step"]) / f - 1.0,
+                                                       4)
 
 
 def gated_batch(wl, seed, dev, alpha=1.0, layer_skip=0.0, keep=288):
@@ -640,7 +714,8 @@ def run_gated_workloads(args, svl, llava_model, dev, pk):
     bts = [synth.make_batch(wl_m, SEED + 301 + i, device=dev) for i in range(2)]
     outs = [llava_model.alloc_outputs(bt) for bt in bts]
     ms, live, clk, _ = timed_steps(svl, llava_model, bts, outs, t_steps, w_steps)
-    res["mixed"] = dict(pass_summary(svl, llava_model, dims, bts, outs, ms, live, pk), clocks=clk)
+    res["mixed"] = dict(pass_summary(svl, llava_model, dims, bts, outs, ms, live, pk,
+                                     step_mhz=clk.pop("step_sm_mhz")), clocks=clk)
     del outs
     # gating sweep at fixed k
     points = [("alpha", 1.0, 0.0), ("alpha", 0.75, 0.0), ("alpha", 0.5, 0.0), ("alpha", 0.25, 0.0),
@@ -650,14 +725,17 @@ def run_gated_workloads(args, svl, llava_model, dev, pk):
         bt = gated_batch(wl_m, SEED + 401, dev, alpha=alpha, layer_skip=skip)
         out = [llava_model.alloc_outputs(bt)]
         ms, live, clk, _ = timed_steps(svl, llava_model, [bt], out, max(3, t_steps // 2), 2)
-        r = pass_summary(svl, llava_model, dims, [bt], out, ms, live, pk)["rows"][0]
-        r.update({"point": f"{kind} {alpha if kind == 'alpha' else skip}", "sm_mhz": clk.get("sm_mhz")})
+        r = pass_summary(svl, llava_model, dims, [bt], out, ms, live, pk, step_mhz=clk.pop("step_sm_mhz"))["rows"][0]
+        r["point"] = f"{kind} {alpha if kind == 'alpha' else skip}"
         rows.append(r)
     ref = rows[0]
     for r in rows:
         r["t_over_t1"] = round(r["ms_per_step"] / ref["ms_per_step"], 4)
         r["f_over_f1"] = round(r["exec_tflop_per_step"] / ref["exec_tflop_per_step"], 4)
         r["time_vs_flops_ratio_minus_1"] = round(r["t_over_t1"] / r["f_over_f1"] - 1.0, 4)
+        if r.get("mcycles_per_step") and ref.get("mcycles_per_step"):
+            r["cycles_vs_flops_ratio_minus_1"] = round(
+                (r["mcycles_per_step"] / ref["mcycles_per_step"]) / r["f_over_f1"] - 1.0, 4)
     res["gating_sweep"] = {"batch": "mixed shape, B=64, keep 288 of 576, layer gates on unless skipped",
                            "rows": rows}
     # video
@@ -666,7 +744,8 @@ def run_gated_workloads(args, svl, llava_model, dev, pk):
     outs = [llava_model.alloc_outputs(bt) for bt in bts]
     ms, live, clk, _ = timed_steps(svl, llava_model, bts, outs, 2 * len(bts), w_steps,
                                    live_tags=("gateup_gemm", "attention"))
-    v = pass_summary(svl, llava_model, dims, bts, outs, ms, live, pk, "budget", list(wl_v.budgets))
+    v = pass_summary(svl, llava_model, dims, bts, outs, ms, live, pk, "budget", list(wl_v.budgets),
+                     step_mhz=clk.pop("step_sm_mhz"))
     scaling_vs(v["rows"], "budget", 0.5)
     v["clocks"] = clk
     res["video"] = v
@@ -678,7 +757,8 @@ def run_gated_workloads(args, svl, llava_model, dev, pk):
     bts = [synth.make_batch(wl_q, SEED + 601 + i, device=dev) for i in range(2)]
     outs = [mq.alloc_outputs(bt) for bt in bts]
     ms, live, clk, _ = timed_steps(svl, mq, bts, outs, t_steps, w_steps)
-    res["qwen"] = dict(pass_summary(svl, mq, wl_q.dims, bts, outs, ms, live, pk), clocks=clk)
+    res["qwen"] = dict(pass_summary(svl, mq, wl_q.dims, bts, outs, ms, live, pk, step_mhz=clk.pop("step_sm_mhz")),
+                       clocks=clk)
     mq.close()
     del wq, outs, mq
     torch.cuda.empty_cache()
@@ -687,9 +767,11 @@ def run_gated_workloads(args, svl, llava_model, dev, pk):
 
 def compact_summary(line, gated):
     """The figures a reader needs first, small enough for a log tail."""
-    s = {"per_budget": [[p["budget"], round(p["ms_per_step"], 2), round(p.get("time_vs_flops_ratio_minus_1", 0), 4)]
+    s = {"per_budget": [[p["budget"], round(p["ms_per_step"], 2), round(p.get("time_vs_flops_ratio_minus_1", 0), 4),
+                         p.get("sm_mhz"), round(p["cycles_vs_flops_ratio_minus_1"], 4)
+                         if p.get("cycles_vs_flops_ratio_minus_1") is not None else None]
                         for p in line["per_budget"]],
-         "per_budget_cols": ["budget", "ms_per_step", "t_vs_F_minus_1"]}
+         "per_budget_cols": ["budget", "ms_per_step", "t_vs_F_minus_1", "sm_mhz", "cycles_vs_F_minus_1"]}
     kern = line.get("kernels", {})
     s["tflops"] = {t: round(kern[t]["tflops"]) for t in ("qkv_gemm", "o_gemm", "gateup_gemm", "down_gemm", "attention")
                    if t in kern and "tflops" in kern[t]}
@@ -699,10 +781,11 @@ def compact_summary(line, gated):
     if gated:
         m = gated["mixed"]
         s["mixed"] = [m["tokens_per_s"], m["exec_tflops"], m.get("roofline", {}).get("frac")]
-        s["gating_sweep"] = [[r["point"], r["t_over_t1"], r["f_over_f1"], r["time_vs_flops_ratio_minus_1"]]
-                             for r in gated["gating_sweep"]["rows"]]
+        s["gating_sweep"] = [[r["point"], r["t_over_t1"], r["f_over_f1"], r["time_vs_flops_ratio_minus_1"],
+                              r.get("cycles_vs_flops_ratio_minus_1")] for r in gated["gating_sweep"]["rows"]]
         v = gated["video"]
-        s["video"] = [[r["budget"], r["ms_per_step"], r.get("time_vs_flops_ratio_minus_1")] for r in v["rows"]]
+        s["video"] = [[r["budget"], r["ms_per_step"], r.get("time_vs_flops_ratio_minus_1"),
+                       r.get("cycles_vs_flops_ratio_minus_1")] for r in v["rows"]]
         s["video_attention_tflops"] = v.get("attention_roofline", {}).get("achieved")
         q = gated["qwen"]
         s["qwen"] = [q["tokens_per_s"], q["exec_tflops"], q.get("roofline", {}).get("frac")]
