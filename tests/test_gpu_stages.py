@@ -1,5 +1,6 @@
-"""Per-stage GPU parity of one decoder layer at LLaVA-1.5-7B widths against
-the oracle's bf16-emulated stages (Sec. 3.2 attention and MLP blocks).
+"""Per-stage GPU parity of one decoder layer at LLaVA-1.5-7B widths (and
+Qwen2-VL-7B's GQA widths) against the oracle's bf16-emulated stages (Sec. 3.2
+attention and MLP blocks).
 
 Each stage runs alone through svl_layer_stage -- the same kernels and launch
 configuration the prefill uses -- on inputs the GPU stored, and the oracle
@@ -74,10 +75,11 @@ def check_close(name, got, ref, extra=0.0, l2_bar=1e-3):
 
 
 class Layer:
-    """One LLaVA-7B-width decoder layer on the GPU and the oracle's view."""
+    """One decoder layer of a workload's widths (LLaVA-7B by default) on the
+    GPU and the oracle's view."""
 
-    def __init__(self, seed, gemm_format=svl.SVL_GEMM_BF16, random_gains=False):
-        wl = synth.WORKLOADS["llava"]
+    def __init__(self, seed, gemm_format=svl.SVL_GEMM_BF16, random_gains=False, workload="llava"):
+        wl = synth.WORKLOADS[workload]
         self.dims = dims = synth.reduced(wl.dims, n_layers=1, vocab=512)
         w = synth.make_weights(dims, seed)
         if random_gains:
@@ -290,6 +292,16 @@ def run_layer_checks(L):
 
 def test_stages_bf16_llava_width():
     L = Layer(seed=301)
+    run_layer_checks(L)
+    L.close()
+
+
+def test_stages_bf16_qwen_width_gqa():
+    """Qwen2-VL-7B widths: d 3584, GQA 28 query / 4 KV heads (one KV head per
+    group, 7 query heads sharing it), FFN 18,944 (4,736 channels per group),
+    RoPE theta 1e6, RMSNorm eps 1e-6; groups off as in the LLaVA case, so a
+    gated-off group removes one KV head and its seven query heads."""
+    L = Layer(seed=311, workload="qwen")
     run_layer_checks(L)
     L.close()
 
