@@ -201,7 +201,7 @@ PreLayout pre_layout(const svl_model_desc& d, int B, int64_t t_cap) {
   L.gu = b.take(sizeof(int4) * nl * L.gu_cap);
   L.dn = b.take(sizeof(int4) * nl * L.dn_cap);
   L.attn = b.take(sizeof(int4) * nl * L.attn_cap);
-  L.counts = b.take(sizeof(int) * 5 * nl);
+  L.counts = b.take(sizeof(int) * 6 * nl);  // five tile/item counts and the attention unit counters
   // e4m3: the quantised rows of the current GEMM input and their scales
   if (d.gemm_format == SVL_GEMM_E4M3) {
     const int64_t o_cols = static_cast<int64_t>(G) * round128(static_cast<int>(hq / G));
@@ -890,6 +890,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   sa.attn_items = at<int4>(ws, L.attn);
   sa.attn_cap = L.attn_cap;
   sa.attn_count = counts + 4 * nl;
+  sa.attn_next = counts + 5 * nl;
   sa.ks_info = at<int>(ws, L.ks_info);
   sa.ks_units = m->ks_resident ? L.ks_units : 0;
   sa.status = m->d_status;
@@ -1133,6 +1134,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
       }
       aa.items = sa.attn_items + static_cast<size_t>(l) * L.attn_cap;
       aa.count = counts + 4 * nl + l;
+      aa.next_unit = counts + 5 * nl + l;
       Launch L1(m, SVL_TAG_ATTENTION, s);
       if (launch_attention_tc(aa, gemm_grid(m, L.attn_cap), s) != cudaSuccess) return SVL_ERR_CUDA;
     }

@@ -4,25 +4,31 @@
 // Persistent kernel, one CTA per SM, two independent query-block pipelines
 // ("slots") per CTA. A unit of work is one block of up to 128 queries of one
 // (sample, active head); every item of the device schedule (up to 256
-// queries) gives two units, its two 128-query halves, and slot s of CTA c
-// takes units 2c + s, 2c + s + 2G, ... of the list [all first halves][all
-// second halves], so neither slot ever waits for the other's chain. Keys come
-// in tiles of 64. Per slot and tile:
+// queries) gives two units, its two 128-query halves, later half first. The
+// schedule lists one head's items next to each other, latest first, and each
+// slot takes the next unit from a counter in global memory when it is ready
+// for one: the units of a head run at about the same time on several SMs and
+// share its keys and values in L2, the heaviest units start first, and no
+// slot idles while units are left. Neither slot ever waits for the other's
+// chain. Keys come in tiles of 64. Per slot and tile:
 //   S = Q K^T      tcgen05.mma M=128 N=64 K=d_head into one of two S buffers
 //                  in TMEM, so S of tile j+1 is computed while the softmax
 //                  works on tile j;
-//   softmax        one query row per thread: row max, P = exp2(S*scale - m)
-//                  rounded to bf16 and written back over the tile's own S
-//                  columns in TMEM (tcgen05.st, two keys per column), row sum;
+//   softmax        one query row per thread: P = exp2(S*scale - m) rounded
+//                  to bf16 and written back over the tile's own S columns in
+//                  TMEM (tcgen05.st, two keys per column), row sum;
 //   O += P V       tcgen05.mma M=128 N=d_head K=64 into the slot's O columns,
 //                  A = P read from tensor memory, B = the V^T tile.
 // P never touches shared memory, and the softmax of tile j+1 does not wait
 // for the P V of tile j: the next S MMA into the same buffer is issued after
 // that P V, and the tensor core executes one thread's MMAs in order.
-// The running max m is only moved when a tile's max exceeds it by more than
-// 2^8 (then O and the row sum are rescaled in place); otherwise P is formed
-// against the stale max, its entries stay below 256 and O needs no per-tile
-// correction. O / rowsum is written out once per unit.
+// The running max m is the row max of the unit's first tile. Later tiles form
+// P against it and only check their row sum: while it stays at most 2^14
+// (every entry of P is then at most 2^14, far from any overflow) O needs no
+// correction and no tile max is computed. A row whose sum exceeds that (or is
+// not finite) takes the tile's max as the new m, O and the row sum are
+// rescaled in place and the tile's P is formed again. O / rowsum is written
+// out once per unit.
 //
 // V arrives transposed (V^T, keys contiguous) so that both operands are
 // K-major. K and V^T tiles go through the slot's own 4-stage ring, which the
@@ -35,7 +41,9 @@
 // the slot's output staging buffer and a TMA tensor store per 64 columns when
 // all 32 rows exist, with per-thread stores otherwise.
 //
-// Warps: 0 / 6 TMA producers of slot 0 / 1; 1 / 7 MMA issuers (warp 1 also
+// Warps: 0 / 6 TMA producers of slot 0 / 1 (the producer also takes the
+// slot's units from the counter and passes them to the other warps of the
+// slot through a small ring in shared memory); 1 / 7 MMA issuers (warp 1 also
 // owns the TMEM allocation: slot s uses columns 256 s .. 256 s + 255 for S0,
 // S1 and O); 2-5 / 8-11 softmax and output of slot 0 / 1. Every barrier
 // completes at most once ahead of its waiter; every wait is bounded.
@@ -43,7 +51,7 @@
 
 namespace svl {
 
-constexpr float kRescaleLog2 = 8.f;  // move the running max when it grows by more than 2^8
+constexpr float kTileSumMax = 16384.f;  // largest row sum of a tile's P formed against the running max
 static_assert(kAttnQ == 256, "an attention item is two blocks of 128 queries");
 
 SVL_DEVINL void attn_abort(volatile int* abort, uint32_t* status) {
@@ -86,42 +94,37 @@ SVL_DEVINL float hi2(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(
 SVL_DEVINL int pos_k(int j) { return j == 0 ? 0 : 2 * j - 1; }
 SVL_DEVINL int pos_v(int m, int n) { return m + 1 < n ? 2 * m + 2 : 2 * m + 1; }
 
-// Row max of 64 scores, masked to [lo, lo + span) unless `full`.
-SVL_DEVINL float row_max64(const uint32_t* sv, int base, bool full, int lo, unsigned span, float m) {
-  float m0 = m, m1 = -INFINITY;
-  if (full) {
+// Scores outside the valid keys [lo, lo + span) of the tile set to -inf.
+SVL_DEVINL void mask64(uint32_t* sv, int lo, unsigned span) {
 #pragma unroll
-    for (int e = 0; e < 64; e += 4) {
-      m0 = max3(m0, __uint_as_float(sv[e]), __uint_as_float(sv[e + 1]));
-      m1 = max3(m1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
-    }
-  } else {
-#pragma unroll
-    for (int e = 0; e < 64; e += 2) {
-      const float a = static_cast<unsigned>(base + e - lo) < span ? __uint_as_float(sv[e]) : -INFINITY;
-      const float b = static_cast<unsigned>(base + e + 1 - lo) < span ? __uint_as_float(sv[e + 1]) : -INFINITY;
-      if (e & 2) m1 = max3(m1, a, b); else m0 = max3(m0, a, b);
-    }
-  }
-  return fmaxf(m0, m1);
+  for (int e = 0; e < 64; ++e)
+    if (static_cast<unsigned>(e - lo) >= span) sv[e] = 0xff800000u;
 }
 
-// P = exp2(S*scale - m) for 64 keys, rounded to bf16 and packed two keys per
-// 32-bit word (lower key in the low half) into pk[32], the layout of the A
-// operand in tensor memory; returns the row sum of the unrounded values.
-SVL_DEVINL float exp_pack64(const uint32_t* sv, int base, bool full, int lo, unsigned span, uint64_t sc2,
-                            uint64_t nm2, uint32_t* pk) {
+// Row max of 64 scores, in four independent chains.
+SVL_DEVINL float row_max64(const uint32_t* sv) {
+  float m0 = -INFINITY, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
+#pragma unroll
+  for (int e = 0; e < 64; e += 8) {
+    m0 = max3(m0, __uint_as_float(sv[e]), __uint_as_float(sv[e + 1]));
+    m1 = max3(m1, __uint_as_float(sv[e + 2]), __uint_as_float(sv[e + 3]));
+    m2 = max3(m2, __uint_as_float(sv[e + 4]), __uint_as_float(sv[e + 5]));
+    m3 = max3(m3, __uint_as_float(sv[e + 6]), __uint_as_float(sv[e + 7]));
+  }
+  return fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
+}
+
+// P = exp2(S*scale - m) for 64 keys (masked scores are -inf and give 0),
+// rounded to bf16 and packed two keys per 32-bit word (lower key in the low
+// half) into pk[32], the layout of the A operand in tensor memory; returns
+// the row sum of the unrounded values.
+SVL_DEVINL float exp_pack64(const uint32_t* sv, uint64_t sc2, uint64_t nm2, uint32_t* pk) {
   uint64_t acc0 = 0, acc1 = 0;
 #pragma unroll
   for (int e2 = 0; e2 < 32; ++e2) {
     const int e = 2 * e2;
     const uint64_t xv = fma2(f2(__uint_as_float(sv[e]), __uint_as_float(sv[e + 1])), sc2, nm2);
-    float x0 = lo2(xv), x1 = hi2(xv);
-    if (!full) {
-      if (static_cast<unsigned>(base + e - lo) >= span) x0 = -INFINITY;
-      if (static_cast<unsigned>(base + e + 1 - lo) >= span) x1 = -INFINITY;
-    }
-    const float p0 = ex2(x0), p1 = ex2(x1);
+    const float p0 = ex2(lo2(xv)), p1 = ex2(hi2(xv));
     if (e2 & 1) acc1 = add2(acc1, f2(p0, p1)); else acc0 = add2(acc0, f2(p0, p1));
     pk[e2] = pack_bf16x2(p0, p1);
   }
@@ -132,6 +135,7 @@ SVL_DEVINL float exp_pack64(const uint32_t* sv, int base, bool full, int lo, uns
 constexpr int kPipeThreads = 384;
 constexpr int kPipeKeys = 64;
 constexpr int kPipeRing = 4;
+constexpr int kUnitRing = 4;   // units handed from a slot's producer to its MMA and softmax warps
 
 template <int DH>
 struct PipeSmem {
@@ -145,19 +149,23 @@ struct PipeSmem {
   static constexpr int r0 = p0 + kP;
   static constexpr int slot = r0 + kPipeRing * kKV;   // bytes per slot (multiple of 1024)
   static constexpr int bars = 2 * slot;
-  static constexpr int total = bars + 512 + 1024;
+  static constexpr int total = bars + 1024 + 1024;
 };
 static_assert(PipeSmem<128>::total <= 232448, "pipelined attention shared memory");
 
 struct PipeBars {
   uint64_t q_full, q_empty, r_full[kPipeRing], r_empty[kPipeRing], s_full[2], p_full[2], pv_done[2];
+  uint64_t unit_full[kUnitRing], unit_empty[kUnitRing];
+  int4 item[kUnitRing];  // the unit's schedule item
+  int unit[kUnitRing];   // unit index, or -1: no units left
 };
+static_assert(2 * sizeof(PipeBars) + 8 <= 1024, "attention barriers");
 
-// Unit u of the list [first halves][second halves] of n_items items.
-SVL_DEVINL bool pipe_unit(const AttnTcArgs& a, int n_items, int u, int4& it, int& qb0, int& qend, int& ntiles) {
-  const int item = u < n_items ? u : u - n_items;
-  const int half = u < n_items ? 0 : 1;
-  it = a.items[item];
+// Unit u: half 1 - (u & 1) of item `it` = item u / 2 of the schedule (an
+// item's later half first). False for an empty half (the short last item of
+// a sample).
+SVL_DEVINL bool unit_rows(const int4& it, int u, int& qb0, int& qend, int& ntiles) {
+  const int half = (u & 1) ^ 1;
   qb0 = it.x + 128 * half;
   qend = min(qb0 + 128, it.y);
   if (qend <= qb0) return false;
@@ -190,6 +198,10 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
         mbar_init(&b->p_full[i], 128);
         mbar_init(&b->pv_done[i], 1);
       }
+      for (int i = 0; i < kUnitRing; ++i) {
+        mbar_init(&b->unit_full[i], 1);
+        mbar_init(&b->unit_empty[i], 5);  // the MMA thread and the four softmax warps
+      }
     }
     *abort = 0;
     fence_barrier_init();
@@ -208,22 +220,44 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
   const int n_items = min(*a.count, a.cap);
   const int n_units = 2 * n_items;
   const int group = a.A / a.Akv;
+  int kunit = 0;  // units taken from (or, producer, put into) the slot's ring
   const int slot = warp < 6 ? 0 : 1;
   const int role = warp < 6 ? warp : warp - 6;  // 0 producer, 1 MMA, 2-5 softmax
   PipeBars* bar = bars + slot;
   uint8_t* ss = sm + slot * L::slot;
   const uint32_t tbase = tmem + 256 * slot;      // S0, S1 at +0, +64; O at +128
-  const int worker = 2 * blockIdx.x + slot, stride = 2 * gridDim.x;
 
   if (role == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       int g = 0, nq = 0;
       bool ok = true;
-      for (int u = worker; u < n_units && ok; u += stride) {
-        int4 it;
-        int qb0, qend, n;
-        if (!pipe_unit(a, n_items, u, it, qb0, qend, n)) continue;
+      // passes unit u (-1: none left) and its item to the MMA and softmax
+      // warps of the slot
+      auto post = [&](int u, const int4& it) -> bool {
+        const int i = kunit % kUnitRing;
+        if (!mbar_wait(&bar->unit_empty[i], ((kunit / kUnitRing) & 1) ^ 1, abort)) return false;
+        bar->unit[i] = u;
+        bar->item[i] = it;
+        mbar_arrive(&bar->unit_full[i]);  // release: the stores above are seen by the waiters
+        ++kunit;
+        return true;
+      };
+      // the next non-empty unit from the counter (u >= n_units: none left)
+      auto take = [&](int& u, int4& it, int& qb0, int& qend, int& n) {
+        for (;;) {
+          u = atomicAdd(a.next_unit, 1);
+          if (u >= n_units) return;
+          it = a.items[u >> 1];
+          if (unit_rows(it, u, qb0, qend, n)) return;
+        }
+      };
+      int u, qb0 = 0, qend = 0, n = 0;
+      int4 it = make_int4(0, 0, 0, 0);
+      take(u, it, qb0, qend, n);
+      while (ok) {
+        if (!post(u < n_units ? u : -1, it)) { ok = false; break; }
+        if (u >= n_units) break;
         const int kvh = it.w / group, key_base = it.z & ~7;
         if (!mbar_wait(&bar->q_empty, (nq & 1) ^ 1, abort)) { ok = false; break; }
         ++nq;
@@ -245,6 +279,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
             tma_load_2d(dst, &a.mapVt, &bar->r_full[st], key0, kvh * DH);
           }
         }
+        // the next unit, taken while this one's tiles are in flight
+        if (ok) take(u, it, qb0, qend, n);
       }
       if (!ok) attn_abort(abort, a.status);
     }
@@ -278,10 +314,17 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
           tc_mma_bf16_ts(tbase + 128, tbase + 64 * b + 8 * kk, dv + ((kk * 32) >> 4), id_o, (acc || kk > 0) ? 1u : 0u);
         tc_commit(&bar->pv_done[b]);
       };
-      for (int u = worker; u < n_units && ok; u += stride) {
-        int4 it;
+      while (ok) {
+        const int i = kunit % kUnitRing;
+        ok = mbar_wait(&bar->unit_full[i], (kunit / kUnitRing) & 1, abort);
+        if (!ok) break;
+        const int u = *reinterpret_cast<volatile int*>(&bar->unit[i]);
+        const int4 it = bar->item[i];  // after the acquiring wait (the asm is a compiler barrier)
+        mbar_arrive(&bar->unit_empty[i]);
+        ++kunit;
+        if (u < 0) break;
         int qb0, qend, n;
-        if (!pipe_unit(a, n_items, u, it, qb0, qend, n)) continue;
+        unit_rows(it, u, qb0, qend, n);
         ok = mbar_wait(&bar->q_full, nq & 1, abort);
         ++nq;
         if (!ok) break;
@@ -333,10 +376,17 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
       __syncwarp();
       return __all_sync(0xffffffffu, got);
     };
-    for (int u = worker; u < n_units && ok; u += stride) {
-      int4 it;
+    while (ok) {
+      const int i = kunit % kUnitRing;
+      if (!wait_all(&bar->unit_full[i], (kunit / kUnitRing) & 1)) { ok = false; break; }
+      const int u = *reinterpret_cast<volatile int*>(&bar->unit[i]);
+      const int4 it = bar->item[i];  // after the acquiring wait (the asm is a compiler barrier)
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar->unit_empty[i]);
+      ++kunit;
+      if (u < 0) break;
       int qb0, qend, n;
-      if (!pipe_unit(a, n_items, u, it, qb0, qend, n)) continue;
+      unit_rows(it, u, qb0, qend, n);
       const int qg = qb0 + row;
       const int key_base = it.z & ~7;
       float m_run = -INFINITY, l_run = 0.f;
@@ -362,20 +412,27 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
         tmem_ld32_async(tbase + 64 * b + 32 + lane_off, sv + 32);
         tmem_ld_wait32(sv);
         tmem_ld_wait32(sv + 32);
-        const float m_tile = row_max64(sv, 0, full, lo, span, -INFINITY) * sc;
-        if (j == 0) {
-          m_run = m_tile;
-        } else {
-          const bool need = m_tile > m_run + kRescaleLog2;
-          if (__any_sync(0xffffffffu, need)) {
-            // O must hold P V of every earlier tile before it is rescaled
-            if (!wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
-            tc_fence_after();
-            const float corr = need ? ex2(m_run - m_tile) : 1.f;
-            if (need) {
+        if (!full) mask64(sv, lo, span);
+        if (j == 0) m_run = row_max64(sv) * sc;
+        uint32_t pk[32];
+        float l_tile = exp_pack64(sv, sc2, f2(m_run == -INFINITY ? 0.f : -m_run, m_run == -INFINITY ? 0.f : -m_run), pk);
+        const bool need = !(l_tile <= kTileSumMax);  // also true for inf / NaN
+        if (__any_sync(0xffffffffu, need)) {
+          // a row of this tile grew past the running max: move it to the
+          // tile's max, rescale the row's O and sum, form P again
+          float corr = 1.f;
+          if (need) {
+            const float m_tile = row_max64(sv) * sc;
+            if (m_tile > m_run) {
+              corr = ex2(m_run - m_tile);
               l_run *= corr;
               m_run = m_tile;
             }
+          }
+          if (j > 0) {
+            // O must hold P V of every earlier tile before it is rescaled
+            if (!wait_all(&bar->pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) { ok = false; break; }
+            tc_fence_after();
 #pragma unroll 1
             for (int cc = 0; cc < DH; cc += 32) {
               uint32_t ov[32];
@@ -387,11 +444,10 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
             }
             tmem_st_wait();
           }
+          const float mref = m_run == -INFINITY ? 0.f : m_run;
+          l_tile = exp_pack64(sv, sc2, f2(-mref, -mref), pk);
         }
-        const float mref = (m_run == -INFINITY) ? 0.f : m_run;
-        const uint64_t nm2 = f2(-mref, -mref);
-        uint32_t pk[32];
-        l_run += exp_pack64(sv, 0, full, lo, span, sc2, nm2, pk);
+        l_run += l_tile;
         // P over the first 32 columns of this tile's S buffer (its S values
         // are in registers already)
         tmem_st32(tbase + 64 * b + lane_off, pk);
@@ -412,24 +468,23 @@ __global__ void __launch_bounds__(kPipeThreads, 1) attn_tc_kernel(const __grid_c
         uint8_t* prow = ss + L::p0 + row * 128;
 #pragma unroll 1
         for (int h = 0; h < DH / 64; ++h) {
+          uint32_t ov[64];
+          tmem_ld32_async(t_o + 64 * h, ov);
+          tmem_ld32_async(t_o + 64 * h + 32, ov + 32);
           // the previous store from these rows (this unit's or the last one's)
           // has left shared memory
           if (lane == 0) bulk_wait_read0();
           __syncwarp();
-#pragma unroll 1
-          for (int c2 = 0; c2 < 2; ++c2) {
-            uint32_t ov[32];
-            tmem_ld32_async(t_o + 64 * h + 32 * c2, ov);
-            tmem_ld_wait32(ov);
+          tmem_ld_wait32(ov);
+          tmem_ld_wait32(ov + 32);
 #pragma unroll
-            for (int d = 0; d < 32; d += 8) {
-              const int chunk = (32 * c2 + d) / 8;  // 16-byte chunk of the 128-byte row
-              *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) = make_uint4(
-                  pack_bf16x2(__uint_as_float(ov[d]) * inv, __uint_as_float(ov[d + 1]) * inv),
-                  pack_bf16x2(__uint_as_float(ov[d + 2]) * inv, __uint_as_float(ov[d + 3]) * inv),
-                  pack_bf16x2(__uint_as_float(ov[d + 4]) * inv, __uint_as_float(ov[d + 5]) * inv),
-                  pack_bf16x2(__uint_as_float(ov[d + 6]) * inv, __uint_as_float(ov[d + 7]) * inv));
-            }
+          for (int d = 0; d < 64; d += 8) {
+            const int chunk = d / 8;  // 16-byte chunk of the 128-byte row
+            *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) = make_uint4(
+                pack_bf16x2(__uint_as_float(ov[d]) * inv, __uint_as_float(ov[d + 1]) * inv),
+                pack_bf16x2(__uint_as_float(ov[d + 2]) * inv, __uint_as_float(ov[d + 3]) * inv),
+                pack_bf16x2(__uint_as_float(ov[d + 4]) * inv, __uint_as_float(ov[d + 5]) * inv),
+                pack_bf16x2(__uint_as_float(ov[d + 6]) * inv, __uint_as_float(ov[d + 7]) * inv));
           }
           fence_proxy_async();  // generic-proxy writes, read by the TMA unit
           __syncwarp();

@@ -267,7 +267,9 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __syncthreads();
   if (tid == 0) a.gu_count[l] = off;
 
-  // ---- attention items: per active sample, blocks of kAttnQ queries (latest first), active heads
+  // ---- attention items: per active sample and active head, blocks of kAttnQ
+  // queries, latest first (the kernel takes units from the front of the list,
+  // so one head's blocks run at about the same time and share its keys in L2)
   off = 0;
   int4* items = a.attn_items + static_cast<size_t>(l) * a.attn_cap;
   const int hpg = a.A / G;
@@ -294,8 +296,8 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
       const int nq = (r1 - r0 + kAttnQ - 1) / kAttnQ;
       const int total = nq * nh;
       for (int t = tid; t < total; t += blockDim.x) {
-        const int qi = nq - 1 - t / nh;
-        const int h = s_heads[t % nh];
+        const int qi = nq - 1 - t % nq;
+        const int h = s_heads[t / nq];
         const int q0 = r0 + qi * kAttnQ;
         const int idx = off + t;
         if (idx < a.attn_cap) items[idx] = make_int4(q0, min(q0 + kAttnQ, r1), r0, h);
@@ -305,7 +307,10 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     }
     __syncthreads();
   }
-  if (tid == 0) a.attn_count[l] = min(off, a.attn_cap);
+  if (tid == 0) {
+    a.attn_count[l] = min(off, a.attn_cap);
+    a.attn_next[l] = 0;
+  }
 }
 
 void launch_schedule(const ScheduleArgs& a, cudaStream_t s) {

@@ -152,6 +152,7 @@ struct ScheduleArgs {
   int4* gu_tiles; int gu_cap; int* gu_count;
   int4* dn_tiles; int dn_cap; int* dn_count;
   int4* attn_items; int attn_cap; int* attn_count;
+  int* attn_next;           // [L] attention unit counters, zeroed here
   int* ks_info;             // [L][2][4]: K-split tail of the O (0) and down (1) lists, see GemmParams
   int ks_units;             // most tail shares the partial buffer holds
   uint32_t* status;
@@ -232,6 +233,7 @@ struct AttnTcArgs {
   CUtensorMap mapO;         // O   [T_cap, A*dh]      boxes 64 x 32 (output stores)
   const int4* items;        // {q0, q_end, r0, head}
   const int* count;
+  int* next_unit;           // unit counter, zero at launch (the schedule zeroes it)
   int cap;
   int A, Akv, dh;
   float scale_log2;         // log2(e) / sqrt(dh)
