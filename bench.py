@@ -237,17 +237,27 @@ def executed_flops(svl, desc, k, s_text, n_vis, lg, gg):
     return tot
 
 
+TRAFFIC_SOURCES = ("gemm.cu", "decoder.cu", "kernels.cuh")  # the GEMM and its tile order
+
+
+def traffic_source_hash():
+    h = hashlib.sha256()
+    for f in TRAFFIC_SOURCES:
+        with open(os.path.join(ROOT, "paper_2607_20357_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
 def gemm_traffic_record():
     """Per-launch DRAM bytes of the dominant GEMM from the committed ncu
-    summary, if it was taken on the current kernel source."""
+    summary, if it was taken on the current source of the kernel and of the
+    schedule that orders its tiles."""
     path = os.path.join(ROOT, "profiles", "gemm_traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as fh:
         rec = json.load(fh)
-    src = os.path.join(ROOT, "paper_2607_20357_gb300", "csrc", "gemm.cu")
-    h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    return rec if rec.get("gemm_cu_sha256_16") == h else None
+    return rec if rec.get("source_sha256_16") == traffic_source_hash() else None
 
 
 # --------------------------------------------------------------------------- CPU oracle sample

@@ -7,7 +7,16 @@ namespace svl {
 
 constexpr int kSelectThreads = 512;
 constexpr int kAttnQ = 256;       // query rows per attention work item (the kernel runs its two 128-row halves as units)
-constexpr int kNBand = 8;         // n-tiles per raster band in the tile lists
+// n-tiles per raster band of a tile list. A band sweeps all m-tiles while its
+// weight columns stay in L2, so the input rows are read once per band: wider
+// bands read them fewer times until the band's weights (band x 256 rows x K)
+// no longer stay in L2. At LLaVA-7B widths the QKV list has 48 n-tiles and
+// the gate/up list 86; 16 and 20 minimise their DRAM traffic (gate/up: 1.32
+// GB per b = 1 launch with bands of 8, 0.85 GB with 20, 2.0 GB with 32).
+constexpr int kNBand = 8;         // down list (16 n-tiles of 256 x 11,008 weights)
+constexpr int kNBandO = 16;       // O list (16 n-tiles of 256 x 4,096 weights: one band)
+constexpr int kNBandQkv = 16;
+constexpr int kNBandGateUp = 20;
 constexpr int kBM_SCHED = 128;    // tile rows (the GEMM's M)
 
 struct SelectArgs {
