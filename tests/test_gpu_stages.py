@@ -78,7 +78,8 @@ class Layer:
     """One decoder layer of a workload's widths (LLaVA-7B by default) on the
     GPU and the oracle's view."""
 
-    def __init__(self, seed, gemm_format=svl.SVL_GEMM_BF16, random_gains=False, workload="llava"):
+    def __init__(self, seed, gemm_format=svl.SVL_GEMM_BF16, random_gains=False, workload="llava", lengths=None,
+                 gg=None):
         wl = synth.WORKLOADS[workload]
         self.dims = dims = synth.reduced(wl.dims, n_layers=1, vocab=512)
         w = synth.make_weights(dims, seed)
@@ -92,8 +93,9 @@ class Layer:
         wd["layers"] = [{k: v.cuda() for k, v in l.items()} for l in w["layers"]]
         self.w = wd
         self.model = svl.GatedPrefill(dims, wd, max_seq=1024, gemm_format=gemm_format)
-        self.B = B = len(LENGTHS)
-        self.cu = np.concatenate([[0], np.cumsum(LENGTHS)]).astype(np.int64)
+        lengths = LENGTHS if lengths is None else lengths
+        self.B = B = len(lengths)
+        self.cu = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int64)
         self.T = int(self.cu[-1])
         self.t_cap = self.T + 5  # rows past the packed batch must stay untouched
         self.t_pad = (self.t_cap + 7) // 8 * 8
@@ -101,13 +103,14 @@ class Layer:
         X = torch.zeros(self.t_cap, dims.d_model)
         X[:self.T] = torch.randn(self.T, dims.d_model, generator=gen) * (0.5 + torch.rand(self.T, 1, generator=gen))
         self.X = X.to(torch.bfloat16).cuda()
-        self.pos = torch.cat([torch.arange(n) for n in LENGTHS] + [torch.zeros(5, dtype=torch.int64)]).to(
+        self.pos = torch.cat([torch.arange(n) for n in lengths] + [torch.zeros(5, dtype=torch.int64)]).to(
             torch.int32).cuda()
         self.cu_d = torch.tensor(self.cu, dtype=torch.int32).cuda()
         G = dims.n_groups
-        gg = np.ones((B, 1, G), np.uint8)
-        gg[1, 0, 2] = 0              # one group off in sample 1
-        gg[2, 0, 0] = gg[2, 0, 3] = 0  # two groups off in sample 2
+        if gg is None:
+            gg = np.ones((B, 1, G), np.uint8)
+            gg[1, 0, 2] = 0              # one group off in sample 1
+            gg[2, 0, 0] = gg[2, 0, 3] = 0  # two groups off in sample 2
         self.gg = gg
         self.group_gate = torch.tensor(gg).cuda()
         self.layer_gate = torch.ones(B, 1, dtype=torch.uint8).cuda()
@@ -175,6 +178,34 @@ def _rope_pair_sum(e, heads, dh):
     return np.concatenate([s, s], axis=-1).reshape(e.shape[0], heads * dh)
 
 
+def check_attention(L, qg, kg, vg, aog):
+    """Attention of every sample against the oracle on the GPU's own Q, K, V:
+    the exact definition and the bf16-P variant, per element; gated-off heads
+    stay NaN."""
+    d = L.dims
+    A, Akv, dh = d.n_heads, d.n_kv_heads, d.d_head
+    store = O.round_bf16
+    for b in range(L.B):
+        r = L.rows(b)
+        S = r.stop - r.start
+        cq = L.head_cols(b, A)
+        if not cq.any():  # every group of the sample off: nothing is computed or stored
+            assert np.isnan(aog[r]).all()
+            continue
+        groups = L.gg[b, 0]
+        qb, kb, vb = qg[r].reshape(S, A, dh), kg[r].reshape(S, Akv, dh), vg[r].reshape(S, Akv, dh)
+        exact = O.attention_heads(qb, kb, vb, groups, d, lambda a: a)
+        var = O.attention_heads(qb, kb, vb, groups, d, lambda a: a, p_bf16=True)
+        # W = sum_j p_j |v_j| / sum_j p_j per (query, head, dim): the weighted mean of |v|
+        W = O.attention_heads(qb, kb, np.abs(vb), groups, d, lambda a: a)
+        got = aog[r][:, cq]
+        check_close(f"attn s{b} vs exact", got, store(exact)[:, cq], (2.0 ** -8 * (1 + 1e-3) + ACC) * W[:, cq],
+                    l2_bar=4e-3)
+        check_close(f"attn s{b} vs bf16-P variant", got, store(var)[:, cq], (2.0 ** -7 * (1 + 1e-3) + ACC) * W[:, cq],
+                    l2_bar=4e-3)
+        assert np.isnan(aog[r][:, ~cq]).all()
+
+
 def run_layer_checks(L):
     d = L.dims
     A, Akv, dh, G = d.n_heads, d.n_kv_heads, d.d_head, d.n_groups
@@ -223,22 +254,7 @@ def run_layer_checks(L):
     ao = torch.full((L.t_cap, hq), nan, dtype=torch.bfloat16, device="cuda")
     L.stage(svl.SVL_LAYER_ATTN, L.X, q=q, k=k, vt=vt, ao=ao)
     aog = np64(ao)
-    for b in range(L.B):
-        r = L.rows(b)
-        S = r.stop - r.start
-        groups = L.gg[b, 0]
-        qb, kb, vb = qg[r].reshape(S, A, dh), kg[r].reshape(S, Akv, dh), vg[r].reshape(S, Akv, dh)
-        exact = O.attention_heads(qb, kb, vb, groups, d, lambda a: a)
-        var = O.attention_heads(qb, kb, vb, groups, d, lambda a: a, p_bf16=True)
-        # W = sum_j p_j |v_j| / sum_j p_j per (query, head, dim): the weighted mean of |v|
-        W = O.attention_heads(qb, kb, np.abs(vb), groups, d, lambda a: a)
-        cq = L.head_cols(b, A)
-        got = aog[r][:, cq]
-        check_close(f"attn s{b} vs exact", got, store(exact)[:, cq], (2.0 ** -8 * (1 + 1e-3) + ACC) * W[:, cq],
-                    l2_bar=4e-3)
-        check_close(f"attn s{b} vs bf16-P variant", got, store(var)[:, cq], (2.0 ** -7 * (1 + 1e-3) + ACC) * W[:, cq],
-                    l2_bar=4e-3)
-        assert np.isnan(aog[r][:, ~cq]).all()
+    check_attention(L, qg, kg, vg, aog)
 
     # ---- O projection + residual (gated-off heads of ao hold NaN: never read)
     Xo = L.X.clone()
@@ -349,3 +365,31 @@ def test_quantize_with_gain_bit_exact():
     got = dst.cpu().view(torch.float8_e4m3fn).to(torch.float64).numpy()
     np.testing.assert_array_equal(got, codes)
     np.testing.assert_array_equal(scale.cpu().numpy(), sc.astype(np.float32))
+
+
+def test_attention_many_ragged_samples():
+    """Attention at LLaVA-7B widths over 16 ragged samples: single-row
+    samples, sample starts off the 8-row alignment of the key tiles, lengths
+    around the 128-query unit and the 256-query item (units whose later half
+    is empty), one sample with every group off and random groups elsewhere.
+    The kernel takes its units from a counter; every unit's output is checked
+    against the oracle, and rows of gated-off heads stay NaN."""
+    lengths = [1, 7, 8, 9, 127, 128, 129, 255, 256, 257, 3, 200, 64, 1, 300, 17]
+    rng = np.random.default_rng(7)
+    gg = (rng.random((len(lengths), 1, 4)) < 0.6).astype(np.uint8)
+    gg[:, 0, 1] = 1        # at least one group on ...
+    gg[5, 0, :] = 0        # ... except in sample 5
+    L = Layer(seed=401, lengths=lengths, gg=gg)
+    d = L.dims
+    hq, dkv = d.n_heads * d.d_head, d.n_kv_heads * d.d_head
+    nan = float("nan")
+    q = torch.full((L.t_cap, hq), nan, dtype=torch.bfloat16, device="cuda")
+    k = torch.full((L.t_cap, dkv), nan, dtype=torch.bfloat16, device="cuda")
+    vt = torch.zeros(dkv, L.t_pad, dtype=torch.bfloat16, device="cuda")
+    L.stage(svl.SVL_LAYER_QKV, L.X, q=q, k=k, vt=vt)
+    ao = torch.full((L.t_cap, hq), nan, dtype=torch.bfloat16, device="cuda")
+    L.stage(svl.SVL_LAYER_ATTN, L.X, q=q, k=k, vt=vt, ao=ao)
+    check_attention(L, np64(q), np64(k), np64(vt).T, np64(ao))
+    assert np.isnan(np64(ao)[L.T:]).all()  # rows past the packed batch untouched
+    L.close()
+
