@@ -344,7 +344,7 @@ def controller_gate_logits(dims, weights, h_prefix, kappa: float) -> np.ndarray:
 
 
 def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_count=-1, gates_override=None,
-                       project=True):
+                       project=True, kept=None):
     """The inference path with the compute controller in the loop (Sec. 3.2,
     Sec. 3.3): tokens with z > 0 survive (keep_count >= 0 overrides), the
     sequence is [kept visual][text][budget token] with positions 0..S, the
@@ -353,7 +353,8 @@ def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_cou
     0, then projected onto the budget for b < 1 unless ``project`` is False),
     and the logits come from the last row -- the budget token, which the
     answer follows. ``gates_override`` ([L, G]) replaces the controller's
-    decision (to replay another implementation's gates).
+    decision (to replay another implementation's gates); ``kept`` replaces
+    the top-k selection as in forward_sample.
     """
     store = make_store(mode)
     L, G, P = dims.n_layers, dims.n_groups, dims.n_prefix
@@ -361,7 +362,7 @@ def forward_controlled(dims, weights, x, text_ids, budget, mode="fp32", keep_cou
     z = token_logits(x, e_b, weights["ctrl_w1"], weights["ctrl_w2"], weights["ctrl_c2"])
     kappa = survival_rate(z)
     k = min(int(keep_count), x.shape[0]) if keep_count >= 0 else int(np.sum(z > 0))
-    kept = select_kept(z, k)
+    kept = select_kept(z, k) if kept is None else np.asarray(kept, dtype=np.int64)
     X, pos = pack_sample(dims, weights, x, kept, text_ids, store)
     tok = store(budget_embedding(float(np.float32(budget)), weights["llm_bud_w1"], weights["llm_bud_w2"]))
     X = np.concatenate([X, tok[None, :]], axis=0)
@@ -545,17 +546,21 @@ def pack_sample(dims, weights, x, kept, text_ids, store):
 
 
 def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
-                   keep_count=-1, mode="fp32", n_layers=None, qws=None):
+                   keep_count=-1, mode="fp32", n_layers=None, qws=None, kept=None):
     """Token controller + pack + gated decoder + final norm + last-row logits.
 
     ``n_layers`` (default: all) runs only the first layers -- used to bound
     the oracle's time; the final norm and LM head then apply after them.
     ``qws`` passes the per-layer e4m3 weights of the fp8 modes when the
-    caller has them already (they depend on the weights only).
+    caller has them already (they depend on the weights only). ``kept``
+    (ascending token indices) replaces the top-k selection downstream: the
+    pack and the decoder then run on that set, e.g. another valid top-k when
+    logits tie.
     """
     store = make_store(mode)
-    z, k, flags, kept = score_select_sample(dims, weights, x, budget, len(text_ids),
-                                            layer_gate, group_gate, keep_count)
+    z, k, flags, sel = score_select_sample(dims, weights, x, budget, len(text_ids),
+                                           layer_gate, group_gate, keep_count)
+    kept = sel if kept is None else np.asarray(kept, dtype=np.int64)
     X, pos = pack_sample(dims, weights, x, kept, text_ids, store)
     e = effective_groups(layer_gate, group_gate, dims.n_prefix)
     nl = dims.n_layers if n_layers is None else n_layers
@@ -570,16 +575,18 @@ def forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate,
     return {"z": z, "k": k, "flags": flags, "kept": kept, "hidden": X, "logits": logits}
 
 
-def decode_reference(dims, weights, x, text_ids, budget, layer_gate, group_gate, fed, keep_count=-1, mode="fp32"):
+def decode_reference(dims, weights, x, text_ids, budget, layer_gate, group_gate, fed, keep_count=-1, mode="fp32",
+                     kept=None):
     """Prompt forward, then one forward per fed token over the extended
     sequence (the definition a KV cache must reproduce). Returns the prompt's
     result and the list of per-step results (``logits`` of the new position,
-    ``hidden`` of all rows)."""
-    first = forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate, keep_count, mode)
+    ``hidden`` of all rows). ``kept`` as in forward_sample."""
+    first = forward_sample(dims, weights, x, text_ids, budget, layer_gate, group_gate, keep_count, mode, kept=kept)
     steps = []
     for n in range(1, len(fed) + 1):
         ids = np.concatenate([np.asarray(text_ids), np.asarray(fed[:n])])
-        steps.append(forward_sample(dims, weights, x, ids, budget, layer_gate, group_gate, first["k"], mode))
+        steps.append(forward_sample(dims, weights, x, ids, budget, layer_gate, group_gate, first["k"], mode,
+                                    kept=first["kept"]))
     return first, steps
 
 

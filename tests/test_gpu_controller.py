@@ -83,11 +83,14 @@ def test_controller_gates_and_forward(prefix):
         assert rel_err(lg_gpu, ref["gate_logits"]) < bar, (i, rel_err(lg_gpu, ref["gate_logits"]), bar)
         # the forward under the GPU's gates
         gk = out["kept_idx"][kept_off[i]:kept_off[i + 1]].numpy()
-        if v1 > v0 and not check_selection(out["scores"][v0:v1].numpy(), gk,
-                                           {"k": k, "kept": O.select_kept(ref["z"], k), "z": ref["z"]}):
-            continue
-        r32 = O.forward_controlled(dims, case.w_np, x, ids, budgets[i], mode="fp32", keep_count=k, gates_override=want)
-        r16 = O.forward_controlled(dims, case.w_np, x, ids, budgets[i], mode="bf16", keep_count=k, gates_override=want)
+        # on a tie-band swap the oracle runs on the GPU's (valid) kept set
+        same = v1 == v0 or check_selection(out["scores"][v0:v1].numpy(), gk,
+                                           {"k": k, "kept": O.select_kept(ref["z"], k), "z": ref["z"]})
+        kov = None if same else gk
+        r32 = O.forward_controlled(dims, case.w_np, x, ids, budgets[i], mode="fp32", keep_count=k, gates_override=want,
+                                   kept=kov)
+        r16 = O.forward_controlled(dims, case.w_np, x, ids, budgets[i], mode="bf16", keep_count=k, gates_override=want,
+                                   kept=kov)
         hid = out["X"][cu[i]:cu[i + 1]].double().numpy()
         assert rel_err(hid, r32["hidden"]) < bar_for(r32, r16, "hidden"), i
         assert l2_err(hid, r32["hidden"]) < bar_for(r32, r16, "hidden", l2_err), i

@@ -114,24 +114,31 @@ def _compare(case, out, n_samples, min_compared):
     for i in range(n_samples):
         v0, v1 = case.b_np["vis_off"][i], case.b_np["vis_off"][i + 1]
         kept = out["kept_idx"][out["kept_off"][i]:out["kept_off"][i + 1]].numpy()
-        if not check_selection(out["scores"][v0:v1].numpy(), kept, refs["fp32"][i]):
-            continue
+        ref = {m: refs[m][i] for m in refs}
+        if not check_selection(out["scores"][v0:v1].numpy(), kept, ref["fp32"]):
+            # a tie-band swap: the oracle's forwards on the GPU's (valid) kept set
+            bn = case.b_np
+            t0, t1 = bn["text_off"][i], bn["text_off"][i + 1]
+            args = (case.dims, case.w_np, bn["vis"][v0:v1], bn["text_ids"][t0:t1], bn["budget"][i],
+                    bn["layer_gate"][i], bn["group_gate"][i], int(bn["keep_count"][i]))
+            ref = {m: O.forward_sample(*args, mode=m, kept=kept) for m in refs}
+            print(f"sample {i}: GPU selection differs inside the tie band; compared on the GPU's kept set")
         hid = out["X"][cu[i]:cu[i + 1]].double().numpy()
         lg = out["logits"][i].double().numpy()
         for key, got in (("hidden", hid), ("logits", lg)):
-            bar = fp8_bar(refs["fp8"][i], refs["fp8_s32"][i], key)
-            e8 = rel_err(got, refs["fp8"][i][key])
+            bar = fp8_bar(ref["fp8"], ref["fp8_s32"], key)
+            e8 = rel_err(got, ref["fp8"][key])
             assert e8 < bar, (i, key, e8, bar)
         # the layers' update: closer to the fp8 definition than to the bf16 one
         t0, t1 = case.b_np["text_off"][i], case.b_np["text_off"][i + 1]
-        x0, _ = O.pack_sample(case.dims, case.w_np, case.b_np["vis"][v0:v1], refs["fp32"][i]["kept"],
+        x0, _ = O.pack_sample(case.dims, case.w_np, case.b_np["vis"][v0:v1], kept,
                               case.b_np["text_ids"][t0:t1], O.round_bf16)
         d_got = hid - x0
-        e8 = l2_err(d_got, refs["fp8"][i]["hidden"] - x0)
-        e16 = l2_err(d_got, refs["bf16"][i]["hidden"] - x0)
+        e8 = l2_err(d_got, ref["fp8"]["hidden"] - x0)
+        e16 = l2_err(d_got, ref["bf16"]["hidden"] - x0)
         assert e8 < e16, (i, e8, e16)
         # and within 1.5x the definition's own storage sensitivity on the update
-        sens = l2_err(refs["fp8_s32"][i]["hidden"] - x0, refs["fp8"][i]["hidden"] - x0)
+        sens = l2_err(ref["fp8_s32"]["hidden"] - x0, ref["fp8"]["hidden"] - x0)
         assert e8 < 1.5 * sens, (i, e8, sens)
         compared += 1
     assert compared >= min_compared
@@ -210,7 +217,9 @@ def test_fp8_decode_matches_extended_prefill():
         r32, s32 = O.decode_reference(*args, mode="fp32")
         kept = outc["kept_idx"][outc["kept_off"][i]:outc["kept_off"][i + 1]].numpy()
         if not check_selection(outc["scores"][v0:v1].numpy(), kept, r32):
-            continue
+            # a tie-band swap: the oracle on the GPU's (valid) kept set
+            r8, s8 = O.decode_reference(*args, mode="fp8", kept=kept)
+            r8s, s8s = O.decode_reference(*args, mode="fp8_s32", kept=kept)
         for t in range(steps):
             e8 = rel_err(got[t][i].double().numpy(), s8[t]["logits"])
             assert e8 < fp8_bar(s8[t], s8s[t], "logits"), (i, t, e8)

@@ -376,6 +376,27 @@ def test_kept_subset_equals_dense_on_shortened_sequence():
     np.testing.assert_allclose(out["hidden"], hid, rtol=1e-10, atol=1e-10)
 
 
+def test_kept_override_runs_the_given_set():
+    """forward_sample(kept=...) runs the downstream on the given set: the
+    oracle's own selection reproduces the plain call exactly, and another set
+    equals the library dense forward on that set's packed rows."""
+    dims = SMALL
+    w = np_weights(dims)
+    x, ids = _sample(dims, 6, n_vis=30)
+    L, G = dims.n_layers, dims.n_groups
+    args = (dims, w, x, ids, 0.6, np.ones(L, np.uint8), np.ones((L, G), np.uint8))
+    out = O.forward_sample(*args, mode="fp64")
+    same = O.forward_sample(*args, mode="fp64", kept=out["kept"])
+    assert np.array_equal(same["hidden"], out["hidden"]) and np.array_equal(same["logits"], out["logits"])
+    # one kept token swapped for one that was not kept (same k)
+    other = np.sort(np.concatenate([np.sort(out["kept"])[1:], np.setdiff1d(np.arange(30), out["kept"])[:1]]))
+    alt = O.forward_sample(*args, mode="fp64", kept=other)
+    assert np.array_equal(alt["kept"], other) and alt["k"] == out["k"]
+    hid, _ = dense_forward(_packed_rows(dims, w, x, other, ids), w["layers"], w["final_norm"], w["lm_head"], dims)
+    np.testing.assert_allclose(alt["hidden"], hid, rtol=1e-10, atol=1e-10)
+    assert not np.allclose(alt["hidden"], out["hidden"])
+
+
 def test_storage_modes_are_close_and_ordered():
     dims = SMALL
     w = np_weights(dims)
