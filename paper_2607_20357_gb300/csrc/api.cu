@@ -918,9 +918,10 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   // gated GEMMs with A boxes of kThinRows rows and deeper stages
   const bool thin = t_cap <= kThinRows;
   const uint32_t a_rows = thin ? kThinRows : 128;
-  CUtensorMap map_x, map_xn, map_ao, map_hm;
+  CUtensorMap map_x, map_xn, map_ao, map_hm, map_xr;
   if (!make_map(&map_x, X, t_cap, d.d_model, a_rows) || !make_map(&map_xn, xn, t_cap, d.d_model) ||
-      !make_map(&map_ao, ao, t_cap, hq, a_rows) || !make_map(&map_hm, hm, t_cap, d.d_ffn, a_rows))
+      !make_map(&map_ao, ao, t_cap, hq, a_rows) || !make_map(&map_hm, hm, t_cap, d.d_ffn, a_rows) ||
+      !make_map(&map_xr, X, t_cap, d.d_model, 32))  // residual stream, 32-row boxes (residual epilogues)
     return SVL_ERR_CUDA;
   // e4m3: every gated GEMM reads the quantised rows of its input (aq, with
   // per-row scales as) -- X for QKV and gate/up, the attention output for
@@ -1157,6 +1158,8 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     }
     p.out[0] = X;
     p.ld[0] = d.d_model;
+    p.mapR = map_xr;
+    p.resid_tma = 1;
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
@@ -1210,6 +1213,8 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     }
     p.out[0] = X;
     p.ld[0] = d.d_model;
+    p.mapR = map_xr;
+    p.resid_tma = 1;
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8 + 4;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;

@@ -631,19 +631,106 @@ SVL_DEVINL bool ksplit_tile(const GemmParams& p, const TileInfo& ti, int lrow, u
   return true;
 }
 
-template <int KIND, bool F8>
+// EPI_RESID through shared memory, for a warp whose 32 rows of the tile all
+// exist: 64 columns at a time, the chunk of X that TMA brought into one of
+// the warp's two buffers gets the accumulator added in place (bf16, with the
+// row's sums of squares of the rounded values for the next norm), and a TMA
+// store writes it back. The first two chunks were requested before the
+// accumulator was ready; chunk h + 2 is requested once the store of chunk h
+// has read its buffer. Bit b of `rpar` is the parity of buffer b's next wait.
+template <bool F8>
+SVL_DEVINL bool resid_tile_tma(const GemmParams& p, const TileInfo& ti, int q, uint32_t taddr, uint8_t* wst,
+                               uint64_t* wbar, uint32_t& rpar, volatile int* abort) {
+  const int lane = threadIdx.x & 31;
+  const int row = ti.m0 + q * 32 + lane;
+  const int nch = ti.ncols / 64;
+  const float af = F8 ? p.a_scale[row] : 1.f;
+  float hss = 0.f;
+  for (int h = 0; h < nch; ++h) {
+    const int b = h & 1;
+    const bool got = mbar_wait(&wbar[b], (rpar >> b) & 1, abort);
+    rpar ^= 1u << b;
+    __syncwarp();
+    if (!__all_sync(0xffffffffu, got)) return false;
+    float v[32], w[32];
+    tmem_ld32(taddr + 64 * h, v);
+    tmem_ld32(taddr + 64 * h + 32, w);
+    if constexpr (F8) {
+      scale_cols(v, p.b_scale[0] + ti.n0 + 64 * h, af);
+      scale_cols(w, p.b_scale[0] + ti.n0 + 64 * h + 32, af);
+    }
+    uint8_t* prow = wst + b * kResidChunk + lane * 128;
+    float ss[2] = {0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      // 16-byte chunk c of the row, where the 128-byte swizzle put it
+      uint4* slot = reinterpret_cast<uint4*>(prow + ((c ^ (lane & 7)) << 4));
+      const uint4 x = *slot;
+      const float* a = c < 4 ? v + 8 * c : w + 8 * (c - 4);
+      const uint32_t xw[4] = {x.x, x.y, x.z, x.w};
+      uint32_t o[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float2 f = unpack_bf16x2(xw[k]);
+        o[k] = pack_bf16x2(a[2 * k] + f.x, a[2 * k + 1] + f.y);
+        const float2 g = unpack_bf16x2(o[k]);
+        ss[c >> 2] = fmaf(g.x, g.x, fmaf(g.y, g.y, ss[c >> 2]));
+      }
+      *slot = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+    if (p.ss_out) {
+      // one partial per 128 columns of the residual stream, its 32-column
+      // sums added in column order
+      hss += ss[0];
+      hss += ss[1];
+      if (((64 * h + 64) & 127) == 0 || h + 1 == nch) {
+        p.ss_out[static_cast<size_t>((ti.n0 + 64 * h) >> 7) * p.ss_ld + row] = hss;
+        hss = 0.f;
+      }
+    }
+    fence_proxy_async();  // generic-proxy writes, read by the TMA unit
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(&p.mapR, wst + b * kResidChunk, ti.n0 + 64 * h, ti.m0 + q * 32);
+      bulk_commit();
+      if (h + 2 < nch) {
+        bulk_wait_read0();  // the store just issued has read this buffer
+        mbar_arrive_expect_tx(&wbar[b], kResidChunk);
+        tma_load_2d(wst + b * kResidChunk, &p.mapR, &wbar[b], ti.n0 + 64 * (h + 2), ti.m0 + q * 32);
+      }
+    }
+  }
+  return true;
+}
+
+template <int KIND, bool F8, bool THIN>
 SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem,
-                              volatile int* abort, KsSync& ks) {
+                              volatile int* abort, KsSync& ks, uint8_t* rstage, uint64_t* rbar) {
   const int ntiles = num_tiles(p);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;  // TMEM lane quarter this warp may access
+  constexpr bool kStaged = KIND == EPI_RESID && !THIN;  // residual through shared memory
+  uint8_t* wst = kStaged ? rstage + q * 2 * kResidChunk : nullptr;
+  uint64_t* wbar = kStaged ? rbar + 2 * q : nullptr;
+  uint32_t rpar = 0;
   int it = 0;
   for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
     TileInfo ti = get_tile(p, t);
     if (!ti.valid) continue;
     const int acc = it & 1;
     const uint32_t aph = (it >> 1) & 1;
-    if constexpr (KIND == EPI_RESID) {
+    const bool staged = kStaged && p.resid_tma && ti.nsplit == 1 && (ti.ncols & 63) == 0 &&
+                        ti.m0 + q * 32 + 32 <= ti.m_end;
+    if (staged) {
+      // the first two chunks of this warp's rows of X, while the main loop runs
+      if (lane == 0) {
+        bulk_wait_read0();  // the previous tile's stores have read both buffers
+        for (int h = 0; h < 2 && 64 * h < ti.ncols; ++h) {
+          mbar_arrive_expect_tx(&wbar[h], kResidChunk);
+          tma_load_2d(wst + h * kResidChunk, &p.mapR, &wbar[h], ti.n0 + 64 * h, ti.m0 + q * 32);
+        }
+      }
+    } else if constexpr (KIND == EPI_RESID) {
       // pull this row's residual segment toward L2 while the main loop runs
       const int prow = ti.m0 + q * 32 + lane;
       if (prow < ti.m_end) {
@@ -672,6 +759,11 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
           set_abort(abort, p.status);
           return;
         }
+      } else if (staged) {
+        if (!resid_tile_tma<F8>(p, ti, q, taddr, wst, wbar, rpar, abort)) {
+          set_abort(abort, p.status);
+          return;
+        }
       } else {
         epilogue_tile<KIND, F8>(p, ti, row, rv, taddr);
       }
@@ -682,6 +774,7 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
     mbar_arrive(&tempty[acc]);
     ++it;
   }
+  if (kStaged && lane == 0) bulk_wait0();  // this warp's residual stores are complete
 }
 
 // ------------------------------------------------------------------ kernel
@@ -699,6 +792,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * NST + 4);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
   KsSync ks{bars + 2 * NST + 5, bars + 2 * NST + 6, reinterpret_cast<volatile int*>(bars + 2 * NST + 7), 0};
+  // EPI_RESID: the epilogue warps' residual chunk buffers and their barriers
+  constexpr bool kStaged = KIND == EPI_RESID && !THIN;
+  uint64_t* rbar = bars + 2 * NST + 8;
+  uint8_t* rstage = stages + NST * SBYTES + 1024;
+  static_assert(!kStaged || (2 * NST + 16) * 8 <= 256, "barriers of the staged residual epilogue");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -712,6 +810,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
     }
     mbar_init(ks.gather, 4 * 32);
     mbar_init(ks.done, 1);
+    if (kStaged)
+      for (int i = 0; i < 8; ++i) mbar_init(&rbar[i], 1);
     *abort = 0;
     fence_barrier_init();
     fence_proxy_async();
@@ -736,7 +836,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   } else if (warp == 1) {
     if (lane == 0) mma_loop<NST, SBYTES, ABYTES, F8>(p, stages, full, empty, tfull, tempty, tmem, abort);
   } else {
-    epilogue_loop<KIND, F8>(p, tfull, tempty, tmem, abort, ks);
+    epilogue_loop<KIND, F8, THIN>(p, tfull, tempty, tmem, abort, ks, rstage, rbar);
   }
 
   __syncwarp();
@@ -1035,9 +1135,18 @@ int gemm_pair_max_clusters(EpiKind kind) {
   return e == cudaSuccess ? n : 0;
 }
 
+// Dynamic shared memory of gemm_kernel: the stages, the alignment slack and
+// the barriers, and for the staged residual epilogue its chunk buffers (at
+// the next 1024-byte boundary after the barriers).
+template <int KIND, bool THIN>
+constexpr int gemm_smem() {
+  return StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256 +
+         ((KIND == EPI_RESID && !THIN) ? 1024 - 256 + kResidStageBytes : 0);
+}
+
 template <int KIND, bool F8 = false, bool THIN = false>
 static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t stream) {
-  constexpr int smem = StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256;
+  constexpr int smem = gemm_smem<KIND, THIN>();
   static_assert(smem <= 232448, "shared memory per CTA");
   static bool configured = false;
   if (!configured) {
@@ -1051,7 +1160,7 @@ static cudaError_t launch_kind(const GemmParams& p, int grid, cudaStream_t strea
 
 template <int KIND, bool F8, bool THIN>
 static int blocks_per_sm_kind() {
-  constexpr int smem = StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256;
+  constexpr int smem = gemm_smem<KIND, THIN>();
   int n = 0;
   if (cudaFuncSetAttribute(gemm_kernel<KIND, F8, THIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
           cudaSuccess ||
