@@ -585,7 +585,7 @@ __global__ void rope_table_kernel(float2* cs, int max_seq, int dh, double theta)
   const int half = dh / 2;
   const long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x;
   if (i >= static_cast<long long>(max_seq) * half) return;
-  const int p = static_cast<int>(i / half), f = static_cast<int>(i % half);
+  const int f = static_cast<int>(i / max_seq), p = static_cast<int>(i % max_seq);
   const double ang = static_cast<double>(p) * pow(theta, -2.0 * f / dh);
   cs[i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
 }

@@ -314,7 +314,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
         report(p.status, SVL_DEV_BAD_INDEX);
         prow = 0;
       }
-      const float2* cs = p.rope_cs + static_cast<size_t>(prow) * half;
+      const float2* cs = p.rope_cs + prow;  // frequency i at cs[i * rope_rows]
       float w[32];
       for (int hb = 0; hb < ti.ncols; hb += dh) {
         for (int i0 = 0; i0 < half; i0 += 32) {
@@ -327,7 +327,7 @@ SVL_DEVINL void epilogue_tile(const GemmParams& p, const TileInfo& ti, int row, 
             }
 #pragma unroll
             for (int j = 0; j < 32; ++j) {
-              const float2 c = cs[i0 + j];
+              const float2 c = cs[static_cast<size_t>(i0 + j) * p.rope_rows];
               const float x1 = v[j] * rs, x2 = w[j] * rs;
               v[j] = x1 * c.x - x2 * c.y;
               w[j] = x2 * c.x + x1 * c.y;

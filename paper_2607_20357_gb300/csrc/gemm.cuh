@@ -67,7 +67,7 @@ struct GemmParams {
   int ld[3];
   const int* row_map;
   const int* pos;
-  const float2* rope_cs;  // [rope_rows, d_head/2] (cos, sin)
+  const float2* rope_cs;  // [d_head/2, rope_rows] (cos, sin), position fastest
   int rope_rows;
   int d_head;
   const float* e_b;       // [B, H]

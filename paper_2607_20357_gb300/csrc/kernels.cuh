@@ -255,7 +255,9 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, int grid, cudaStream_t s);
 // One bounded wait on a barrier nobody arrives on (time-out self-test).
 void launch_selftest_wait(uint32_t* status, long long cycles, cudaStream_t s);
 
-// RoPE table: cs[p * half + i] = (cos, sin)(p * theta^(-2i/dh)), double precision.
+// RoPE table: cs[i * max_seq + p] = (cos, sin)(p * theta^(-2i/dh)), double
+// precision, position fastest (the lanes of a warp hold consecutive rows, so
+// their reads of one frequency are contiguous).
 void launch_rope_table(float2* cs, int max_seq, int dh, double theta, cudaStream_t s);
 
 }  // namespace svl
