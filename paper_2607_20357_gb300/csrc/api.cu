@@ -918,10 +918,11 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   // gated GEMMs with A boxes of kThinRows rows and deeper stages
   const bool thin = t_cap <= kThinRows;
   const uint32_t a_rows = thin ? kThinRows : 128;
-  CUtensorMap map_x, map_xn, map_ao, map_hm, map_xr;
+  CUtensorMap map_x, map_xn, map_ao, map_hm, map_xr, map_hmo;
   if (!make_map(&map_x, X, t_cap, d.d_model, a_rows) || !make_map(&map_xn, xn, t_cap, d.d_model) ||
       !make_map(&map_ao, ao, t_cap, hq, a_rows) || !make_map(&map_hm, hm, t_cap, d.d_ffn, a_rows) ||
-      !make_map(&map_xr, X, t_cap, d.d_model, 32))  // residual stream, 32-row boxes (residual epilogues)
+      !make_map(&map_xr, X, t_cap, d.d_model, 32) ||  // residual stream, 32-row boxes (residual epilogues)
+      !make_map(&map_hmo, hm, t_cap, d.d_ffn, 32))    // SwiGLU outputs, 32-row boxes (gate/up epilogue)
     return SVL_ERR_CUDA;
   // e4m3: every gated GEMM reads the quantised rows of its input (aq, with
   // per-row scales as) -- X for QKV and gate/up, the attention output for
@@ -1159,7 +1160,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.out[0] = X;
     p.ld[0] = d.d_model;
     p.mapR = map_xr;
-    p.resid_tma = 1;
+    p.stage_tma = 1;
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
@@ -1191,6 +1192,8 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.kgroup = d.d_model;
     p.out[0] = hm;
     p.ld[0] = d.d_ffn;
+    p.mapR = map_hmo;
+    p.stage_tma = 1;
     if ((st = pair ? launch_pair(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s)
                    : launch(EPI_SWIGLU, m, SVL_TAG_GATEUP, p, L.gu_cap, s, f8, thin)) != SVL_OK)
       return st;
@@ -1214,7 +1217,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.out[0] = X;
     p.ld[0] = d.d_model;
     p.mapR = map_xr;
-    p.resid_tma = 1;
+    p.stage_tma = 1;
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8 + 4;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;

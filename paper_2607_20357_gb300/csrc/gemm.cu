@@ -703,25 +703,75 @@ SVL_DEVINL bool resid_tile_tma(const GemmParams& p, const TileInfo& ti, int q, u
   return true;
 }
 
+// EPI_SWIGLU through shared memory, for a warp whose 32 rows of the tile all
+// exist: 64 output columns at a time, SiLU(gate) * up goes into one of the
+// warp's two buffers (swizzled like the TMA box) and a TMA store writes it
+// out. The buffers alternate over all of the warp's chunks (`sbuf` counts
+// them), so a buffer is written again once the store before the latest one
+// -- its own previous store -- has read it.
+template <bool F8>
+SVL_DEVINL void swiglu_tile_tma(const GemmParams& p, const TileInfo& ti, int q, uint32_t taddr, uint8_t* wst,
+                                uint32_t& sbuf) {
+  const int lane = threadIdx.x & 31;
+  const int row = ti.m0 + q * 32 + lane;
+  const float af = F8 ? p.a_scale[row] : 1.f;
+  const float rs = (p.ss_in ? row_rms_scale(p, row) : 1.f) * af;
+  const int nch = ti.ncols / 64;
+  for (int h = 0; h < nch; ++h) {
+    const int b = sbuf++ & 1;
+    if (lane == 0) bulk_wait_read1();  // the store before the latest one (from this buffer) has read it
+    __syncwarp();
+    uint8_t* prow = wst + b * kResidChunk + lane * 128;
+#pragma unroll 1
+    for (int c2 = 0; c2 < 2; ++c2) {
+      float v[32], u[32];
+      tmem_ld32(taddr + 64 * h + 32 * c2, v);
+      tmem_ld32(taddr + kBHalf + 64 * h + 32 * c2, u);
+      if constexpr (F8) {
+        scale_cols(v, p.b_scale[0] + ti.n0 + 64 * h + 32 * c2, 1.f);
+        scale_cols(u, p.b_scale[1] + ti.n0 + 64 * h + 32 * c2, 1.f);
+      }
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j] * rs) * (u[j] * rs);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int c = 4 * c2 + i;  // 16-byte chunk of the 128-byte row
+        *reinterpret_cast<uint4*>(prow + ((c ^ (lane & 7)) << 4)) =
+            make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                       pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+      }
+    }
+    fence_proxy_async();  // generic-proxy writes, read by the TMA unit
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(&p.mapR, wst + b * kResidChunk, ti.n0 + 64 * h, ti.m0 + q * 32);
+      bulk_commit();
+    }
+  }
+}
+
 template <int KIND, bool F8, bool THIN>
 SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem,
                               volatile int* abort, KsSync& ks, uint8_t* rstage, uint64_t* rbar) {
   const int ntiles = num_tiles(p);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;  // TMEM lane quarter this warp may access
-  constexpr bool kStaged = KIND == EPI_RESID && !THIN;  // residual through shared memory
+  // residual (EPI_RESID) or outputs (EPI_SWIGLU) through shared memory
+  constexpr bool kStaged = (KIND == EPI_RESID || KIND == EPI_SWIGLU) && !THIN;
   uint8_t* wst = kStaged ? rstage + q * 2 * kResidChunk : nullptr;
   uint64_t* wbar = kStaged ? rbar + 2 * q : nullptr;
-  uint32_t rpar = 0;
+  uint32_t rpar = 0;  // EPI_RESID: parity of each buffer's next wait
+  uint32_t sbuf = 0;  // EPI_SWIGLU: chunks stored so far (buffer = sbuf & 1)
   int it = 0;
   for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
     TileInfo ti = get_tile(p, t);
     if (!ti.valid) continue;
     const int acc = it & 1;
     const uint32_t aph = (it >> 1) & 1;
-    const bool staged = kStaged && p.resid_tma && ti.nsplit == 1 && (ti.ncols & 63) == 0 &&
+    // (TMA boxes of 64 columns at a 16-byte aligned column)
+    const bool staged = kStaged && p.stage_tma && ti.nsplit == 1 && (ti.ncols & 63) == 0 && (ti.n0 & 7) == 0 &&
                         ti.m0 + q * 32 + 32 <= ti.m_end;
-    if (staged) {
+    if (staged && KIND == EPI_RESID) {
       // the first two chunks of this warp's rows of X, while the main loop runs
       if (lane == 0) {
         bulk_wait_read0();  // the previous tile's stores have read both buffers
@@ -767,6 +817,8 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
       } else {
         epilogue_tile<KIND, F8>(p, ti, row, rv, taddr);
       }
+    } else if (KIND == EPI_SWIGLU && staged) {
+      swiglu_tile_tma<F8>(p, ti, q, taddr, wst, sbuf);
     } else {
       epilogue_tile<KIND, F8>(p, ti, row, rv, taddr);
     }
@@ -774,7 +826,7 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
     mbar_arrive(&tempty[acc]);
     ++it;
   }
-  if (kStaged && lane == 0) bulk_wait0();  // this warp's residual stores are complete
+  if (kStaged && lane == 0) bulk_wait0();  // this warp's staged stores are complete
 }
 
 // ------------------------------------------------------------------ kernel
@@ -792,8 +844,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * NST + 4);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
   KsSync ks{bars + 2 * NST + 5, bars + 2 * NST + 6, reinterpret_cast<volatile int*>(bars + 2 * NST + 7), 0};
-  // EPI_RESID: the epilogue warps' residual chunk buffers and their barriers
-  constexpr bool kStaged = KIND == EPI_RESID && !THIN;
+  // EPI_RESID / EPI_SWIGLU: the epilogue warps' chunk buffers (and, for the
+  // residual loads, their barriers)
+  constexpr bool kStaged = (KIND == EPI_RESID || KIND == EPI_SWIGLU) && !THIN;
   uint64_t* rbar = bars + 2 * NST + 8;
   uint8_t* rstage = stages + NST * SBYTES + 1024;
   static_assert(!kStaged || (2 * NST + 16) * 8 <= 256, "barriers of the staged residual epilogue");
@@ -1141,7 +1194,7 @@ int gemm_pair_max_clusters(EpiKind kind) {
 template <int KIND, bool THIN>
 constexpr int gemm_smem() {
   return StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256 +
-         ((KIND == EPI_RESID && !THIN) ? 1024 - 256 + kResidStageBytes : 0);
+         (((KIND == EPI_RESID || KIND == EPI_SWIGLU) && !THIN) ? 1024 - 256 + kResidStageBytes : 0);
 }
 
 template <int KIND, bool F8 = false, bool THIN = false>

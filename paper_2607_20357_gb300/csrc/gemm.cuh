@@ -24,7 +24,7 @@ constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA + TMEM, warps 2-5 e
 constexpr int kAccCols = 256;      // fp32 columns per accumulator
 constexpr int kTmemCols = 512;     // two accumulators (epilogue overlaps the next tile)
 constexpr int kGemmSmem = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
-constexpr int kResidChunk = 32 * 128;             // one warp's 32 rows x 64 columns of bf16
+constexpr int kResidChunk = 32 * 128;             // one warp's 32 rows x 64 columns of bf16 (staged epilogues)
 constexpr int kResidStageBytes = 4 * 2 * kResidChunk;  // two chunk buffers per epilogue warp
 
 enum EpiKind : int {
@@ -99,12 +99,14 @@ struct GemmParams {
   // are readable 32 floats past their last column.
   const float* a_scale;
   const float* b_scale[3];
-  // EPI_RESID: the residual stream (out[0]) as a tensor map with boxes of 64
-  // columns x 32 rows. When resid_tma is set, each epilogue warp whose 32 rows
-  // of a tile all exist stages them through shared memory: TMA load of X,
-  // accumulator added, TMA store back (per-thread loads and stores otherwise).
+  // out[0] as a tensor map with boxes of 64 columns x 32 rows (EPI_RESID:
+  // the residual stream; EPI_SWIGLU: the hidden rows). When stage_tma is set,
+  // each epilogue warp whose 32 rows of a tile all exist stages them through
+  // shared memory: EPI_RESID loads X with TMA, adds the accumulator and stores
+  // back; EPI_SWIGLU writes its outputs and stores them with TMA (per-thread
+  // loads and stores otherwise).
   CUtensorMap mapR;
-  int resid_tma;
+  int stage_tma;
   uint32_t* status;
 };
 
