@@ -924,6 +924,8 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
       !make_map(&map_xr, X, t_cap, d.d_model, 32) ||  // residual stream, 32-row boxes (residual epilogues)
       !make_map(&map_hmo, hm, t_cap, d.d_ffn, 32))    // SwiGLU outputs, 32-row boxes (gate/up epilogue)
     return SVL_ERR_CUDA;
+  CUtensorMap map_q32, map_k32;  // Q and K, 32-row boxes (QKV epilogue)
+  if (!make_map(&map_q32, qb, t_cap, hq, 32) || !make_map(&map_k32, kb, t_cap, dkv, 32)) return SVL_ERR_CUDA;
   // e4m3: every gated GEMM reads the quantised rows of its input (aq, with
   // per-row scales as) -- X for QKV and gate/up, the attention output for
   // O, the SwiGLU output for down (both group-padded to whole K blocks)
@@ -1083,6 +1085,9 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.rope_cs = m->rope_cs;
     p.rope_rows = d.max_seq;
     p.d_head = dh;
+    p.mapR = map_q32;
+    p.mapR2 = map_k32;
+    p.stage_tma = 1;
     if ((st = pair ? launch_pair(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s)
                    : launch(EPI_QKV_ROPE, m, SVL_TAG_QKV, p, L.qkv_cap, s, f8, thin)) != SVL_OK)
       return st;

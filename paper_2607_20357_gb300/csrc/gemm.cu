@@ -750,14 +750,79 @@ SVL_DEVINL void swiglu_tile_tma(const GemmParams& p, const TileInfo& ti, int q, 
   }
 }
 
+// 32 bf16 values of this lane's row at column c (a multiple of 32) of the
+// warp's staging buffers: buffer c / 64, swizzled like the TMA box.
+SVL_DEVINL void stage_row32(uint8_t* wst, int c, const float* v) {
+  const int lane = threadIdx.x & 31;
+  uint8_t* prow = wst + (c >> 6) * kResidChunk + lane * 128;
+  const int pos0 = (c & 63) >> 3;
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    *reinterpret_cast<uint4*>(prow + (((pos0 + i) ^ (lane & 7)) << 4)) =
+        make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                   pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+}
+
+// EPI_QKV_ROPE, Q and K, through shared memory, for a warp whose 32 rows of
+// the tile all exist and heads of a multiple of 64 columns: per head, the
+// rotated rows go into the warp's buffers (head columns [0, 64) in the
+// first, [64, 128) in the second) and one TMA store per 64 columns writes
+// them, once the previous head's stores have read the buffers.
+template <bool F8>
+SVL_DEVINL void qkv_tile_tma(const GemmParams& p, const TileInfo& ti, int q, uint32_t taddr, uint8_t* wst) {
+  const int lane = threadIdx.x & 31;
+  const int row = ti.m0 + q * 32 + lane;
+  const float af = F8 ? p.a_scale[row] : 1.f;
+  const float rs = (p.ss_in ? row_rms_scale(p, row) : 1.f) * af;
+  const float* bsc = F8 ? p.b_scale[ti.mat] + ti.n0 : nullptr;
+  const CUtensorMap* map = ti.mat == 0 ? &p.mapR : &p.mapR2;
+  const int dh = p.d_head, half = dh / 2;
+  int prow = p.pos[row];
+  if (prow < 0 || prow >= p.rope_rows) {  // longer than the model's max_seq
+    report(p.status, SVL_DEV_BAD_INDEX);
+    prow = 0;
+  }
+  const float2* cs = p.rope_cs + prow;  // frequency i at cs[i * rope_rows]
+  for (int hb = 0; hb < ti.ncols; hb += dh) {
+    if (lane == 0) bulk_wait_read0();  // the previous head's stores have read the buffers
+    __syncwarp();
+#pragma unroll 1
+    for (int i0 = 0; i0 < half; i0 += 32) {
+      float v[32], w[32];
+      tmem_ld32(taddr + hb + i0, v);
+      tmem_ld32(taddr + hb + half + i0, w);
+      if constexpr (F8) {
+        scale_cols(v, bsc + hb + i0, 1.f);
+        scale_cols(w, bsc + hb + half + i0, 1.f);
+      }
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const float2 c = cs[static_cast<size_t>(i0 + j) * p.rope_rows];
+        const float x1 = v[j] * rs, x2 = w[j] * rs;
+        v[j] = x1 * c.x - x2 * c.y;
+        w[j] = x2 * c.x + x1 * c.y;
+      }
+      stage_row32(wst, i0, v);
+      stage_row32(wst, half + i0, w);
+    }
+    fence_proxy_async();  // generic-proxy writes, read by the TMA unit
+    __syncwarp();
+    if (lane == 0) {
+      for (int k = 0; k < dh / 64; ++k)
+        tma_store_2d(map, wst + k * kResidChunk, ti.n0 + hb + 64 * k, ti.m0 + q * 32);
+      bulk_commit();
+    }
+  }
+}
+
 template <int KIND, bool F8, bool THIN>
 SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* tempty, uint32_t tmem,
                               volatile int* abort, KsSync& ks, uint8_t* rstage, uint64_t* rbar) {
   const int ntiles = num_tiles(p);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int q = warp & 3;  // TMEM lane quarter this warp may access
-  // residual (EPI_RESID) or outputs (EPI_SWIGLU) through shared memory
-  constexpr bool kStaged = (KIND == EPI_RESID || KIND == EPI_SWIGLU) && !THIN;
+  // residual (EPI_RESID) or outputs (EPI_SWIGLU, EPI_QKV_ROPE) through shared memory
+  constexpr bool kStaged = (KIND == EPI_RESID || KIND == EPI_SWIGLU || KIND == EPI_QKV_ROPE) && !THIN;
   uint8_t* wst = kStaged ? rstage + q * 2 * kResidChunk : nullptr;
   uint64_t* wbar = kStaged ? rbar + 2 * q : nullptr;
   uint32_t rpar = 0;  // EPI_RESID: parity of each buffer's next wait
@@ -819,6 +884,8 @@ SVL_DEVINL void epilogue_loop(const GemmParams& p, uint64_t* tfull, uint64_t* te
       }
     } else if (KIND == EPI_SWIGLU && staged) {
       swiglu_tile_tma<F8>(p, ti, q, taddr, wst, sbuf);
+    } else if (KIND == EPI_QKV_ROPE && staged && ti.mat < 2 && (p.d_head & 63) == 0) {
+      qkv_tile_tma<F8>(p, ti, q, taddr, wst);
     } else {
       epilogue_tile<KIND, F8>(p, ti, row, rv, taddr);
     }
@@ -844,9 +911,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1) gemm_kernel(const __grid_cons
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * NST + 4);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
   KsSync ks{bars + 2 * NST + 5, bars + 2 * NST + 6, reinterpret_cast<volatile int*>(bars + 2 * NST + 7), 0};
-  // EPI_RESID / EPI_SWIGLU: the epilogue warps' chunk buffers (and, for the
-  // residual loads, their barriers)
-  constexpr bool kStaged = (KIND == EPI_RESID || KIND == EPI_SWIGLU) && !THIN;
+  // EPI_RESID / EPI_SWIGLU / EPI_QKV_ROPE: the epilogue warps' chunk buffers
+  // (and, for the residual loads, their barriers)
+  constexpr bool kStaged = (KIND == EPI_RESID || KIND == EPI_SWIGLU || KIND == EPI_QKV_ROPE) && !THIN;
   uint64_t* rbar = bars + 2 * NST + 8;
   uint8_t* rstage = stages + NST * SBYTES + 1024;
   static_assert(!kStaged || (2 * NST + 16) * 8 <= 256, "barriers of the staged residual epilogue");
@@ -1194,7 +1261,8 @@ int gemm_pair_max_clusters(EpiKind kind) {
 template <int KIND, bool THIN>
 constexpr int gemm_smem() {
   return StageCfg<KIND, THIN>::stages * StageCfg<KIND, THIN>::bytes + 1024 + 256 +
-         (((KIND == EPI_RESID || KIND == EPI_SWIGLU) && !THIN) ? 1024 - 256 + kResidStageBytes : 0);
+         (((KIND == EPI_RESID || KIND == EPI_SWIGLU || KIND == EPI_QKV_ROPE) && !THIN) ? 1024 - 256 + kResidStageBytes
+                                                                                      : 0);
 }
 
 template <int KIND, bool F8 = false, bool THIN = false>

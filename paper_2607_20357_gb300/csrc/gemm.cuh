@@ -100,12 +100,14 @@ struct GemmParams {
   const float* a_scale;
   const float* b_scale[3];
   // out[0] as a tensor map with boxes of 64 columns x 32 rows (EPI_RESID:
-  // the residual stream; EPI_SWIGLU: the hidden rows). When stage_tma is set,
-  // each epilogue warp whose 32 rows of a tile all exist stages them through
-  // shared memory: EPI_RESID loads X with TMA, adds the accumulator and stores
-  // back; EPI_SWIGLU writes its outputs and stores them with TMA (per-thread
-  // loads and stores otherwise).
+  // the residual stream; EPI_SWIGLU: the hidden rows; EPI_QKV_ROPE: Q, and K
+  // in mapR2). When stage_tma is set, each epilogue warp whose 32 rows of a
+  // tile all exist stages them through shared memory: EPI_RESID loads X with
+  // TMA, adds the accumulator and stores back; EPI_SWIGLU and EPI_QKV_ROPE (Q
+  // and K) write their outputs and store them with TMA (per-thread loads and
+  // stores otherwise, and for V^T).
   CUtensorMap mapR;
+  CUtensorMap mapR2;  // EPI_QKV_ROPE: mapR holds Q (mat 0), mapR2 K (mat 1)
   int stage_tma;
   uint32_t* status;
 };
