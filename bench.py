@@ -237,7 +237,7 @@ def executed_flops(svl, desc, k, s_text, n_vis, lg, gg):
     return tot
 
 
-TRAFFIC_SOURCES = ("gemm.cu", "decoder.cu", "kernels.cuh")  # the GEMM and its tile order
+TRAFFIC_SOURCES = ("gemm.cu", "decoder.cu", "kernels.cuh", "api.cu")  # the GEMM and its tile order
 
 
 def traffic_source_hash():

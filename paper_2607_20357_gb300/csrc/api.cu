@@ -870,6 +870,10 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
   sa.dh = dh;
   sa.D = d.d_model;
   sa.Di = d.d_ffn;
+  {
+    const long long row_bytes = static_cast<long long>(sa.nsparse_rows) * d.d_model * (m->e4m3 ? 1 : 2);
+    sa.mband = static_cast<int>(std::max<long long>(1, kMBandBytes / row_bytes));
+  }
   sa.cu_seqlens = cu_seqlens;
   sa.layer_gate = layer_gate;
   sa.group_gate = group_gate;
@@ -1166,6 +1170,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ld[0] = d.d_model;
     p.mapR = map_xr;
     p.stage_tma = 1;
+    p.a_evict_first = 1;  // n-band list: the weights stay in L2, the input rows stream
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l) * L.ks_units;
@@ -1223,6 +1228,7 @@ svl_status prefill_impl(svl_model* m, int32_t B, int32_t t_cap, void* X, const i
     p.ld[0] = d.d_model;
     p.mapR = map_xr;
     p.stage_tma = 1;
+    p.a_evict_first = 1;  // n-band list: the weights stay in L2, the input rows stream
     p.ks_info = sa.ks_info + static_cast<size_t>(l) * 8 + 4;
     p.ks_part = at<float>(ws, L.ks_part);
     p.ks_ticket = ks_ticket + static_cast<size_t>(2 * l + 1) * L.ks_units;

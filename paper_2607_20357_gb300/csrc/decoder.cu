@@ -39,19 +39,30 @@ SVL_DEVINL int build_runs(NTile* out, int cnt, int mask, int G, int width, int s
   return cnt;
 }
 
-// Emits mt x nt tiles of one segment, n-tiles in bands of `nband` (a band
-// sweeps all m-tiles before the next band starts, so concurrent CTAs share
-// the same weight columns in L2).
+// Emits mt x nt tiles of one segment in raster bands. mband > 0: bands of
+// `mband` m-tiles, each sweeping all n-tiles while its input rows stay in L2
+// (the tiles of one n-tile follow each other, so concurrent CTAs share its
+// weights too). Otherwise bands of `nband` n-tiles, each sweeping all m-tiles
+// while its weight columns stay in L2.
 __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const NTile* nt, int n_nt, int kmask,
-                           uint32_t* status, int bm = kBM_SCHED, int nband = kNBand) {
+                           uint32_t* status, int bm = kBM_SCHED, int nband = kNBand, int mband = 0) {
   const int mt = (r1 - r0 + bm - 1) / bm;
   const int total = mt * n_nt;
   for (int t = threadIdx.x; t < total; t += blockDim.x) {
-    const int band = t / (mt * nband);
-    const int rem = t - band * mt * nband;
-    const int bw = min(nband, n_nt - band * nband);
-    const int mi = rem / bw;
-    const int ni = band * nband + rem % bw;
+    int mi, ni;
+    if (mband > 0) {
+      const int band = t / (mband * n_nt);
+      const int rem = t - band * mband * n_nt;
+      const int bh = min(mband, mt - band * mband);
+      ni = rem / bh;
+      mi = band * mband + rem % bh;
+    } else {
+      const int band = t / (mt * nband);
+      const int rem = t - band * mt * nband;
+      const int bw = min(nband, n_nt - band * nband);
+      mi = rem / bw;
+      ni = band * nband + rem % bw;
+    }
     const int m0 = r0 + mi * bm;
     const int idx = base + t;
     if (idx >= cap) {
@@ -124,7 +135,7 @@ SVL_DEVINL bool group_on(const SchedShared& sh, int b, int j) { return (sh.mask[
 // Called by the whole block; thread 0 walks groups and samples.
 template <class Cols>
 __device__ int emit_group_runs(const ScheduleArgs& a, const SchedShared& sh, int4* tiles, int cap, NTile* nt,
-                               int* s_nnt, int* s_run, Cols cols, int nband) {
+                               int* s_nnt, int* s_run, Cols cols) {
   const int tid = threadIdx.x, B = a.B, G = a.G;
   int off = 0;
   int j0 = 0;
@@ -165,7 +176,7 @@ __device__ int emit_group_runs(const ScheduleArgs& a, const SchedShared& sh, int
       __syncthreads();
       const int r0 = s_run[0], r1 = s_run[1];
       if (r0 < 0) break;
-      emit_tiles(tiles, off, cap, r0, r1, nt, *s_nnt, 0, a.status, a.nsparse_rows, nband);
+      emit_tiles(tiles, off, cap, r0, r1, nt, *s_nnt, 0, a.status, a.nsparse_rows, 0, a.mband);
       off += ((r1 - r0 + a.nsparse_rows - 1) / a.nsparse_rows) * *s_nnt;
       __syncthreads();
     }
@@ -227,7 +238,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     return build_runs(out, c, mask, G, hk, 256, 2);
   };
   int off = emit_group_runs(a, sh, a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, a.qkv_cap, nt, &s_nnt, s_run,
-                            qkv_cols, kNBandQkv);
+                            qkv_cols);
   __syncthreads();
   if (tid == 0)
     a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, a.nsparse_wave, a.dh);
@@ -264,8 +275,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     const int mask = ((1 << (j1 + 1)) - 1) & ~((1 << j0) - 1);
     return build_runs(out, 0, mask, G, a.Di / G, 128, 0);
   };
-  off = emit_group_runs(a, sh, a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, a.gu_cap, nt, &s_nnt, s_run, gu_cols,
-                        kNBandGateUp);
+  off = emit_group_runs(a, sh, a.gu_tiles + static_cast<size_t>(l) * a.gu_cap, a.gu_cap, nt, &s_nnt, s_run, gu_cols);
   __syncthreads();
   if (tid == 0) a.gu_count[l] = off;
 

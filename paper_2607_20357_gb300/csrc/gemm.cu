@@ -143,6 +143,7 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
   constexpr int BK = F8 ? kBK8 : kBK;
   const int ntiles = num_tiles(p);
   const int nkb = p.K / BK, kgb = p.kgroup / BK;
+  const uint64_t pol = l2_evict_first_policy();
   int s = 0;
   uint32_t ph = 0;
   for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
@@ -167,7 +168,10 @@ SVL_DEVINL void producer_loop(const GemmParams& p, uint8_t* stages, uint64_t* fu
       uint8_t* sa = stages + s * SBYTES;
       uint8_t* sb = sa + ABYTES;
       mbar_arrive_expect_tx(&full[s], bytes);
-      tma_load_2d(sa, &p.mapA, &full[s], kb * BK, ti.m0);
+      if (p.a_evict_first)
+        tma_load_2d_hint(sa, &p.mapA, &full[s], kb * BK, ti.m0, pol);
+      else
+        tma_load_2d(sa, &p.mapA, &full[s], kb * BK, ti.m0);
       tma_load_2d(sb, mb0, &full[s], kb * BK, ti.n0);
       if (halves == 2) tma_load_2d(sb + kBHalfBytes, mb1, &full[s], kb * BK, y1);
       if (++s == NST) {

@@ -109,6 +109,10 @@ struct GemmParams {
   CUtensorMap mapR;
   CUtensorMap mapR2;  // EPI_QKV_ROPE: mapR holds Q (mat 0), mapR2 K (mat 1)
   int stage_tma;
+  // 1: A loads with the L2 evict_first policy. The n-band lists of the
+  // residual GEMMs keep a band of weights in L2 while the input rows stream
+  // through; this keeps the rows from pushing the band out.
+  int a_evict_first;
   uint32_t* status;
 };
 

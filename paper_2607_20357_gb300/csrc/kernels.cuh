@@ -7,16 +7,21 @@ namespace svl {
 
 constexpr int kSelectThreads = 512;
 constexpr int kAttnQ = 256;       // query rows per attention work item (the kernel runs its two 128-row halves as units)
-// n-tiles per raster band of a tile list. A band sweeps all m-tiles while its
-// weight columns stay in L2, so the input rows are read once per band: wider
-// bands read them fewer times until the band's weights (band x 256 rows x K)
-// no longer stay in L2. At LLaVA-7B widths the QKV list has 48 n-tiles and
-// the gate/up list 86; 16 and 20 minimise their DRAM traffic (gate/up: 1.32
-// GB per b = 1 launch with bands of 8, 0.85 GB with 20, 2.0 GB with 32).
+// n-tiles per raster band of the residual GEMMs' tile lists (O, down). A band
+// sweeps all m-tiles while its weight columns stay in L2, so the input rows
+// are read once per band: wider bands read them fewer times until the band's
+// weights (band x 256 rows x K) no longer stay in L2 (about 45 MB).
 constexpr int kNBand = 8;         // down list (16 n-tiles of 256 x 11,008 weights)
 constexpr int kNBandO = 16;       // O list (16 n-tiles of 256 x 4,096 weights: one band)
-constexpr int kNBandQkv = 16;
-constexpr int kNBandGateUp = 20;
+// The N-sparse lists (QKV, gate/up) run in bands of m-tiles whose input rows
+// total at most this many bytes: a band sweeps all n-tiles while its rows
+// stay in L2, so the rows are read once and the weights once per band. At
+// LLaVA-7B widths and b = 1 the 84 MB of rows make two bands (gate/up: 0.71
+// GB of DRAM traffic per launch, against 0.87 GB in bands of 20 n-tiles and
+// 0.84 GB with 27 MB of rows per band); a batch whose rows fit in one band
+// reads everything once. 100 MB of rows in one band no longer stay in L2
+// (4.2 GB).
+constexpr long long kMBandBytes = 40ll << 20;
 constexpr int kBM_SCHED = 128;    // tile rows (the GEMM's M)
 
 struct SelectArgs {
@@ -149,6 +154,7 @@ struct ScheduleArgs {
   int num_sms;              // CTAs of the persistent GEMM (one wave of tiles)
   int nsparse_rows;         // rows per tile of the QKV and gate/up lists (128, or 256 for CTA pairs)
   int nsparse_wave;         // tiles of those lists that run at once (CTAs, or CTA pairs)
+  int mband;                // m-tiles per raster band of those lists (see kMBandBytes)
   int A, Akv, dh, D, Di;
   const int* cu_seqlens;
   const uint8_t* layer_gate;
