@@ -78,21 +78,40 @@ __device__ void emit_tiles(int4* tiles, int base, int cap, int r0, int r1, const
 // at most half full, each of its tiles is cut into two half-width tiles
 // (which then still fit in one wave and finish in about half the time).
 // `head` > 0: halves must hold whole heads of that width (RoPE epilogue).
-// Runs on one thread after the list is complete; returns the new count.
-__device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head) {
+// Called by the whole block once the list is complete; the appended halves
+// keep the order of their tiles (a ballot prefix over the eligible ones).
+// s_scan: blockDim.x / 32 ints of shared memory. Returns the new count.
+__device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head, int* s_scan) {
   const int r = count % num_sms;
   if (r == 0 || 2 * r > num_sms) return count;
-  int added = 0;
-  for (int i = count - r; i < count; ++i) {
-    const int4 t = tiles[i];
-    const int nc = t.w & 0xFFFF;
-    const int half = nc / 2;
-    if (nc < 64 || (half & 15) || (head > 0 && half % head) || count + added >= cap) continue;
-    tiles[i] = make_int4(t.x, t.y, t.z, (t.w & ~0xFFFF) | half);
-    tiles[count + added] = make_int4(t.x, t.y, t.z + half, (t.w & ~0xFFFF) | (nc - half));
-    ++added;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  int eligible = 0;  // in the chunks before this one
+  for (int c0 = count - r; c0 < count; c0 += blockDim.x) {
+    const int i = c0 + static_cast<int>(threadIdx.x);
+    int4 t = make_int4(0, 0, 0, 0);
+    bool e = false;
+    if (i < count) {
+      t = tiles[i];
+      const int nc = t.w & 0xFFFF, half = nc / 2;
+      e = nc >= 64 && !(half & 15) && !(head > 0 && half % head);
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, e);
+    if (lane == 0) s_scan[warp] = __popc(bal);
+    __syncthreads();
+    int before = eligible + __popc(bal & ((1u << lane) - 1u)), chunk = 0;
+    for (int w = 0; w < nw; ++w) {
+      if (w < warp) before += s_scan[w];
+      chunk += s_scan[w];
+    }
+    __syncthreads();  // s_scan is reused by the next chunk
+    if (e && count + before < cap) {
+      const int nc = t.w & 0xFFFF, half = nc / 2;
+      tiles[i] = make_int4(t.x, t.y, t.z, (t.w & ~0xFFFF) | half);
+      tiles[count + before] = make_int4(t.x, t.y, t.z + half, (t.w & ~0xFFFF) | (nc - half));
+    }
+    eligible += chunk;
   }
-  return count + added;
+  return count + min(eligible, cap - count);
 }
 
 // Residual GEMMs (O, down) cut the tiles of a last wave that is at most half
@@ -100,20 +119,20 @@ __device__ int split_tail(int4* tiles, int count, int cap, int num_sms, int head
 // num_sms / r, at most 8, within the list capacity and the partial buffer),
 // the copies compute shares of the tile's K blocks side by side in that wave
 // and the last to finish sums them. Full-width tiles keep the tensor core's
-// widest MMAs. Writes {first copy index, r, s} to info; returns the count.
+// widest MMAs. Called by the whole block once the list is complete; thread 0
+// writes {first copy index, r, s} to info. Returns the count.
 __device__ int split_k_tail(int4* tiles, int count, int cap, int num_sms, int units, int* info) {
-  info[0] = count;
-  info[1] = 0;
-  info[2] = 1;
   const int sp = ksplit_shares(count, cap, num_sms, units);
-  if (sp < 2) return count;
-  const int r = count % num_sms;
+  const int r = sp < 2 ? 0 : count % num_sms;
   const int first = count - r;
-  for (int part = 1; part < sp; ++part)
-    for (int i = 0; i < r; ++i) tiles[count + (part - 1) * r + i] = tiles[first + i];
-  info[0] = first;
-  info[1] = r;
-  info[2] = sp;
+  if (threadIdx.x == 0) {
+    info[0] = first;
+    info[1] = r;
+    info[2] = sp < 2 ? 1 : sp;
+  }
+  if (sp < 2) return count;
+  // copy `part` (1 .. sp-1) of tail tile i goes to count + (part - 1) r + i
+  for (int idx = threadIdx.x; idx < r * (sp - 1); idx += blockDim.x) tiles[count + idx] = tiles[first + idx % r];
   return count + r * (sp - 1);
 }
 
@@ -191,6 +210,7 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   __shared__ int s_nseg, s_nnt;
   __shared__ int s_heads[256];
   __shared__ int s_run[4];
+  __shared__ int s_scan[8];  // per-warp counts of split_tail (256 threads)
   pdl_trigger();
   pdl_wait();
   extern __shared__ int sched_dyn[];
@@ -240,8 +260,8 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
   int off = emit_group_runs(a, sh, a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, a.qkv_cap, nt, &s_nnt, s_run,
                             qkv_cols);
   __syncthreads();
-  if (tid == 0)
-    a.qkv_count[l] = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, a.nsparse_wave, a.dh);
+  off = split_tail(a.qkv_tiles + static_cast<size_t>(l) * a.qkv_cap, off, a.qkv_cap, a.nsparse_wave, a.dh, s_scan);
+  if (tid == 0) a.qkv_count[l] = off;
 
   // ---- O projection (K-sparse: kmask = segment mask), all D columns
   off = 0;
@@ -254,9 +274,9 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
   }
   __syncthreads();
-  if (tid == 0)
-    a.o_count[l] = split_k_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms,
-                                a.ks_units, a.ks_info + static_cast<size_t>(l) * 8);
+  off = split_k_tail(a.o_tiles + static_cast<size_t>(l) * a.o_cap, min(off, a.o_cap), a.o_cap, a.num_sms, a.ks_units,
+                     a.ks_info + static_cast<size_t>(l) * 8);
+  if (tid == 0) a.o_count[l] = off;
   // ---- down projection: same tiles shape as O
   off = 0;
   for (int s = 0; s < nseg; ++s) {
@@ -265,9 +285,9 @@ __global__ void __launch_bounds__(256) schedule_kernel(ScheduleArgs a) {
     off += ((sg.y - sg.x + kBM_SCHED - 1) / kBM_SCHED) * s_nnt;
   }
   __syncthreads();
-  if (tid == 0)
-    a.dn_count[l] = split_k_tail(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, min(off, a.dn_cap), a.dn_cap,
-                                 a.num_sms, a.ks_units, a.ks_info + static_cast<size_t>(l) * 8 + 4);
+  off = split_k_tail(a.dn_tiles + static_cast<size_t>(l) * a.dn_cap, min(off, a.dn_cap), a.dn_cap, a.num_sms,
+                     a.ks_units, a.ks_info + static_cast<size_t>(l) * 8 + 4);
+  if (tid == 0) a.dn_count[l] = off;
   __syncthreads();
 
   // ---- gate/up (N-sparse over active FFN channels, 128 per tile, per group block)
